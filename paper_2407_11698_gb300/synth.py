@@ -1,0 +1,36 @@
+"""Seeded synthetic inputs shared by the tests, the smoke check and the benchmark.
+
+Holds none of the method's arithmetic: only the recipe for the integer images
+and labels that stand in for MNIST / FashionMNIST / CIFAR-10 (Sec. 4 shapes:
+28x28x1 and 32x32x3 images, G = 10 classes).  Images are int8 uniform on
+[-128, 127]; labels uniform on [0, G).  Batch ``step`` of a run seeded with
+``seed`` comes from numpy's PCG64 seeded by the pair (seed, step), so any step
+can be regenerated on its own.
+"""
+import numpy as np
+
+
+def _rng(seed: int, step: int, stream: int) -> np.random.Generator:
+    return np.random.Generator(np.random.PCG64(np.random.SeedSequence([seed, step, stream])))
+
+
+def images(seed: int, step: int, batch: int, shape) -> np.ndarray:
+    """int8 images of shape (batch, *shape), NHWC, uniform on [-128, 127]."""
+    return _rng(seed, step, 0).integers(-128, 128, size=(batch, *shape), dtype=np.int8)
+
+
+def labels(seed: int, step: int, batch: int, num_classes: int = 10) -> np.ndarray:
+    """int32 class labels uniform on [0, num_classes)."""
+    return _rng(seed, step, 1).integers(0, num_classes, size=(batch,), dtype=np.int32)
+
+
+def gaussian_images(seed: int, step: int, batch: int, shape, sigma: float = 64.0) -> np.ndarray:
+    """int8 images drawn as round(N(0, sigma^2)) clamped to [-128, 127]: the
+    distribution App. A's preprocessing aims for (mean 0, sigma 64)."""
+    x = np.rint(_rng(seed, step, 2).normal(0.0, sigma, size=(batch, *shape)))
+    return np.clip(x, -128, 127).astype(np.int8)
+
+
+def int_tensor(seed: int, shape, lo: int, hi: int, stream: int = 3) -> np.ndarray:
+    """int64 tensor uniform on [lo, hi] (inclusive), for kernel-level tests."""
+    return _rng(seed, 0, stream).integers(lo, hi + 1, size=shape, dtype=np.int64)
