@@ -1,0 +1,383 @@
+#!/usr/bin/env python
+"""Benchmark of the NITRO-D integer training step on GB300.
+
+One step = forward of every block, every block's local backward and every
+IntegerSGD update (the full local-loss block step) on one batch of synthetic
+int8 images resident in HBM, for the VGG-style workload (3 blocks of two 3x3
+convs 64/128/256 with max-pool + an output block, batch 128, 32x32x3 inputs).
+
+Prints ONE JSON line on rank 0.  Multi-GPU runs (torchrun) train independent
+replicas, one per GPU (the step has no exchange; weak scaling).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+"""
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "int training images/s at 1 GB300; int conv TOPS as % of dense int8 peak"
+WORKLOAD = "vgg_64_128_256_b128"
+L2_FLUSH_BYTES = 512 << 20          # > 129 MB L2
+
+
+def parse():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=20)
+    p.add_argument("--warmup", type=int, default=5)
+    p.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    p.add_argument("--workload", default=WORKLOAD)
+    p.add_argument("--no-graph", action="store_true")
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--profile-steps", type=int, default=3)
+    return p.parse_args()
+
+
+def measured_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return json.load(f), "measured"
+    except OSError:
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}, "fallback"
+
+
+# ------------------------------------------------------------------ clocks
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+        self.lines = []
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), "--query-gpu=" + self.FIELDS,
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except OSError:
+            self.proc = None
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def __exit__(self, *a):
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in self.lines:
+            parts = [t.strip() for t in line.split(",")]
+            if len(parts) < 7:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                mx.append(float(parts[1]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[3:7]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ------------------------------------------------------------------ our step
+class GpuNet:
+    def __init__(self, wl, seed, torch, nb):
+        self.torch, self.nb = torch, nb
+        B = wl["batch"]
+        self.B = B
+        self.blocks = [nb.Block(b["layers"], b["in_features"], seed=seed + i, max_batch=B)
+                       for i, b in enumerate(wl["blocks"])]
+        from paper_2407_11698_gb300 import synth
+        x = synth.images(seed, 0, B, wl["input_shape"]).reshape(B, -1)
+        y = synth.labels(seed, 0, B)
+        self.x = torch.from_numpy(x).cuda()
+        self.y = torch.from_numpy(y).cuda()
+        self.acts = [self.x]
+        for g in self.blocks:
+            self.acts.append(torch.empty((B, g.out_features), dtype=torch.int8, device="cuda")
+                             if g.layers else self.acts[-1])
+        self.loss = torch.zeros((len(self.blocks),), dtype=torch.int64, device="cuda")
+        self.in_bytes = self.x.numel() + 4 * self.y.numel()
+
+    def step(self, x=None, y=None, loss=None):
+        x = self.x if x is None else x
+        y = self.y if y is None else y
+        loss = self.loss if loss is None else loss
+        acts = [x] + self.acts[1:]
+        for i, g in enumerate(self.blocks):
+            g.forward(acts[i], acts[i + 1] if g.layers else None)
+        for i, g in enumerate(self.blocks):
+            g.backward(acts[i], y, loss[i:i + 1])
+        for g in self.blocks:
+            g.sgd()
+
+
+def kernel_profile(nb):
+    import ctypes
+    L = nb.lib()
+    out = {}
+    for k in range(L.nitro_profile_kernel_count()):
+        n, ms, ops, by = ctypes.c_uint64(), ctypes.c_double(), ctypes.c_double(), ctypes.c_double()
+        st = L.nitro_profile_read(k, ctypes.byref(n), ctypes.byref(ms), ctypes.byref(ops), ctypes.byref(by))
+        if st == 0 and n.value:
+            out[L.nitro_profile_kernel_name(k).decode()] = dict(
+                launches=n.value, ms=ms.value, ops=ops.value, bytes=by.value)
+    return out
+
+
+def run_ours(args, rank, world, local_rank):
+    import torch
+    import torch.distributed as dist
+    from paper_2407_11698_gb300 import binding as nb
+    from paper_2407_11698_gb300 import workloads as WL
+
+    torch.cuda.set_device(local_rank)
+    nb.lib()
+    wl = WL.WORKLOADS[args.workload]
+    net = GpuNet(wl, 20240716 + 7 * rank, torch, nb)
+    stream = torch.cuda.current_stream()
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device="cuda")
+
+    for _ in range(args.warmup):
+        net.step()
+    torch.cuda.synchronize()
+
+    # launches per step (host-side counter around one eager step)
+    L = nb.lib()
+    c0 = L.nitro_kernel_launches()
+    net.step()
+    torch.cuda.synchronize()
+    launches_per_step = L.nitro_kernel_launches() - c0
+
+    graph = None
+    if not args.no_graph:
+        graph = torch.cuda.CUDAGraph()
+        side = torch.cuda.Stream()
+        side.wait_stream(stream)
+        with torch.cuda.stream(side):
+            with torch.cuda.graph(graph, stream=side):
+                net.step()
+        stream.wait_stream(side)
+        for _ in range(2):
+            graph.replay()
+        torch.cuda.synchronize()
+
+    def one():
+        if graph is not None:
+            graph.replay()
+        else:
+            net.step()
+
+    # ---------------- headline timed region: K steps, L2 flushed between steps
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(args.steps)]
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(local_rank) as clocks:
+        t_wall = time.perf_counter()
+        for i in range(args.steps):
+            flush.zero_()
+            ev[i][0].record(stream)
+            one()
+            ev[i][1].record(stream)
+        torch.cuda.synchronize()
+        t_wall = time.perf_counter() - t_wall
+        if t_wall < 1.0:      # keep sampling long enough for a clock reading
+            time.sleep(1.0 - t_wall)
+    if world > 1:
+        dist.barrier()
+    step_ms = [a.elapsed_time(b) for a, b in ev]
+    total_ms = sum(step_ms)
+    t = torch.tensor([total_ms], dtype=torch.float64, device="cuda")
+    if world > 1:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    total_ms = float(t.item())
+    value = world * net.B * args.steps / (total_ms / 1e3)
+
+    # ---------------- end to end through the public API, host buffers
+    from paper_2407_11698_gb300 import synth
+    xh = torch.from_numpy(synth.images(3, 0, net.B, wl["input_shape"]).reshape(net.B, -1)).pin_memory()
+    yh = torch.from_numpy(synth.labels(3, 0, net.B)).pin_memory()
+    lh = torch.empty((len(net.blocks),), dtype=torch.int64).pin_memory()
+    xd, yd = torch.empty_like(net.x), torch.empty_like(net.y)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        xd.copy_(xh, non_blocking=True)
+        yd.copy_(yh, non_blocking=True)
+        net.step(xd, yd)
+        lh.copy_(net.loss, non_blocking=True)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = e0.elapsed_time(e1)
+    t = torch.tensor([e2e_ms], dtype=torch.float64, device="cuda")
+    if world > 1:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    e2e_value = world * net.B * args.steps / (float(t.item()) / 1e3)
+
+    # ---------------- per-kernel device time inside eager steps (roofline)
+    L.nitro_profile_reset()
+    L.nitro_profile_enable(1)
+    for _ in range(args.profile_steps):
+        flush.zero_()
+        net.step()
+    torch.cuda.synchronize()
+    L.nitro_profile_enable(0)
+    prof = kernel_profile(nb)
+    L.nitro_profile_reset()
+
+    if rank != 0:
+        return None
+    peaks, peak_src = measured_peaks()
+    total_k = sum(v["ms"] for v in prof.values()) or 1.0
+    dom_name, dom = max(prof.items(), key=lambda kv: kv[1]["ms"])
+    per_launch_ms = dom["ms"] / dom["launches"]
+    if dom["ops"] > 0:
+        if dom_name.startswith("tc_"):
+            bound, peak, unit = "tensor", peaks["bf16_tflops_sustained"], "TFLOP/s"
+            peak_note = "bf16 dense, %s (sustained): the contraction runs as exact bf16 MMAs" % peak_src
+        else:
+            # CUDA-core int64 MACs: 152 SMs x 64 IMAD/clk x 2 ops x 2.07 GHz
+            bound, peak, unit = "alu", 152 * 64 * 2 * 2.07e9 / 1e12, "TOPS"
+            peak_note = "derived: 152 SMs x 64 int32 IMAD/clk x 2 ops x 2070 MHz"
+        achieved = dom["ops"] / dom["launches"] / (per_launch_ms / 1e3) / 1e12
+    else:
+        bound, peak, unit = "hbm", peaks["hbm_gbs"], "GB/s"
+        peak_note = "HBM copy, %s" % peak_src
+        achieved = dom["bytes"] / dom["launches"] / (per_launch_ms / 1e3) / 1e9
+    conv_ops = sum(v["ops"] for k, v in prof.items() if "conv" in k)
+    conv_ms = sum(v["ms"] for k, v in prof.items() if "conv" in k)
+    line = {
+        "metric": METRIC,
+        "value": round(value, 2),
+        "unit": "images/s",
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": round(total_ms / args.steps, 4),
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "int8/int32->int64",
+        "data": "synthetic",
+        "config": {"workload": args.workload, "batch": net.B,
+                   "input": "x".join(str(v) for v in wl["input_shape"]) + " int8 uniform [-128,127]",
+                   "blocks": len(wl["blocks"]), "cuda_graph": graph is not None,
+                   "l2": "flushed (512 MiB write) between timed steps",
+                   "parallelism": "replicas" if world > 1 else "single"},
+        "e2e": {"value": round(e2e_value, 2), "unit": "images/s",
+                "h2d_bytes_per_step": int(net.in_bytes),
+                "d2h_bytes_per_step": int(8 * len(net.blocks))},
+        "gpu_launches": int(launches_per_step * args.steps),
+        "roofline": {"bound": bound, "kernel": dom_name, "achieved": round(achieved, 3),
+                     "peak": round(peak, 2), "unit": unit, "frac": round(achieved / peak, 4),
+                     "traffic": None, "peak_source": peak_note,
+                     "per_launch_ms": round(per_launch_ms, 5),
+                     "share_of_kernel_time": round(dom["ms"] / total_k, 4)},
+        "conv_tops": round(conv_ops / (conv_ms / 1e3) / 1e12, 3) if conv_ms else None,
+        "kernels": {k: {"launches": v["launches"], "ms": round(v["ms"], 4),
+                        "share": round(v["ms"] / total_k, 4)} for k, v in sorted(prof.items())},
+        "clocks": clocks.summary(),
+    }
+    return line
+
+
+# ------------------------------------------------------------------ oracle (CPU)
+def oracle_rate(wl_name, sample_batch, steps, warmup=0):
+    """images/s of the CPU oracle training `steps` steps of the workload at a
+    reduced batch (the sample); returns (value, seconds, threads)."""
+    import numpy as np
+    import oracle as O
+    from paper_2407_11698_gb300 import synth
+    from paper_2407_11698_gb300 import workloads as WL
+    wl = WL.WORKLOADS[wl_name]
+    blocks = [O.OracleBlock([O.LayerDesc(*l) for l in b["layers"]], in_features=b["in_features"],
+                            seed=20240716 + i) for i, b in enumerate(wl["blocks"])]
+    for s in range(warmup + steps):
+        if s == warmup:
+            t0 = time.perf_counter()
+        x = synth.images(1, s, sample_batch, wl["input_shape"]).astype(np.int64)
+        y = synth.labels(1, s, sample_batch).astype(np.int64)
+        O.train_step(blocks, x, y)
+    dt = time.perf_counter() - t0
+    return sample_batch * steps / dt, dt, O.num_threads()
+
+
+def main():
+    args = parse()
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        if rank != 0:
+            return 0
+        # the oracle as it stands, on the host cores, each step a bounded
+        # sample (batch 8 of the workload's 128)
+        sample_b = 8
+        value, dt, cores = oracle_rate(args.workload, sample_b, args.steps, args.warmup)
+        line = {"impl": "reference", "metric": METRIC, "value": round(value, 4), "unit": "images/s",
+                "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+                "ms_per_step": round(dt / args.steps * 1e3, 2), "higher_is_better": True,
+                "scaling": "weak", "vs_baseline": None, "dtype": "int64", "data": "synthetic",
+                "config": {"workload": args.workload, "sample_batch": sample_b},
+                "cpu_baseline": {"value": round(value, 4), "unit": "images/s", "cores": cores,
+                                 "kind": "oracle",
+                                 "sample": "%d training steps at batch %d of %s" % (args.steps, sample_b, args.workload)},
+                "e2e": {"value": round(value, 4), "unit": "images/s", "h2d_bytes_per_step": 0,
+                        "d2h_bytes_per_step": 0}}
+        print(json.dumps(line), flush=True)
+        return 0
+
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+        torch.cuda.set_device(local_rank)
+        dist.init_process_group("nccl")
+    line = run_ours(args, rank, world, local_rank)
+    if rank == 0:
+        if not args.no_cpu_baseline:
+            sample_b = 16
+            v, dt, cores = oracle_rate(args.workload, sample_b, 1)
+            line["cpu_baseline"] = {"value": round(v, 4), "unit": "images/s", "cores": cores,
+                                    "kind": "oracle",
+                                    "sample": "1 training step at batch %d of %s (%.1f s)" % (sample_b, args.workload, dt)}
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+        dist.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,198 @@
+/*
+ * nitro.h - C ABI of the GB300 library for the NITRO-D local-loss block
+ * training step (arXiv 2407.11698, Sec. 3.2 architecture, Sec. 3.3 learning
+ * algorithm).
+ *
+ * One handle = one integer local-loss block: its forward layers (3x3 conv or
+ * linear, each followed by NITRO-Scaling, NITRO-ReLU and an optional 2x2
+ * max-pool) and its learning layer (IntLinear to G classes + NITRO-Scaling,
+ * trained on the RSS loss).  A block with zero forward layers is the network's
+ * output block.  A network is a chain of handles; the caller runs every
+ * block's forward, then every block's backward (they are independent, Sec.
+ * 3.3), then every block's IntegerSGD step.
+ *
+ * Conventions
+ *   activations   int8, NHWC  a[((b*H + y)*W + x)*C + c]; linear: a[b*In + i]
+ *   conv weights  int32, OHWI w[((co*3 + ky)*3 + kx)*Cin + ci]
+ *   linear / learning weights int32 w[o*In + i]; learning input is the block
+ *                 output flattened in (h, w, c) order
+ *   weight gradients int64, same layout as the weights
+ *   gradients delta and the loss gradient int32
+ *   labels        int32 in [0, G)
+ *   streams       `stream` is a cudaStream_t passed as void* (NULL = legacy
+ *                 default stream)
+ *
+ * Ownership: the caller owns every pointer argument and the stream; device
+ * pointers must stay valid until the work queued on `stream` has run.  The
+ * library owns everything inside a handle (weights, weight gradients, cached
+ * forward state, workspace), allocated once by nitro_init_block for
+ * `max_batch` samples and freed by nitro_destroy_block.
+ *
+ * Errors: every call checks its arguments on the host and returns
+ * NITRO_ERR_ARG / NITRO_ERR_UNSUPPORTED before queuing anything.  Compute
+ * calls are asynchronous: conditions found on the device (a value that does
+ * not fit its storage type, a label outside [0, G), a bounded wait that gave
+ * up) are latched in a per-block device status word and reported by
+ * nitro_block_status or nitro_block_get_tensor, which synchronise.  No
+ * exception crosses the ABI and no call traps the device.
+ */
+#ifndef NITRO_H
+#define NITRO_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    NITRO_OK = 0,
+    NITRO_ERR_ARG = 1,          /* bad argument, or a label outside [0, G) */
+    NITRO_ERR_OVERFLOW = 2,     /* a value did not fit its storage type     */
+    NITRO_ERR_TIMEOUT = 3,      /* a bounded device wait gave up            */
+    NITRO_ERR_CUDA = 4,         /* a CUDA runtime call failed               */
+    NITRO_ERR_UNSUPPORTED = 5   /* valid but not supported by this build    */
+} nitro_status;
+
+typedef enum { NITRO_ROUND_FLOOR = 0, NITRO_ROUND_TRUNC = 1 } nitro_round;
+typedef enum { NITRO_CONV3X3 = 0, NITRO_LINEAR = 1 } nitro_layer_kind;
+
+/* Bits of the device status word (nitro_block_status_bits). */
+#define NITRO_STATUS_BIT_OVERFLOW  1u
+#define NITRO_STATUS_BIT_BAD_LABEL 2u
+#define NITRO_STATUS_BIT_TIMEOUT   4u
+
+/* One forward layer (Sec. 3.2.1, Table 1): 3x3 conv with stride 1 and zero
+ * padding 1, or linear; then NITRO-Scaling with SF = 2^8*9*cin (conv) or
+ * 2^8*cin (linear), NITRO-ReLU, and a 2x2 stride-2 max-pool if pool2x2
+ * (conv only; output size floor(h/2) x floor(w/2)).  h, w: input size
+ * (1, 1 for linear).  A linear layer after a conv layer reads its input
+ * flattened in (h, w, c) order, so cin = h'*w'*c of that output. */
+typedef struct {
+    int kind;        /* nitro_layer_kind */
+    int cin, cout;
+    int h, w;
+    int pool2x2;
+} nitro_layer_desc;
+
+/* One local-loss block (Sec. 3.2, Sec. 3.3; hyper-parameters of App. B). */
+typedef struct {
+    int n_layers;                    /* 0 = output block                     */
+    const nitro_layer_desc* layers;  /* n_layers entries, copied at init     */
+    int in_features;                 /* flattened input size per sample      */
+    int num_classes;                 /* G, 1..64                             */
+    int alpha_inv;                   /* NITRO-ReLU 1/alpha, >= 2             */
+    int64_t gamma_inv_lr;            /* learning / output layers; forward
+                                        layers use AF*gamma_inv_lr with
+                                        AF = 2^6*G (Sec. 3.3.5)              */
+    int64_t eta_inv_fw, eta_inv_lr;  /* weight-decay thresholds, 0 = off     */
+    int sgd_round;                   /* nitro_round for IntegerSGD           */
+    int max_batch;                   /* workspace is sized for this          */
+} nitro_block_desc;
+
+typedef struct nitro_block nitro_block;
+
+/* Creates a block on the current CUDA device and initialises every weight
+ * tensor with the integer Kaiming rule (Sec. 3.3.1): b = floor(128*1732 /
+ * (isqrt(fan_in)*1000)), weights uniform on {-b..b}.  Element e of tensor t
+ * (t = layer index, 255 for the learning layer) is -b + u mod (2b+1), u being
+ * output number t*2^40 + e of SplitMix64 seeded with `seed`.  Weights are
+ * uploaded on `stream`.  Returns NITRO_ERR_ARG for inconsistent shapes,
+ * NITRO_ERR_CUDA if allocation fails (nothing is leaked). */
+nitro_status nitro_init_block(const nitro_block_desc* desc, uint64_t seed, void* stream,
+                              nitro_block** out);
+
+/* Forward layers of the block (Sec. 3.3, first phase): for each layer
+ * z = conv/linear(a, W) (exact integer sum), z* = floor(z / SF) (Eq. 1),
+ * NITRO-ReLU (Sec. 3.2.2), optional max-pool.  a_in: device int8
+ * [batch x in_features]; a_out: device int8 [batch x out_features] of the
+ * last layer, or NULL.  Caches what backward needs.  0 <= batch <= max_batch.
+ * For an output block this only records the batch. */
+nitro_status nitro_block_forward(nitro_block* blk, const int8_t* a_in, int batch,
+                                 int8_t* a_out, void* stream);
+
+/* Local backward of the block (Sec. 3.3, second phase): learning layer
+ * y_hat = floor(a W_lr^T / (2^8 d)), scaled one-hot target y (32 at the label,
+ * Sec. 3.3.4 and App. A), grad_L = y_hat - y, RSS loss; weight gradient of
+ * the learning layer; delta_fw = grad_L W_lr (pre-update W_lr, Sec. 3.3.5);
+ * then through each forward layer, last to first: max-pool backward (to the
+ * recorded window maximum), NITRO-ReLU backward (per piece), straight-through
+ * NITRO-Scaling (Sec. 3.2.1), weight gradient, input gradient.  Must follow
+ * nitro_block_forward with the same a_in and batch.  labels: device int32
+ * [batch]; loss_dev: device int64 [1] receiving floor(SSE/2), or NULL. */
+nitro_status nitro_block_backward(nitro_block* blk, const int8_t* a_in, const int32_t* labels,
+                                  int batch, int64_t* loss_dev, void* stream);
+
+/* IntegerSGD (Algorithm 1) on every weight tensor of the block using the
+ * weight gradients of the last backward: d = R(dW, gamma_inv), plus
+ * R(W, eta_inv) if eta_inv != 0, W -= d; R = floor or trunc per sgd_round.
+ * Forward layers use gamma_inv^fw = 2^6*G*gamma_inv_lr and eta_inv_fw; the
+ * learning layer gamma_inv_lr and eta_inv_lr. */
+nitro_status nitro_integersgd_step(nitro_block* blk, void* stream);
+
+/* Tensors readable / writable through get/set_tensor.  Batch-shaped tensors
+ * hold the last forward/backward batch. */
+typedef enum {
+    NITRO_T_W = 0,       /* layer weights, int32                               */
+    NITRO_T_DW = 1,      /* layer weight gradient, int64                       */
+    NITRO_T_WLR = 2,     /* learning/output weights [G x d], int32 (layer = 0) */
+    NITRO_T_DWLR = 3,    /* learning weight gradient, int64 (layer = 0)        */
+    NITRO_T_ACT = 4,     /* layer output after pool, int8 [batch x out]        */
+    NITRO_T_REGION = 5,  /* NITRO-ReLU piece 0..3 per pre-pool output, int8    */
+    NITRO_T_ARGMAX = 6,  /* max-pool window position 0..3 per output, int8     */
+    NITRO_T_DELTA = 7,   /* gradient at the layer's pre-activation, int32      */
+    NITRO_T_GRAD_L = 8,  /* loss gradient [batch x G], int32 (layer = 0)       */
+    NITRO_T_SSE = 9      /* sum of squared errors, int64 [1] (layer = 0)       */
+} nitro_tensor;
+
+/* Size in bytes of tensor (which, layer) at the current batch. */
+nitro_status nitro_block_tensor_bytes(const nitro_block* blk, int which, int layer,
+                                      size_t* bytes);
+
+/* Synchronises the device, copies the tensor to host memory host_dst (which
+ * must hold exactly `bytes` = nitro_block_tensor_bytes), and returns the
+ * latched device status (NITRO_OK if none). */
+nitro_status nitro_block_get_tensor(nitro_block* blk, int which, int layer, void* host_dst,
+                                    size_t bytes);
+
+/* Synchronises the device and overwrites a weight tensor (NITRO_T_W,
+ * NITRO_T_DW, NITRO_T_WLR, NITRO_T_DWLR) from host memory; used to resume
+ * from a checkpoint.  Bit-exact: all state is integer. */
+nitro_status nitro_block_set_tensor(nitro_block* blk, int which, int layer,
+                                    const void* host_src, size_t bytes);
+
+/* Synchronises the device and returns the latched status as nitro_status
+ * (TIMEOUT before OVERFLOW before a bad label = ARG); clears it if clear. */
+nitro_status nitro_block_status(nitro_block* blk, int clear);
+
+/* Synchronises the device and returns the raw NITRO_STATUS_BIT_* word. */
+uint32_t nitro_block_status_bits(nitro_block* blk);
+
+/* Releases every device buffer of the block.  NULL is ignored. */
+void nitro_destroy_block(nitro_block* blk);
+
+/* ---- Diagnostics (not part of the training step) -------------------------
+ * Every kernel launch of the library is counted.  With profiling on, each
+ * launch is also bracketed by CUDA events recorded on its own stream and
+ * tagged with its kernel class and algorithmic work (integer ops = 2 x MACs;
+ * bytes for the HBM-bound update).  Profile eager calls only: events are not
+ * recorded into CUDA-graph captures. */
+uint64_t nitro_kernel_launches(void);            /* launches issued since load */
+void nitro_profile_enable(int on);
+void nitro_profile_reset(void);                  /* drops recorded launches  */
+int nitro_profile_kernel_count(void);            /* number of kernel classes */
+const char* nitro_profile_kernel_name(int id);   /* static string            */
+/* Synchronises on the recorded events of class `id` and returns their count,
+ * summed device time (ms) and summed algorithmic ops and bytes. */
+nitro_status nitro_profile_read(int id, uint64_t* launches, double* ms, double* ops,
+                                double* bytes);
+
+/* Static, human-readable name of a status code. */
+const char* nitro_status_str(nitro_status s);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* NITRO_H */

@@ -1,0 +1,250 @@
+"""ctypes binding of ``libnitro.so`` (declared in ``include/nitro.h``).
+
+Argument marshalling only: every step of the block training step runs in the
+library's CUDA kernels.  The module-level functions carry the C-ABI names and
+return its status codes; ``Block`` wraps one handle for callers that hold
+their activations and labels in torch CUDA tensors.  There is no CPU path:
+loading fails loudly when the library has not been built.
+"""
+import ctypes
+import os
+
+import numpy as np
+
+from . import build as _build
+
+NITRO_OK, NITRO_ERR_ARG, NITRO_ERR_OVERFLOW, NITRO_ERR_TIMEOUT, NITRO_ERR_CUDA, \
+    NITRO_ERR_UNSUPPORTED = range(6)
+NITRO_CONV3X3, NITRO_LINEAR = 0, 1
+NITRO_ROUND_FLOOR, NITRO_ROUND_TRUNC = 0, 1
+STATUS_BIT_OVERFLOW, STATUS_BIT_BAD_LABEL, STATUS_BIT_TIMEOUT = 1, 2, 4
+(NITRO_T_W, NITRO_T_DW, NITRO_T_WLR, NITRO_T_DWLR, NITRO_T_ACT, NITRO_T_REGION,
+ NITRO_T_ARGMAX, NITRO_T_DELTA, NITRO_T_GRAD_L, NITRO_T_SSE) = range(10)
+
+TENSOR_DTYPE = {
+    NITRO_T_W: np.int32, NITRO_T_DW: np.int64, NITRO_T_WLR: np.int32, NITRO_T_DWLR: np.int64,
+    NITRO_T_ACT: np.int8, NITRO_T_REGION: np.int8, NITRO_T_ARGMAX: np.int8,
+    NITRO_T_DELTA: np.int32, NITRO_T_GRAD_L: np.int32, NITRO_T_SSE: np.int64,
+}
+
+
+class nitro_layer_desc(ctypes.Structure):
+    _fields_ = [("kind", ctypes.c_int), ("cin", ctypes.c_int), ("cout", ctypes.c_int),
+                ("h", ctypes.c_int), ("w", ctypes.c_int), ("pool2x2", ctypes.c_int)]
+
+
+class nitro_block_desc(ctypes.Structure):
+    _fields_ = [("n_layers", ctypes.c_int), ("layers", ctypes.POINTER(nitro_layer_desc)),
+                ("in_features", ctypes.c_int), ("num_classes", ctypes.c_int),
+                ("alpha_inv", ctypes.c_int), ("gamma_inv_lr", ctypes.c_int64),
+                ("eta_inv_fw", ctypes.c_int64), ("eta_inv_lr", ctypes.c_int64),
+                ("sgd_round", ctypes.c_int), ("max_batch", ctypes.c_int)]
+
+
+class NitroError(RuntimeError):
+    def __init__(self, status, what=""):
+        self.status = int(status)
+        super().__init__("%s: %s (status %d)" % (what, status_str(status), int(status)))
+
+
+_lib = None
+_VP = ctypes.c_void_p
+
+
+def lib():
+    """The loaded ``libnitro.so``; raises if it has not been built."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(_build.LIB):
+        raise RuntimeError("libnitro.so is missing (%s): build it with "
+                           "paper_2407_11698_gb300.build.build() first" % _build.LIB)
+    L = ctypes.CDLL(_build.LIB)
+    L.nitro_init_block.argtypes = [ctypes.POINTER(nitro_block_desc), ctypes.c_uint64, _VP,
+                                   ctypes.POINTER(_VP)]
+    L.nitro_block_forward.argtypes = [_VP, _VP, ctypes.c_int, _VP, _VP]
+    L.nitro_block_backward.argtypes = [_VP, _VP, _VP, ctypes.c_int, _VP, _VP]
+    L.nitro_integersgd_step.argtypes = [_VP, _VP]
+    L.nitro_block_tensor_bytes.argtypes = [_VP, ctypes.c_int, ctypes.c_int,
+                                           ctypes.POINTER(ctypes.c_size_t)]
+    L.nitro_block_get_tensor.argtypes = [_VP, ctypes.c_int, ctypes.c_int, _VP, ctypes.c_size_t]
+    L.nitro_block_set_tensor.argtypes = [_VP, ctypes.c_int, ctypes.c_int, _VP, ctypes.c_size_t]
+    L.nitro_block_status.argtypes = [_VP, ctypes.c_int]
+    L.nitro_block_status_bits.argtypes = [_VP]
+    L.nitro_block_status_bits.restype = ctypes.c_uint32
+    L.nitro_destroy_block.argtypes = [_VP]
+    L.nitro_destroy_block.restype = None
+    L.nitro_status_str.argtypes = [ctypes.c_int]
+    L.nitro_status_str.restype = ctypes.c_char_p
+    L.nitro_kernel_launches.argtypes = []
+    L.nitro_kernel_launches.restype = ctypes.c_uint64
+    L.nitro_profile_enable.argtypes = [ctypes.c_int]
+    L.nitro_profile_enable.restype = None
+    L.nitro_profile_reset.argtypes = []
+    L.nitro_profile_reset.restype = None
+    L.nitro_profile_kernel_count.argtypes = []
+    L.nitro_profile_kernel_count.restype = ctypes.c_int
+    L.nitro_profile_kernel_name.argtypes = [ctypes.c_int]
+    L.nitro_profile_kernel_name.restype = ctypes.c_char_p
+    _PD = ctypes.POINTER(ctypes.c_double)
+    L.nitro_profile_read.argtypes = [ctypes.c_int, ctypes.POINTER(ctypes.c_uint64), _PD, _PD, _PD]
+    L.nitro_profile_read.restype = ctypes.c_int
+    for name in ("nitro_init_block", "nitro_block_forward", "nitro_block_backward",
+                 "nitro_integersgd_step", "nitro_block_tensor_bytes", "nitro_block_get_tensor",
+                 "nitro_block_set_tensor", "nitro_block_status"):
+        getattr(L, name).restype = ctypes.c_int
+    _lib = L
+    return L
+
+
+def status_str(s):
+    try:
+        return lib().nitro_status_str(int(s)).decode()
+    except RuntimeError:
+        return "status"
+
+
+# ---------------------------------------------------------------- C-ABI names
+def nitro_init_block(desc, seed, stream=None):
+    """Returns (status, handle)."""
+    h = _VP()
+    st = lib().nitro_init_block(ctypes.byref(desc), int(seed) & (2**64 - 1), stream, ctypes.byref(h))
+    return st, h
+
+
+def nitro_block_forward(blk, a_in, batch, a_out, stream=None):
+    return lib().nitro_block_forward(blk, a_in, int(batch), a_out, stream)
+
+
+def nitro_block_backward(blk, a_in, labels, batch, loss_dev, stream=None):
+    return lib().nitro_block_backward(blk, a_in, labels, int(batch), loss_dev, stream)
+
+
+def nitro_integersgd_step(blk, stream=None):
+    return lib().nitro_integersgd_step(blk, stream)
+
+
+def nitro_block_tensor_bytes(blk, which, layer=0):
+    n = ctypes.c_size_t()
+    st = lib().nitro_block_tensor_bytes(blk, int(which), int(layer), ctypes.byref(n))
+    return st, n.value
+
+
+def nitro_block_get_tensor(blk, which, layer, host_ptr, nbytes):
+    return lib().nitro_block_get_tensor(blk, int(which), int(layer), host_ptr, int(nbytes))
+
+
+def nitro_block_set_tensor(blk, which, layer, host_ptr, nbytes):
+    return lib().nitro_block_set_tensor(blk, int(which), int(layer), host_ptr, int(nbytes))
+
+
+def nitro_block_status(blk, clear=False):
+    return lib().nitro_block_status(blk, 1 if clear else 0)
+
+
+def nitro_block_status_bits(blk):
+    return lib().nitro_block_status_bits(blk)
+
+
+def nitro_destroy_block(blk):
+    lib().nitro_destroy_block(blk)
+
+
+# ---------------------------------------------------------------- helpers
+def make_block_desc(layers, in_features, num_classes=10, alpha_inv=10, gamma_inv_lr=512,
+                    eta_inv_fw=0, eta_inv_lr=0, sgd_round=NITRO_ROUND_FLOOR, max_batch=1):
+    """Build a ``nitro_block_desc`` from layer tuples (kind, cin, cout, h, w, pool).
+    Returns (desc, keepalive) - keep the second value alive while desc is used."""
+    arr = (nitro_layer_desc * max(1, len(layers)))()
+    for i, l in enumerate(layers):
+        arr[i] = nitro_layer_desc(*[int(v) for v in l])
+    d = nitro_block_desc(len(layers), arr if layers else None, int(in_features), int(num_classes),
+                         int(alpha_inv), int(gamma_inv_lr), int(eta_inv_fw), int(eta_inv_lr),
+                         int(sgd_round), int(max_batch))
+    return d, arr
+
+
+def _stream_ptr(stream):
+    if stream is None:
+        import torch
+        stream = torch.cuda.current_stream()
+    return _VP(stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream))
+
+
+def _ptr(t):
+    return None if t is None else _VP(t.data_ptr())
+
+
+class Block:
+    """One local-loss block handle.  Activations / labels / loss are torch CUDA
+    tensors (int8 / int32 / int64); calls queue work on the given (or current)
+    torch stream."""
+
+    def __init__(self, layers, in_features, seed=0, max_batch=1, stream=None, **hyper):
+        self.layers = [tuple(int(v) for v in l) for l in layers]
+        self.desc, self._keep = make_block_desc(self.layers, in_features, max_batch=max_batch,
+                                                **hyper)
+        st, self.h = nitro_init_block(self.desc, seed, _stream_ptr(stream))
+        if st != NITRO_OK:
+            raise NitroError(st, "nitro_init_block")
+        self.in_features = int(in_features)
+        self.num_classes = self.desc.num_classes
+        if self.layers:
+            k, cin, cout, h, w, pool = self.layers[-1]
+            self.out_features = (h // 2) * (w // 2) * cout if pool else h * w * cout
+        else:
+            self.out_features = 0
+
+    def forward(self, a_in, a_out=None, stream=None):
+        st = nitro_block_forward(self.h, _ptr(a_in), a_in.shape[0], _ptr(a_out), _stream_ptr(stream))
+        if st != NITRO_OK:
+            raise NitroError(st, "nitro_block_forward")
+        return a_out
+
+    def backward(self, a_in, labels, loss=None, stream=None):
+        st = nitro_block_backward(self.h, _ptr(a_in), _ptr(labels), labels.shape[0], _ptr(loss),
+                                  _stream_ptr(stream))
+        if st != NITRO_OK:
+            raise NitroError(st, "nitro_block_backward")
+        return loss
+
+    def sgd(self, stream=None):
+        st = nitro_integersgd_step(self.h, _stream_ptr(stream))
+        if st != NITRO_OK:
+            raise NitroError(st, "nitro_integersgd_step")
+
+    def get(self, which, layer=0, check=True):
+        """Host copy of a tensor as a flat numpy array (synchronises)."""
+        st, n = nitro_block_tensor_bytes(self.h, which, layer)
+        if st != NITRO_OK:
+            raise NitroError(st, "nitro_block_tensor_bytes")
+        dt = np.dtype(TENSOR_DTYPE[which])
+        out = np.empty(n // dt.itemsize, dtype=dt)
+        st = nitro_block_get_tensor(self.h, which, layer, out.ctypes.data_as(_VP), n)
+        if check and st not in (NITRO_OK,):
+            raise NitroError(st, "nitro_block_get_tensor")
+        return out
+
+    def set(self, which, layer, values):
+        dt = np.dtype(TENSOR_DTYPE[which])
+        arr = np.ascontiguousarray(values, dtype=dt)
+        st = nitro_block_set_tensor(self.h, which, layer, arr.ctypes.data_as(_VP), arr.nbytes)
+        if st != NITRO_OK:
+            raise NitroError(st, "nitro_block_set_tensor")
+
+    def status(self, clear=False):
+        return nitro_block_status(self.h, clear)
+
+    def status_bits(self):
+        return nitro_block_status_bits(self.h)
+
+    def close(self):
+        if getattr(self, "h", None):
+            nitro_destroy_block(self.h)
+            self.h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass

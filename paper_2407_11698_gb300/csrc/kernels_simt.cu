@@ -1,0 +1,453 @@
+// CUDA-core kernels of the NITRO-D block step: an exact int64 implicit GEMM
+// for every contraction shape (conv 3x3 fwd / dgrad / wgrad, linear fwd /
+// dgrad / wgrad), and the element-wise stages fused around it (NITRO-Scaling,
+// NITRO-ReLU and max-pool forward; max-pool, NITRO-ReLU backward and STE;
+// learning layer and RSS loss; IntegerSGD).
+//
+// These serve the layers whose contraction is too narrow for the tensor-core
+// path (first layers with 1 or 3 input channels, MLP layers, learning layers
+// with G = 10 outputs) and are the exactness reference on the device.
+#include "nitro_internal.cuh"
+#include "prof.cuh"
+
+namespace nitro {
+namespace {
+
+constexpr int kTile = 64;   // M and N tile
+constexpr int kTK = 16;     // K slab
+constexpr unsigned kFull = 0xffffffffu;
+
+struct GemmParams {
+    const int8_t* act;
+    const int32_t* grad;
+    const int32_t* wts;
+    int64_t* out;
+    int M, N, K;
+    int B, H, W, Cin, Cout;
+    int k_split;
+};
+
+// Operand element A[m][k] / B[n][k] of each contraction (see GemmMode).
+template <int MODE>
+__device__ __forceinline__ int32_t load_a(const GemmParams& p, int m, int k) {
+    if (MODE == GM_CONV_FWD || MODE == GM_CONV_DGRAD) {
+        const int hw = p.H * p.W;
+        const int b = m / hw, r = m - b * hw, y = r / p.W, x = r - y * p.W;
+        const int C = MODE == GM_CONV_FWD ? p.Cin : p.Cout;
+        const int t = k / C, c = k - t * C, ky = t / 3, kx = t - 3 * ky;
+        // forward reads input (y+ky-1, x+kx-1); dgrad reads output (y-ky+1, x-kx+1)
+        const int iy = MODE == GM_CONV_FWD ? y + ky - 1 : y - ky + 1;
+        const int ix = MODE == GM_CONV_FWD ? x + kx - 1 : x - kx + 1;
+        if (iy < 0 || iy >= p.H || ix < 0 || ix >= p.W) return 0;
+        const int64_t idx = ((int64_t)(b * p.H + iy) * p.W + ix) * C + c;
+        return MODE == GM_CONV_FWD ? (int32_t)p.act[idx] : p.grad[idx];
+    } else if (MODE == GM_CONV_WGRAD) {
+        return p.grad[(int64_t)k * p.Cout + m];
+    } else if (MODE == GM_LIN_FWD) {
+        return p.act[(int64_t)m * p.Cin + k];
+    } else if (MODE == GM_LIN_DGRAD) {
+        return p.grad[(int64_t)m * p.Cout + k];
+    } else {  // GM_LIN_WGRAD
+        return p.grad[(int64_t)k * p.Cout + m];
+    }
+}
+
+template <int MODE>
+__device__ __forceinline__ int32_t load_b(const GemmParams& p, int n, int k) {
+    if (MODE == GM_CONV_FWD) {
+        return p.wts[(int64_t)n * 9 * p.Cin + k];
+    } else if (MODE == GM_CONV_DGRAD) {
+        const int t = k / p.Cout, co = k - t * p.Cout;
+        return p.wts[((int64_t)co * 9 + t) * p.Cin + n];
+    } else if (MODE == GM_CONV_WGRAD) {
+        const int t = n / p.Cin, ci = n - t * p.Cin, ky = t / 3, kx = t - 3 * ky;
+        const int hw = p.H * p.W;
+        const int b = k / hw, r = k - b * hw, y = r / p.W, x = r - y * p.W;
+        const int iy = y + ky - 1, ix = x + kx - 1;
+        if (iy < 0 || iy >= p.H || ix < 0 || ix >= p.W) return 0;
+        return p.act[((int64_t)(b * p.H + iy) * p.W + ix) * p.Cin + ci];
+    } else if (MODE == GM_LIN_FWD) {
+        return p.wts[(int64_t)n * p.Cin + k];
+    } else if (MODE == GM_LIN_DGRAD) {
+        return p.wts[(int64_t)k * p.Cin + n];
+    } else {  // GM_LIN_WGRAD
+        return p.act[(int64_t)k * p.Cin + n];
+    }
+}
+
+// 64x64 output tile per CTA, 4x4 per thread, int64 accumulators.  With
+// gridDim.z > 1 each CTA sums one K slice and adds it into a zeroed `out`
+// with 64-bit integer atomics (exact and order-independent).
+template <int MODE>
+__global__ void __launch_bounds__(256) k_gemm(GemmParams p) {
+    __shared__ int32_t As[kTK][kTile + 4];
+    __shared__ int32_t Bs[kTK][kTile + 4];
+    const int m0 = blockIdx.y * kTile, n0 = blockIdx.x * kTile;
+    const int kb = blockIdx.z * p.k_split;
+    const int ke = min(p.K, kb + p.k_split);
+    const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
+    int64_t acc[4][4];
+#pragma unroll
+    for (int r = 0; r < 4; ++r)
+#pragma unroll
+        for (int c = 0; c < 4; ++c) acc[r][c] = 0;
+
+    for (int k0 = kb; k0 < ke; k0 += kTK) {
+        for (int i = threadIdx.x; i < kTile * kTK; i += 256) {
+            const int mm = i / kTK, kk = i - mm * kTK;
+            const int k = k0 + kk;
+            const int m = m0 + mm, n = n0 + mm;
+            As[kk][mm] = (m < p.M && k < ke) ? load_a<MODE>(p, m, k) : 0;
+            Bs[kk][mm] = (n < p.N && k < ke) ? load_b<MODE>(p, n, k) : 0;
+        }
+        __syncthreads();
+#pragma unroll
+        for (int kk = 0; kk < kTK; ++kk) {
+            int32_t a[4], b[4];
+#pragma unroll
+            for (int r = 0; r < 4; ++r) a[r] = As[kk][ty + 16 * r];
+#pragma unroll
+            for (int c = 0; c < 4; ++c) b[c] = Bs[kk][tx + 16 * c];
+#pragma unroll
+            for (int r = 0; r < 4; ++r)
+#pragma unroll
+                for (int c = 0; c < 4; ++c) acc[r][c] += (int64_t)a[r] * b[c];
+        }
+        __syncthreads();
+    }
+#pragma unroll
+    for (int r = 0; r < 4; ++r)
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+            const int m = m0 + ty + 16 * r, n = n0 + tx + 16 * c;
+            if (m < p.M && n < p.N) {
+                int64_t* o = p.out + (int64_t)m * p.N + n;
+                if (gridDim.z > 1)
+                    atomicAdd(reinterpret_cast<unsigned long long*>(o),
+                              (unsigned long long)acc[r][c]);
+                else
+                    *o = acc[r][c];
+            }
+        }
+}
+
+// ---------------------------------------------------------------------------
+// Forward epilogue: one thread per pooling window (or per element).
+// ---------------------------------------------------------------------------
+__global__ void k_fwd_epilogue(const int64_t* __restrict__ z, LayerGeom g, int B,
+                               int alpha_inv, int mu, int64_t kdiv, int8_t* __restrict__ out,
+                               int8_t* __restrict__ out2, int8_t* __restrict__ region,
+                               int8_t* __restrict__ argmax) {
+    const int C = g.cout;
+    if (!g.pool) {
+        const int64_t n = (int64_t)B * g.h * g.w * C;
+        for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
+             i += (int64_t)gridDim.x * blockDim.x) {
+            const int64_t zs = scale_floor(z[i], kdiv);
+            region[i] = (int8_t)relu_region(zs);
+            const int8_t v = (int8_t)relu_value(zs, alpha_inv, mu);
+            out[i] = v;
+            if (out2) out2[i] = v;
+        }
+        return;
+    }
+    // windows over ceil(h/2) x ceil(w/2); partial windows (odd edges) only
+    // record region codes of the positions the floor-sized pool drops.
+    const int wy_n = (g.h + 1) / 2, wx_n = (g.w + 1) / 2;
+    const int64_t n = (int64_t)B * wy_n * wx_n * C;
+    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        const int c = (int)(i % C);
+        int64_t r = i / C;
+        const int wx = (int)(r % wx_n);
+        r /= wx_n;
+        const int wy = (int)(r % wy_n);
+        const int b = (int)(r / wy_n);
+        int best = 0, bestv = 0;
+        bool full = (2 * wy + 1 < g.h) && (2 * wx + 1 < g.w);
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            const int iy = 2 * wy + (k >> 1), ix = 2 * wx + (k & 1);
+            if (iy >= g.h || ix >= g.w) continue;
+            const int64_t pi = ((int64_t)(b * g.h + iy) * g.w + ix) * C + c;
+            const int64_t zs = scale_floor(z[pi], kdiv);
+            region[pi] = (int8_t)relu_region(zs);
+            const int v = relu_value(zs, alpha_inv, mu);
+            if (k == 0 || v > bestv) { bestv = v; best = k; }
+        }
+        if (full) {
+            const int64_t oi = ((int64_t)(b * g.oh + wy) * g.ow + wx) * C + c;
+            out[oi] = (int8_t)bestv;
+            if (out2) out2[oi] = (int8_t)bestv;
+            argmax[oi] = (int8_t)best;
+        }
+    }
+}
+
+// ---------------------------------------------------------------------------
+// Learning layer forward + RSS loss: one CTA per sample.
+// ---------------------------------------------------------------------------
+constexpr int kGChunk = 16;
+
+__global__ void __launch_bounds__(256) k_learn_fwd(const int8_t* __restrict__ a,
+                                                   const int32_t* __restrict__ wlr,
+                                                   const int32_t* __restrict__ labels, int d,
+                                                   int G, int32_t* __restrict__ grad_l,
+                                                   unsigned long long* sse, uint32_t* maxabs_gl,
+                                                   uint32_t* status) {
+    __shared__ int64_t red[8][kGChunk];
+    const int b = blockIdx.x;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int lab = labels[b];
+    const bool bad = lab < 0 || lab >= G;
+    if (bad && threadIdx.x == 0) atomicOr(status, ST_BAD_LABEL);
+    const int8_t* arow = a + (int64_t)b * d;
+    for (int g0 = 0; g0 < G; g0 += kGChunk) {
+        int64_t acc[kGChunk];
+#pragma unroll
+        for (int q = 0; q < kGChunk; ++q) acc[q] = 0;
+        for (int j = threadIdx.x; j < d; j += 256) {
+            const int32_t av = arow[j];
+#pragma unroll
+            for (int q = 0; q < kGChunk; ++q)
+                if (g0 + q < G) acc[q] += (int64_t)av * wlr[(int64_t)(g0 + q) * d + j];
+        }
+#pragma unroll
+        for (int q = 0; q < kGChunk; ++q) {
+#pragma unroll
+            for (int off = 16; off; off >>= 1) acc[q] += __shfl_xor_sync(kFull, acc[q], off);
+            if (lane == 0) red[warp][q] = acc[q];
+        }
+        __syncthreads();
+        if (threadIdx.x < kGChunk && g0 + threadIdx.x < G) {
+            const int q = threadIdx.x, gi = g0 + q;
+            int64_t zsum = 0;
+            for (int w = 0; w < 8; ++w) zsum += red[w][q];
+            const int64_t yhat = scale_floor(zsum, d);       // NITRO-Scaling, SF = 2^8 d
+            const int64_t v = yhat - ((!bad && gi == lab) ? 32 : 0);
+            if (!fits_i32(v)) atomicOr(status, ST_OVERFLOW);
+            const int32_t s = (int32_t)v;
+            grad_l[(int64_t)b * G + gi] = s;
+            atomicAdd(sse, (unsigned long long)((int64_t)s * s));
+            atomicMax(maxabs_gl, abs_u32(s));
+        }
+        __syncthreads();
+    }
+}
+
+// dW_lr[g][j] = sum_b grad_l[b][g] * a[b][j]
+__global__ void k_learn_dw(const int8_t* __restrict__ a, const int32_t* __restrict__ grad_l,
+                           int B, int d, int G, int64_t* __restrict__ dwlr) {
+    const int j = blockIdx.x * blockDim.x + threadIdx.x;
+    const int g = blockIdx.y;
+    if (j >= d) return;
+    int64_t s = 0;
+    for (int b = 0; b < B; ++b) s += (int64_t)grad_l[(int64_t)b * G + g] * a[(int64_t)b * d + j];
+    dwlr[(int64_t)g * d + j] = s;
+}
+
+// ---------------------------------------------------------------------------
+// Gradient at a layer output -> delta at its pre-activation.
+// ---------------------------------------------------------------------------
+__global__ void k_grad_to_delta(DeltaSrc src, LayerGeom g, int B, int alpha_inv,
+                                const int8_t* __restrict__ region,
+                                const int8_t* __restrict__ argmax, int32_t* __restrict__ delta,
+                                uint32_t* maxabs_delta, uint32_t* status) {
+    const int64_t out_f = (int64_t)g.oh * g.ow * g.cout;
+    const int64_t n = (int64_t)B * out_f;
+    if (blockIdx.x == 0 && threadIdx.x == 0 &&
+        int64_bound_exceeded(*src.maxabs_a, *src.maxabs_b, src.bound_k))
+        atomicOr(status, ST_OVERFLOW);
+    uint32_t mx = 0;
+    bool ovf = false;
+    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t b = i / out_f, q = i - b * out_f;
+        int64_t gv;
+        if (src.wlr) {
+            uint64_t acc = 0;  // modulo 2^64, exact below the bound
+            for (int k = 0; k < src.G; ++k)
+                acc += (uint64_t)(int64_t)src.grad_l[b * src.G + k] *
+                       (uint64_t)(int64_t)src.wlr[(int64_t)k * out_f + q];
+            gv = (int64_t)acc;
+        } else {
+            gv = src.g64[i];
+        }
+        ovf |= !fits_i32(gv);
+        const int32_t gs = (int32_t)gv;
+        if (g.pool) {
+            const int c = (int)(q % g.cout);
+            const int64_t r = q / g.cout;
+            const int ox = (int)(r % g.ow), oy = (int)(r / g.ow);
+            const int am = argmax[i];
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                const int iy = 2 * oy + (k >> 1), ix = 2 * ox + (k & 1);
+                const int64_t pi = ((b * g.h + iy) * g.w + ix) * g.cout + c;
+                const int32_t dv = (k == am) ? relu_backward(gs, region[pi], alpha_inv) : 0;
+                delta[pi] = dv;
+                mx = max(mx, abs_u32(dv));
+            }
+        } else {
+            const int32_t dv = relu_backward(gs, region[i], alpha_inv);
+            delta[i] = dv;
+            mx = max(mx, abs_u32(dv));
+        }
+    }
+#pragma unroll
+    for (int off = 16; off; off >>= 1) mx = max(mx, __shfl_xor_sync(kFull, mx, off));
+    ovf = __any_sync(kFull, ovf);
+    if ((threadIdx.x & 31) == 0) {
+        if (mx) atomicMax(maxabs_delta, mx);
+        if (ovf) atomicOr(status, ST_OVERFLOW);
+    }
+}
+
+// ---------------------------------------------------------------------------
+// IntegerSGD (Algorithm 1); blockIdx.y selects the tensor.
+// ---------------------------------------------------------------------------
+__global__ void k_integersgd(SgdBatch bt) {
+    const SgdTensor t = bt.t[blockIdx.y];
+    uint32_t mx = 0;
+    bool ovf = false;
+    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < t.n;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t w = t.w[i];
+        int64_t d = bt.round_trunc ? tdiv64(t.dw[i], t.gamma_inv) : fdiv64(t.dw[i], t.gamma_inv);
+        if (t.eta_inv != 0) d += bt.round_trunc ? tdiv64(w, t.eta_inv) : fdiv64(w, t.eta_inv);
+        const int64_t nw = w - d;
+        ovf |= !fits_i32(nw);
+        const int32_t s = (int32_t)nw;
+        t.w[i] = s;
+        mx = max(mx, abs_u32(s));
+    }
+#pragma unroll
+    for (int off = 16; off; off >>= 1) mx = max(mx, __shfl_xor_sync(kFull, mx, off));
+    ovf = __any_sync(kFull, ovf);
+    if ((threadIdx.x & 31) == 0) {
+        if (mx) atomicMax(t.maxabs_w, mx);
+        if (ovf) atomicOr(bt.status, ST_OVERFLOW);
+    }
+}
+
+__global__ void k_finish_loss(const unsigned long long* sse, int64_t* loss) {
+    loss[0] = fdiv64((int64_t)sse[0], 2);
+}
+
+inline int grid_for(int64_t n, int threads, int cap = 152 * 16) {
+    int64_t g = (n + threads - 1) / threads;
+    return (int)(g < 1 ? 1 : (g > cap ? cap : g));
+}
+
+}  // namespace
+
+cudaError_t simt_gemm(int mode, const int8_t* act, const int32_t* grad, const int32_t* wts,
+                      int64_t* out, int B, int H, int W, int Cin, int Cout, cudaStream_t s) {
+    GemmParams p{act, grad, wts, out, 0, 0, 0, B, H, W, Cin, Cout, 0};
+    const int P = B * H * W;
+    switch (mode) {
+        case GM_CONV_FWD: p.M = P; p.N = Cout; p.K = 9 * Cin; break;
+        case GM_CONV_DGRAD: p.M = P; p.N = Cin; p.K = 9 * Cout; break;
+        case GM_CONV_WGRAD: p.M = Cout; p.N = 9 * Cin; p.K = P; break;
+        case GM_LIN_FWD: p.M = B; p.N = Cout; p.K = Cin; break;
+        case GM_LIN_DGRAD: p.M = B; p.N = Cin; p.K = Cout; break;
+        case GM_LIN_WGRAD: p.M = Cout; p.N = Cin; p.K = B; break;
+        default: return cudaErrorInvalidValue;
+    }
+    if (p.M <= 0 || p.N <= 0) return cudaSuccess;
+    const int tiles_m = (p.M + kTile - 1) / kTile, tiles_n = (p.N + kTile - 1) / kTile;
+    int splits = 1;
+    if (mode == GM_CONV_WGRAD || mode == GM_LIN_WGRAD) {
+        const int64_t tiles = (int64_t)tiles_m * tiles_n;
+        const int64_t want = (4 * 152 + tiles - 1) / tiles;
+        const int64_t maxs = (p.K + 255) / 256;
+        splits = (int)(want < maxs ? want : maxs);
+        if (splits < 1) splits = 1;
+    }
+    p.k_split = ((p.K + splits - 1) / splits + kTK - 1) / kTK * kTK;
+    if (p.k_split == 0) p.k_split = kTK;
+    splits = p.K > 0 ? (p.K + p.k_split - 1) / p.k_split : 1;
+    if (splits > 1 || p.K == 0) {
+        cudaError_t e = cudaMemsetAsync(out, 0, sizeof(int64_t) * (size_t)p.M * p.N, s);
+        if (e != cudaSuccess) return e;
+        if (p.K == 0) return cudaSuccess;
+    }
+    dim3 grid(tiles_n, tiles_m, splits);
+    static const int kIds[6] = {K_SIMT_CONV_FWD, K_SIMT_CONV_DGRAD, K_SIMT_CONV_WGRAD,
+                                K_SIMT_LIN_FWD, K_SIMT_LIN_DGRAD, K_SIMT_LIN_WGRAD};
+    ProfScope ps(kIds[mode], s, 2.0 * p.M * p.N * p.K, 0.0);
+    switch (mode) {
+        case GM_CONV_FWD: k_gemm<GM_CONV_FWD><<<grid, 256, 0, s>>>(p); break;
+        case GM_CONV_DGRAD: k_gemm<GM_CONV_DGRAD><<<grid, 256, 0, s>>>(p); break;
+        case GM_CONV_WGRAD: k_gemm<GM_CONV_WGRAD><<<grid, 256, 0, s>>>(p); break;
+        case GM_LIN_FWD: k_gemm<GM_LIN_FWD><<<grid, 256, 0, s>>>(p); break;
+        case GM_LIN_DGRAD: k_gemm<GM_LIN_DGRAD><<<grid, 256, 0, s>>>(p); break;
+        default: k_gemm<GM_LIN_WGRAD><<<grid, 256, 0, s>>>(p); break;
+    }
+    return cudaGetLastError();
+}
+
+cudaError_t simt_fwd_epilogue(const int64_t* z, const LayerGeom& g, int B, int alpha_inv,
+                              int mu, int8_t* out, int8_t* out2, int8_t* region,
+                              int8_t* argmax, cudaStream_t s) {
+    if (B <= 0) return cudaSuccess;
+    const int64_t kdiv = g.kind == NITRO_CONV3X3 ? 9LL * g.cin : (int64_t)g.cin;
+    const int64_t n = g.pool ? (int64_t)B * ((g.h + 1) / 2) * ((g.w + 1) / 2) * g.cout
+                             : (int64_t)B * g.h * g.w * g.cout;
+    ProfScope ps(K_FWD_EPILOGUE, s, 0.0, 0.0);
+    k_fwd_epilogue<<<grid_for(n, 256), 256, 0, s>>>(z, g, B, alpha_inv, mu, kdiv, out, out2,
+                                                    region, argmax);
+    return cudaGetLastError();
+}
+
+cudaError_t simt_learn_fwd(const int8_t* a, const int32_t* wlr, const int32_t* labels, int B,
+                           int d, int G, int32_t* grad_l, unsigned long long* sse,
+                           uint32_t* maxabs_gl, uint32_t* status, cudaStream_t s) {
+    if (B <= 0) return cudaSuccess;
+    ProfScope ps(K_LEARN_FWD, s, 2.0 * B * d * G, 0.0);
+    k_learn_fwd<<<B, 256, 0, s>>>(a, wlr, labels, d, G, grad_l, sse, maxabs_gl, status);
+    return cudaGetLastError();
+}
+
+cudaError_t simt_learn_dw(const int8_t* a, const int32_t* grad_l, int B, int d, int G,
+                          int64_t* dwlr, cudaStream_t s) {
+    dim3 grid((d + 255) / 256, G);
+    ProfScope ps(K_LEARN_DW, s, 2.0 * B * d * G, 0.0);
+    k_learn_dw<<<grid, 256, 0, s>>>(a, grad_l, B, d, G, dwlr);
+    return cudaGetLastError();
+}
+
+cudaError_t simt_grad_to_delta(const DeltaSrc& src, const LayerGeom& g, int B, int alpha_inv,
+                               const int8_t* region, const int8_t* argmax, int32_t* delta,
+                               uint32_t* maxabs_delta, uint32_t* status, cudaStream_t s) {
+    if (B <= 0) return cudaSuccess;
+    if (g.pool && ((g.h & 1) || (g.w & 1))) {
+        cudaError_t e = cudaMemsetAsync(delta, 0, sizeof(int32_t) * (size_t)B * g.h * g.w * g.cout, s);
+        if (e != cudaSuccess) return e;
+    }
+    const int64_t n = (int64_t)B * g.oh * g.ow * g.cout;
+    ProfScope ps(K_GRAD_TO_DELTA, s, 0.0, 0.0);
+    k_grad_to_delta<<<grid_for(n, 256), 256, 0, s>>>(src, g, B, alpha_inv, region, argmax, delta,
+                                                     maxabs_delta, status);
+    return cudaGetLastError();
+}
+
+cudaError_t simt_integersgd(const SgdBatch& b, cudaStream_t s) {
+    if (b.count <= 0) return cudaSuccess;
+    int64_t nmax = 0;
+    for (int i = 0; i < b.count; ++i) nmax = b.t[i].n > nmax ? b.t[i].n : nmax;
+    dim3 grid(grid_for(nmax, 256, 152 * 4), b.count);
+    double bytes = 0;
+    for (int i = 0; i < b.count; ++i) bytes += 16.0 * b.t[i].n;   // W r+w, dW r
+    ProfScope ps(K_INTEGERSGD, s, 0.0, bytes);
+    k_integersgd<<<grid, 256, 0, s>>>(b);
+    return cudaGetLastError();
+}
+
+cudaError_t simt_finish_loss(const unsigned long long* sse, int64_t* loss, cudaStream_t s) {
+    ProfScope ps(K_FINISH_LOSS, s, 0.0, 0.0);
+    k_finish_loss<<<1, 1, 0, s>>>(sse, loss);
+    return cudaGetLastError();
+}
+
+}  // namespace nitro

@@ -1,0 +1,481 @@
+// C ABI of the NITRO-D block step (declared in include/nitro.h): argument
+// checks, device memory of a block, and the launch sequence of forward,
+// backward and IntegerSGD on the caller's stream.
+#include <cstdio>
+#include <cstdlib>
+#include <algorithm>
+#include <cstring>
+#include <new>
+#include <vector>
+
+#include "nitro_internal.cuh"
+#include "tc_conv.cuh"
+
+using namespace nitro;
+
+namespace {
+
+constexpr int kLearningTensorId = 255;
+constexpr int kMaxLayers = kMaxSgdTensors - 1;
+
+struct Layer {
+    LayerGeom g;
+    int64_t in_f, out_f, pre_f;  // per-sample sizes: input, output (post-pool), pre-pool
+    int64_t wcount;
+    int32_t* W = nullptr;
+    int64_t* dW = nullptr;
+    int8_t* act = nullptr;       // [max_batch x out_f]
+    int8_t* region = nullptr;    // [max_batch x pre_f]
+    int8_t* argmax = nullptr;    // [max_batch x out_f] if pool
+    int32_t* delta = nullptr;    // [max_batch x pre_f]
+    TcLayer tc;                  // tensor-core state (limb planes, maps)
+};
+
+}  // namespace
+
+struct nitro_block {
+    nitro_block_desc desc{};
+    std::vector<Layer> L;
+    int G = 0, mu = 0;
+    int64_t d = 0;
+    int32_t* Wlr = nullptr;
+    int64_t* dWlr = nullptr;
+    int32_t* grad_l = nullptr;      // [max_batch x G]
+    int64_t* z64 = nullptr;         // scratch, int64 pre-activations / dgrad outputs
+    size_t z64_elems = 0;
+    uint32_t* words = nullptr;      // [0] status [1] max|grad_l| [2] max|W_lr|
+                                    // [3 + i] max|W_i|  [3 + n + i] max|delta_i|
+    unsigned long long* sse = nullptr;
+    int batch = 0;
+    std::vector<void*> allocs;
+    TcWorkspace tcw;
+};
+
+namespace {
+
+uint32_t* w_status(nitro_block* b) { return b->words; }
+uint32_t* w_gl(nitro_block* b) { return b->words + 1; }
+uint32_t* w_wlr(nitro_block* b) { return b->words + 2; }
+uint32_t* w_w(nitro_block* b, int i) { return b->words + 3 + i; }
+uint32_t* w_delta(nitro_block* b, int i) { return b->words + 3 + (int)b->L.size() + i; }
+int n_words(int n_layers) { return 3 + 2 * n_layers; }
+
+template <typename T>
+bool dalloc(nitro_block* b, T** p, size_t count) {
+    void* q = nullptr;
+    if (count == 0) count = 1;
+    if (cudaMalloc(&q, count * sizeof(T)) != cudaSuccess) return false;
+    b->allocs.push_back(q);
+    *p = static_cast<T*>(q);
+    return true;
+}
+
+void free_all(nitro_block* b) {
+    for (void* p : b->allocs) cudaFree(p);
+    b->allocs.clear();
+}
+
+uint64_t splitmix64_at(uint64_t seed, uint64_t index) {
+    uint64_t z = seed + (index + 1ULL) * 0x9E3779B97F4A7C15ULL;
+    z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ULL;
+    z = (z ^ (z >> 27)) * 0x94D049BB133111EBULL;
+    return z ^ (z >> 31);
+}
+
+int64_t isqrt64(int64_t n) {
+    if (n <= 0) return 0;
+    int64_t r = 0;
+    for (int64_t bit = (int64_t)1 << 62; bit; bit >>= 2) {  // digit-by-digit
+        if (n >= r + bit) { n -= r + bit; r = (r >> 1) + bit; } else { r >>= 1; }
+    }
+    return r;
+}
+
+// Integer Kaiming bound (Sec. 3.3.1)
+int64_t kaiming_bound(int64_t fan_in) { return fdiv64(128 * 1732, isqrt64(fan_in) * 1000); }
+
+std::vector<int32_t> draw_weights(int64_t n, int64_t fan_in, uint64_t seed, uint64_t tensor_id) {
+    const int64_t b = kaiming_bound(fan_in);
+    const uint64_t span = (uint64_t)(2 * b + 1);
+    std::vector<int32_t> w((size_t)n);
+    for (int64_t e = 0; e < n; ++e)
+        w[(size_t)e] = (int32_t)((int64_t)(splitmix64_at(seed, (tensor_id << 40) + (uint64_t)e) % span) - b);
+    return w;
+}
+
+uint32_t host_maxabs(const int32_t* p, size_t n) {
+    uint32_t m = 0;
+    for (size_t i = 0; i < n; ++i) m = abs_u32(p[i]) > m ? abs_u32(p[i]) : m;
+    return m;
+}
+
+nitro_status cuda_fail(cudaError_t e) {
+    return e == cudaSuccess ? NITRO_OK : NITRO_ERR_CUDA;
+}
+
+#define NITRO_TRY(expr)                                \
+    do {                                               \
+        cudaError_t _e = (expr);                       \
+        if (_e != cudaSuccess) return NITRO_ERR_CUDA;  \
+    } while (0)
+
+nitro_status validate(const nitro_block_desc* d) {
+    if (!d) return NITRO_ERR_ARG;
+    if (d->n_layers < 0 || d->n_layers > kMaxLayers) return NITRO_ERR_ARG;
+    if (d->n_layers > 0 && !d->layers) return NITRO_ERR_ARG;
+    if (d->num_classes < 1 || d->num_classes > 64) return NITRO_ERR_ARG;
+    if (d->alpha_inv < 2 || d->alpha_inv > (1 << 20)) return NITRO_ERR_ARG;
+    if (d->gamma_inv_lr < 1 || d->gamma_inv_lr > ((int64_t)1 << 48)) return NITRO_ERR_ARG;
+    if (d->eta_inv_fw < 0 || d->eta_inv_lr < 0) return NITRO_ERR_ARG;
+    if (d->sgd_round != NITRO_ROUND_FLOOR && d->sgd_round != NITRO_ROUND_TRUNC) return NITRO_ERR_ARG;
+    if (d->max_batch < 0 || d->max_batch > (1 << 20)) return NITRO_ERR_ARG;
+    if (d->in_features < 1 || d->in_features > (1 << 24)) return NITRO_ERR_ARG;
+    int64_t prev_out = d->in_features;
+    for (int i = 0; i < d->n_layers; ++i) {
+        const nitro_layer_desc& l = d->layers[i];
+        if (l.cin < 1 || l.cout < 1 || l.cin > (1 << 20) || l.cout > (1 << 20)) return NITRO_ERR_ARG;
+        if (l.pool2x2 != 0 && l.pool2x2 != 1) return NITRO_ERR_ARG;
+        int64_t in_f, out_f, pre_f;
+        if (l.kind == NITRO_CONV3X3) {
+            if (l.h < 1 || l.w < 1) return NITRO_ERR_ARG;
+            if (l.pool2x2 && (l.h < 2 || l.w < 2)) return NITRO_ERR_ARG;
+            in_f = (int64_t)l.h * l.w * l.cin;
+            pre_f = (int64_t)l.h * l.w * l.cout;
+            out_f = l.pool2x2 ? (int64_t)(l.h / 2) * (l.w / 2) * l.cout : pre_f;
+            // wgrad sums B*h*w terms of |delta| < 2^31 times |a| <= 2^7
+            if ((int64_t)d->max_batch * l.h * l.w > ((int64_t)1 << 24)) return NITRO_ERR_ARG;
+        } else if (l.kind == NITRO_LINEAR) {
+            if (l.h != 1 || l.w != 1 || l.pool2x2) return NITRO_ERR_ARG;
+            in_f = l.cin;
+            pre_f = out_f = l.cout;
+        } else {
+            return NITRO_ERR_ARG;
+        }
+        if (in_f != prev_out) return NITRO_ERR_ARG;
+        if (pre_f > (1 << 24) || in_f > (1 << 24)) return NITRO_ERR_ARG;
+        if ((int64_t)d->max_batch * (pre_f > in_f ? pre_f : in_f) >= ((int64_t)1 << 31)) return NITRO_ERR_ARG;
+        prev_out = out_f;
+    }
+    if ((int64_t)d->max_batch * prev_out >= ((int64_t)1 << 31)) return NITRO_ERR_ARG;
+    return NITRO_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* nitro_status_str(nitro_status s) {
+    switch (s) {
+        case NITRO_OK: return "ok";
+        case NITRO_ERR_ARG: return "invalid argument";
+        case NITRO_ERR_OVERFLOW: return "integer overflow";
+        case NITRO_ERR_TIMEOUT: return "device wait timed out";
+        case NITRO_ERR_CUDA: return "CUDA error";
+        case NITRO_ERR_UNSUPPORTED: return "unsupported";
+    }
+    return "unknown status";
+}
+
+nitro_status nitro_init_block(const nitro_block_desc* desc, uint64_t seed, void* stream,
+                              nitro_block** out) {
+    if (!out) return NITRO_ERR_ARG;
+    *out = nullptr;
+    nitro_status st = validate(desc);
+    if (st != NITRO_OK) return st;
+    cudaStream_t s = (cudaStream_t)stream;
+    nitro_block* b = new (std::nothrow) nitro_block();
+    if (!b) return NITRO_ERR_CUDA;
+    b->desc = *desc;
+    b->desc.layers = nullptr;
+    b->G = desc->num_classes;
+    {
+        // mu_int8: floor-average of the four segment means (Sec. 3.2.2)
+        const int a = desc->alpha_inv;
+        b->mu = (int)fdiv64(fdiv64(-127, a) + fdiv64(-127, 2 * a) + 63 + 127, 4);
+    }
+    const int MB = desc->max_batch;
+    size_t z_need = 0;
+    bool ok = true;
+    std::vector<std::vector<int32_t>> host_w;
+    for (int i = 0; i < desc->n_layers && ok; ++i) {
+        const nitro_layer_desc& l = desc->layers[i];
+        Layer ly;
+        ly.g.kind = l.kind; ly.g.cin = l.cin; ly.g.cout = l.cout;
+        ly.g.h = l.h; ly.g.w = l.w; ly.g.pool = l.pool2x2;
+        ly.g.oh = l.pool2x2 ? l.h / 2 : l.h;
+        ly.g.ow = l.pool2x2 ? l.w / 2 : l.w;
+        ly.in_f = (int64_t)l.h * l.w * l.cin;
+        ly.pre_f = (int64_t)l.h * l.w * l.cout;
+        ly.out_f = (int64_t)ly.g.oh * ly.g.ow * l.cout;
+        const int64_t fan_in = l.kind == NITRO_CONV3X3 ? 9LL * l.cin : (int64_t)l.cin;
+        ly.wcount = (int64_t)l.cout * fan_in;
+        ok = ok && dalloc(b, &ly.W, ly.wcount) && dalloc(b, &ly.dW, ly.wcount) &&
+             dalloc(b, &ly.act, (size_t)MB * ly.out_f) &&
+             dalloc(b, &ly.region, (size_t)MB * ly.pre_f) &&
+             dalloc(b, &ly.delta, (size_t)MB * ly.pre_f);
+        if (ok && l.pool2x2) ok = dalloc(b, &ly.argmax, (size_t)MB * ly.out_f);
+        z_need = std::max(z_need, (size_t)MB * (size_t)ly.pre_f);
+        z_need = std::max(z_need, (size_t)MB * (size_t)ly.in_f);
+        host_w.push_back(draw_weights(ly.wcount, fan_in, seed, (uint64_t)i));
+        b->L.push_back(ly);
+    }
+    b->d = desc->n_layers ? b->L.back().out_f : desc->in_features;
+    ok = ok && dalloc(b, &b->Wlr, (size_t)b->G * b->d) && dalloc(b, &b->dWlr, (size_t)b->G * b->d) &&
+         dalloc(b, &b->grad_l, (size_t)MB * b->G) && dalloc(b, &b->z64, z_need) &&
+         dalloc(b, &b->words, n_words(desc->n_layers)) && dalloc(b, &b->sse, 1);
+    b->z64_elems = z_need;
+    if (ok) ok = tc_block_init(b->tcw, b->allocs, desc->max_batch);
+    for (int i = 0; ok && i < desc->n_layers; ++i)
+        ok = tc_layer_init(b->L[i].tc, b->L[i].g, desc->max_batch, b->tcw, b->allocs);
+    if (!ok) {
+        free_all(b);
+        delete b;
+        return NITRO_ERR_CUDA;
+    }
+    std::vector<int32_t> wlr = draw_weights((int64_t)b->G * b->d, b->d, seed, kLearningTensorId);
+    std::vector<uint32_t> words(n_words(desc->n_layers), 0);
+    words[2] = host_maxabs(wlr.data(), wlr.size());
+    cudaError_t e = cudaSuccess;
+    for (int i = 0; i < desc->n_layers && e == cudaSuccess; ++i) {
+        words[3 + i] = host_maxabs(host_w[i].data(), host_w[i].size());
+        e = cudaMemcpyAsync(b->L[i].W, host_w[i].data(), host_w[i].size() * 4, cudaMemcpyHostToDevice, s);
+        if (e == cudaSuccess) e = cudaMemsetAsync(b->L[i].dW, 0, (size_t)b->L[i].wcount * 8, s);
+    }
+    if (e == cudaSuccess) e = cudaMemcpyAsync(b->Wlr, wlr.data(), wlr.size() * 4, cudaMemcpyHostToDevice, s);
+    if (e == cudaSuccess) e = cudaMemsetAsync(b->dWlr, 0, (size_t)b->G * b->d * 8, s);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(b->words, words.data(), words.size() * 4, cudaMemcpyHostToDevice, s);
+    if (e == cudaSuccess) e = cudaMemsetAsync(b->sse, 0, 8, s);
+    for (int i = 0; e == cudaSuccess && i < desc->n_layers; ++i)
+        e = tc_refresh_weights(b->L[i].tc, b->L[i].g, b->L[i].W, w_w(b, i), s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) {
+        free_all(b);
+        delete b;
+        return NITRO_ERR_CUDA;
+    }
+    *out = b;
+    return NITRO_OK;
+}
+
+void nitro_destroy_block(nitro_block* b) {
+    if (!b) return;
+    cudaDeviceSynchronize();
+    free_all(b);
+    delete b;
+}
+
+nitro_status nitro_block_forward(nitro_block* b, const int8_t* a_in, int batch, int8_t* a_out,
+                                 void* stream) {
+    if (!b || batch < 0 || batch > b->desc.max_batch) return NITRO_ERR_ARG;
+    if (batch > 0 && !a_in) return NITRO_ERR_ARG;
+    cudaStream_t s = (cudaStream_t)stream;
+    b->batch = batch;
+    if (batch == 0) return NITRO_OK;
+    const int n = (int)b->L.size();
+    const int8_t* x = a_in;
+    for (int i = 0; i < n; ++i) {
+        Layer& ly = b->L[i];
+        const LayerGeom& g = ly.g;
+        int8_t* out2 = (i == n - 1) ? a_out : nullptr;
+        bool done = false;
+        NITRO_TRY(tc_conv_forward(ly.tc, g, x, batch, b->desc.alpha_inv, b->mu, ly.act, out2,
+                                  ly.region, ly.argmax, b->tcw, s, &done));
+        if (!done) {
+            const int mode = g.kind == NITRO_CONV3X3 ? GM_CONV_FWD : GM_LIN_FWD;
+            NITRO_TRY(simt_gemm(mode, x, nullptr, ly.W, b->z64, batch, g.h, g.w, g.cin, g.cout, s));
+            NITRO_TRY(simt_fwd_epilogue(b->z64, g, batch, b->desc.alpha_inv, b->mu, ly.act, out2,
+                                        ly.region, ly.argmax, s));
+        }
+        x = ly.act;
+    }
+    return NITRO_OK;
+}
+
+nitro_status nitro_block_backward(nitro_block* b, const int8_t* a_in, const int32_t* labels,
+                                  int batch, int64_t* loss_dev, void* stream) {
+    if (!b || batch < 0 || batch != b->batch) return NITRO_ERR_ARG;
+    if (batch > 0 && (!labels || !a_in)) return NITRO_ERR_ARG;
+    cudaStream_t s = (cudaStream_t)stream;
+    const int n = (int)b->L.size();
+    const int G = b->G;
+    const int64_t d = b->d;
+    // reset per-step accumulators and range words
+    NITRO_TRY(cudaMemsetAsync(b->sse, 0, sizeof(unsigned long long), s));
+    NITRO_TRY(cudaMemsetAsync(w_gl(b), 0, 4, s));
+    if (n) NITRO_TRY(cudaMemsetAsync(w_delta(b, 0), 0, 4 * n, s));
+    if (batch == 0) {
+        NITRO_TRY(cudaMemsetAsync(b->dWlr, 0, (size_t)G * d * 8, s));
+        for (int i = 0; i < n; ++i) NITRO_TRY(cudaMemsetAsync(b->L[i].dW, 0, (size_t)b->L[i].wcount * 8, s));
+        if (loss_dev) NITRO_TRY(cudaMemsetAsync(loss_dev, 0, 8, s));
+        return NITRO_OK;
+    }
+    const int8_t* a_last = n ? b->L[n - 1].act : a_in;
+    NITRO_TRY(simt_learn_fwd(a_last, b->Wlr, labels, batch, (int)d, G, b->grad_l, b->sse, w_gl(b),
+                             w_status(b), s));
+    NITRO_TRY(simt_learn_dw(a_last, b->grad_l, batch, (int)d, G, b->dWlr, s));
+    if (loss_dev) NITRO_TRY(simt_finish_loss(b->sse, loss_dev, s));
+    if (n == 0) return NITRO_OK;
+    // delta_fw = grad_L W_lr (pre-update), into the last layer
+    {
+        Layer& ly = b->L[n - 1];
+        DeltaSrc src{};
+        src.grad_l = b->grad_l; src.wlr = b->Wlr; src.G = G;
+        src.maxabs_a = w_gl(b); src.maxabs_b = w_wlr(b); src.bound_k = G;
+        NITRO_TRY(simt_grad_to_delta(src, ly.g, batch, b->desc.alpha_inv, ly.region, ly.argmax,
+                                     ly.delta, w_delta(b, n - 1), w_status(b), s));
+    }
+    for (int i = n - 1; i >= 0; --i) {
+        Layer& ly = b->L[i];
+        const LayerGeom& g = ly.g;
+        const int8_t* x = i ? b->L[i - 1].act : a_in;
+        bool done = false;
+        NITRO_TRY(tc_conv_wgrad(ly.tc, g, x, ly.delta, w_delta(b, i), batch, ly.dW, b->tcw, s, &done));
+        if (!done) {
+            const int mode = g.kind == NITRO_CONV3X3 ? GM_CONV_WGRAD : GM_LIN_WGRAD;
+            NITRO_TRY(simt_gemm(mode, x, ly.delta, nullptr, ly.dW, batch, g.h, g.w, g.cin, g.cout, s));
+        }
+        if (i == 0) break;
+        done = false;
+        NITRO_TRY(tc_conv_dgrad(ly.tc, g, ly.delta, w_delta(b, i), batch, b->z64, b->tcw, s, &done));
+        if (!done) {
+            const int mode = g.kind == NITRO_CONV3X3 ? GM_CONV_DGRAD : GM_LIN_DGRAD;
+            NITRO_TRY(simt_gemm(mode, nullptr, ly.delta, ly.W, b->z64, batch, g.h, g.w, g.cin, g.cout, s));
+        }
+        Layer& lo = b->L[i - 1];
+        DeltaSrc src{};
+        src.g64 = b->z64;
+        src.maxabs_a = w_delta(b, i); src.maxabs_b = w_w(b, i);
+        src.bound_k = g.kind == NITRO_CONV3X3 ? 9LL * g.cout : (int64_t)g.cout;
+        NITRO_TRY(simt_grad_to_delta(src, lo.g, batch, b->desc.alpha_inv, lo.region, lo.argmax,
+                                     lo.delta, w_delta(b, i - 1), w_status(b), s));
+    }
+    return NITRO_OK;
+}
+
+nitro_status nitro_integersgd_step(nitro_block* b, void* stream) {
+    if (!b) return NITRO_ERR_ARG;
+    cudaStream_t s = (cudaStream_t)stream;
+    const int n = (int)b->L.size();
+    // gamma_inv^fw = AF * gamma_inv^lr, AF = 2^6 * G (Sec. 3.3.5)
+    const int64_t gamma_fw = 64LL * b->G * b->desc.gamma_inv_lr;
+    SgdBatch bt{};
+    bt.round_trunc = b->desc.sgd_round == NITRO_ROUND_TRUNC;
+    bt.status = w_status(b);
+    for (int i = 0; i < n; ++i)
+        bt.t[bt.count++] = SgdTensor{b->L[i].W, b->L[i].dW, b->L[i].wcount, gamma_fw,
+                                     b->desc.eta_inv_fw, w_w(b, i)};
+    bt.t[bt.count++] = SgdTensor{b->Wlr, b->dWlr, (int64_t)b->G * b->d, b->desc.gamma_inv_lr,
+                                 b->desc.eta_inv_lr, w_wlr(b)};
+    NITRO_TRY(cudaMemsetAsync(w_wlr(b), 0, 4, s));
+    if (n) NITRO_TRY(cudaMemsetAsync(w_w(b, 0), 0, 4 * n, s));
+    NITRO_TRY(simt_integersgd(bt, s));
+    for (int i = 0; i < n; ++i)
+        NITRO_TRY(tc_refresh_weights(b->L[i].tc, b->L[i].g, b->L[i].W, w_w(b, i), s));
+    return NITRO_OK;
+}
+
+nitro_status nitro_block_tensor_bytes(const nitro_block* b, int which, int layer, size_t* bytes) {
+    if (!b || !bytes) return NITRO_ERR_ARG;
+    const int n = (int)b->L.size();
+    const bool per_layer = which == NITRO_T_W || which == NITRO_T_DW || which == NITRO_T_ACT ||
+                           which == NITRO_T_REGION || which == NITRO_T_ARGMAX || which == NITRO_T_DELTA;
+    if (per_layer && (layer < 0 || layer >= n)) return NITRO_ERR_ARG;
+    if (!per_layer && layer != 0) return NITRO_ERR_ARG;
+    const size_t B = (size_t)b->batch;
+    switch (which) {
+        case NITRO_T_W: *bytes = (size_t)b->L[layer].wcount * 4; break;
+        case NITRO_T_DW: *bytes = (size_t)b->L[layer].wcount * 8; break;
+        case NITRO_T_WLR: *bytes = (size_t)b->G * b->d * 4; break;
+        case NITRO_T_DWLR: *bytes = (size_t)b->G * b->d * 8; break;
+        case NITRO_T_ACT: *bytes = B * b->L[layer].out_f; break;
+        case NITRO_T_REGION: *bytes = B * b->L[layer].pre_f; break;
+        case NITRO_T_ARGMAX:
+            if (!b->L[layer].g.pool) return NITRO_ERR_ARG;
+            *bytes = B * b->L[layer].out_f;
+            break;
+        case NITRO_T_DELTA: *bytes = B * b->L[layer].pre_f * 4; break;
+        case NITRO_T_GRAD_L: *bytes = B * b->G * 4; break;
+        case NITRO_T_SSE: *bytes = 8; break;
+        default: return NITRO_ERR_ARG;
+    }
+    return NITRO_OK;
+}
+
+static const void* tensor_ptr(nitro_block* b, int which, int layer) {
+    switch (which) {
+        case NITRO_T_W: return b->L[layer].W;
+        case NITRO_T_DW: return b->L[layer].dW;
+        case NITRO_T_WLR: return b->Wlr;
+        case NITRO_T_DWLR: return b->dWlr;
+        case NITRO_T_ACT: return b->L[layer].act;
+        case NITRO_T_REGION: return b->L[layer].region;
+        case NITRO_T_ARGMAX: return b->L[layer].argmax;
+        case NITRO_T_DELTA: return b->L[layer].delta;
+        case NITRO_T_GRAD_L: return b->grad_l;
+        case NITRO_T_SSE: return b->sse;
+    }
+    return nullptr;
+}
+
+static nitro_status latched(uint32_t bits) {
+    if (bits & ST_TIMEOUT) return NITRO_ERR_TIMEOUT;
+    if (bits & ST_OVERFLOW) return NITRO_ERR_OVERFLOW;
+    if (bits & ST_BAD_LABEL) return NITRO_ERR_ARG;
+    return NITRO_OK;
+}
+
+uint32_t nitro_block_status_bits(nitro_block* b) {
+    if (!b) return 0;
+    uint32_t bits = 0;
+    if (cudaDeviceSynchronize() != cudaSuccess) return 0xffffffffu;
+    if (cudaMemcpy(&bits, b->words, 4, cudaMemcpyDeviceToHost) != cudaSuccess) return 0xffffffffu;
+    return bits;
+}
+
+nitro_status nitro_block_status(nitro_block* b, int clear) {
+    if (!b) return NITRO_ERR_ARG;
+    const uint32_t bits = nitro_block_status_bits(b);
+    if (bits == 0xffffffffu) return NITRO_ERR_CUDA;
+    if (clear && cudaMemset(b->words, 0, 4) != cudaSuccess) return NITRO_ERR_CUDA;
+    if (clear && cudaDeviceSynchronize() != cudaSuccess) return NITRO_ERR_CUDA;
+    return latched(bits);
+}
+
+nitro_status nitro_block_get_tensor(nitro_block* b, int which, int layer, void* host_dst,
+                                    size_t bytes) {
+    size_t need = 0;
+    nitro_status st = nitro_block_tensor_bytes(b, which, layer, &need);
+    if (st != NITRO_OK) return st;
+    if (bytes != need || (need && !host_dst)) return NITRO_ERR_ARG;
+    if (cudaDeviceSynchronize() != cudaSuccess) return NITRO_ERR_CUDA;
+    if (need && cudaMemcpy(host_dst, tensor_ptr(b, which, layer), need, cudaMemcpyDeviceToHost) != cudaSuccess)
+        return NITRO_ERR_CUDA;
+    uint32_t bits = 0;
+    if (cudaMemcpy(&bits, b->words, 4, cudaMemcpyDeviceToHost) != cudaSuccess) return NITRO_ERR_CUDA;
+    return latched(bits);
+}
+
+nitro_status nitro_block_set_tensor(nitro_block* b, int which, int layer, const void* host_src,
+                                    size_t bytes) {
+    if (which != NITRO_T_W && which != NITRO_T_DW && which != NITRO_T_WLR && which != NITRO_T_DWLR)
+        return NITRO_ERR_ARG;
+    size_t need = 0;
+    nitro_status st = nitro_block_tensor_bytes(b, which, layer, &need);
+    if (st != NITRO_OK) return st;
+    if (bytes != need || !host_src) return NITRO_ERR_ARG;
+    if (cudaDeviceSynchronize() != cudaSuccess) return NITRO_ERR_CUDA;
+    if (cudaMemcpy((void*)tensor_ptr(b, which, layer), host_src, need, cudaMemcpyHostToDevice) != cudaSuccess)
+        return NITRO_ERR_CUDA;
+    if (which == NITRO_T_W || which == NITRO_T_WLR) {
+        const uint32_t m = host_maxabs(static_cast<const int32_t*>(host_src), need / 4);
+        uint32_t* word = which == NITRO_T_W ? w_w(b, layer) : w_wlr(b);
+        if (cudaMemcpy(word, &m, 4, cudaMemcpyHostToDevice) != cudaSuccess) return NITRO_ERR_CUDA;
+        if (which == NITRO_T_W &&
+            tc_refresh_weights(b->L[layer].tc, b->L[layer].g, b->L[layer].W, word, 0) != cudaSuccess)
+            return NITRO_ERR_CUDA;
+    }
+    if (cudaDeviceSynchronize() != cudaSuccess) return NITRO_ERR_CUDA;
+    return NITRO_OK;
+}
+
+}  // extern "C"

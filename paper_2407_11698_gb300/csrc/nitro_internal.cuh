@@ -1,0 +1,146 @@
+// Internal declarations of the GB300 NITRO-D library (not part of the ABI).
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "nitro.h"
+
+namespace nitro {
+
+// ---------------------------------------------------------------------------
+// Integer helpers, device and host.  fdiv is the paper's \intdiv (floor).
+// ---------------------------------------------------------------------------
+__host__ __device__ __forceinline__ int64_t fdiv64(int64_t x, int64_t d) {
+    int64_t q = x / d;
+    return (x % d < 0) ? q - 1 : q;
+}
+__host__ __device__ __forceinline__ int32_t fdiv32(int32_t x, int32_t d) {
+    int32_t q = x / d;
+    return (x % d < 0) ? q - 1 : q;
+}
+__host__ __device__ __forceinline__ int64_t tdiv64(int64_t x, int64_t d) { return x / d; }
+
+// floor(z / (256 * k)) = floor(floor(z / 256) / k) for k > 0; the first step
+// is an arithmetic shift.
+__host__ __device__ __forceinline__ int64_t scale_floor(int64_t z, int64_t k) {
+    return fdiv64(z >> 8, k);
+}
+
+__host__ __device__ __forceinline__ bool fits_i32(int64_t v) {
+    return v >= INT32_MIN && v <= INT32_MAX;
+}
+
+// NITRO-ReLU piece of x: 0 x<-127, 1 -127<=x<0, 2 0<=x<=127, 3 x>127.
+__host__ __device__ __forceinline__ int relu_region(int64_t x) {
+    return x < -127 ? 0 : (x < 0 ? 1 : (x <= 127 ? 2 : 3));
+}
+// NITRO-ReLU forward value (Sec. 3.2.2).
+__host__ __device__ __forceinline__ int relu_value(int64_t x, int alpha_inv, int mu) {
+    if (x < 0) {
+        int c = x < -127 ? -127 : (int)x;
+        return fdiv32(c, alpha_inv) - mu;
+    }
+    return (x > 127 ? 127 : (int)x) - mu;
+}
+// NITRO-ReLU backward per piece.
+__host__ __device__ __forceinline__ int32_t relu_backward(int32_t g, int region, int alpha_inv) {
+    return region == 1 ? fdiv32(g, alpha_inv) : (region == 2 ? g : 0);
+}
+
+__host__ __device__ __forceinline__ uint32_t abs_u32(int32_t v) {
+    return v < 0 ? (uint32_t)(-(int64_t)v) : (uint32_t)v;
+}
+
+// max|A| * max|B| * k >= 2^63 : int64 exactness of an int32 x int32
+// contraction of length k is no longer guaranteed.
+__host__ __device__ __forceinline__ bool int64_bound_exceeded(uint32_t ma, uint32_t mb, int64_t k) {
+    unsigned __int128 p = (unsigned __int128)ma * mb * (unsigned __int128)k;
+    return p >= ((unsigned __int128)1 << 63);
+}
+
+// ---------------------------------------------------------------------------
+// Layer geometry as the kernels see it.
+// ---------------------------------------------------------------------------
+struct LayerGeom {
+    int kind;       // NITRO_CONV3X3 / NITRO_LINEAR
+    int cin, cout;  // linear: cin = in features, cout = out features
+    int h, w;       // input spatial (1 for linear)
+    int pool;       // 2x2 max-pool after NITRO-ReLU
+    int oh, ow;     // output spatial after the optional pool
+};
+
+// Device status word bits (same values as the ABI's NITRO_STATUS_BIT_*).
+enum : uint32_t { ST_OVERFLOW = 1u, ST_BAD_LABEL = 2u, ST_TIMEOUT = 4u };
+
+// ---------------------------------------------------------------------------
+// CUDA-core kernels (kernels_simt.cu).  All launch on `s`, return the launch
+// error, and do nothing for empty problems.
+// ---------------------------------------------------------------------------
+enum GemmMode : int {
+    GM_CONV_FWD = 0,    // C[p][co]      = sum_(t,ci) a[p + tap t][ci] * W[co][t][ci]
+    GM_CONV_DGRAD = 1,  // C[p][ci]      = sum_(t,co) g[p - tap t][co] * W[co][t][ci]
+    GM_CONV_WGRAD = 2,  // C[co][(t,ci)] = sum_p g[p][co] * a[p + tap t][ci]
+    GM_LIN_FWD = 3,     // C[b][o] = sum_i a[b][i] * W[o][i]
+    GM_LIN_DGRAD = 4,   // C[b][i] = sum_o g[b][o] * W[o][i]
+    GM_LIN_WGRAD = 5    // C[o][i] = sum_b g[b][o] * a[b][i]
+};
+
+// Exact int64 implicit GEMM on CUDA cores.  act: int8 activations, grad:
+// int32 gradients, wts: int32 weights; out: int64, row-major C (overwritten).
+cudaError_t simt_gemm(int mode, const int8_t* act, const int32_t* grad, const int32_t* wts,
+                      int64_t* out, int B, int H, int W, int Cin, int Cout, cudaStream_t s);
+
+// z (int64, pre-pool NHWC) -> NITRO-Scaling -> NITRO-ReLU -> region codes,
+// optional 2x2 max-pool with argmax codes, int8 outputs (out2 may be NULL).
+cudaError_t simt_fwd_epilogue(const int64_t* z, const LayerGeom& g, int B, int alpha_inv,
+                              int mu, int8_t* out, int8_t* out2, int8_t* region,
+                              int8_t* argmax, cudaStream_t s);
+
+// Learning layer forward + loss: grad_l = floor(a W^T / (256 d)) - 32 onehot,
+// sse += sum grad_l^2 (mod 2^64), words[1] = max|grad_l|, status bits.
+cudaError_t simt_learn_fwd(const int8_t* a, const int32_t* wlr, const int32_t* labels, int B,
+                           int d, int G, int32_t* grad_l, unsigned long long* sse,
+                           uint32_t* maxabs_gl, uint32_t* status, cudaStream_t s);
+
+// dW_lr[g][j] = sum_b grad_l[b][g] a[b][j]
+cudaError_t simt_learn_dw(const int8_t* a, const int32_t* grad_l, int B, int d, int G,
+                          int64_t* dwlr, cudaStream_t s);
+
+// Gradient at the output of layer g (post-pool) -> delta at its
+// pre-activation: max-pool backward, NITRO-ReLU backward, STE.  The source
+// is either delta_fw = grad_l W_lr (lr_wlr != NULL) or an int64 dgrad output.
+struct DeltaSrc {
+    const int32_t* grad_l;   // [B][G]   (learning-layer source)
+    const int32_t* wlr;      // [G][d]
+    int G;
+    const uint32_t* maxabs_a;  // bound check operands: max|grad| and max|W|
+    const uint32_t* maxabs_b;
+    int64_t bound_k;           // contraction length for the bound
+    const int64_t* g64;      // [B][out features of the layer] (dgrad source)
+};
+cudaError_t simt_grad_to_delta(const DeltaSrc& src, const LayerGeom& g, int B, int alpha_inv,
+                               const int8_t* region, const int8_t* argmax, int32_t* delta,
+                               uint32_t* maxabs_delta, uint32_t* status, cudaStream_t s);
+
+// IntegerSGD (Algorithm 1) over up to kMaxSgdTensors tensors in one launch.
+constexpr int kMaxSgdTensors = 16;
+struct SgdTensor {
+    int32_t* w;
+    const int64_t* dw;
+    int64_t n;
+    int64_t gamma_inv, eta_inv;
+    uint32_t* maxabs_w;
+};
+struct SgdBatch {
+    SgdTensor t[kMaxSgdTensors];
+    int count;
+    int round_trunc;
+    uint32_t* status;
+};
+cudaError_t simt_integersgd(const SgdBatch& b, cudaStream_t s);
+
+// loss = floor(int64(sse) / 2)
+cudaError_t simt_finish_loss(const unsigned long long* sse, int64_t* loss, cudaStream_t s);
+
+}  // namespace nitro

@@ -1,0 +1,107 @@
+"""Host-side checks of the C-ABI library (no GPU needed).
+
+Builds libnitro.so if needed (cross-compiling needs no GPU), loads it, and
+checks that every function include/*.h declares is exported, and that
+argument checks that run before any device call reject bad input.
+"""
+import ctypes
+import glob
+import os
+import re
+import subprocess
+
+import pytest
+
+from paper_2407_11698_gb300 import binding as nb
+from paper_2407_11698_gb300 import build as nbuild
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _declared_functions():
+    names = set()
+    for h in glob.glob(os.path.join(ROOT, "include", "*.h")):
+        text = open(h).read()
+        text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+        for m in re.finditer(r"^\s*[A-Za-z_][\w\s\*]*?\b(nitro_\w+)\s*\(", text, flags=re.M):
+            names.add(m.group(1))
+    return sorted(names)
+
+
+@pytest.fixture(scope="module")
+def lib():
+    nbuild.build()
+    return nb.lib()
+
+
+def test_header_declares_the_four_step_entry_points():
+    names = _declared_functions()
+    for fn in ("nitro_init_block", "nitro_block_forward", "nitro_block_backward",
+               "nitro_integersgd_step"):
+        assert fn in names
+
+
+def test_every_declared_symbol_is_exported(lib):
+    out = subprocess.run(["nm", "-D", "--defined-only", nbuild.LIB], capture_output=True,
+                         text=True, check=True).stdout
+    exported = {line.split()[-1] for line in out.splitlines() if " T " in line}
+    missing = [n for n in _declared_functions() if n not in exported]
+    assert not missing, missing
+    for n in _declared_functions():
+        assert hasattr(lib, n)
+
+
+def test_status_strings(lib):
+    assert nb.status_str(nb.NITRO_OK) == "ok"
+    assert nb.status_str(nb.NITRO_ERR_OVERFLOW) == "integer overflow"
+    assert nb.status_str(99) == "unknown status"
+
+
+def _bad(**kw):
+    base = dict(layers=[(nb.NITRO_CONV3X3, 1, 4, 6, 6, 1)], in_features=36, max_batch=2)
+    base.update(kw)
+    layers = base.pop("layers")
+    in_f = base.pop("in_features")
+    d, keep = nb.make_block_desc(layers, in_f, **base)
+    st, h = nb.nitro_init_block(d, 1, None)
+    return st, h, keep
+
+
+@pytest.mark.parametrize("kw", [
+    dict(alpha_inv=1),                                      # int8 output range needs alpha_inv >= 2
+    dict(num_classes=0),
+    dict(gamma_inv_lr=0),
+    dict(eta_inv_fw=-1),
+    dict(sgd_round=2),
+    dict(max_batch=-1),
+    dict(in_features=35),                                   # chain mismatch
+    dict(layers=[(nb.NITRO_LINEAR, 36, 4, 2, 1, 0)]),       # linear takes h = w = 1
+    dict(layers=[(nb.NITRO_LINEAR, 36, 4, 1, 1, 1)]),       # no pool after linear
+    dict(layers=[(7, 1, 4, 6, 6, 0)]),                      # unknown kind
+    dict(layers=[(nb.NITRO_CONV3X3, 1, 4, 6, 6, 1), (nb.NITRO_LINEAR, 37, 3, 1, 1, 0)]),
+    dict(layers=[], in_features=0),
+])
+def test_init_rejects_bad_descriptors(lib, kw):
+    st, h, _ = _bad(**kw)
+    assert st == nb.NITRO_ERR_ARG and not h.value
+
+
+def test_null_handle_calls_are_rejected(lib):
+    assert nb.nitro_block_forward(None, None, 0, None) == nb.NITRO_ERR_ARG
+    assert nb.nitro_block_backward(None, None, None, 0, None) == nb.NITRO_ERR_ARG
+    assert nb.nitro_integersgd_step(None) == nb.NITRO_ERR_ARG
+    assert nb.nitro_block_status(None) == nb.NITRO_ERR_ARG
+    nb.nitro_destroy_block(None)
+    st, _ = nb.nitro_block_tensor_bytes(None, nb.NITRO_T_W, 0)
+    assert st == nb.NITRO_ERR_ARG
+
+
+def test_oracle_library_builds_independently():
+    from oracle import build as obuild
+    path = obuild.build()
+    lib_o = ctypes.CDLL(path)
+    assert hasattr(lib_o, "nor_conv3x3_fwd")
+    # the oracle and the GPU library share no symbols
+    out = subprocess.run(["nm", "-D", "--defined-only", path], capture_output=True, text=True,
+                         check=True).stdout
+    assert not any(" nitro_" in l for l in out.splitlines())
