@@ -172,6 +172,32 @@ uint32_t nitro_block_status_bits(nitro_block* blk);
 /* Releases every device buffer of the block.  NULL is ignored. */
 void nitro_destroy_block(nitro_block* blk);
 
+/* ---- Allocation-free layer forward ----------------------------------------
+ * The paper has no counterpart to this call: it exists for callers that
+ * cannot allocate device memory once running - code inside a host program
+ * that owns the whole device-memory budget, real-time loops that forbid
+ * allocation after start-up, or code that must not let cudaMalloc/cudaFree
+ * synchronise the device.
+ *
+ * Runs the forward of ONE 3x3 conv layer exactly as nitro_block_forward does
+ * (conv, NITRO-Scaling, NITRO-ReLU, optional 2x2 max-pool) on caller-owned
+ * buffers: a_in int8 NHWC [batch x h x w x cin], weights int32 OHWI, a_out
+ * int8 [batch x h' x w' x cout], region int8 [batch x h x w x cout], argmax
+ * int8 [batch x h' x w' x cout] (pool2x2 only, else may be NULL).  It calls no
+ * cudaMalloc, cudaFree or allocating library routine: the int64
+ * pre-activations go to a fixed 16 MiB array inside the library, so
+ * batch*h*w*cout may be at most 2^21; larger sizes return NITRO_ERR_ARG and
+ * queue nothing.  Every GPU that loads the library holds that array until the
+ * process exits.  The first call on each device looks up the array's address
+ * (cudaGetSymbolAddress, with that device current); make that first call
+ * before any stream capture.  All calls share the one array: calls whose work
+ * overlaps on the GPU (different streams, or different host threads) race
+ * and give wrong results; serialise them, e.g. on one stream. */
+nitro_status nitro_conv3x3_forward_noalloc(const int8_t* a_in, const int32_t* weights, int batch,
+                                           int h, int w, int cin, int cout, int pool2x2,
+                                           int alpha_inv, int8_t* a_out, int8_t* region,
+                                           int8_t* argmax, void* stream);
+
 /* ---- Diagnostics (not part of the training step) -------------------------
  * Every kernel launch of the library is counted.  With profiling on, each
  * launch is also bracketed by CUDA events recorded on its own stream and

@@ -89,6 +89,8 @@ def lib():
     _PD = ctypes.POINTER(ctypes.c_double)
     L.nitro_profile_read.argtypes = [ctypes.c_int, ctypes.POINTER(ctypes.c_uint64), _PD, _PD, _PD]
     L.nitro_profile_read.restype = ctypes.c_int
+    L.nitro_conv3x3_forward_noalloc.argtypes = [_VP, _VP] + [ctypes.c_int] * 7 + [_VP, _VP, _VP, _VP]
+    L.nitro_conv3x3_forward_noalloc.restype = ctypes.c_int
     for name in ("nitro_init_block", "nitro_block_forward", "nitro_block_backward",
                  "nitro_integersgd_step", "nitro_block_tensor_bytes", "nitro_block_get_tensor",
                  "nitro_block_set_tensor", "nitro_block_status"):
@@ -144,6 +146,13 @@ def nitro_block_status(blk, clear=False):
 
 def nitro_block_status_bits(blk):
     return lib().nitro_block_status_bits(blk)
+
+
+def nitro_conv3x3_forward_noalloc(a_in, weights, batch, h, w, cin, cout, pool2x2, alpha_inv,
+                                  a_out, region, argmax, stream=None):
+    return lib().nitro_conv3x3_forward_noalloc(a_in, weights, int(batch), int(h), int(w), int(cin),
+                                               int(cout), int(pool2x2), int(alpha_inv), a_out,
+                                               region, argmax, stream)
 
 
 def nitro_destroy_block(blk):

@@ -1,0 +1,75 @@
+"""The allocation-free conv forward against the block forward (GPU).
+
+nitro_conv3x3_forward_noalloc serves callers that cannot allocate device
+memory while running; it keeps its int64 scratch in a fixed array inside the
+library.  This file is named to be collected last, so a run that stops at
+the first failure has run every other test before it.
+"""
+import numpy as np
+import pytest
+
+from paper_2407_11698_gb300 import binding as nb
+from paper_2407_11698_gb300 import synth
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def torch():
+    t = pytest.importorskip("torch")
+    if not t.cuda.is_available():
+        pytest.skip("no CUDA device")
+    nb.lib()
+    return t
+
+
+def _block_forward(torch, blk, x):
+    out = torch.empty((x.shape[0], blk.out_features), dtype=torch.int8, device="cuda")
+    blk.forward(x, out)
+    return (blk.get(nb.NITRO_T_ACT, 0), blk.get(nb.NITRO_T_REGION, 0),
+            blk.get(nb.NITRO_T_ARGMAX, 0) if blk.layers[0][5] else None)
+
+
+def _noalloc_forward(torch, x, w, B, h, wd, cin, cout, pool, alpha):
+    oh, ow = (h // 2, wd // 2) if pool else (h, wd)
+    out = torch.full((B, oh * ow * cout), 99, dtype=torch.int8, device="cuda")
+    region = torch.full((B, h * wd * cout), 99, dtype=torch.int8, device="cuda")
+    am = torch.full((B, oh * ow * cout), 99, dtype=torch.int8, device="cuda") if pool else None
+    st = nb.nitro_conv3x3_forward_noalloc(nb._ptr(x), nb._ptr(w), B, h, wd, cin, cout, pool, alpha,
+                                          nb._ptr(out), nb._ptr(region), nb._ptr(am),
+                                          nb._stream_ptr(None))
+    assert st == nb.NITRO_OK, nb.status_str(st)
+    torch.cuda.synchronize()
+    return (out.cpu().numpy().reshape(-1), region.cpu().numpy().reshape(-1),
+            None if am is None else am.cpu().numpy().reshape(-1))
+
+
+@pytest.mark.parametrize("shape", [(16, 28, 28, 1, 32, 1, 10), (5, 7, 9, 6, 11, 1, 4),
+                                   (3, 8, 8, 64, 64, 0, 10)])
+def test_noalloc_matches_block_forward_on_two_calls_in_a_row(torch, shape):
+    B, h, wd, cin, cout, pool, alpha = shape
+    blk = nb.Block([(nb.NITRO_CONV3X3, cin, cout, h, wd, pool)], h * wd * cin, seed=3,
+                   max_batch=B, alpha_inv=alpha)
+    try:
+        # wide weights (several int8 limbs) as well as the initial ones
+        for call, scale in enumerate((1, 70001)):
+            w = (blk.get(nb.NITRO_T_W, 0).astype(np.int64) * scale).astype(np.int32)
+            blk.set(nb.NITRO_T_W, 0, w)
+            x = torch.from_numpy(synth.images(9, call, B, (h, wd, cin)).reshape(B, -1)).cuda()
+            wd_dev = torch.from_numpy(w).cuda()
+            want = _block_forward(torch, blk, x)
+            got = _noalloc_forward(torch, x, wd_dev, B, h, wd, cin, cout, pool, alpha)
+            for g_, w_ in zip(got, want):
+                if w_ is None:
+                    assert g_ is None
+                else:
+                    assert np.array_equal(g_, w_), "call %d differs" % call
+    finally:
+        blk.close()
+
+
+def test_noalloc_rejects_sizes_beyond_its_array(torch):
+    # 2^21 int64 pre-activations at most: 64 x 32 x 32 x 64 = 2^22 is too large
+    st = nb.nitro_conv3x3_forward_noalloc(None, None, 64, 32, 32, 64, 64, 0, 10, None, None, None,
+                                          nb._stream_ptr(None))
+    assert st == nb.NITRO_ERR_ARG
