@@ -48,7 +48,6 @@ struct nitro_block {
     unsigned long long* sse = nullptr;
     int batch = 0;
     std::vector<void*> allocs;
-    TcWorkspace tcw;
 };
 
 namespace {
@@ -224,9 +223,8 @@ nitro_status nitro_init_block(const nitro_block_desc* desc, uint64_t seed, void*
          dalloc(b, &b->grad_l, (size_t)MB * b->G) && dalloc(b, &b->z64, z_need) &&
          dalloc(b, &b->words, n_words(desc->n_layers)) && dalloc(b, &b->sse, 1);
     b->z64_elems = z_need;
-    if (ok) ok = tc_block_init(b->tcw, b->allocs, desc->max_batch);
     for (int i = 0; ok && i < desc->n_layers; ++i)
-        ok = tc_layer_init(b->L[i].tc, b->L[i].g, desc->max_batch, b->tcw, b->allocs);
+        ok = tc_layer_init(b->L[i].tc, b->L[i].g, desc->max_batch, i > 0, b->allocs);
     if (!ok) {
         free_all(b);
         delete b;
@@ -278,14 +276,14 @@ nitro_status nitro_block_forward(nitro_block* b, const int8_t* a_in, int batch, 
         const LayerGeom& g = ly.g;
         int8_t* out2 = (i == n - 1) ? a_out : nullptr;
         bool done = false;
-        NITRO_TRY(tc_conv_forward(ly.tc, g, x, batch, b->desc.alpha_inv, b->mu, ly.act, out2,
-                                  ly.region, ly.argmax, b->tcw, s, &done));
+        NITRO_TRY(tc_pack_input(ly.tc, g, x, batch, s));
+        NITRO_TRY(tc_conv_forward(ly.tc, g, batch, b->z64, w_status(b), s, &done));
         if (!done) {
             const int mode = g.kind == NITRO_CONV3X3 ? GM_CONV_FWD : GM_LIN_FWD;
             NITRO_TRY(simt_gemm(mode, x, nullptr, ly.W, b->z64, batch, g.h, g.w, g.cin, g.cout, s));
-            NITRO_TRY(simt_fwd_epilogue(b->z64, g, batch, b->desc.alpha_inv, b->mu, ly.act, out2,
-                                        ly.region, ly.argmax, s));
         }
+        NITRO_TRY(simt_fwd_epilogue(b->z64, g, batch, b->desc.alpha_inv, b->mu, ly.act, out2,
+                                    ly.region, ly.argmax, s));
         x = ly.act;
     }
     return NITRO_OK;
@@ -329,14 +327,14 @@ nitro_status nitro_block_backward(nitro_block* b, const int8_t* a_in, const int3
         const LayerGeom& g = ly.g;
         const int8_t* x = i ? b->L[i - 1].act : a_in;
         bool done = false;
-        NITRO_TRY(tc_conv_wgrad(ly.tc, g, x, ly.delta, w_delta(b, i), batch, ly.dW, b->tcw, s, &done));
+        NITRO_TRY(tc_conv_wgrad(ly.tc, g, ly.delta, w_delta(b, i), batch, ly.dW, w_status(b), s, &done));
         if (!done) {
             const int mode = g.kind == NITRO_CONV3X3 ? GM_CONV_WGRAD : GM_LIN_WGRAD;
             NITRO_TRY(simt_gemm(mode, x, ly.delta, nullptr, ly.dW, batch, g.h, g.w, g.cin, g.cout, s));
         }
         if (i == 0) break;
         done = false;
-        NITRO_TRY(tc_conv_dgrad(ly.tc, g, ly.delta, w_delta(b, i), batch, b->z64, b->tcw, s, &done));
+        NITRO_TRY(tc_conv_dgrad(ly.tc, g, batch, b->z64, w_status(b), s, &done));
         if (!done) {
             const int mode = g.kind == NITRO_CONV3X3 ? GM_CONV_DGRAD : GM_LIN_DGRAD;
             NITRO_TRY(simt_gemm(mode, nullptr, ly.delta, ly.W, b->z64, batch, g.h, g.w, g.cin, g.cout, s));

@@ -1,30 +1,776 @@
-// Tensor-core conv path (tcgen05).  Not yet enabled: every entry declines.
+// tcgen05 implicit-GEMM kernels for the 3x3 conv forward, weight gradient
+// and input gradient, plus the kernels that split operands into bf16 limb
+// planes.  See tc_conv.cuh for the exactness argument and the layouts.
+//
+// One CTA computes one 128 x N output tile over a range of K-blocks (64
+// elements each).  Warp 0 issues TMA loads into an S-stage shared-memory ring,
+// warp 1 allocates TMEM and issues the MMAs, warps 2..9 drain the fp32 TMEM
+// accumulator every <= 16 K-blocks into int64 registers (two warps per TMEM
+// lane quadrant, each owning half of the N columns).  Two TMEM accumulators
+// alternate so the MMAs of the next chunk overlap the drain of the last.
+// Every wait on an mbarrier is bounded in time; on expiry the kernel raises
+// the TIMEOUT status bit, lets the other roles leave, frees TMEM and returns.
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cudaTypedefs.h>
+
+#include <mutex>
+
+#include "prof.cuh"
 #include "tc_conv.cuh"
 
 namespace nitro {
+namespace {
 
-bool tc_block_init(TcWorkspace& ws, std::vector<void*>&, int max_batch) {
-    ws.max_batch = max_batch;
+enum TcMode : int { TC_FWD = 0, TC_WGRAD = 1, TC_DGRAD = 2 };
+
+constexpr int kBM = 128;              // rows per tile (TMEM lanes)
+constexpr int kBK = 64;               // K elements per block (one 128-byte row)
+constexpr int kChunkBlocks = 16;      // 16 x 64 = 1024 products per exact chunk
+constexpr int kThreads = 320;         // 10 warps
+constexpr uint64_t kWaitNs = 2000000000ull;   // 2 s bound on any wait
+
+// ------------------------------------------------------------------ PTX
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
+                 : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+        " selp.u32 %0, 1, 0, p;\n}\n"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+__device__ __forceinline__ uint64_t global_ns() {
+    uint64_t t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+// Bounded wait: false when the time limit passed (TIMEOUT raised) or another
+// role of this CTA gave up.
+__device__ __noinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag,
+                                       uint32_t* status) {
+    if (mbar_try_wait(bar, parity)) return true;
+    const uint64_t t0 = global_ns();
+    for (uint32_t i = 1;; ++i) {
+        if (mbar_try_wait(bar, parity)) return true;
+        if ((i & 63) == 0) {
+            if (*abort_flag) return false;
+            if (global_ns() - t0 > kWaitNs) {
+                *abort_flag = 1;
+                atomicOr(status, ST_TIMEOUT);
+                return false;
+            }
+        }
+    }
+}
+
+__device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap* m, uint32_t bar,
+                                            int c0, int c1, int c2) {
+    asm volatile(
+        "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%3, %4, %5}], [%2];" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(m)), "r"(bar), "r"(c0), "r"(c1), "r"(c2)
+        : "memory");
+}
+__device__ __forceinline__ void tma_load_4d(uint32_t dst, const CUtensorMap* m, uint32_t bar,
+                                            int c0, int c1, int c2, int c3) {
+    asm volatile(
+        "cp.async.bulk.tensor.4d.shared::cluster.global.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%3, %4, %5, %6}], [%2];" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(m)), "r"(bar), "r"(c0), "r"(c1), "r"(c2), "r"(c3)
+        : "memory");
+}
+__device__ __forceinline__ void tma_load_5d(uint32_t dst, const CUtensorMap* m, uint32_t bar,
+                                            int c0, int c1, int c2, int c3, int c4) {
+    asm volatile(
+        "cp.async.bulk.tensor.5d.shared::cluster.global.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%3, %4, %5, %6, %7}], [%2];" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(m)), "r"(bar), "r"(c0), "r"(c1), "r"(c2), "r"(c3),
+        "r"(c4)
+        : "memory");
+}
+
+__device__ __forceinline__ void tc_fence_before() {
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+
+// Shared-memory matrix descriptor, K-major operand, 128-byte swizzle: rows of
+// 128 bytes, 8-row groups 1024 bytes apart (stride byte offset), version 1.
+__device__ __forceinline__ uint64_t desc_sw128(uint32_t saddr) {
+    uint64_t d = 0;
+    d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);
+    d |= (uint64_t)1 << 16;               // leading byte offset (unused here)
+    d |= (uint64_t)(1024 >> 4) << 32;     // stride byte offset
+    d |= (uint64_t)1 << 46;               // descriptor version
+    d |= (uint64_t)2 << 61;               // 128-byte swizzle
+    return d;
+}
+
+// Instruction descriptor: kind::f16, A = B = bf16, D = f32, both K-major.
+__host__ __device__ constexpr uint32_t idesc_bf16(int m, int n) {
+    return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(n >> 3) << 17) |
+           ((uint32_t)(m >> 4) << 24);
+}
+
+__device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc,
+                                          uint32_t accumulate) {
+    asm volatile(
+        "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+        " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
+        "l"(a), "l"(b), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+__device__ __forceinline__ void umma_commit(uint32_t bar) {
+    asm volatile(
+        "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+        : "memory");
+}
+
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, "
+        "%11, %12, %13, %14, %15}, [%16];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+          "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+// ------------------------------------------------------------------ kernel
+struct TcArgs {
+    int B, H, W, Cin, Cout, Bp;
+    int ntx, nty;          // pixel tiles along x and y (forward / dgrad)
+    int wb, hb, bb;        // pixel box (forward / dgrad): wb * hb * bb = 128
+    int kb_total, kb_per_split;
+    const int* limbs_a;    // limb counts (nullptr = 1)
+    const int* limbs_b;
+    int64_t* out;
+    uint32_t* status;
+    int atomic_out;
+};
+
+template <int N>
+struct TcCfg {
+    static constexpr int A_BYTES = kBM * kBK * 2;
+    static constexpr int B_BYTES = N * kBK * 2;
+    static constexpr int STAGE = A_BYTES + B_BYTES;
+    static constexpr int S = N >= 128 ? 6 : 8;
+    static constexpr int SMEM = 1024 + S * STAGE + 256;
+};
+
+template <int MODE, int N>
+__global__ void __launch_bounds__(kThreads, 1)
+    k_tc_gemm(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+              const TcArgs args) {
+    using C = TcCfg<N>;
+    constexpr int S = C::S;
+    constexpr int NH = N / 2;            // columns per epilogue warp
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + S * C::STAGE);
+    // bars[0..S) full, [S..2S) empty, [2S..2S+2) tmem full, [2S+2..2S+4) tmem empty
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * S + 4);
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const uint32_t bar0 = smem_u32(bars);
+    auto full_bar = [&](int s) { return bar0 + 8u * s; };
+    auto empty_bar = [&](int s) { return bar0 + 8u * (S + s); };
+    auto tfull_bar = [&](int b) { return bar0 + 8u * (2 * S + b); };
+    auto tempty_bar = [&](int b) { return bar0 + 8u * (2 * S + 2 + b); };
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < S; ++s) {
+            mbar_init(full_bar(s), 1);
+            mbar_init(empty_bar(s), 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(tfull_bar(b), 1);
+            mbar_init(tempty_bar(b), 8);
+        }
+        *abort_flag = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    if (warp == 1) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                         smem_u32(tmem_slot)),
+                     "r"(2 * N)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+
+    const int mt = blockIdx.x, nt = blockIdx.y;
+    const int n0 = nt * N;
+    const int kb0 = blockIdx.z * args.kb_per_split;
+    const int kb1 = min(args.kb_total, kb0 + args.kb_per_split);
+    const int nkb = kb1 - kb0;
+    int LA = args.limbs_a ? *args.limbs_a : 1;
+    int LB = args.limbs_b ? *args.limbs_b : 1;
+    LA = LA < 1 ? 1 : (LA > kMaxLimbs ? kMaxLimbs : LA);
+    LB = LB < 1 ? 1 : (LB > kMaxLimbs ? kMaxLimbs : LB);
+    const int passes = LA * LB;
+    const int cpp = (nkb + kChunkBlocks - 1) / kChunkBlocks;   // chunks per pass
+
+    // pixel tile origin (forward / dgrad)
+    const int tx = mt % args.ntx, ty = (mt / args.ntx) % args.nty, tb = mt / (args.ntx * args.nty);
+    const int x0 = tx * args.wb, y0 = ty * args.hb, b0 = tb * args.bb;
+
+    if (warp == 0) {
+        if (lane == 0 && nkb > 0) {
+            // ---------------- TMA producer
+            int it = 0;
+            for (int p = 0; p < passes; ++p) {
+                const int la = p / LB, lb = p % LB;
+                for (int kb = kb0; kb < kb1; ++kb, ++it) {
+                    const int s = it % S;
+                    if (!mbar_wait(empty_bar(s), ((it / S) & 1) ^ 1, abort_flag, args.status))
+                        goto producer_done;
+                    const uint32_t fb = full_bar(s);
+                    const uint32_t a_dst = smem_u32(smem + s * C::STAGE);
+                    const uint32_t b_dst = a_dst + C::A_BYTES;
+                    mbar_expect_tx(fb, C::STAGE);
+                    if (MODE == TC_FWD) {
+                        const int nc = args.Cin / kBK;
+                        const int t = kb / nc, cb = kb - t * nc, ky = t / 3, kx = t - 3 * ky;
+                        tma_load_4d(a_dst, &tmA, fb, cb * kBK, x0 + kx - 1, y0 + ky - 1, b0);
+                        tma_load_3d(b_dst, &tmB, fb, t * args.Cin + cb * kBK, n0, lb);
+                    } else if (MODE == TC_DGRAD) {
+                        const int nc = args.Cout / kBK;
+                        const int t = kb / nc, cb = kb - t * nc, ky = t / 3, kx = t - 3 * ky;
+                        tma_load_5d(a_dst, &tmA, fb, cb * kBK, x0 - kx + 1, y0 - ky + 1, b0, la);
+                        tma_load_4d(b_dst, &tmB, fb, cb * kBK, n0, t, lb);
+                    } else {  // TC_WGRAD: rows (tap, ci), K = (y, x, b)
+                        const int nbb = (args.Bp + kBK - 1) / kBK;
+                        const int pos = kb / nbb, bbk = kb - pos * nbb;
+                        const int y = pos / args.W, x = pos - y * args.W;
+#pragma unroll
+                        for (int j = 0; j < 2; ++j) {
+                            const int m = mt * kBM + j * 64;
+                            int t = m / args.Cin, ci0 = m - t * args.Cin;
+                            if (t >= 9) { t = 0; ci0 = args.Cin; }   // fully out of range: zeros
+                            const int ky = t / 3, kx = t - 3 * ky;
+                            tma_load_4d(a_dst + j * (64 * 128), &tmA, fb, bbk * kBK, x + kx - 1,
+                                        y + ky - 1, ci0);
+                        }
+                        tma_load_4d(b_dst, &tmB, fb, bbk * kBK, x, y, lb * args.Cout + n0);
+                    }
+                }
+            }
+        producer_done:;
+        }
+    } else if (warp == 1) {
+        if (lane == 0 && nkb > 0) {
+            // ---------------- MMA issuer
+            constexpr uint32_t idesc = idesc_bf16(kBM, N);
+            int it = 0, chunk = 0;
+            for (int p = 0; p < passes; ++p) {
+                for (int c = 0; c < cpp; ++c, ++chunk) {
+                    const int buf = chunk & 1;
+                    if (!mbar_wait(tempty_bar(buf), ((chunk >> 1) & 1) ^ 1, abort_flag, args.status))
+                        goto mma_done;
+                    tc_fence_after();
+                    const uint32_t d = tmem + (uint32_t)(buf * N);
+                    const int c0 = kb0 + c * kChunkBlocks;
+                    const int c1 = min(kb1, c0 + kChunkBlocks);
+                    for (int kb = c0; kb < c1; ++kb, ++it) {
+                        const int s = it % S;
+                        if (!mbar_wait(full_bar(s), (it / S) & 1, abort_flag, args.status))
+                            goto mma_done;
+                        tc_fence_after();
+                        const uint32_t a_addr = smem_u32(smem + s * C::STAGE);
+                        const uint32_t b_addr = a_addr + C::A_BYTES;
+#pragma unroll
+                        for (int k = 0; k < kBK / 16; ++k)
+                            umma_bf16(d, desc_sw128(a_addr + 32 * k), desc_sw128(b_addr + 32 * k),
+                                      idesc, (kb > c0 || k > 0) ? 1u : 0u);
+                        umma_commit(empty_bar(s));
+                    }
+                    umma_commit(tfull_bar(buf));
+                }
+            }
+        mma_done:;
+        }
+    } else {
+        // ---------------- epilogue: warps 2..9
+        const int q = warp & 3;             // TMEM lane quadrant this warp may read
+        const int half = (warp - 2) >> 2;   // which half of the N columns
+        uint64_t acc[NH];
+#pragma unroll
+        for (int i = 0; i < NH; ++i) acc[i] = 0;
+        bool ok = nkb > 0;
+        int chunk = 0;
+        for (int p = 0; ok && p < passes; ++p) {
+            const int shift = 8 * (p / LB + p % LB);
+            for (int c = 0; c < cpp; ++c, ++chunk) {
+                const int buf = chunk & 1;
+                if (!mbar_wait(tfull_bar(buf), (chunk >> 1) & 1, abort_flag, args.status)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t base = tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(buf * N + half * NH);
+#pragma unroll
+                for (int j = 0; j < NH / 16; ++j) {
+                    uint32_t r[16];
+                    tmem_ld16(base + 16 * j, r);
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) {
+                        const int v = __float2int_rz(__uint_as_float(r[i]));   // exact integer
+                        acc[16 * j + i] += (uint64_t)(int64_t)v << shift;
+                    }
+                }
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(tempty_bar(buf));
+            }
+        }
+        if (ok) {
+            const int r = 32 * q + lane;   // output row of this thread
+            const int col0 = n0 + half * NH;
+            if (MODE == TC_WGRAD) {
+                const int m = mt * kBM + r;
+                const int t = m / args.Cin, ci = m - t * args.Cin;
+                if (t < 9) {
+                    int64_t* o = args.out + (int64_t)t * args.Cin + ci;
+                    const int64_t cstride = 9LL * args.Cin;
+#pragma unroll
+                    for (int i = 0; i < NH; ++i) {
+                        unsigned long long* dst =
+                            reinterpret_cast<unsigned long long*>(o + (int64_t)(col0 + i) * cstride);
+                        if (args.atomic_out) atomicAdd(dst, (unsigned long long)acc[i]);
+                        else *dst = acc[i];
+                    }
+                }
+            } else {
+                const int xx = r % args.wb, yy = (r / args.wb) % args.hb, bbx = r / (args.wb * args.hb);
+                const int x = x0 + xx, y = y0 + yy, b = b0 + bbx;
+                if (x < args.W && y < args.H && b < args.B) {
+                    const int ncols = MODE == TC_FWD ? args.Cout : args.Cin;
+                    int64_t* o = args.out + (((int64_t)b * args.H + y) * args.W + x) * ncols + col0;
+#pragma unroll
+                    for (int i = 0; i < NH; i += 2) {
+                        longlong2 v;
+                        v.x = (long long)acc[i];
+                        v.y = (long long)acc[i + 1];
+                        *reinterpret_cast<longlong2*>(o + i) = v;
+                    }
+                }
+            }
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(2 * N)
+                     : "memory");
+    }
+}
+
+// ------------------------------------------------------------------ limb packing
+__device__ __forceinline__ int limb_count(uint32_t m) {
+    // top limb in [-128, 128]: ranges of 1..4 signed-digit limbs
+    return m <= 128u ? 1 : (m <= 32895u ? 2 : (m <= 8421375u ? 3 : 4));
+}
+__device__ __forceinline__ uint16_t bf16_bits(int v) {
+    return __bfloat16_as_ushort(__float2bfloat16_rn((float)v));   // exact for |v| <= 256
+}
+// limb l of x given L limbs (signed digits below the top, remainder on top)
+__device__ __forceinline__ int limb_of(int64_t x, int l, int L) {
+    for (int i = 0; i < L - 1; ++i) {
+        const int64_t d = ((x + 128) & 255) - 128;
+        if (i == l) return (int)d;
+        x = (x - d) >> 8;
+    }
+    return (int)x;
+}
+
+// int8 NHWC -> bf16 NHWC copy
+__global__ void k_pack_act_nhwc(const int8_t* __restrict__ x, int64_t n, uint16_t* __restrict__ out) {
+    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
+         i += (int64_t)gridDim.x * blockDim.x)
+        out[i] = bf16_bits(x[i]);
+}
+
+// [B][HW][C] int (int8 or int32 with limbs) -> [L][C][HW][Bp] bf16, zero for b >= B.
+template <typename T>
+__global__ void k_pack_transposed(const T* __restrict__ x, int B, int HW, int C, int Bp,
+                                  const uint32_t* maxabs, uint16_t* __restrict__ out) {
+    __shared__ int tile[32][33];
+    const int pos = blockIdx.x;                 // pixel (y, x)
+    const int c0 = blockIdx.y * 32, b0 = blockIdx.z * 32;
+    const int L = maxabs ? limb_count(*maxabs) : 1;
+    for (int k = threadIdx.y; k < 32; k += blockDim.y) {     // read: b = b0 + k, c = c0 + tx
+        const int b = b0 + k, c = c0 + threadIdx.x;
+        tile[k][threadIdx.x] = (b < B && c < C) ? (int)x[((int64_t)b * HW + pos) * C + c] : 0;
+    }
+    __syncthreads();
+    const int64_t plane = (int64_t)C * HW * Bp;
+    for (int k = threadIdx.y; k < 32; k += blockDim.y) {     // write: c = c0 + k, b = b0 + tx
+        const int c = c0 + k, b = b0 + threadIdx.x;
+        if (c >= C || b >= Bp) continue;
+        const int64_t v = tile[threadIdx.x][k];
+        const int64_t o = ((int64_t)c * HW + pos) * Bp + b;
+        for (int l = 0; l < L; ++l) out[l * plane + o] = bf16_bits(limb_of(v, l, L));
+    }
+}
+
+// int32 delta NHWC -> limb planes [L][B][H][W][C]; also records the limb count.
+__global__ void k_pack_delta_nhwc(const int32_t* __restrict__ d, int64_t n,
+                                  const uint32_t* maxabs, uint16_t* __restrict__ out) {
+    const int L = limb_count(*maxabs);
+    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        int64_t x = d[i];
+        for (int l = 0; l < L - 1; ++l) {
+            const int64_t dg = ((x + 128) & 255) - 128;
+            out[l * n + i] = bf16_bits((int)dg);
+            x = (x - dg) >> 8;
+        }
+        out[(int64_t)(L - 1) * n + i] = bf16_bits((int)x);
+    }
+}
+
+__global__ void k_set_limbs(const uint32_t* maxabs, int* limbs) {
+    *limbs = limb_count(*maxabs);
+}
+
+// W [Cout][9][Cin] -> w_planes [L][Cout][9][Cin] and wt_planes [L][9][Cin][Cout]
+__global__ void k_pack_weights(const int32_t* __restrict__ W, int Cout, int Cin,
+                               const uint32_t* maxabs, uint16_t* __restrict__ wp,
+                               uint16_t* __restrict__ wtp) {
+    const int L = limb_count(*maxabs);
+    const int64_t n = (int64_t)Cout * 9 * Cin;
+    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        const int ci = (int)(i % Cin);
+        const int t = (int)((i / Cin) % 9);
+        const int co = (int)(i / (9LL * Cin));
+        int64_t x = W[i];
+        const int64_t it = ((int64_t)t * Cin + ci) * Cout + co;
+        for (int l = 0; l < L; ++l) {
+            int v;
+            if (l < L - 1) {
+                const int64_t dg = ((x + 128) & 255) - 128;
+                v = (int)dg;
+                x = (x - dg) >> 8;
+            } else {
+                v = (int)x;
+            }
+            const uint16_t bits = bf16_bits(v);
+            if (wp) wp[l * n + i] = bits;
+            if (wtp) wtp[l * n + it] = bits;
+        }
+    }
+}
+
+// ------------------------------------------------------------------ host side
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                             &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+    });
+    return fn;
+}
+
+// bf16 tensor map, dims innermost first; strides in elements for dims 1..r-1.
+bool make_map(CUtensorMap* m, const void* base, int rank, const uint64_t* dims,
+              const uint64_t* strides_elems, const uint32_t* box) {
+    auto fn = encode_fn();
+    if (!fn) return false;
+    cuuint64_t gdim[5], gstride[4];
+    cuuint32_t bdim[5], estr[5];
+    for (int i = 0; i < rank; ++i) {
+        gdim[i] = dims[i];
+        bdim[i] = box[i];
+        estr[i] = 1;
+    }
+    for (int i = 0; i < rank - 1; ++i) gstride[i] = strides_elems[i] * 2;
+    CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, (cuuint32_t)rank, const_cast<void*>(base),
+                    gdim, gstride, bdim, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                    CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
+template <int MODE, int N>
+cudaError_t launch_gemm(const CUtensorMap& a, const CUtensorMap& b, const TcArgs& args, dim3 grid,
+                        cudaStream_t s) {
+    using C = TcCfg<N>;
+    static bool attr_set = false;
+    if (!attr_set) {
+        cudaError_t e = cudaFuncSetAttribute(k_tc_gemm<MODE, N>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+        if (e != cudaSuccess) return e;
+        attr_set = true;
+    }
+    k_tc_gemm<MODE, N><<<grid, kThreads, C::SMEM, s>>>(a, b, args);
+    return cudaGetLastError();
+}
+
+template <int MODE>
+cudaError_t launch_gemm_n(int n, const CUtensorMap& a, const CUtensorMap& b, const TcArgs& args,
+                          dim3 grid, cudaStream_t s) {
+    return n == 128 ? launch_gemm<MODE, 128>(a, b, args, grid, s)
+                    : launch_gemm<MODE, 64>(a, b, args, grid, s);
+}
+
+int pick_n(int cols) { return cols % 128 == 0 ? 128 : 64; }
+
+void pixel_tiling(const LayerGeom& g, int batch, TcArgs& a, int* tiles_m) {
+    if (g.w > 8) { a.wb = 16; a.hb = 8; a.bb = 1; }
+    else { a.wb = 8; a.hb = 8; a.bb = 2; }
+    a.ntx = (g.w + a.wb - 1) / a.wb;
+    a.nty = (g.h + a.hb - 1) / a.hb;
+    *tiles_m = a.ntx * a.nty * ((batch + a.bb - 1) / a.bb);
+}
+
+inline int grid1d(int64_t n) {
+    int64_t g = (n + 255) / 256;
+    return (int)(g < 1 ? 1 : (g > 152 * 8 ? 152 * 8 : g));
+}
+
+template <typename T>
+bool dalloc(std::vector<void*>& allocs, T** p, size_t count) {
+    void* q = nullptr;
+    if (cudaMalloc(&q, (count ? count : 1) * sizeof(T)) != cudaSuccess) return false;
+    allocs.push_back(q);
+    *p = static_cast<T*>(q);
     return true;
 }
-bool tc_layer_init(TcLayer&, const LayerGeom&, int, TcWorkspace&, std::vector<void*>&) { return true; }
-cudaError_t tc_refresh_weights(TcLayer&, const LayerGeom&, const int32_t*, const uint32_t*, cudaStream_t) {
+
+}  // namespace
+
+bool tc_layer_init(TcLayer& t, const LayerGeom& g, int max_batch, bool has_dgrad,
+                   std::vector<void*>& allocs) {
+    t = TcLayer();
+    if (g.kind != NITRO_CONV3X3 || max_batch < 1 || !encode_fn()) return true;
+    const bool chan_ok = g.cin % 64 == 0 && g.cout % 64 == 0;
+    const bool pix_ok = g.h >= 8 && g.w >= 8;
+    t.fwd = chan_ok && pix_ok;
+    t.dgrad = has_dgrad && chan_ok && pix_ok;
+    t.wgrad = chan_ok;
+    if (!t.fwd && !t.wgrad && !t.dgrad) return true;
+    t.max_bp = (max_batch + 7) / 8 * 8;
+    const size_t hw = (size_t)g.h * g.w;
+    const size_t nw = (size_t)g.cout * 9 * g.cin;
+    bool ok = dalloc(allocs, &t.limbs, 2);
+    if (ok && t.fwd) ok = dalloc(allocs, &t.act_nhwc, (size_t)max_batch * hw * g.cin);
+    if (ok && t.wgrad) ok = dalloc(allocs, &t.act_t, (size_t)g.cin * hw * t.max_bp);
+    if (ok && t.wgrad) ok = dalloc(allocs, &t.d_t, (size_t)kMaxLimbs * g.cout * hw * t.max_bp);
+    if (ok && t.dgrad) ok = dalloc(allocs, &t.d_nhwc, (size_t)kMaxLimbs * max_batch * hw * g.cout);
+    if (ok && t.fwd) ok = dalloc(allocs, &t.w_planes, (size_t)kMaxLimbs * nw);
+    if (ok && t.dgrad) ok = dalloc(allocs, &t.wt_planes, (size_t)kMaxLimbs * nw);
+    if (ok) ok = cudaMemset(t.limbs, 0, 2 * sizeof(int)) == cudaSuccess;
+    return ok;
+}
+
+cudaError_t tc_refresh_weights(TcLayer& t, const LayerGeom& g, const int32_t* W,
+                               const uint32_t* maxabs_w, cudaStream_t s) {
+    if (!t.fwd && !t.dgrad) return cudaSuccess;
+    const int64_t n = (int64_t)g.cout * 9 * g.cin;
+    {
+        ProfScope ps(K_TC_PACK, s, 0.0, (double)n * 4 * 2);
+        k_pack_weights<<<grid1d(n), 256, 0, s>>>(W, g.cout, g.cin, maxabs_w, t.w_planes, t.wt_planes);
+    }
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    ProfScope ps(K_TC_PACK, s, 0.0, 0.0);
+    k_set_limbs<<<1, 1, 0, s>>>(maxabs_w, t.limbs);
+    return cudaGetLastError();
+}
+
+cudaError_t tc_pack_input(TcLayer& t, const LayerGeom& g, const int8_t* x, int batch,
+                          cudaStream_t s) {
+    if (batch <= 0 || (!t.fwd && !t.wgrad)) return cudaSuccess;
+    const int hw = g.h * g.w;
+    if (t.fwd) {
+        const int64_t n = (int64_t)batch * hw * g.cin;
+        ProfScope ps(K_TC_PACK, s, 0.0, (double)n * 3);
+        k_pack_act_nhwc<<<grid1d(n), 256, 0, s>>>(x, n, t.act_nhwc);
+        cudaError_t e = cudaGetLastError();
+        if (e != cudaSuccess) return e;
+    }
+    if (t.wgrad) {
+        const int bp = (batch + 7) / 8 * 8;
+        dim3 grid(hw, (g.cin + 31) / 32, (bp + 31) / 32);
+        ProfScope ps(K_TC_PACK, s, 0.0, (double)batch * hw * g.cin * 3);
+        k_pack_transposed<int8_t><<<grid, dim3(32, 8), 0, s>>>(x, batch, hw, g.cin, bp, nullptr,
+                                                               t.act_t);
+        return cudaGetLastError();
+    }
     return cudaSuccess;
 }
-cudaError_t tc_conv_forward(TcLayer&, const LayerGeom&, const int8_t*, int, int, int, int8_t*, int8_t*,
-                            int8_t*, int8_t*, TcWorkspace&, cudaStream_t, bool* done) {
+
+cudaError_t tc_conv_forward(TcLayer& t, const LayerGeom& g, int batch, int64_t* z,
+                            uint32_t* status, cudaStream_t s, bool* done) {
     *done = false;
-    return cudaSuccess;
+    if (!t.fwd || batch <= 0) return cudaSuccess;
+    TcArgs a{};
+    a.B = batch; a.H = g.h; a.W = g.w; a.Cin = g.cin; a.Cout = g.cout;
+    a.Bp = (batch + 7) / 8 * 8;
+    int tiles_m = 0;
+    pixel_tiling(g, batch, a, &tiles_m);
+    const int n = pick_n(g.cout);
+    a.kb_total = 9 * (g.cin / kBK);
+    a.kb_per_split = a.kb_total;
+    a.limbs_a = nullptr;
+    a.limbs_b = t.limbs;
+    a.out = z;
+    a.status = status;
+    a.atomic_out = 0;
+    CUtensorMap ma, mb;
+    const uint64_t da[4] = {(uint64_t)g.cin, (uint64_t)g.w, (uint64_t)g.h, (uint64_t)batch};
+    const uint64_t sa[3] = {(uint64_t)g.cin, (uint64_t)g.w * g.cin, (uint64_t)g.h * g.w * g.cin};
+    const uint32_t ba[4] = {64, (uint32_t)a.wb, (uint32_t)a.hb, (uint32_t)a.bb};
+    const uint64_t db[3] = {(uint64_t)9 * g.cin, (uint64_t)g.cout, (uint64_t)kMaxLimbs};
+    const uint64_t sb[2] = {(uint64_t)9 * g.cin, (uint64_t)9 * g.cin * g.cout};
+    const uint32_t bb[3] = {64, (uint32_t)n, 1};
+    if (!make_map(&ma, t.act_nhwc, 4, da, sa, ba) || !make_map(&mb, t.w_planes, 3, db, sb, bb))
+        return cudaErrorInvalidValue;
+    dim3 grid(tiles_m, g.cout / n, 1);
+    const double ops = 2.0 * batch * g.h * g.w * g.cout * 9.0 * g.cin;
+    ProfScope ps(K_TC_CONV_FWD, s, ops, 0.0);
+    cudaError_t e = launch_gemm_n<TC_FWD>(n, ma, mb, a, grid, s);
+    if (e == cudaSuccess) *done = true;
+    return e;
 }
-cudaError_t tc_conv_wgrad(TcLayer&, const LayerGeom&, const int8_t*, const int32_t*, const uint32_t*,
-                          int, int64_t*, TcWorkspace&, cudaStream_t, bool* done) {
+
+cudaError_t tc_conv_wgrad(TcLayer& t, const LayerGeom& g, const int32_t* delta,
+                          const uint32_t* maxabs_delta, int batch, int64_t* dW,
+                          uint32_t* status, cudaStream_t s, bool* done) {
     *done = false;
-    return cudaSuccess;
+    if (batch <= 0 || (!t.wgrad && !t.dgrad)) return cudaSuccess;
+    const int hw = g.h * g.w;
+    const int bp = (batch + 7) / 8 * 8;
+    // limb planes of delta in the layouts the tensor-core passes read
+    if (t.dgrad) {
+        const int64_t n = (int64_t)batch * hw * g.cout;
+        ProfScope ps(K_TC_PACK, s, 0.0, (double)n * 4 * 2);
+        k_pack_delta_nhwc<<<grid1d(n), 256, 0, s>>>(delta, n, maxabs_delta, t.d_nhwc);
+        cudaError_t e = cudaGetLastError();
+        if (e != cudaSuccess) return e;
+    }
+    if (t.wgrad) {
+        dim3 grid(hw, (g.cout + 31) / 32, (bp + 31) / 32);
+        ProfScope ps(K_TC_PACK, s, 0.0, (double)batch * hw * g.cout * 4 * 2);
+        k_pack_transposed<int32_t><<<grid, dim3(32, 8), 0, s>>>(delta, batch, hw, g.cout, bp,
+                                                                maxabs_delta, t.d_t);
+        cudaError_t e = cudaGetLastError();
+        if (e != cudaSuccess) return e;
+    }
+    {
+        ProfScope ps(K_TC_PACK, s, 0.0, 0.0);
+        k_set_limbs<<<1, 1, 0, s>>>(maxabs_delta, t.limbs + 1);
+        cudaError_t e = cudaGetLastError();
+        if (e != cudaSuccess) return e;
+    }
+    if (!t.wgrad) return cudaSuccess;
+    TcArgs a{};
+    a.B = batch; a.H = g.h; a.W = g.w; a.Cin = g.cin; a.Cout = g.cout; a.Bp = bp;
+    a.ntx = a.nty = 1; a.wb = a.hb = a.bb = 1;
+    const int n = pick_n(g.cout);
+    const int tiles_m = (9 * g.cin + kBM - 1) / kBM, tiles_n = g.cout / n;
+    const int nbb = (bp + kBK - 1) / kBK;
+    a.kb_total = hw * nbb;
+    // split K so that about one wave of CTAs runs, each with >= one exact chunk
+    const int tiles = tiles_m * tiles_n;
+    int splits = (152 + tiles - 1) / tiles;
+    const int max_splits = (a.kb_total + kChunkBlocks - 1) / kChunkBlocks;
+    splits = splits < 1 ? 1 : (splits > max_splits ? max_splits : splits);
+    a.kb_per_split = (a.kb_total + splits - 1) / splits;
+    splits = (a.kb_total + a.kb_per_split - 1) / a.kb_per_split;
+    a.limbs_a = nullptr;
+    a.limbs_b = t.limbs + 1;
+    a.out = dW;
+    a.status = status;
+    a.atomic_out = splits > 1;
+    CUtensorMap ma, mb;
+    const uint64_t da[4] = {(uint64_t)bp, (uint64_t)g.w, (uint64_t)g.h, (uint64_t)g.cin};
+    const uint64_t sa[3] = {(uint64_t)bp, (uint64_t)g.w * bp, (uint64_t)hw * bp};
+    const uint32_t ba[4] = {64, 1, 1, 64};
+    const uint64_t db[4] = {(uint64_t)bp, (uint64_t)g.w, (uint64_t)g.h, (uint64_t)g.cout * kMaxLimbs};
+    const uint32_t bb[4] = {64, 1, 1, (uint32_t)n};
+    if (!make_map(&ma, t.act_t, 4, da, sa, ba) || !make_map(&mb, t.d_t, 4, db, sa, bb))
+        return cudaErrorInvalidValue;
+    if (a.atomic_out) {
+        cudaError_t e = cudaMemsetAsync(dW, 0, sizeof(int64_t) * 9 * g.cin * g.cout, s);
+        if (e != cudaSuccess) return e;
+    }
+    dim3 grid(tiles_m, tiles_n, splits);
+    const double ops = 2.0 * batch * hw * g.cout * 9.0 * g.cin;
+    ProfScope ps(K_TC_CONV_WGRAD, s, ops, 0.0);
+    cudaError_t e = launch_gemm_n<TC_WGRAD>(n, ma, mb, a, grid, s);
+    if (e == cudaSuccess) *done = true;
+    return e;
 }
-cudaError_t tc_conv_dgrad(TcLayer&, const LayerGeom&, const int32_t*, const uint32_t*, int, int64_t*,
-                          TcWorkspace&, cudaStream_t, bool* done) {
+
+cudaError_t tc_conv_dgrad(TcLayer& t, const LayerGeom& g, int batch, int64_t* g64,
+                          uint32_t* status, cudaStream_t s, bool* done) {
     *done = false;
-    return cudaSuccess;
+    if (!t.dgrad || batch <= 0) return cudaSuccess;
+    TcArgs a{};
+    a.B = batch; a.H = g.h; a.W = g.w; a.Cin = g.cin; a.Cout = g.cout;
+    a.Bp = (batch + 7) / 8 * 8;
+    int tiles_m = 0;
+    pixel_tiling(g, batch, a, &tiles_m);
+    const int n = pick_n(g.cin);
+    a.kb_total = 9 * (g.cout / kBK);
+    a.kb_per_split = a.kb_total;
+    a.limbs_a = t.limbs + 1;
+    a.limbs_b = t.limbs;
+    a.out = g64;
+    a.status = status;
+    a.atomic_out = 0;
+    CUtensorMap ma, mb;
+    const uint64_t da[5] = {(uint64_t)g.cout, (uint64_t)g.w, (uint64_t)g.h, (uint64_t)batch,
+                            (uint64_t)kMaxLimbs};
+    // limb planes are batch-sized at this call's batch
+    const uint64_t plane = (uint64_t)batch * g.h * g.w * g.cout;
+    const uint64_t sa[4] = {(uint64_t)g.cout, (uint64_t)g.w * g.cout, (uint64_t)g.h * g.w * g.cout,
+                            plane};
+    const uint32_t ba[5] = {64, (uint32_t)a.wb, (uint32_t)a.hb, (uint32_t)a.bb, 1};
+    const uint64_t db[4] = {(uint64_t)g.cout, (uint64_t)g.cin, 9, (uint64_t)kMaxLimbs};
+    const uint64_t sb[3] = {(uint64_t)g.cout, (uint64_t)g.cin * g.cout, (uint64_t)9 * g.cin * g.cout};
+    const uint32_t bb[4] = {64, (uint32_t)n, 1, 1};
+    if (!make_map(&ma, t.d_nhwc, 5, da, sa, ba) || !make_map(&mb, t.wt_planes, 4, db, sb, bb))
+        return cudaErrorInvalidValue;
+    dim3 grid(tiles_m, g.cin / n, 1);
+    const double ops = 2.0 * batch * g.h * g.w * g.cin * 9.0 * g.cout;
+    ProfScope ps(K_TC_CONV_DGRAD, s, ops, 0.0);
+    cudaError_t e = launch_gemm_n<TC_DGRAD>(n, ma, mb, a, grid, s);
+    if (e == cudaSuccess) *done = true;
+    return e;
 }
 
 }  // namespace nitro

@@ -1,7 +1,21 @@
-// Tensor-core (tcgen05) path of the conv contractions: state kept per layer
-// and per block, and the entry points the ABI calls.  Each entry point sets
-// *done = false when it does not take the layer, and the caller then runs the
-// CUDA-core kernels.
+// Tensor-core (tcgen05) path of the 3x3 conv contractions.
+//
+// Every operand is split exactly into signed 8-bit limbs, x = sum_l 2^(8l) x_l
+// with x_l in [-128, 127] and the top limb in [-128, 128], each held as a
+// bf16 value (exact).  A contraction runs one pass per (A limb, B limb) pair
+// on the bf16 tensor pipe with fp32 accumulation in TMEM; every partial sum
+// over at most 1024 products of magnitude <= 2^14 is an integer below 2^24 and
+// therefore exact, so chunks of 1024 are drained to integers and the passes
+// are combined in int64 (modulo 2^64) with shifts 8 (la + lb).
+//
+// Layouts (bf16, limb planes outermost):
+//   act_nhwc  [B][H][W][Cin]           forward A  (pixels x taps*channels)
+//   act_t     [Cin][H][W][Bp]          wgrad A    ((tap, ci) x (y, x, b))
+//   d_nhwc    [L][B][H][W][Cout]       dgrad A
+//   d_t       [L][Cout][H][W][Bp]      wgrad B
+//   w_planes  [L][Cout][9][Cin]        forward B
+//   wt_planes [L][9][Cin][Cout]        dgrad B
+// Bp = batch rounded up to 8 (TMA strides are multiples of 16 bytes).
 #pragma once
 
 #include <vector>
@@ -10,27 +24,47 @@
 
 namespace nitro {
 
+constexpr int kMaxLimbs = 4;
+
 struct TcLayer {
-    bool fwd = false, wgrad = false, dgrad = false;   // which passes run on tcgen05
+    bool fwd = false, wgrad = false, dgrad = false;   // passes that run on tcgen05
+    int max_bp = 0;
+    uint16_t* act_nhwc = nullptr;
+    uint16_t* act_t = nullptr;
+    uint16_t* d_nhwc = nullptr;
+    uint16_t* d_t = nullptr;
+    uint16_t* w_planes = nullptr;
+    uint16_t* wt_planes = nullptr;
+    int* limbs = nullptr;   // device: [0] weight limbs, [1] delta limbs
 };
 
-struct TcWorkspace {
-    int max_batch = 0;
-};
-
-bool tc_block_init(TcWorkspace& ws, std::vector<void*>& allocs, int max_batch);
-bool tc_layer_init(TcLayer& t, const LayerGeom& g, int max_batch, TcWorkspace& ws,
+// Decides which passes of a layer run on tensor cores and allocates their
+// buffers (recorded in `allocs`).  `has_dgrad`: the layer is not the block's
+// first, so its input gradient is needed.
+bool tc_layer_init(TcLayer& t, const LayerGeom& g, int max_batch, bool has_dgrad,
                    std::vector<void*>& allocs);
+
+// Re-splits the layer's int32 weights into limb planes (after init, an update
+// or a checkpoint load); the limb count follows *maxabs_w.
 cudaError_t tc_refresh_weights(TcLayer& t, const LayerGeom& g, const int32_t* W,
                                const uint32_t* maxabs_w, cudaStream_t s);
-cudaError_t tc_conv_forward(TcLayer& t, const LayerGeom& g, const int8_t* x, int batch,
-                            int alpha_inv, int mu, int8_t* act, int8_t* out2, int8_t* region,
-                            int8_t* argmax, TcWorkspace& ws, cudaStream_t s, bool* done);
-cudaError_t tc_conv_wgrad(TcLayer& t, const LayerGeom& g, const int8_t* x, const int32_t* delta,
-                          const uint32_t* maxabs_delta, int batch, int64_t* dW, TcWorkspace& ws,
-                          cudaStream_t s, bool* done);
-cudaError_t tc_conv_dgrad(TcLayer& t, const LayerGeom& g, const int32_t* delta,
-                          const uint32_t* maxabs_delta, int batch, int64_t* g64, TcWorkspace& ws,
-                          cudaStream_t s, bool* done);
+
+// bf16 copies of the layer's int8 input for the forward and wgrad operands.
+cudaError_t tc_pack_input(TcLayer& t, const LayerGeom& g, const int8_t* x, int batch,
+                          cudaStream_t s);
+
+// z[p][co] (int64) = forward contraction; *done = false if not on tcgen05.
+cudaError_t tc_conv_forward(TcLayer& t, const LayerGeom& g, int batch, int64_t* z,
+                            uint32_t* status, cudaStream_t s, bool* done);
+
+// Splits delta into limb planes (both layouts as needed) and, if wgrad runs on
+// tcgen05, dW = sum_p delta (x) im2col(a).  Must precede tc_conv_dgrad.
+cudaError_t tc_conv_wgrad(TcLayer& t, const LayerGeom& g, const int32_t* delta,
+                          const uint32_t* maxabs_delta, int batch, int64_t* dW,
+                          uint32_t* status, cudaStream_t s, bool* done);
+
+// g[p][ci] (int64) = sum_(t,co) delta[p - tap t][co] W[co][t][ci].
+cudaError_t tc_conv_dgrad(TcLayer& t, const LayerGeom& g, int batch, int64_t* g64,
+                          uint32_t* status, cudaStream_t s, bool* done);
 
 }  // namespace nitro

@@ -1,0 +1,89 @@
+"""Tensor-core (tcgen05) conv path: bit-exact against the oracle through the
+C-ABI on shapes that exercise ragged tiles, batch padding and 1..4 limb
+operands.  Every block has two conv layers, so fwd, wgrad and dgrad of the
+second layer and the fwd of the first all run on tensor cores when the
+channel counts are multiples of 64."""
+import numpy as np
+import pytest
+
+from paper_2407_11698_gb300 import binding as nb
+from paper_2407_11698_gb300 import synth
+
+from netpair import NetPair
+
+pytestmark = pytest.mark.gpu
+C = nb.NITRO_CONV3X3
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _cuda():
+    torch = pytest.importorskip("torch")
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    nb.lib()
+
+
+def _two_conv_block(B, h, w, c0, c1, c2, pool):
+    oh, ow = (h // 2, w // 2) if pool else (h, w)
+    return [{"layers": [(C, c0, c1, h, w, 0), (C, c1, c2, h, w, int(pool))],
+             "in_features": h * w * c0},
+            {"layers": [], "in_features": oh * ow * c2}]
+
+
+def _widen(pair, scale):
+    """Multiply every forward weight by `scale` on both sides (more limbs)."""
+    for g, o in zip(pair.gb, pair.ob):
+        for i in range(len(o.layers)):
+            w = (o.W[i] * scale).astype(np.int64)
+            assert np.abs(w).max() < 2**31
+            o.W[i] = w
+            g.set(nb.NITRO_T_W, i, w.astype(np.int32))
+
+
+@pytest.mark.parametrize("B,h,w,c0,c1,c2,pool,scale", [
+    (8, 8, 8, 64, 64, 64, True, 1),
+    (3, 12, 9, 64, 128, 64, True, 1),          # ragged tiles in x and y, batch pad
+    (5, 8, 8, 192, 64, 128, False, 3),         # N = 64 tiles, 2-image pixel tiles
+    (8, 16, 16, 64, 128, 128, True, 1000),     # two-limb weights
+    (4, 8, 8, 64, 64, 64, True, 70001),        # three-limb weights
+    (4, 8, 8, 64, 64, 64, False, 2**22),       # four-limb weights
+    (130, 8, 16, 64, 64, 64, True, 1),         # batch over 128 (wgrad batch blocks)
+])
+def test_two_conv_block_parity(B, h, w, c0, c1, c2, pool, scale):
+    blocks = _two_conv_block(B, h, w, c0, c1, c2, pool)
+    pair = NetPair(blocks, B, seed=31)
+    try:
+        if scale != 1:
+            _widen(pair, scale)
+        for s in range(3):
+            x = synth.images(13, s, B, (h, w, c0))
+            y = synth.labels(13, s, B)
+            gl, ol = pair.step(x, y)
+            assert gl == ol, (s, gl, ol)
+            pair.compare("step %d" % s)
+    finally:
+        pair.close()
+
+
+def test_tensor_core_kernels_ran():
+    """The tc kernels are the ones launched for a 64-channel layer."""
+    torch = pytest.importorskip("torch")
+    import ctypes
+    L = nb.lib()
+    blocks = _two_conv_block(8, 8, 8, 64, 64, 64, True)
+    pair = NetPair(blocks, 8, seed=2)
+    try:
+        L.nitro_profile_reset()
+        L.nitro_profile_enable(1)
+        pair.step_gpu(synth.images(1, 0, 8, (8, 8, 64)), synth.labels(1, 0, 8))
+        L.nitro_profile_enable(0)
+        names = {}
+        for k in range(L.nitro_profile_kernel_count()):
+            n, ms, ops, by = ctypes.c_uint64(), ctypes.c_double(), ctypes.c_double(), ctypes.c_double()
+            L.nitro_profile_read(k, ctypes.byref(n), ctypes.byref(ms), ctypes.byref(ops), ctypes.byref(by))
+            names[L.nitro_profile_kernel_name(k).decode()] = n.value
+        L.nitro_profile_reset()
+        assert names["tc_conv_fwd"] == 2 and names["tc_conv_wgrad"] == 2 and names["tc_conv_dgrad"] == 1
+        assert names["simt_conv_fwd"] == 0 and names["simt_conv_wgrad"] == 0
+    finally:
+        pair.close()
