@@ -185,53 +185,110 @@ __global__ void k_fwd_epilogue(const int64_t* __restrict__ z, LayerGeom g, int B
 }
 
 // ---------------------------------------------------------------------------
-// Learning layer forward + RSS loss: one CTA per sample.
+// Learning layer forward + RSS loss, in two kernels.
+// k_learn_partial: CTA (d-slice, group of kLrSamples samples) adds its partial
+// sums of z[b][g] = sum_j a[b][j] W_lr[g][j] into zsum with int64 atomics
+// (exact, order independent).  k_learn_finish: one CTA turns zsum into
+// y_hat = floor(z / (256 d)), grad_L = y_hat - 32 onehot, SSE and the loss.
 // ---------------------------------------------------------------------------
 constexpr int kGChunk = 16;
+constexpr int kLrSamples = 4;
+constexpr int kLrSlice = 1024;
 
-__global__ void __launch_bounds__(256) k_learn_fwd(const int8_t* __restrict__ a,
-                                                   const int32_t* __restrict__ wlr,
-                                                   const int32_t* __restrict__ labels, int d,
-                                                   int G, int32_t* __restrict__ grad_l,
-                                                   unsigned long long* sse, uint32_t* maxabs_gl,
-                                                   uint32_t* status) {
-    __shared__ int64_t red[8][kGChunk];
-    const int b = blockIdx.x;
+__global__ void __launch_bounds__(256) k_learn_partial(const int8_t* __restrict__ a,
+                                                       const int32_t* __restrict__ wlr, int B,
+                                                       int d, int G,
+                                                       unsigned long long* __restrict__ zsum) {
+    __shared__ int64_t red[8][kLrSamples * kGChunk];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int lab = labels[b];
-    const bool bad = lab < 0 || lab >= G;
-    if (bad && threadIdx.x == 0) atomicOr(status, ST_BAD_LABEL);
-    const int8_t* arow = a + (int64_t)b * d;
+    const int j0 = blockIdx.x * kLrSlice, j1 = min(d, j0 + kLrSlice);
+    const int b0 = blockIdx.y * kLrSamples;
     for (int g0 = 0; g0 < G; g0 += kGChunk) {
-        int64_t acc[kGChunk];
+        int64_t acc[kLrSamples][kGChunk];
 #pragma unroll
-        for (int q = 0; q < kGChunk; ++q) acc[q] = 0;
-        for (int j = threadIdx.x; j < d; j += 256) {
-            const int32_t av = arow[j];
+        for (int u = 0; u < kLrSamples; ++u)
 #pragma unroll
-            for (int q = 0; q < kGChunk; ++q)
-                if (g0 + q < G) acc[q] += (int64_t)av * wlr[(int64_t)(g0 + q) * d + j];
+            for (int q = 0; q < kGChunk; ++q) acc[u][q] = 0;
+        for (int j = j0 + threadIdx.x; j < j1; j += 256) {
+            int32_t av[kLrSamples];
+#pragma unroll
+            for (int u = 0; u < kLrSamples; ++u)
+                av[u] = (b0 + u < B) ? (int32_t)a[(int64_t)(b0 + u) * d + j] : 0;
+#pragma unroll
+            for (int q = 0; q < kGChunk; ++q) {
+                if (g0 + q < G) {
+                    const int64_t w = wlr[(int64_t)(g0 + q) * d + j];
+#pragma unroll
+                    for (int u = 0; u < kLrSamples; ++u) acc[u][q] += w * av[u];
+                }
+            }
         }
 #pragma unroll
-        for (int q = 0; q < kGChunk; ++q) {
+        for (int u = 0; u < kLrSamples; ++u)
 #pragma unroll
-            for (int off = 16; off; off >>= 1) acc[q] += __shfl_xor_sync(kFull, acc[q], off);
-            if (lane == 0) red[warp][q] = acc[q];
+            for (int q = 0; q < kGChunk; ++q) {
+                int64_t v = acc[u][q];
+#pragma unroll
+                for (int off = 16; off; off >>= 1) v += __shfl_xor_sync(kFull, v, off);
+                if (lane == 0) red[warp][u * kGChunk + q] = v;
+            }
+        __syncthreads();
+        if (threadIdx.x < kLrSamples * kGChunk) {
+            const int u = threadIdx.x / kGChunk, q = threadIdx.x % kGChunk;
+            if (b0 + u < B && g0 + q < G) {
+                int64_t v = 0;
+                for (int w = 0; w < 8; ++w) v += red[w][threadIdx.x];
+                atomicAdd(&zsum[(int64_t)(b0 + u) * G + g0 + q], (unsigned long long)v);
+            }
         }
         __syncthreads();
-        if (threadIdx.x < kGChunk && g0 + threadIdx.x < G) {
-            const int q = threadIdx.x, gi = g0 + q;
-            int64_t zsum = 0;
-            for (int w = 0; w < 8; ++w) zsum += red[w][q];
-            const int64_t yhat = scale_floor(zsum, d);       // NITRO-Scaling, SF = 2^8 d
-            const int64_t v = yhat - ((!bad && gi == lab) ? 32 : 0);
-            if (!fits_i32(v)) atomicOr(status, ST_OVERFLOW);
-            const int32_t s = (int32_t)v;
-            grad_l[(int64_t)b * G + gi] = s;
-            atomicAdd(sse, (unsigned long long)((int64_t)s * s));
-            atomicMax(maxabs_gl, abs_u32(s));
-        }
-        __syncthreads();
+    }
+}
+
+__global__ void __launch_bounds__(1024) k_learn_finish(const unsigned long long* __restrict__ zsum,
+                                                       const int32_t* __restrict__ labels, int B,
+                                                       int d, int G, int32_t* __restrict__ grad_l,
+                                                       unsigned long long* sse, int64_t* loss,
+                                                       uint32_t* maxabs_gl, uint32_t* status) {
+    __shared__ unsigned long long red_s[32];
+    __shared__ uint32_t red_m[32];
+    __shared__ int flags;
+    if (threadIdx.x == 0) flags = 0;
+    __syncthreads();
+    unsigned long long ss = 0;
+    uint32_t mx = 0;
+    int fl = 0;
+    const int64_t n = (int64_t)B * G;
+    for (int64_t i = threadIdx.x; i < n; i += blockDim.x) {
+        const int b = (int)(i / G), g = (int)(i - (int64_t)b * G);
+        const int lab = labels[b];
+        const bool bad = lab < 0 || lab >= G;
+        if (bad && g == 0) fl |= ST_BAD_LABEL;
+        const int64_t yhat = scale_floor((int64_t)zsum[i], d);     // NITRO-Scaling, SF = 2^8 d
+        const int64_t v = yhat - ((!bad && g == lab) ? 32 : 0);
+        if (!fits_i32(v)) fl |= ST_OVERFLOW;
+        const int32_t sv = (int32_t)v;
+        grad_l[i] = sv;
+        ss += (unsigned long long)((int64_t)sv * sv);
+        mx = max(mx, abs_u32(sv));
+    }
+#pragma unroll
+    for (int off = 16; off; off >>= 1) {
+        ss += __shfl_xor_sync(kFull, ss, off);
+        mx = max(mx, __shfl_xor_sync(kFull, mx, off));
+    }
+    if (fl) atomicOr(&flags, fl);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (lane == 0) { red_s[warp] = ss; red_m[warp] = mx; }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        unsigned long long t = 0;
+        uint32_t m = 0;
+        for (int w = 0; w < (int)(blockDim.x >> 5); ++w) { t += red_s[w]; m = max(m, red_m[w]); }
+        *sse = t;                                            // modulo 2^64
+        if (loss) *loss = fdiv64((int64_t)t, 2);
+        atomicMax(maxabs_gl, m);
+        if (flags) atomicOr(status, (uint32_t)flags);
     }
 }
 
@@ -330,10 +387,6 @@ __global__ void k_integersgd(SgdBatch bt) {
     }
 }
 
-__global__ void k_finish_loss(const unsigned long long* sse, int64_t* loss) {
-    loss[0] = fdiv64((int64_t)sse[0], 2);
-}
-
 inline int grid_for(int64_t n, int threads, int cap = 152 * 16) {
     int64_t g = (n + threads - 1) / threads;
     return (int)(g < 1 ? 1 : (g > cap ? cap : g));
@@ -401,11 +454,22 @@ cudaError_t simt_fwd_epilogue(const int64_t* z, const LayerGeom& g, int B, int a
 }
 
 cudaError_t simt_learn_fwd(const int8_t* a, const int32_t* wlr, const int32_t* labels, int B,
-                           int d, int G, int32_t* grad_l, unsigned long long* sse,
-                           uint32_t* maxabs_gl, uint32_t* status, cudaStream_t s) {
+                           int d, int G, int64_t* zsum, int32_t* grad_l, unsigned long long* sse,
+                           int64_t* loss, uint32_t* maxabs_gl, uint32_t* status, cudaStream_t s) {
     if (B <= 0) return cudaSuccess;
-    ProfScope ps(K_LEARN_FWD, s, 2.0 * B * d * G, 0.0);
-    k_learn_fwd<<<B, 256, 0, s>>>(a, wlr, labels, d, G, grad_l, sse, maxabs_gl, status);
+    cudaError_t e = cudaMemsetAsync(zsum, 0, sizeof(int64_t) * (size_t)B * G, s);
+    if (e != cudaSuccess) return e;
+    {
+        dim3 grid((d + kLrSlice - 1) / kLrSlice, (B + kLrSamples - 1) / kLrSamples);
+        ProfScope ps(K_LEARN_FWD, s, 2.0 * B * d * G, 0.0);
+        k_learn_partial<<<grid, 256, 0, s>>>(a, wlr, B, d, G,
+                                             reinterpret_cast<unsigned long long*>(zsum));
+        e = cudaGetLastError();
+        if (e != cudaSuccess) return e;
+    }
+    ProfScope ps(K_FINISH_LOSS, s, 0.0, 0.0);
+    k_learn_finish<<<1, 1024, 0, s>>>(reinterpret_cast<const unsigned long long*>(zsum), labels, B,
+                                      d, G, grad_l, sse, loss, maxabs_gl, status);
     return cudaGetLastError();
 }
 
@@ -444,10 +508,5 @@ cudaError_t simt_integersgd(const SgdBatch& b, cudaStream_t s) {
     return cudaGetLastError();
 }
 
-cudaError_t simt_finish_loss(const unsigned long long* sse, int64_t* loss, cudaStream_t s) {
-    ProfScope ps(K_FINISH_LOSS, s, 0.0, 0.0);
-    k_finish_loss<<<1, 1, 0, s>>>(sse, loss);
-    return cudaGetLastError();
-}
 
 }  // namespace nitro

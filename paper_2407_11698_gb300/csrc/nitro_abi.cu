@@ -41,6 +41,7 @@ struct nitro_block {
     int32_t* Wlr = nullptr;
     int64_t* dWlr = nullptr;
     int32_t* grad_l = nullptr;      // [max_batch x G]
+    int64_t* zsum = nullptr;        // [max_batch x G] learning-layer pre-activations
     int64_t* z64 = nullptr;         // scratch, int64 pre-activations / dgrad outputs
     size_t z64_elems = 0;
     uint32_t* words = nullptr;      // [0] status [1] max|grad_l| [2] max|W_lr|
@@ -108,9 +109,6 @@ uint32_t host_maxabs(const int32_t* p, size_t n) {
     return m;
 }
 
-nitro_status cuda_fail(cudaError_t e) {
-    return e == cudaSuccess ? NITRO_OK : NITRO_ERR_CUDA;
-}
 
 #define NITRO_TRY(expr)                                \
     do {                                               \
@@ -220,7 +218,7 @@ nitro_status nitro_init_block(const nitro_block_desc* desc, uint64_t seed, void*
     }
     b->d = desc->n_layers ? b->L.back().out_f : desc->in_features;
     ok = ok && dalloc(b, &b->Wlr, (size_t)b->G * b->d) && dalloc(b, &b->dWlr, (size_t)b->G * b->d) &&
-         dalloc(b, &b->grad_l, (size_t)MB * b->G) && dalloc(b, &b->z64, z_need) &&
+         dalloc(b, &b->grad_l, (size_t)MB * b->G) && dalloc(b, &b->zsum, (size_t)MB * b->G) && dalloc(b, &b->z64, z_need) &&
          dalloc(b, &b->words, n_words(desc->n_layers)) && dalloc(b, &b->sse, 1);
     b->z64_elems = z_need;
     for (int i = 0; ok && i < desc->n_layers; ++i)
@@ -271,19 +269,27 @@ nitro_status nitro_block_forward(nitro_block* b, const int8_t* a_in, int batch, 
     if (batch == 0) return NITRO_OK;
     const int n = (int)b->L.size();
     const int8_t* x = a_in;
+    bool nhwc_done = false;
     for (int i = 0; i < n; ++i) {
         Layer& ly = b->L[i];
         const LayerGeom& g = ly.g;
         int8_t* out2 = (i == n - 1) ? a_out : nullptr;
-        bool done = false;
-        NITRO_TRY(tc_pack_input(ly.tc, g, x, batch, s));
-        NITRO_TRY(tc_conv_forward(ly.tc, g, batch, b->z64, w_status(b), s, &done));
+        bool done = false, fused = false;
+        NITRO_TRY(tc_pack_input(ly.tc, g, x, batch, nhwc_done, s));
+        // the epilogue also writes the next layer's bf16 forward operand
+        uint16_t* next_nhwc = nullptr;
+        if (i + 1 < n && b->L[i + 1].tc.fwd && b->L[i + 1].tc.cin8 == g.cout)
+            next_nhwc = b->L[i + 1].tc.act_nhwc;
+        TcFwdOut fo{b->desc.alpha_inv, b->mu, ly.act, out2, ly.region, ly.argmax, next_nhwc};
+        NITRO_TRY(tc_conv_forward(ly.tc, g, batch, b->z64, &fo, w_status(b), s, &done, &fused));
         if (!done) {
             const int mode = g.kind == NITRO_CONV3X3 ? GM_CONV_FWD : GM_LIN_FWD;
             NITRO_TRY(simt_gemm(mode, x, nullptr, ly.W, b->z64, batch, g.h, g.w, g.cin, g.cout, s));
         }
-        NITRO_TRY(simt_fwd_epilogue(b->z64, g, batch, b->desc.alpha_inv, b->mu, ly.act, out2,
-                                    ly.region, ly.argmax, s));
+        if (!fused)
+            NITRO_TRY(simt_fwd_epilogue(b->z64, g, batch, b->desc.alpha_inv, b->mu, ly.act, out2,
+                                        ly.region, ly.argmax, s));
+        nhwc_done = fused && next_nhwc != nullptr;
         x = ly.act;
     }
     return NITRO_OK;
@@ -308,10 +314,9 @@ nitro_status nitro_block_backward(nitro_block* b, const int8_t* a_in, const int3
         return NITRO_OK;
     }
     const int8_t* a_last = n ? b->L[n - 1].act : a_in;
-    NITRO_TRY(simt_learn_fwd(a_last, b->Wlr, labels, batch, (int)d, G, b->grad_l, b->sse, w_gl(b),
-                             w_status(b), s));
+    NITRO_TRY(simt_learn_fwd(a_last, b->Wlr, labels, batch, (int)d, G, b->zsum, b->grad_l, b->sse,
+                             loss_dev, w_gl(b), w_status(b), s));
     NITRO_TRY(simt_learn_dw(a_last, b->grad_l, batch, (int)d, G, b->dWlr, s));
-    if (loss_dev) NITRO_TRY(simt_finish_loss(b->sse, loss_dev, s));
     if (n == 0) return NITRO_OK;
     // delta_fw = grad_L W_lr (pre-update), into the last layer
     {

@@ -27,6 +27,43 @@ __host__ __device__ __forceinline__ int64_t scale_floor(int64_t z, int64_t k) {
     return fdiv64(z >> 8, k);
 }
 
+// Floor division by an invariant positive integer d through a multiply-high,
+// after Granlund & Montgomery, "Division by invariant integers using
+// multiplication" (PLDI 1994), Fig. 4.1 (N = 64): with l = ceil(log2 d),
+// m = floor(2^64 (2^l - d) / d) + 1, sh1 = min(l, 1), sh2 = max(l - 1, 0),
+// floor(n / d) = (t + ((n - t) >> sh1)) >> sh2 with t = mulhi(m, n), for every
+// unsigned 64-bit n.  Negative x use floor(x / d) = -floor((-x - 1) / d) - 1.
+struct FloorDiv {
+    uint64_t m;
+    int sh1, sh2;
+    __host__ static FloorDiv make(uint64_t d) {
+        int l = 0;
+        while (l < 64 && ((uint64_t)1 << l) < d) ++l;
+        FloorDiv f;
+        const unsigned __int128 two_l = (unsigned __int128)1 << l;
+        f.m = (uint64_t)((((unsigned __int128)1 << 64) * (two_l - d)) / d + 1);
+        f.sh1 = l < 1 ? l : 1;
+        f.sh2 = l > 1 ? l - 1 : 0;
+        return f;
+    }
+    __host__ __device__ __forceinline__ uint64_t udiv(uint64_t n) const {
+#ifdef __CUDA_ARCH__
+        const uint64_t t = __umul64hi(m, n);
+#else
+        const uint64_t t = (uint64_t)(((unsigned __int128)m * n) >> 64);
+#endif
+        return (t + ((n - t) >> sh1)) >> sh2;
+    }
+    __host__ __device__ __forceinline__ int64_t floor_div(int64_t x) const {
+        if (x >= 0) return (int64_t)udiv((uint64_t)x);
+        return -(int64_t)udiv((uint64_t)(-(x + 1))) - 1;
+    }
+    __host__ __device__ __forceinline__ int64_t trunc_div(int64_t x) const {
+        if (x >= 0) return (int64_t)udiv((uint64_t)x);
+        return -(int64_t)udiv((uint64_t)(-(x + 1)) + 1);
+    }
+};
+
 __host__ __device__ __forceinline__ bool fits_i32(int64_t v) {
     return v >= INT32_MIN && v <= INT32_MAX;
 }
@@ -40,6 +77,14 @@ __host__ __device__ __forceinline__ int relu_value(int64_t x, int alpha_inv, int
     if (x < 0) {
         int c = x < -127 ? -127 : (int)x;
         return fdiv32(c, alpha_inv) - mu;
+    }
+    return (x > 127 ? 127 : (int)x) - mu;
+}
+// Same, with the slope division through a precomputed divider.
+__host__ __device__ __forceinline__ int relu_value(int64_t x, const FloorDiv& alpha, int mu) {
+    if (x < 0) {
+        int64_t c = x < -127 ? -127 : x;
+        return (int)alpha.floor_div(c) - mu;
     }
     return (x > 127 ? 127 : (int)x) - mu;
 }
@@ -98,10 +143,11 @@ cudaError_t simt_fwd_epilogue(const int64_t* z, const LayerGeom& g, int B, int a
                               int8_t* argmax, cudaStream_t s);
 
 // Learning layer forward + loss: grad_l = floor(a W^T / (256 d)) - 32 onehot,
-// sse += sum grad_l^2 (mod 2^64), words[1] = max|grad_l|, status bits.
+// sse = sum grad_l^2 (mod 2^64), loss = floor(sse / 2) (if loss != NULL),
+// max|grad_l| into *maxabs_gl, status bits.  zsum: int64 scratch [B x G].
 cudaError_t simt_learn_fwd(const int8_t* a, const int32_t* wlr, const int32_t* labels, int B,
-                           int d, int G, int32_t* grad_l, unsigned long long* sse,
-                           uint32_t* maxabs_gl, uint32_t* status, cudaStream_t s);
+                           int d, int G, int64_t* zsum, int32_t* grad_l, unsigned long long* sse,
+                           int64_t* loss, uint32_t* maxabs_gl, uint32_t* status, cudaStream_t s);
 
 // dW_lr[g][j] = sum_b grad_l[b][g] a[b][j]
 cudaError_t simt_learn_dw(const int8_t* a, const int32_t* grad_l, int B, int d, int G,
@@ -140,7 +186,5 @@ struct SgdBatch {
 };
 cudaError_t simt_integersgd(const SgdBatch& b, cudaStream_t s);
 
-// loss = floor(int64(sse) / 2)
-cudaError_t simt_finish_loss(const unsigned long long* sse, int64_t* loss, cudaStream_t s);
 
 }  // namespace nitro

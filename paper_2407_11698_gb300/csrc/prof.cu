@@ -37,8 +37,8 @@ cudaEvent_t take_event() {
 
 const char* const kNames[K_COUNT] = {
     "simt_conv_fwd", "simt_conv_dgrad", "simt_conv_wgrad", "simt_linear_fwd",
-    "simt_linear_dgrad", "simt_linear_wgrad", "fwd_epilogue", "learn_fwd_loss",
-    "learn_dw", "grad_to_delta", "integersgd", "finish_loss", "tc_conv_fwd",
+    "simt_linear_dgrad", "simt_linear_wgrad", "fwd_epilogue", "learn_partial",
+    "learn_dw", "grad_to_delta", "integersgd", "learn_finish_loss", "tc_conv_fwd",
     "tc_conv_wgrad", "tc_conv_dgrad", "tc_pack_limbs", "tc_finish"};
 
 }  // namespace

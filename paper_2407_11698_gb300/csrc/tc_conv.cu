@@ -158,15 +158,45 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
 // ------------------------------------------------------------------ kernel
 struct TcArgs {
     int B, H, W, Cin, Cout, Bp;
+    int cin_k;             // channels per tap in the K index (Cin rounded up to 64)
     int ntx, nty;          // pixel tiles along x and y (forward / dgrad)
     int wb, hb, bb;        // pixel box (forward / dgrad): wb * hb * bb = 128
+    int tiles_m, tiles_n, total_tiles;
     int kb_total, kb_per_split;
+    int ncols;             // valid output columns (Cout for fwd/wgrad, Cin for dgrad)
     const int* limbs_a;    // limb counts (nullptr = 1)
     const int* limbs_b;
     int64_t* out;
     uint32_t* status;
     int atomic_out;
+    // forward with fused NITRO-Scaling / NITRO-ReLU / max-pool epilogue
+    int fuse;
+    FloorDiv sf, alpha;    // divide by SF = 2^8 * 9 * Cin, and by alpha_inv
+    int mu, pool, oh, ow;
+    int8_t* act;           // layer output (post-pool) int8 NHWC
+    int8_t* out2;          // optional second copy of the output (caller's buffer)
+    int8_t* region;        // NITRO-ReLU piece per pre-pool output
+    int8_t* argmax;        // window position per pooled output
+    uint16_t* next_nhwc;   // bf16 copy of the output for the next layer's forward, or null
 };
+
+// 16 int8 values (4 packed words) -> one 16-byte store
+__device__ __forceinline__ void st16(int8_t* dst, const uint32_t* w) {
+    *reinterpret_cast<uint4*>(dst) = make_uint4(w[0], w[1], w[2], w[3]);
+}
+// 16 int8 values (4 packed words) -> 16 bf16 values (two 16-byte stores)
+__device__ __forceinline__ void st16_bf16(uint16_t* dst, const uint32_t* w) {
+    uint32_t o[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+        const int lo = (int8_t)(w[k >> 1] >> (16 * (k & 1)));
+        const int hi = (int8_t)(w[k >> 1] >> (16 * (k & 1) + 8));
+        o[k] = (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn((float)lo)) |
+               ((uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn((float)hi)) << 16);
+    }
+    reinterpret_cast<uint4*>(dst)[0] = make_uint4(o[0], o[1], o[2], o[3]);
+    reinterpret_cast<uint4*>(dst)[1] = make_uint4(o[4], o[5], o[6], o[7]);
+}
 
 template <int N>
 struct TcCfg {
@@ -177,6 +207,23 @@ struct TcCfg {
     static constexpr int SMEM = 1024 + S * STAGE + 256;
 };
 
+struct Tile {
+    int mt, nt, kb0, kb1;
+};
+__device__ __forceinline__ Tile decode_tile(const TcArgs& a, int tile) {
+    Tile t;
+    t.nt = tile % a.tiles_n;
+    const int r = tile / a.tiles_n;
+    t.mt = r % a.tiles_m;
+    const int split = r / a.tiles_m;
+    t.kb0 = split * a.kb_per_split;
+    t.kb1 = min(a.kb_total, t.kb0 + a.kb_per_split);
+    return t;
+}
+
+// Persistent: CTA c handles tiles c, c + gridDim.x, ...; the TMA ring, the
+// MMA chunk sequence and the two TMEM accumulators run on across tiles, so
+// one tile's epilogue overlaps the next tile's loads and MMAs.
 template <int MODE, int N>
 __global__ void __launch_bounds__(kThreads, 1)
     k_tc_gemm(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
@@ -223,93 +270,96 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
 
-    const int mt = blockIdx.x, nt = blockIdx.y;
-    const int n0 = nt * N;
-    const int kb0 = blockIdx.z * args.kb_per_split;
-    const int kb1 = min(args.kb_total, kb0 + args.kb_per_split);
-    const int nkb = kb1 - kb0;
     int LA = args.limbs_a ? *args.limbs_a : 1;
     int LB = args.limbs_b ? *args.limbs_b : 1;
     LA = LA < 1 ? 1 : (LA > kMaxLimbs ? kMaxLimbs : LA);
     LB = LB < 1 ? 1 : (LB > kMaxLimbs ? kMaxLimbs : LB);
     const int passes = LA * LB;
-    const int cpp = (nkb + kChunkBlocks - 1) / kChunkBlocks;   // chunks per pass
-
-    // pixel tile origin (forward / dgrad)
-    const int tx = mt % args.ntx, ty = (mt / args.ntx) % args.nty, tb = mt / (args.ntx * args.nty);
-    const int x0 = tx * args.wb, y0 = ty * args.hb, b0 = tb * args.bb;
 
     if (warp == 0) {
-        if (lane == 0 && nkb > 0) {
+        if (lane == 0) {
             // ---------------- TMA producer
             int it = 0;
-            for (int p = 0; p < passes; ++p) {
-                const int la = p / LB, lb = p % LB;
-                for (int kb = kb0; kb < kb1; ++kb, ++it) {
-                    const int s = it % S;
-                    if (!mbar_wait(empty_bar(s), ((it / S) & 1) ^ 1, abort_flag, args.status))
-                        goto producer_done;
-                    const uint32_t fb = full_bar(s);
-                    const uint32_t a_dst = smem_u32(smem + s * C::STAGE);
-                    const uint32_t b_dst = a_dst + C::A_BYTES;
-                    mbar_expect_tx(fb, C::STAGE);
-                    if (MODE == TC_FWD) {
-                        const int nc = args.Cin / kBK;
-                        const int t = kb / nc, cb = kb - t * nc, ky = t / 3, kx = t - 3 * ky;
-                        tma_load_4d(a_dst, &tmA, fb, cb * kBK, x0 + kx - 1, y0 + ky - 1, b0);
-                        tma_load_3d(b_dst, &tmB, fb, t * args.Cin + cb * kBK, n0, lb);
-                    } else if (MODE == TC_DGRAD) {
-                        const int nc = args.Cout / kBK;
-                        const int t = kb / nc, cb = kb - t * nc, ky = t / 3, kx = t - 3 * ky;
-                        tma_load_5d(a_dst, &tmA, fb, cb * kBK, x0 - kx + 1, y0 - ky + 1, b0, la);
-                        tma_load_4d(b_dst, &tmB, fb, cb * kBK, n0, t, lb);
-                    } else {  // TC_WGRAD: rows (tap, ci), K = (y, x, b)
-                        const int nbb = (args.Bp + kBK - 1) / kBK;
-                        const int pos = kb / nbb, bbk = kb - pos * nbb;
-                        const int y = pos / args.W, x = pos - y * args.W;
+            for (int tile = blockIdx.x; tile < args.total_tiles; tile += gridDim.x) {
+                const Tile T = decode_tile(args, tile);
+                const int n0 = T.nt * N;
+                const int tx = T.mt % args.ntx, ty = (T.mt / args.ntx) % args.nty;
+                const int tb = T.mt / (args.ntx * args.nty);
+                const int x0 = tx * args.wb, y0 = ty * args.hb, b0 = tb * args.bb;
+                for (int p = 0; p < passes; ++p) {
+                    const int la = p / LB, lb = p % LB;
+                    for (int kb = T.kb0; kb < T.kb1; ++kb, ++it) {
+                        const int s = it % S;
+                        if (!mbar_wait(empty_bar(s), ((it / S) & 1) ^ 1, abort_flag, args.status))
+                            goto producer_done;
+                        const uint32_t fb = full_bar(s);
+                        const uint32_t a_dst = smem_u32(smem + s * C::STAGE);
+                        const uint32_t b_dst = a_dst + C::A_BYTES;
+                        mbar_expect_tx(fb, C::STAGE);
+                        if (MODE == TC_FWD) {
+                            const int nc = args.cin_k / kBK;
+                            const int t = kb / nc, cb = kb - t * nc, ky = t / 3, kx = t - 3 * ky;
+                            tma_load_4d(a_dst, &tmA, fb, cb * kBK, x0 + kx - 1, y0 + ky - 1, b0);
+                            tma_load_3d(b_dst, &tmB, fb, t * args.cin_k + cb * kBK, n0, lb);
+                        } else if (MODE == TC_DGRAD) {
+                            const int nc = (args.Cout + kBK - 1) / kBK;
+                            const int t = kb / nc, cb = kb - t * nc, ky = t / 3, kx = t - 3 * ky;
+                            tma_load_5d(a_dst, &tmA, fb, cb * kBK, x0 - kx + 1, y0 - ky + 1, b0, la);
+                            tma_load_4d(b_dst, &tmB, fb, cb * kBK, n0, t, lb);
+                        } else {  // TC_WGRAD: rows (tap, ci), K = (y, x, b)
+                            const int nbb = (args.Bp + kBK - 1) / kBK;
+                            const int pos = kb / nbb, bbk = kb - pos * nbb;
+                            const int y = pos / args.W, x = pos - y * args.W;
 #pragma unroll
-                        for (int j = 0; j < 2; ++j) {
-                            const int m = mt * kBM + j * 64;
-                            int t = m / args.Cin, ci0 = m - t * args.Cin;
-                            if (t >= 9) { t = 0; ci0 = args.Cin; }   // fully out of range: zeros
-                            const int ky = t / 3, kx = t - 3 * ky;
-                            tma_load_4d(a_dst + j * (64 * 128), &tmA, fb, bbk * kBK, x + kx - 1,
-                                        y + ky - 1, ci0);
+                            for (int j = 0; j < 2; ++j) {
+                                const int m = T.mt * kBM + j * 64;
+                                int t = m / args.cin_k, ci0 = m - t * args.cin_k;
+                                if (t >= 9) { t = 0; ci0 = args.cin_k; }   // past the last tap: zeros
+                                const int ky = t / 3, kx = t - 3 * ky;
+                                tma_load_4d(a_dst + j * (64 * 128), &tmA, fb, bbk * kBK, x + kx - 1,
+                                            y + ky - 1, ci0);
+                            }
+                            tma_load_5d(b_dst, &tmB, fb, bbk * kBK, x, y, n0, lb);
                         }
-                        tma_load_4d(b_dst, &tmB, fb, bbk * kBK, x, y, lb * args.Cout + n0);
                     }
                 }
             }
         producer_done:;
         }
     } else if (warp == 1) {
-        if (lane == 0 && nkb > 0) {
+        if (lane == 0) {
             // ---------------- MMA issuer
             constexpr uint32_t idesc = idesc_bf16(kBM, N);
             int it = 0, chunk = 0;
-            for (int p = 0; p < passes; ++p) {
-                for (int c = 0; c < cpp; ++c, ++chunk) {
-                    const int buf = chunk & 1;
-                    if (!mbar_wait(tempty_bar(buf), ((chunk >> 1) & 1) ^ 1, abort_flag, args.status))
-                        goto mma_done;
-                    tc_fence_after();
-                    const uint32_t d = tmem + (uint32_t)(buf * N);
-                    const int c0 = kb0 + c * kChunkBlocks;
-                    const int c1 = min(kb1, c0 + kChunkBlocks);
-                    for (int kb = c0; kb < c1; ++kb, ++it) {
-                        const int s = it % S;
-                        if (!mbar_wait(full_bar(s), (it / S) & 1, abort_flag, args.status))
+            for (int tile = blockIdx.x; tile < args.total_tiles; tile += gridDim.x) {
+                const Tile T = decode_tile(args, tile);
+                const int cpp = (T.kb1 - T.kb0 + kChunkBlocks - 1) / kChunkBlocks;
+                for (int p = 0; p < passes; ++p) {
+                    for (int c = 0; c < cpp; ++c, ++chunk) {
+                        const int buf = chunk & 1;
+                        if (!mbar_wait(tempty_bar(buf), ((chunk >> 1) & 1) ^ 1, abort_flag,
+                                       args.status))
                             goto mma_done;
                         tc_fence_after();
-                        const uint32_t a_addr = smem_u32(smem + s * C::STAGE);
-                        const uint32_t b_addr = a_addr + C::A_BYTES;
+                        const uint32_t d = tmem + (uint32_t)(buf * N);
+                        const int c0 = T.kb0 + c * kChunkBlocks;
+                        const int c1 = min(T.kb1, c0 + kChunkBlocks);
+                        for (int kb = c0; kb < c1; ++kb, ++it) {
+                            const int s = it % S;
+                            if (!mbar_wait(full_bar(s), (it / S) & 1, abort_flag, args.status))
+                                goto mma_done;
+                            tc_fence_after();
+                            const uint32_t a_addr = smem_u32(smem + s * C::STAGE);
+                            const uint32_t b_addr = a_addr + C::A_BYTES;
 #pragma unroll
-                        for (int k = 0; k < kBK / 16; ++k)
-                            umma_bf16(d, desc_sw128(a_addr + 32 * k), desc_sw128(b_addr + 32 * k),
-                                      idesc, (kb > c0 || k > 0) ? 1u : 0u);
-                        umma_commit(empty_bar(s));
+                            for (int k = 0; k < kBK / 16; ++k)
+                                umma_bf16(d, desc_sw128(a_addr + 32 * k),
+                                          desc_sw128(b_addr + 32 * k), idesc,
+                                          (kb > c0 || k > 0) ? 1u : 0u);
+                            umma_commit(empty_bar(s));
+                        }
+                        umma_commit(tfull_bar(buf));
                     }
-                    umma_commit(tfull_bar(buf));
                 }
             }
         mma_done:;
@@ -318,69 +368,162 @@ __global__ void __launch_bounds__(kThreads, 1)
         // ---------------- epilogue: warps 2..9
         const int q = warp & 3;             // TMEM lane quadrant this warp may read
         const int half = (warp - 2) >> 2;   // which half of the N columns
-        uint64_t acc[NH];
-#pragma unroll
-        for (int i = 0; i < NH; ++i) acc[i] = 0;
-        bool ok = nkb > 0;
         int chunk = 0;
-        for (int p = 0; ok && p < passes; ++p) {
-            const int shift = 8 * (p / LB + p % LB);
-            for (int c = 0; c < cpp; ++c, ++chunk) {
-                const int buf = chunk & 1;
-                if (!mbar_wait(tfull_bar(buf), (chunk >> 1) & 1, abort_flag, args.status)) {
-                    ok = false;
-                    break;
-                }
-                tc_fence_after();
-                const uint32_t base = tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(buf * N + half * NH);
+        for (int tile = blockIdx.x; tile < args.total_tiles; tile += gridDim.x) {
+            const Tile T = decode_tile(args, tile);
+            const int cpp = (T.kb1 - T.kb0 + kChunkBlocks - 1) / kChunkBlocks;
+            uint64_t acc[NH];
 #pragma unroll
-                for (int j = 0; j < NH / 16; ++j) {
-                    uint32_t r[16];
-                    tmem_ld16(base + 16 * j, r);
+            for (int i = 0; i < NH; ++i) acc[i] = 0;
+            for (int p = 0; p < passes; ++p) {
+                const int shift = 8 * (p / LB + p % LB);
+                for (int c = 0; c < cpp; ++c, ++chunk) {
+                    const int buf = chunk & 1;
+                    if (!mbar_wait(tfull_bar(buf), (chunk >> 1) & 1, abort_flag, args.status))
+                        goto epi_done;
+                    tc_fence_after();
+                    const uint32_t base =
+                        tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(buf * N + half * NH);
 #pragma unroll
-                    for (int i = 0; i < 16; ++i) {
-                        const int v = __float2int_rz(__uint_as_float(r[i]));   // exact integer
-                        acc[16 * j + i] += (uint64_t)(int64_t)v << shift;
+                    for (int j = 0; j < NH / 16; ++j) {
+                        uint32_t r[16];
+                        tmem_ld16(base + 16 * j, r);
+#pragma unroll
+                        for (int i = 0; i < 16; ++i) {
+                            const int v = __float2int_rz(__uint_as_float(r[i]));   // exact integer
+                            acc[16 * j + i] += (uint64_t)(int64_t)v << shift;
+                        }
                     }
-                }
-                tc_fence_before();
-                __syncwarp();
-                if (lane == 0) mbar_arrive(tempty_bar(buf));
-            }
-        }
-        if (ok) {
-            const int r = 32 * q + lane;   // output row of this thread
-            const int col0 = n0 + half * NH;
-            if (MODE == TC_WGRAD) {
-                const int m = mt * kBM + r;
-                const int t = m / args.Cin, ci = m - t * args.Cin;
-                if (t < 9) {
-                    int64_t* o = args.out + (int64_t)t * args.Cin + ci;
-                    const int64_t cstride = 9LL * args.Cin;
-#pragma unroll
-                    for (int i = 0; i < NH; ++i) {
-                        unsigned long long* dst =
-                            reinterpret_cast<unsigned long long*>(o + (int64_t)(col0 + i) * cstride);
-                        if (args.atomic_out) atomicAdd(dst, (unsigned long long)acc[i]);
-                        else *dst = acc[i];
-                    }
-                }
-            } else {
-                const int xx = r % args.wb, yy = (r / args.wb) % args.hb, bbx = r / (args.wb * args.hb);
-                const int x = x0 + xx, y = y0 + yy, b = b0 + bbx;
-                if (x < args.W && y < args.H && b < args.B) {
-                    const int ncols = MODE == TC_FWD ? args.Cout : args.Cin;
-                    int64_t* o = args.out + (((int64_t)b * args.H + y) * args.W + x) * ncols + col0;
-#pragma unroll
-                    for (int i = 0; i < NH; i += 2) {
-                        longlong2 v;
-                        v.x = (long long)acc[i];
-                        v.y = (long long)acc[i + 1];
-                        *reinterpret_cast<longlong2*>(o + i) = v;
-                    }
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(tempty_bar(buf));
                 }
             }
+            {
+                const int r = 32 * q + lane;   // output row of this thread
+                const int col0 = T.nt * N + half * NH;
+                if (MODE == TC_WGRAD) {
+                    const int m = T.mt * kBM + r;
+                    const int t = m / args.cin_k, ci = m - t * args.cin_k;
+                    if (t < 9 && ci < args.Cin) {
+                        int64_t* o = args.out + (int64_t)t * args.Cin + ci;
+                        const int64_t cstride = 9LL * args.Cin;
+#pragma unroll
+                        for (int i = 0; i < NH; ++i) {
+                            if (col0 + i >= args.ncols) break;
+                            unsigned long long* dst = reinterpret_cast<unsigned long long*>(
+                                o + (int64_t)(col0 + i) * cstride);
+                            if (args.atomic_out) atomicAdd(dst, (unsigned long long)acc[i]);
+                            else *dst = acc[i];
+                        }
+                    }
+                } else if (MODE == TC_FWD && args.fuse) {
+                    // z* = floor(z / SF), NITRO-ReLU piece and value, optional
+                    // 2x2 max-pool across lanes; int8 outputs straight from
+                    // registers (the 2x2 windows of a tile lie inside one warp:
+                    // x partner lane ^ 1, y partner lane ^ wb).
+                    const int tx = T.mt % args.ntx, ty = (T.mt / args.ntx) % args.nty;
+                    const int tb = T.mt / (args.ntx * args.nty);
+                    const int xx = r % args.wb, yy = (r / args.wb) % args.hb;
+                    const int bbx = r / (args.wb * args.hb);
+                    const int x = tx * args.wb + xx, y = ty * args.hb + yy, b = tb * args.bb + bbx;
+                    const bool valid = x < args.W && y < args.H && b < args.B;
+                    const int C = args.Cout;
+                    uint32_t vpk[NH / 4], rpk[NH / 4];
+#pragma unroll
+                    for (int g4 = 0; g4 < NH / 4; ++g4) {
+                        uint32_t vp = 0, rp = 0;
+#pragma unroll
+                        for (int u = 0; u < 4; ++u) {
+                            const int64_t zs = args.sf.floor_div((int64_t)acc[4 * g4 + u]);
+                            rp |= (uint32_t)relu_region(zs) << (8 * u);
+                            vp |= (uint32_t)(uint8_t)(int8_t)relu_value(zs, args.alpha, args.mu) << (8 * u);
+                        }
+                        vpk[g4] = vp;
+                        rpk[g4] = rp;
+                    }
+                    const int64_t pix = ((int64_t)b * args.H + y) * args.W + x;
+                    if (valid) {
+#pragma unroll
+                        for (int k = 0; k < NH / 16; ++k)
+                            if (col0 + 16 * k < C) st16(args.region + pix * C + col0 + 16 * k, rpk + 4 * k);
+                    }
+                    if (!args.pool) {
+                        if (valid) {
+#pragma unroll
+                            for (int k = 0; k < NH / 16; ++k) {
+                                if (col0 + 16 * k >= C) break;
+                                const int64_t o = pix * C + col0 + 16 * k;
+                                st16(args.act + o, vpk + 4 * k);
+                                if (args.out2) st16(args.out2 + o, vpk + 4 * k);
+                                if (args.next_nhwc) st16_bf16(args.next_nhwc + o, vpk + 4 * k);
+                            }
+                        }
+                    } else {
+                        const int dys = args.wb;
+                        uint32_t opk[NH / 4], apk[NH / 4];
+#pragma unroll
+                        for (int g4 = 0; g4 < NH / 4; ++g4) {
+                            const uint32_t v00 = vpk[g4];
+                            const uint32_t v01 = __shfl_xor_sync(0xffffffffu, v00, 1);
+                            const uint32_t v10 = __shfl_xor_sync(0xffffffffu, v00, dys);
+                            const uint32_t v11 = __shfl_xor_sync(0xffffffffu, v00, dys ^ 1);
+                            uint32_t op = 0, ap = 0;
+#pragma unroll
+                            for (int u = 0; u < 4; ++u) {
+                                // window order (0,0), (0,1), (1,0), (1,1); first maximum wins
+                                int best = (int8_t)(v00 >> (8 * u)), k = 0;
+                                const int c1 = (int8_t)(v01 >> (8 * u));
+                                const int c2 = (int8_t)(v10 >> (8 * u));
+                                const int c3 = (int8_t)(v11 >> (8 * u));
+                                if (c1 > best) { best = c1; k = 1; }
+                                if (c2 > best) { best = c2; k = 2; }
+                                if (c3 > best) { best = c3; k = 3; }
+                                op |= (uint32_t)(uint8_t)best << (8 * u);
+                                ap |= (uint32_t)k << (8 * u);
+                            }
+                            opk[g4] = op;
+                            apk[g4] = ap;
+                        }
+                        if (valid && !(x & 1) && !(y & 1) && x + 1 < args.W && y + 1 < args.H) {
+                            const int64_t opix = ((int64_t)b * args.oh + (y >> 1)) * args.ow + (x >> 1);
+#pragma unroll
+                            for (int k = 0; k < NH / 16; ++k) {
+                                if (col0 + 16 * k >= C) break;
+                                const int64_t o = opix * C + col0 + 16 * k;
+                                st16(args.act + o, opk + 4 * k);
+                                if (args.out2) st16(args.out2 + o, opk + 4 * k);
+                                st16(args.argmax + o, apk + 4 * k);
+                                if (args.next_nhwc) st16_bf16(args.next_nhwc + o, opk + 4 * k);
+                            }
+                        }
+                    }
+                } else {
+                    const int tx = T.mt % args.ntx, ty = (T.mt / args.ntx) % args.nty;
+                    const int tb = T.mt / (args.ntx * args.nty);
+                    const int xx = r % args.wb, yy = (r / args.wb) % args.hb;
+                    const int bbx = r / (args.wb * args.hb);
+                    const int x = tx * args.wb + xx, y = ty * args.hb + yy, b = tb * args.bb + bbx;
+                    if (x < args.W && y < args.H && b < args.B) {
+                        int64_t* o = args.out + (((int64_t)b * args.H + y) * args.W + x) * args.ncols + col0;
+                        if (col0 + NH <= args.ncols && (args.ncols & 1) == 0) {
+#pragma unroll
+                            for (int i = 0; i < NH; i += 2) {
+                                longlong2 v;
+                                v.x = (long long)acc[i];
+                                v.y = (long long)acc[i + 1];
+                                *reinterpret_cast<longlong2*>(o + i) = v;
+                            }
+                        } else {
+#pragma unroll
+                            for (int i = 0; i < NH; ++i)
+                                if (col0 + i < args.ncols) o[i] = (int64_t)acc[i];
+                        }
+                    }
+                }
+            }
         }
+    epi_done:;
     }
     tc_fence_before();
     __syncthreads();
@@ -409,11 +552,16 @@ __device__ __forceinline__ int limb_of(int64_t x, int l, int L) {
     return (int)x;
 }
 
-// int8 NHWC -> bf16 NHWC copy
-__global__ void k_pack_act_nhwc(const int8_t* __restrict__ x, int64_t n, uint16_t* __restrict__ out) {
+// int8 NHWC [P][C] -> bf16 NHWC [P][Cp] copy, zero in channels C..Cp-1
+__global__ void k_pack_act_nhwc(const int8_t* __restrict__ x, int64_t P, int C, int Cp,
+                                uint16_t* __restrict__ out) {
+    const int64_t n = P * Cp;
     for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
-         i += (int64_t)gridDim.x * blockDim.x)
-        out[i] = bf16_bits(x[i]);
+         i += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t p = i / Cp;
+        const int c = (int)(i - p * Cp);
+        out[i] = c < C ? bf16_bits(x[p * C + c]) : (uint16_t)0;
+    }
 }
 
 // [B][HW][C] int (int8 or int32 with limbs) -> [L][C][HW][Bp] bf16, zero for b >= B.
@@ -459,12 +607,14 @@ __global__ void k_set_limbs(const uint32_t* maxabs, int* limbs) {
     *limbs = limb_count(*maxabs);
 }
 
-// W [Cout][9][Cin] -> w_planes [L][Cout][9][Cin] and wt_planes [L][9][Cin][Cout]
-__global__ void k_pack_weights(const int32_t* __restrict__ W, int Cout, int Cin,
+// W [Cout][9][Cin] -> w_planes [L][Cout][9][Ck] (Ck = Cin rounded up to 64,
+// padding left zero) and wt_planes [L][9][Cin][Cout]
+__global__ void k_pack_weights(const int32_t* __restrict__ W, int Cout, int Cin, int Ck,
                                const uint32_t* maxabs, uint16_t* __restrict__ wp,
                                uint16_t* __restrict__ wtp) {
     const int L = limb_count(*maxabs);
     const int64_t n = (int64_t)Cout * 9 * Cin;
+    const int64_t nk = (int64_t)Cout * 9 * Ck;
     for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
          i += (int64_t)gridDim.x * blockDim.x) {
         const int ci = (int)(i % Cin);
@@ -472,6 +622,7 @@ __global__ void k_pack_weights(const int32_t* __restrict__ W, int Cout, int Cin,
         const int co = (int)(i / (9LL * Cin));
         int64_t x = W[i];
         const int64_t it = ((int64_t)t * Cin + ci) * Cout + co;
+        const int64_t ik = ((int64_t)co * 9 + t) * Ck + ci;
         for (int l = 0; l < L; ++l) {
             int v;
             if (l < L - 1) {
@@ -482,7 +633,7 @@ __global__ void k_pack_weights(const int32_t* __restrict__ W, int Cout, int Cin,
                 v = (int)x;
             }
             const uint16_t bits = bf16_bits(v);
-            if (wp) wp[l * n + i] = bits;
+            if (wp) wp[l * nk + ik] = bits;
             if (wtp) wtp[l * n + it] = bits;
         }
     }
@@ -523,8 +674,19 @@ bool make_map(CUtensorMap* m, const void* base, int rank, const uint64_t* dims,
     return r == CUDA_SUCCESS;
 }
 
+int sm_count() {
+    static int n = 0;
+    if (n == 0) {
+        int dev = 0;
+        if (cudaGetDevice(&dev) != cudaSuccess ||
+            cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n < 1)
+            n = 148;
+    }
+    return n;
+}
+
 template <int MODE, int N>
-cudaError_t launch_gemm(const CUtensorMap& a, const CUtensorMap& b, const TcArgs& args, dim3 grid,
+cudaError_t launch_gemm(const CUtensorMap& a, const CUtensorMap& b, const TcArgs& args,
                         cudaStream_t s) {
     using C = TcCfg<N>;
     static bool attr_set = false;
@@ -534,25 +696,25 @@ cudaError_t launch_gemm(const CUtensorMap& a, const CUtensorMap& b, const TcArgs
         if (e != cudaSuccess) return e;
         attr_set = true;
     }
+    const int grid = args.total_tiles < sm_count() ? args.total_tiles : sm_count();
     k_tc_gemm<MODE, N><<<grid, kThreads, C::SMEM, s>>>(a, b, args);
     return cudaGetLastError();
 }
 
 template <int MODE>
 cudaError_t launch_gemm_n(int n, const CUtensorMap& a, const CUtensorMap& b, const TcArgs& args,
-                          dim3 grid, cudaStream_t s) {
-    return n == 128 ? launch_gemm<MODE, 128>(a, b, args, grid, s)
-                    : launch_gemm<MODE, 64>(a, b, args, grid, s);
+                          cudaStream_t s) {
+    return n == 128 ? launch_gemm<MODE, 128>(a, b, args, s) : launch_gemm<MODE, 64>(a, b, args, s);
 }
 
 int pick_n(int cols) { return cols % 128 == 0 ? 128 : 64; }
 
-void pixel_tiling(const LayerGeom& g, int batch, TcArgs& a, int* tiles_m) {
+void pixel_tiling(const LayerGeom& g, int batch, TcArgs& a) {
     if (g.w > 8) { a.wb = 16; a.hb = 8; a.bb = 1; }
     else { a.wb = 8; a.hb = 8; a.bb = 2; }
     a.ntx = (g.w + a.wb - 1) / a.wb;
     a.nty = (g.h + a.hb - 1) / a.hb;
-    *tiles_m = a.ntx * a.nty * ((batch + a.bb - 1) / a.bb);
+    a.tiles_m = a.ntx * a.nty * ((batch + a.bb - 1) / a.bb);
 }
 
 inline int grid1d(int64_t n) {
@@ -569,29 +731,36 @@ bool dalloc(std::vector<void*>& allocs, T** p, size_t count) {
     return true;
 }
 
+inline int round_up(int v, int m) { return (v + m - 1) / m * m; }
+
 }  // namespace
 
 bool tc_layer_init(TcLayer& t, const LayerGeom& g, int max_batch, bool has_dgrad,
                    std::vector<void*>& allocs) {
     t = TcLayer();
     if (g.kind != NITRO_CONV3X3 || max_batch < 1 || !encode_fn()) return true;
-    const bool chan_ok = g.cin % 64 == 0 && g.cout % 64 == 0;
+    // Narrow inputs (Cin < 32, e.g. image channels) stay on the CUDA-core
+    // kernels: zero-padding them to a 64-wide K-block wastes most MMA work.
     const bool pix_ok = g.h >= 8 && g.w >= 8;
-    t.fwd = chan_ok && pix_ok;
-    t.dgrad = has_dgrad && chan_ok && pix_ok;
-    t.wgrad = chan_ok;
-    if (!t.fwd && !t.wgrad && !t.dgrad) return true;
-    t.max_bp = (max_batch + 7) / 8 * 8;
+    const bool wide = g.cin >= 32;
+    t.fwd = pix_ok && wide;
+    t.wgrad = wide;
+    t.dgrad = has_dgrad && pix_ok && g.cout % 8 == 0;
+    t.max_bp = round_up(max_batch, 8);
+    t.cin8 = round_up(g.cin, 8);
+    t.cin_k = round_up(g.cin, 64);
     const size_t hw = (size_t)g.h * g.w;
     const size_t nw = (size_t)g.cout * 9 * g.cin;
+    const size_t nwk = (size_t)g.cout * 9 * t.cin_k;
     bool ok = dalloc(allocs, &t.limbs, 2);
-    if (ok && t.fwd) ok = dalloc(allocs, &t.act_nhwc, (size_t)max_batch * hw * g.cin);
+    if (ok && t.fwd) ok = dalloc(allocs, &t.act_nhwc, (size_t)max_batch * hw * t.cin8);
     if (ok && t.wgrad) ok = dalloc(allocs, &t.act_t, (size_t)g.cin * hw * t.max_bp);
     if (ok && t.wgrad) ok = dalloc(allocs, &t.d_t, (size_t)kMaxLimbs * g.cout * hw * t.max_bp);
     if (ok && t.dgrad) ok = dalloc(allocs, &t.d_nhwc, (size_t)kMaxLimbs * max_batch * hw * g.cout);
-    if (ok && t.fwd) ok = dalloc(allocs, &t.w_planes, (size_t)kMaxLimbs * nw);
+    if (ok && t.fwd) ok = dalloc(allocs, &t.w_planes, (size_t)kMaxLimbs * nwk);
     if (ok && t.dgrad) ok = dalloc(allocs, &t.wt_planes, (size_t)kMaxLimbs * nw);
     if (ok) ok = cudaMemset(t.limbs, 0, 2 * sizeof(int)) == cudaSuccess;
+    if (ok && t.fwd) ok = cudaMemset(t.w_planes, 0, (size_t)kMaxLimbs * nwk * 2) == cudaSuccess;
     return ok;
 }
 
@@ -601,7 +770,8 @@ cudaError_t tc_refresh_weights(TcLayer& t, const LayerGeom& g, const int32_t* W,
     const int64_t n = (int64_t)g.cout * 9 * g.cin;
     {
         ProfScope ps(K_TC_PACK, s, 0.0, (double)n * 4 * 2);
-        k_pack_weights<<<grid1d(n), 256, 0, s>>>(W, g.cout, g.cin, maxabs_w, t.w_planes, t.wt_planes);
+        k_pack_weights<<<grid1d(n), 256, 0, s>>>(W, g.cout, g.cin, t.cin_k, maxabs_w, t.w_planes,
+                                                 t.wt_planes);
     }
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
@@ -611,18 +781,18 @@ cudaError_t tc_refresh_weights(TcLayer& t, const LayerGeom& g, const int32_t* W,
 }
 
 cudaError_t tc_pack_input(TcLayer& t, const LayerGeom& g, const int8_t* x, int batch,
-                          cudaStream_t s) {
+                          bool nhwc_done, cudaStream_t s) {
     if (batch <= 0 || (!t.fwd && !t.wgrad)) return cudaSuccess;
     const int hw = g.h * g.w;
-    if (t.fwd) {
-        const int64_t n = (int64_t)batch * hw * g.cin;
-        ProfScope ps(K_TC_PACK, s, 0.0, (double)n * 3);
-        k_pack_act_nhwc<<<grid1d(n), 256, 0, s>>>(x, n, t.act_nhwc);
+    if (t.fwd && !nhwc_done) {
+        const int64_t P = (int64_t)batch * hw;
+        ProfScope ps(K_TC_PACK, s, 0.0, (double)P * (g.cin + 2 * t.cin8));
+        k_pack_act_nhwc<<<grid1d(P * t.cin8), 256, 0, s>>>(x, P, g.cin, t.cin8, t.act_nhwc);
         cudaError_t e = cudaGetLastError();
         if (e != cudaSuccess) return e;
     }
     if (t.wgrad) {
-        const int bp = (batch + 7) / 8 * 8;
+        const int bp = round_up(batch, 8);
         dim3 grid(hw, (g.cin + 31) / 32, (bp + 31) / 32);
         ProfScope ps(K_TC_PACK, s, 0.0, (double)batch * hw * g.cin * 3);
         k_pack_transposed<int8_t><<<grid, dim3(32, 8), 0, s>>>(x, batch, hw, g.cin, bp, nullptr,
@@ -633,36 +803,57 @@ cudaError_t tc_pack_input(TcLayer& t, const LayerGeom& g, const int8_t* x, int b
 }
 
 cudaError_t tc_conv_forward(TcLayer& t, const LayerGeom& g, int batch, int64_t* z,
-                            uint32_t* status, cudaStream_t s, bool* done) {
+                            const TcFwdOut* fo, uint32_t* status, cudaStream_t s, bool* done,
+                            bool* fused) {
     *done = false;
+    *fused = false;
     if (!t.fwd || batch <= 0) return cudaSuccess;
     TcArgs a{};
     a.B = batch; a.H = g.h; a.W = g.w; a.Cin = g.cin; a.Cout = g.cout;
-    a.Bp = (batch + 7) / 8 * 8;
-    int tiles_m = 0;
-    pixel_tiling(g, batch, a, &tiles_m);
+    a.Bp = round_up(batch, 8);
+    a.cin_k = t.cin_k;
+    pixel_tiling(g, batch, a);
     const int n = pick_n(g.cout);
-    a.kb_total = 9 * (g.cin / kBK);
+    a.tiles_n = (g.cout + n - 1) / n;
+    a.total_tiles = a.tiles_m * a.tiles_n;
+    a.kb_total = 9 * (t.cin_k / kBK);
     a.kb_per_split = a.kb_total;
+    a.ncols = g.cout;
     a.limbs_a = nullptr;
     a.limbs_b = t.limbs;
     a.out = z;
     a.status = status;
     a.atomic_out = 0;
+    if (fo && g.cout % 16 == 0) {
+        a.fuse = 1;
+        a.sf = FloorDiv::make(256ull * 9ull * (uint64_t)g.cin);
+        a.alpha = FloorDiv::make((uint64_t)fo->alpha_inv);
+        a.mu = fo->mu;
+        a.pool = g.pool;
+        a.oh = g.oh;
+        a.ow = g.ow;
+        a.act = fo->act;
+        a.out2 = fo->out2;
+        a.region = fo->region;
+        a.argmax = fo->argmax;
+        a.next_nhwc = fo->next_nhwc;
+    }
     CUtensorMap ma, mb;
-    const uint64_t da[4] = {(uint64_t)g.cin, (uint64_t)g.w, (uint64_t)g.h, (uint64_t)batch};
-    const uint64_t sa[3] = {(uint64_t)g.cin, (uint64_t)g.w * g.cin, (uint64_t)g.h * g.w * g.cin};
+    const uint64_t da[4] = {(uint64_t)t.cin8, (uint64_t)g.w, (uint64_t)g.h, (uint64_t)batch};
+    const uint64_t sa[3] = {(uint64_t)t.cin8, (uint64_t)g.w * t.cin8, (uint64_t)g.h * g.w * t.cin8};
     const uint32_t ba[4] = {64, (uint32_t)a.wb, (uint32_t)a.hb, (uint32_t)a.bb};
-    const uint64_t db[3] = {(uint64_t)9 * g.cin, (uint64_t)g.cout, (uint64_t)kMaxLimbs};
-    const uint64_t sb[2] = {(uint64_t)9 * g.cin, (uint64_t)9 * g.cin * g.cout};
+    const uint64_t db[3] = {(uint64_t)9 * t.cin_k, (uint64_t)g.cout, (uint64_t)kMaxLimbs};
+    const uint64_t sb[2] = {(uint64_t)9 * t.cin_k, (uint64_t)9 * t.cin_k * g.cout};
     const uint32_t bb[3] = {64, (uint32_t)n, 1};
     if (!make_map(&ma, t.act_nhwc, 4, da, sa, ba) || !make_map(&mb, t.w_planes, 3, db, sb, bb))
         return cudaErrorInvalidValue;
-    dim3 grid(tiles_m, g.cout / n, 1);
     const double ops = 2.0 * batch * g.h * g.w * g.cout * 9.0 * g.cin;
     ProfScope ps(K_TC_CONV_FWD, s, ops, 0.0);
-    cudaError_t e = launch_gemm_n<TC_FWD>(n, ma, mb, a, grid, s);
-    if (e == cudaSuccess) *done = true;
+    cudaError_t e = launch_gemm_n<TC_FWD>(n, ma, mb, a, s);
+    if (e == cudaSuccess) {
+        *done = true;
+        *fused = a.fuse != 0;
+    }
     return e;
 }
 
@@ -672,7 +863,7 @@ cudaError_t tc_conv_wgrad(TcLayer& t, const LayerGeom& g, const int32_t* delta,
     *done = false;
     if (batch <= 0 || (!t.wgrad && !t.dgrad)) return cudaSuccess;
     const int hw = g.h * g.w;
-    const int bp = (batch + 7) / 8 * 8;
+    const int bp = round_up(batch, 8);
     // limb planes of delta in the layouts the tensor-core passes read
     if (t.dgrad) {
         const int64_t n = (int64_t)batch * hw * g.cout;
@@ -698,18 +889,22 @@ cudaError_t tc_conv_wgrad(TcLayer& t, const LayerGeom& g, const int32_t* delta,
     if (!t.wgrad) return cudaSuccess;
     TcArgs a{};
     a.B = batch; a.H = g.h; a.W = g.w; a.Cin = g.cin; a.Cout = g.cout; a.Bp = bp;
+    a.cin_k = t.cin_k;
     a.ntx = a.nty = 1; a.wb = a.hb = a.bb = 1;
     const int n = pick_n(g.cout);
-    const int tiles_m = (9 * g.cin + kBM - 1) / kBM, tiles_n = g.cout / n;
+    a.tiles_m = (9 * t.cin_k + kBM - 1) / kBM;
+    a.tiles_n = (g.cout + n - 1) / n;
     const int nbb = (bp + kBK - 1) / kBK;
     a.kb_total = hw * nbb;
     // split K so that about one wave of CTAs runs, each with >= one exact chunk
-    const int tiles = tiles_m * tiles_n;
-    int splits = (152 + tiles - 1) / tiles;
+    const int tiles = a.tiles_m * a.tiles_n;
+    int splits = (sm_count() + tiles - 1) / tiles;
     const int max_splits = (a.kb_total + kChunkBlocks - 1) / kChunkBlocks;
     splits = splits < 1 ? 1 : (splits > max_splits ? max_splits : splits);
     a.kb_per_split = (a.kb_total + splits - 1) / splits;
     splits = (a.kb_total + a.kb_per_split - 1) / a.kb_per_split;
+    a.total_tiles = tiles * splits;
+    a.ncols = g.cout;
     a.limbs_a = nullptr;
     a.limbs_b = t.limbs + 1;
     a.out = dW;
@@ -717,20 +912,21 @@ cudaError_t tc_conv_wgrad(TcLayer& t, const LayerGeom& g, const int32_t* delta,
     a.atomic_out = splits > 1;
     CUtensorMap ma, mb;
     const uint64_t da[4] = {(uint64_t)bp, (uint64_t)g.w, (uint64_t)g.h, (uint64_t)g.cin};
-    const uint64_t sa[3] = {(uint64_t)bp, (uint64_t)g.w * bp, (uint64_t)hw * bp};
+    const uint64_t sa[4] = {(uint64_t)bp, (uint64_t)g.w * bp, (uint64_t)hw * bp,
+                            (uint64_t)g.cout * hw * bp};
     const uint32_t ba[4] = {64, 1, 1, 64};
-    const uint64_t db[4] = {(uint64_t)bp, (uint64_t)g.w, (uint64_t)g.h, (uint64_t)g.cout * kMaxLimbs};
-    const uint32_t bb[4] = {64, 1, 1, (uint32_t)n};
-    if (!make_map(&ma, t.act_t, 4, da, sa, ba) || !make_map(&mb, t.d_t, 4, db, sa, bb))
+    const uint64_t db[5] = {(uint64_t)bp, (uint64_t)g.w, (uint64_t)g.h, (uint64_t)g.cout,
+                            (uint64_t)kMaxLimbs};
+    const uint32_t bb[5] = {64, 1, 1, (uint32_t)n, 1};
+    if (!make_map(&ma, t.act_t, 4, da, sa, ba) || !make_map(&mb, t.d_t, 5, db, sa, bb))
         return cudaErrorInvalidValue;
     if (a.atomic_out) {
         cudaError_t e = cudaMemsetAsync(dW, 0, sizeof(int64_t) * 9 * g.cin * g.cout, s);
         if (e != cudaSuccess) return e;
     }
-    dim3 grid(tiles_m, tiles_n, splits);
     const double ops = 2.0 * batch * hw * g.cout * 9.0 * g.cin;
     ProfScope ps(K_TC_CONV_WGRAD, s, ops, 0.0);
-    cudaError_t e = launch_gemm_n<TC_WGRAD>(n, ma, mb, a, grid, s);
+    cudaError_t e = launch_gemm_n<TC_WGRAD>(n, ma, mb, a, s);
     if (e == cudaSuccess) *done = true;
     return e;
 }
@@ -741,12 +937,15 @@ cudaError_t tc_conv_dgrad(TcLayer& t, const LayerGeom& g, int batch, int64_t* g6
     if (!t.dgrad || batch <= 0) return cudaSuccess;
     TcArgs a{};
     a.B = batch; a.H = g.h; a.W = g.w; a.Cin = g.cin; a.Cout = g.cout;
-    a.Bp = (batch + 7) / 8 * 8;
-    int tiles_m = 0;
-    pixel_tiling(g, batch, a, &tiles_m);
+    a.Bp = round_up(batch, 8);
+    a.cin_k = t.cin_k;
+    pixel_tiling(g, batch, a);
     const int n = pick_n(g.cin);
-    a.kb_total = 9 * (g.cout / kBK);
+    a.tiles_n = (g.cin + n - 1) / n;
+    a.total_tiles = a.tiles_m * a.tiles_n;
+    a.kb_total = 9 * ((g.cout + kBK - 1) / kBK);
     a.kb_per_split = a.kb_total;
+    a.ncols = g.cin;
     a.limbs_a = t.limbs + 1;
     a.limbs_b = t.limbs;
     a.out = g64;
@@ -765,10 +964,9 @@ cudaError_t tc_conv_dgrad(TcLayer& t, const LayerGeom& g, int batch, int64_t* g6
     const uint32_t bb[4] = {64, (uint32_t)n, 1, 1};
     if (!make_map(&ma, t.d_nhwc, 5, da, sa, ba) || !make_map(&mb, t.wt_planes, 4, db, sb, bb))
         return cudaErrorInvalidValue;
-    dim3 grid(tiles_m, g.cin / n, 1);
     const double ops = 2.0 * batch * g.h * g.w * g.cin * 9.0 * g.cout;
     ProfScope ps(K_TC_CONV_DGRAD, s, ops, 0.0);
-    cudaError_t e = launch_gemm_n<TC_DGRAD>(n, ma, mb, a, grid, s);
+    cudaError_t e = launch_gemm_n<TC_DGRAD>(n, ma, mb, a, s);
     if (e == cudaSuccess) *done = true;
     return e;
 }

@@ -9,13 +9,16 @@
 // are combined in int64 (modulo 2^64) with shifts 8 (la + lb).
 //
 // Layouts (bf16, limb planes outermost):
-//   act_nhwc  [B][H][W][Cin]           forward A  (pixels x taps*channels)
+//   act_nhwc  [B][H][W][Cin8]          forward A  (pixels x taps*channels)
 //   act_t     [Cin][H][W][Bp]          wgrad A    ((tap, ci) x (y, x, b))
 //   d_nhwc    [L][B][H][W][Cout]       dgrad A
 //   d_t       [L][Cout][H][W][Bp]      wgrad B
-//   w_planes  [L][Cout][9][Cin]        forward B
+//   w_planes  [L][Cout][9][Cin64]      forward B
 //   wt_planes [L][9][Cin][Cout]        dgrad B
-// Bp = batch rounded up to 8 (TMA strides are multiples of 16 bytes).
+// Bp = batch rounded up to 8 and Cin8 = Cin rounded up to 8 (TMA strides are
+// multiples of 16 bytes); Cin64 = Cin rounded up to 64 so that a K-block of
+// the forward never spans two taps.  Padding holds zeros; tiles that run past
+// a tensor edge read zeros (TMA out-of-bounds fill) and skip their stores.
 #pragma once
 
 #include <vector>
@@ -28,7 +31,9 @@ constexpr int kMaxLimbs = 4;
 
 struct TcLayer {
     bool fwd = false, wgrad = false, dgrad = false;   // passes that run on tcgen05
-    int max_bp = 0;
+    int max_bp = 0;   // batch rounded up to 8
+    int cin8 = 0;     // channels of the NHWC bf16 input copy (Cin rounded up to 8)
+    int cin_k = 0;    // channels per tap in the forward K index (Cin rounded up to 64)
     uint16_t* act_nhwc = nullptr;
     uint16_t* act_t = nullptr;
     uint16_t* d_nhwc = nullptr;
@@ -49,13 +54,28 @@ bool tc_layer_init(TcLayer& t, const LayerGeom& g, int max_batch, bool has_dgrad
 cudaError_t tc_refresh_weights(TcLayer& t, const LayerGeom& g, const int32_t* W,
                                const uint32_t* maxabs_w, cudaStream_t s);
 
-// bf16 copies of the layer's int8 input for the forward and wgrad operands.
+// bf16 copies of the layer's int8 input for the forward and wgrad operands
+// (the forward copy is skipped when the previous layer's epilogue wrote it).
 cudaError_t tc_pack_input(TcLayer& t, const LayerGeom& g, const int8_t* x, int batch,
-                          cudaStream_t s);
+                          bool nhwc_done, cudaStream_t s);
 
-// z[p][co] (int64) = forward contraction; *done = false if not on tcgen05.
+// Outputs of a forward layer for the fused epilogue.
+struct TcFwdOut {
+    int alpha_inv, mu;
+    int8_t* act;          // [B][oh][ow][Cout] int8
+    int8_t* out2;         // optional copy (may be null)
+    int8_t* region;       // [B][h][w][Cout] int8
+    int8_t* argmax;       // [B][oh][ow][Cout] int8 if pooled
+    uint16_t* next_nhwc;  // next layer's bf16 input copy, or null
+};
+
+// Forward contraction on tcgen05; *done = false if the layer does not run
+// there.  With fo != null and Cout % 16 == 0 the epilogue applies
+// NITRO-Scaling, NITRO-ReLU and the max-pool and writes fo's outputs
+// (*fused = true); otherwise z[p][co] (int64) is written.
 cudaError_t tc_conv_forward(TcLayer& t, const LayerGeom& g, int batch, int64_t* z,
-                            uint32_t* status, cudaStream_t s, bool* done);
+                            const TcFwdOut* fo, uint32_t* status, cudaStream_t s, bool* done,
+                            bool* fused);
 
 // Splits delta into limb planes (both layouts as needed) and, if wgrad runs on
 // tcgen05, dW = sum_p delta (x) im2col(a).  Must precede tc_conv_dgrad.
