@@ -191,57 +191,38 @@ __global__ void k_fwd_epilogue(const int64_t* __restrict__ z, LayerGeom g, int B
 // (exact, order independent).  k_learn_finish: one CTA turns zsum into
 // y_hat = floor(z / (256 d)), grad_L = y_hat - 32 onehot, SSE and the loss.
 // ---------------------------------------------------------------------------
-constexpr int kGChunk = 16;
-constexpr int kLrSamples = 4;
-constexpr int kLrSlice = 1024;
+constexpr int kLrSamples = 16;   // samples per CTA
 
+// CTA (feature slice, group of kLrSamples samples): the slice of a and of
+// every row of W_lr is staged in shared memory with coalesced loads (rows
+// padded so that concurrent rows fall in distinct banks), then each thread
+// forms whole dot products for (sample, class) pairs and adds them into zsum.
 __global__ void __launch_bounds__(256) k_learn_partial(const int8_t* __restrict__ a,
                                                        const int32_t* __restrict__ wlr, int B,
-                                                       int d, int G,
+                                                       int d, int G, int slice,
                                                        unsigned long long* __restrict__ zsum) {
-    __shared__ int64_t red[8][kLrSamples * kGChunk];
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int j0 = blockIdx.x * kLrSlice, j1 = min(d, j0 + kLrSlice);
-    const int b0 = blockIdx.y * kLrSamples;
-    for (int g0 = 0; g0 < G; g0 += kGChunk) {
-        int64_t acc[kLrSamples][kGChunk];
-#pragma unroll
-        for (int u = 0; u < kLrSamples; ++u)
-#pragma unroll
-            for (int q = 0; q < kGChunk; ++q) acc[u][q] = 0;
-        for (int j = j0 + threadIdx.x; j < j1; j += 256) {
-            int32_t av[kLrSamples];
-#pragma unroll
-            for (int u = 0; u < kLrSamples; ++u)
-                av[u] = (b0 + u < B) ? (int32_t)a[(int64_t)(b0 + u) * d + j] : 0;
-#pragma unroll
-            for (int q = 0; q < kGChunk; ++q) {
-                if (g0 + q < G) {
-                    const int64_t w = wlr[(int64_t)(g0 + q) * d + j];
-#pragma unroll
-                    for (int u = 0; u < kLrSamples; ++u) acc[u][q] += w * av[u];
-                }
-            }
-        }
-#pragma unroll
-        for (int u = 0; u < kLrSamples; ++u)
-#pragma unroll
-            for (int q = 0; q < kGChunk; ++q) {
-                int64_t v = acc[u][q];
-#pragma unroll
-                for (int off = 16; off; off >>= 1) v += __shfl_xor_sync(kFull, v, off);
-                if (lane == 0) red[warp][u * kGChunk + q] = v;
-            }
-        __syncthreads();
-        if (threadIdx.x < kLrSamples * kGChunk) {
-            const int u = threadIdx.x / kGChunk, q = threadIdx.x % kGChunk;
-            if (b0 + u < B && g0 + q < G) {
-                int64_t v = 0;
-                for (int w = 0; w < 8; ++w) v += red[w][threadIdx.x];
-                atomicAdd(&zsum[(int64_t)(b0 + u) * G + g0 + q], (unsigned long long)v);
-            }
-        }
-        __syncthreads();
+    extern __shared__ int32_t lr_smem[];
+    const int wstride = slice + 1;                    // int32 row stride of the W tile
+    const int astride = slice + 4;                    // byte row stride of the a tile
+    int32_t* ws = lr_smem;
+    int8_t* as = reinterpret_cast<int8_t*>(ws + (size_t)G * wstride);
+    const int j0 = blockIdx.x * slice, n = min(slice, d - j0);
+    const int b0 = blockIdx.y * kLrSamples, nb = min(kLrSamples, B - b0);
+    for (int g = 0; g < G; ++g)
+        for (int j = threadIdx.x; j < n; j += blockDim.x)
+            ws[g * wstride + j] = wlr[(int64_t)g * d + j0 + j];
+    for (int u = 0; u < nb; ++u)
+        for (int j = threadIdx.x; j < n; j += blockDim.x)
+            as[u * astride + j] = a[(int64_t)(b0 + u) * d + j0 + j];
+    __syncthreads();
+    for (int p = threadIdx.x; p < nb * G; p += blockDim.x) {
+        const int u = p / G, g = p - u * G;
+        const int32_t* wr = ws + g * wstride;
+        const int8_t* ar = as + u * astride;
+        int64_t acc = 0;
+#pragma unroll 8
+        for (int j = 0; j < n; ++j) acc += (int64_t)wr[j] * ar[j];
+        atomicAdd(&zsum[(int64_t)(b0 + u) * G + g], (unsigned long long)acc);
     }
 }
 
@@ -460,10 +441,15 @@ cudaError_t simt_learn_fwd(const int8_t* a, const int32_t* wlr, const int32_t* l
     cudaError_t e = cudaMemsetAsync(zsum, 0, sizeof(int64_t) * (size_t)B * G, s);
     if (e != cudaSuccess) return e;
     {
-        dim3 grid((d + kLrSlice - 1) / kLrSlice, (B + kLrSamples - 1) / kLrSamples);
+        // slice sized so the staged tiles fit 48 KB of shared memory
+        int slice = (48 * 1024 - 64) / (4 * G + kLrSamples + 8);
+        slice = slice > 1024 ? 1024 : (slice / 32) * 32;
+        if (slice < 32) slice = 32;
+        const size_t smem = (size_t)G * (slice + 1) * 4 + (size_t)kLrSamples * (slice + 4);
+        dim3 grid((d + slice - 1) / slice, (B + kLrSamples - 1) / kLrSamples);
         ProfScope ps(K_LEARN_FWD, s, 2.0 * B * d * G, 0.0);
-        k_learn_partial<<<grid, 256, 0, s>>>(a, wlr, B, d, G,
-                                             reinterpret_cast<unsigned long long*>(zsum));
+        k_learn_partial<<<grid, 256, smem, s>>>(a, wlr, B, d, G, slice,
+                                                reinterpret_cast<unsigned long long*>(zsum));
         e = cudaGetLastError();
         if (e != cudaSuccess) return e;
     }

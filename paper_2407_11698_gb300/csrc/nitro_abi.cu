@@ -125,7 +125,7 @@ nitro_status validate(const nitro_block_desc* d) {
     if (d->gamma_inv_lr < 1 || d->gamma_inv_lr > ((int64_t)1 << 48)) return NITRO_ERR_ARG;
     if (d->eta_inv_fw < 0 || d->eta_inv_lr < 0) return NITRO_ERR_ARG;
     if (d->sgd_round != NITRO_ROUND_FLOOR && d->sgd_round != NITRO_ROUND_TRUNC) return NITRO_ERR_ARG;
-    if (d->max_batch < 0 || d->max_batch > (1 << 20)) return NITRO_ERR_ARG;
+    if (d->max_batch < 0 || d->max_batch > 1000000) return NITRO_ERR_ARG;
     if (d->in_features < 1 || d->in_features > (1 << 24)) return NITRO_ERR_ARG;
     int64_t prev_out = d->in_features;
     for (int i = 0; i < d->n_layers; ++i) {

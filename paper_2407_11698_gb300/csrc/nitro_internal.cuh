@@ -64,6 +64,33 @@ struct FloorDiv {
     }
 };
 
+// The same method with N = 32 for 32-bit operands (one 32-bit multiply-high).
+struct FloorDiv32 {
+    uint32_t m;
+    int sh1, sh2;
+    __host__ static FloorDiv32 make(uint32_t d) {
+        int l = 0;
+        while (l < 32 && ((uint64_t)1 << l) < d) ++l;
+        FloorDiv32 f;
+        f.m = (uint32_t)((((uint64_t)1 << 32) * (((uint64_t)1 << l) - d)) / d + 1);
+        f.sh1 = l < 1 ? l : 1;
+        f.sh2 = l > 1 ? l - 1 : 0;
+        return f;
+    }
+    __host__ __device__ __forceinline__ uint32_t udiv(uint32_t n) const {
+#ifdef __CUDA_ARCH__
+        const uint32_t t = __umulhi(m, n);
+#else
+        const uint32_t t = (uint32_t)(((uint64_t)m * n) >> 32);
+#endif
+        return (t + ((n - t) >> sh1)) >> sh2;
+    }
+    __host__ __device__ __forceinline__ int32_t floor_div(int32_t x) const {
+        if (x >= 0) return (int32_t)udiv((uint32_t)x);
+        return -(int32_t)udiv((uint32_t)(-(x + 1))) - 1;
+    }
+};
+
 __host__ __device__ __forceinline__ bool fits_i32(int64_t v) {
     return v >= INT32_MIN && v <= INT32_MAX;
 }

@@ -2,11 +2,11 @@
 // and input gradient, plus the kernels that split operands into bf16 limb
 // planes.  See tc_conv.cuh for the exactness argument and the layouts.
 //
-// One CTA computes one 128 x N output tile over a range of K-blocks (64
-// elements each).  Warp 0 issues TMA loads into an S-stage shared-memory ring,
-// warp 1 allocates TMEM and issues the MMAs, warps 2..9 drain the fp32 TMEM
-// accumulator every <= 16 K-blocks into int64 registers (two warps per TMEM
-// lane quadrant, each owning half of the N columns).  Two TMEM accumulators
+// A persistent CTA computes 128 x N output tiles, each over a range of
+// K-blocks (64 elements each).  Warp 0 issues TMA loads into an S-stage shared-memory ring,
+// warp 1 allocates TMEM and issues the MMAs, warps 2..17 drain the fp32 TMEM
+// accumulator every <= 16 K-blocks into int64 registers (four warps per TMEM
+// lane quadrant, each owning a quarter of the N columns).  Two TMEM accumulators
 // alternate so the MMAs of the next chunk overlap the drain of the last.
 // Every wait on an mbarrier is bounded in time; on expiry the kernel raises
 // the TIMEOUT status bit, lets the other roles leave, frees TMEM and returns.
@@ -27,7 +27,8 @@ enum TcMode : int { TC_FWD = 0, TC_WGRAD = 1, TC_DGRAD = 2 };
 constexpr int kBM = 128;              // rows per tile (TMEM lanes)
 constexpr int kBK = 64;               // K elements per block (one 128-byte row)
 constexpr int kChunkBlocks = 16;      // 16 x 64 = 1024 products per exact chunk
-constexpr int kThreads = 320;         // 10 warps
+constexpr int kEpiWarps = 16;         // 4 per TMEM lane quadrant
+constexpr int kThreads = 64 + 32 * kEpiWarps;   // TMA warp, MMA warp, epilogue
 constexpr uint64_t kWaitNs = 2000000000ull;   // 2 s bound on any wait
 
 // ------------------------------------------------------------------ PTX
@@ -144,6 +145,15 @@ __device__ __forceinline__ void umma_commit(uint32_t bar) {
         : "memory");
 }
 
+__device__ __forceinline__ void tmem_ld16_nowait(uint32_t taddr, uint32_t* r) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, "
+        "%11, %12, %13, %14, %15}, [%16];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+          "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr));
+}
 __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
     asm volatile(
         "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, "
@@ -171,7 +181,9 @@ struct TcArgs {
     int atomic_out;
     // forward with fused NITRO-Scaling / NITRO-ReLU / max-pool epilogue
     int fuse;
-    FloorDiv sf, alpha;    // divide by SF = 2^8 * 9 * Cin, and by alpha_inv
+    FloorDiv alpha;        // divide by alpha_inv
+    FloorDiv32 sf32;       // divide by 9 * Cin (after the shift by 8)
+    int64_t z_hi, z_lo;    // z >= 128 SF: piece 3; z < -127 SF: piece 0
     int mu, pool, oh, ow;
     int8_t* act;           // layer output (post-pool) int8 NHWC
     int8_t* out2;          // optional second copy of the output (caller's buffer)
@@ -204,7 +216,7 @@ struct TcCfg {
     static constexpr int B_BYTES = N * kBK * 2;
     static constexpr int STAGE = A_BYTES + B_BYTES;
     static constexpr int S = N >= 128 ? 6 : 8;
-    static constexpr int SMEM = 1024 + S * STAGE + 256;
+    static constexpr int SMEM = 1024 + S * STAGE + 512;
 };
 
 struct Tile {
@@ -230,7 +242,7 @@ __global__ void __launch_bounds__(kThreads, 1)
               const TcArgs args) {
     using C = TcCfg<N>;
     constexpr int S = C::S;
-    constexpr int NH = N / 2;            // columns per epilogue warp
+    constexpr int NH = N / 4;            // columns per epilogue warp
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
@@ -238,6 +250,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     // bars[0..S) full, [S..2S) empty, [2S..2S+2) tmem full, [2S+2..2S+4) tmem empty
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * S + 4);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+    int8_t* relu_tab = reinterpret_cast<int8_t*>(smem + S * C::STAGE + 256);   // 255 entries
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const uint32_t bar0 = smem_u32(bars);
@@ -253,11 +266,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(tfull_bar(b), 1);
-            mbar_init(tempty_bar(b), 8);
+            mbar_init(tempty_bar(b), kEpiWarps);
         }
         *abort_flag = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
+    // NITRO-ReLU value of every z* in [-127, 127] (fused forward epilogue)
+    if (MODE == TC_FWD && args.fuse && threadIdx.x >= 64 && threadIdx.x < 64 + 255)
+        relu_tab[threadIdx.x - 64] = (int8_t)relu_value((int64_t)threadIdx.x - 64 - 127, args.alpha, args.mu);
     if (warp == 1) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
                          smem_u32(tmem_slot)),
@@ -365,9 +381,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         mma_done:;
         }
     } else {
-        // ---------------- epilogue: warps 2..9
+        // ---------------- epilogue: warps 2..17
         const int q = warp & 3;             // TMEM lane quadrant this warp may read
-        const int half = (warp - 2) >> 2;   // which half of the N columns
+        const int half = (warp - 2) >> 2;   // which quarter of the N columns
         int chunk = 0;
         for (int tile = blockIdx.x; tile < args.total_tiles; tile += gridDim.x) {
             const Tile T = decode_tile(args, tile);
@@ -384,15 +400,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                     tc_fence_after();
                     const uint32_t base =
                         tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(buf * N + half * NH);
+                    uint32_t r[NH];
 #pragma unroll
-                    for (int j = 0; j < NH / 16; ++j) {
-                        uint32_t r[16];
-                        tmem_ld16(base + 16 * j, r);
+                    for (int j = 0; j < NH / 16; ++j) tmem_ld16_nowait(base + 16 * j, r + 16 * j);
+                    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 #pragma unroll
-                        for (int i = 0; i < 16; ++i) {
-                            const int v = __float2int_rz(__uint_as_float(r[i]));   // exact integer
-                            acc[16 * j + i] += (uint64_t)(int64_t)v << shift;
-                        }
+                    for (int i = 0; i < NH; ++i) {
+                        const int v = __float2int_rz(__uint_as_float(r[i]));   // exact integer
+                        acc[i] += (uint64_t)(int64_t)v << shift;
                     }
                     tc_fence_before();
                     __syncwarp();
@@ -435,9 +450,24 @@ __global__ void __launch_bounds__(kThreads, 1)
                         uint32_t vp = 0, rp = 0;
 #pragma unroll
                         for (int u = 0; u < 4; ++u) {
-                            const int64_t zs = args.sf.floor_div((int64_t)acc[4 * g4 + u]);
-                            rp |= (uint32_t)relu_region(zs) << (8 * u);
-                            vp |= (uint32_t)(uint8_t)(int8_t)relu_value(zs, args.alpha, args.mu) << (8 * u);
+                            // z* = floor(z / SF): outside [-127, 127] only the
+                            // saturated piece matters; inside, floor((z >> 8) / 9Cin)
+                            // fits 32 bits.
+                            const int64_t z = (int64_t)acc[4 * g4 + u];
+                            int reg, val;
+                            if (z >= args.z_hi) {
+                                reg = 3;
+                                val = relu_tab[254];
+                            } else if (z < args.z_lo) {
+                                reg = 0;
+                                val = relu_tab[0];
+                            } else {
+                                const int zq = args.sf32.floor_div((int32_t)(z >> 8));
+                                reg = zq < 0 ? 1 : 2;
+                                val = relu_tab[zq + 127];
+                            }
+                            rp |= (uint32_t)reg << (8 * u);
+                            vp |= (uint32_t)(uint8_t)(int8_t)val << (8 * u);
                         }
                         vpk[g4] = vp;
                         rpk[g4] = rp;
@@ -542,15 +572,6 @@ __device__ __forceinline__ int limb_count(uint32_t m) {
 __device__ __forceinline__ uint16_t bf16_bits(int v) {
     return __bfloat16_as_ushort(__float2bfloat16_rn((float)v));   // exact for |v| <= 256
 }
-// limb l of x given L limbs (signed digits below the top, remainder on top)
-__device__ __forceinline__ int limb_of(int64_t x, int l, int L) {
-    for (int i = 0; i < L - 1; ++i) {
-        const int64_t d = ((x + 128) & 255) - 128;
-        if (i == l) return (int)d;
-        x = (x - d) >> 8;
-    }
-    return (int)x;
-}
 
 // int8 NHWC [P][C] -> bf16 NHWC [P][Cp] copy, zero in channels C..Cp-1
 __global__ void k_pack_act_nhwc(const int8_t* __restrict__ x, int64_t P, int C, int Cp,
@@ -564,55 +585,92 @@ __global__ void k_pack_act_nhwc(const int8_t* __restrict__ x, int64_t P, int C, 
     }
 }
 
-// [B][HW][C] int (int8 or int32 with limbs) -> [L][C][HW][Bp] bf16, zero for b >= B.
+// [B][HW][C] int (int8, or int32 split into limbs) -> [L][C][HW][Bp] bf16,
+// zero for b >= B.  Tile: one pixel, 32 channels x 64 batch entries; each
+// thread writes two consecutive batch entries per plane (128-byte warp rows).
+// Block (0,0,0) thread 0 records the limb count in *limbs_out if given.
 template <typename T>
-__global__ void k_pack_transposed(const T* __restrict__ x, int B, int HW, int C, int Bp,
-                                  const uint32_t* maxabs, uint16_t* __restrict__ out) {
-    __shared__ int tile[32][33];
-    const int pos = blockIdx.x;                 // pixel (y, x)
-    const int c0 = blockIdx.y * 32, b0 = blockIdx.z * 32;
+__global__ void __launch_bounds__(256) k_pack_transposed(const T* __restrict__ x, int B, int HW,
+                                                         int C, int Bp, const uint32_t* maxabs,
+                                                         uint16_t* __restrict__ out,
+                                                         int* limbs_out) {
+    __shared__ int tile[32][65];
+    const int pos = blockIdx.x;
+    const int c0 = blockIdx.y * 32, b0 = blockIdx.z * 64;
     const int L = maxabs ? limb_count(*maxabs) : 1;
-    for (int k = threadIdx.y; k < 32; k += blockDim.y) {     // read: b = b0 + k, c = c0 + tx
+    if (limbs_out && blockIdx.x == 0 && blockIdx.y == 0 && blockIdx.z == 0 && threadIdx.x == 0 &&
+        threadIdx.y == 0)
+        *limbs_out = L;
+    for (int k = threadIdx.y; k < 64; k += 8) {      // read: b = b0 + k, c = c0 + tx
         const int b = b0 + k, c = c0 + threadIdx.x;
-        tile[k][threadIdx.x] = (b < B && c < C) ? (int)x[((int64_t)b * HW + pos) * C + c] : 0;
+        tile[threadIdx.x][k] = (b < B && c < C) ? (int)x[((int64_t)b * HW + pos) * C + c] : 0;
     }
     __syncthreads();
     const int64_t plane = (int64_t)C * HW * Bp;
-    for (int k = threadIdx.y; k < 32; k += blockDim.y) {     // write: c = c0 + k, b = b0 + tx
-        const int c = c0 + k, b = b0 + threadIdx.x;
+    for (int k = threadIdx.y; k < 32; k += 8) {      // write: c = c0 + k, b = b0 + 2 tx (+1)
+        const int c = c0 + k, b = b0 + 2 * threadIdx.x;
         if (c >= C || b >= Bp) continue;
-        const int64_t v = tile[threadIdx.x][k];
-        const int64_t o = ((int64_t)c * HW + pos) * Bp + b;
-        for (int l = 0; l < L; ++l) out[l * plane + o] = bf16_bits(limb_of(v, l, L));
-    }
-}
-
-// int32 delta NHWC -> limb planes [L][B][H][W][C]; also records the limb count.
-__global__ void k_pack_delta_nhwc(const int32_t* __restrict__ d, int64_t n,
-                                  const uint32_t* maxabs, uint16_t* __restrict__ out) {
-    const int L = limb_count(*maxabs);
-    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
-         i += (int64_t)gridDim.x * blockDim.x) {
-        int64_t x = d[i];
-        for (int l = 0; l < L - 1; ++l) {
-            const int64_t dg = ((x + 128) & 255) - 128;
-            out[l * n + i] = bf16_bits((int)dg);
-            x = (x - dg) >> 8;
+        int64_t v0 = tile[k][2 * threadIdx.x], v1 = tile[k][2 * threadIdx.x + 1];
+        uint32_t* o = reinterpret_cast<uint32_t*>(out + ((int64_t)c * HW + pos) * Bp + b);
+        for (int l = 0; l < L; ++l) {
+            int d0, d1;
+            if (l < L - 1) {
+                d0 = (int)(((v0 + 128) & 255) - 128);
+                d1 = (int)(((v1 + 128) & 255) - 128);
+                v0 = (v0 - d0) >> 8;
+                v1 = (v1 - d1) >> 8;
+            } else {
+                d0 = (int)v0;
+                d1 = (int)v1;
+            }
+            o[l * (plane / 2)] = (uint32_t)bf16_bits(d0) | ((uint32_t)bf16_bits(d1) << 16);
         }
-        out[(int64_t)(L - 1) * n + i] = bf16_bits((int)x);
     }
 }
 
-__global__ void k_set_limbs(const uint32_t* maxabs, int* limbs) {
-    *limbs = limb_count(*maxabs);
+// int32 delta NHWC (n values, n % 8 == 0) -> limb planes [L][n], eight values
+// per thread and one 16-byte store per plane; records the limb count.
+__global__ void __launch_bounds__(256) k_pack_delta_nhwc(const int32_t* __restrict__ d, int64_t n,
+                                                         const uint32_t* maxabs,
+                                                         uint16_t* __restrict__ out,
+                                                         int* limbs_out) {
+    const int L = limb_count(*maxabs);
+    if (limbs_out && blockIdx.x == 0 && threadIdx.x == 0) *limbs_out = L;
+    const int64_t n8 = n / 8;
+    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n8;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        const int4 a0 = reinterpret_cast<const int4*>(d)[2 * i];
+        const int4 a1 = reinterpret_cast<const int4*>(d)[2 * i + 1];
+        int64_t v[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
+        for (int l = 0; l < L; ++l) {
+            uint32_t w[4];
+#pragma unroll
+            for (int k = 0; k < 8; k += 2) {
+                int dg[2];
+#pragma unroll
+                for (int u = 0; u < 2; ++u) {
+                    if (l < L - 1) {
+                        dg[u] = (int)(((v[k + u] + 128) & 255) - 128);
+                        v[k + u] = (v[k + u] - dg[u]) >> 8;
+                    } else {
+                        dg[u] = (int)v[k + u];
+                    }
+                }
+                w[k / 2] = (uint32_t)bf16_bits(dg[0]) | ((uint32_t)bf16_bits(dg[1]) << 16);
+            }
+            reinterpret_cast<uint4*>(out + (int64_t)l * n)[i] = make_uint4(w[0], w[1], w[2], w[3]);
+        }
+    }
 }
+
 
 // W [Cout][9][Cin] -> w_planes [L][Cout][9][Ck] (Ck = Cin rounded up to 64,
 // padding left zero) and wt_planes [L][9][Cin][Cout]
 __global__ void k_pack_weights(const int32_t* __restrict__ W, int Cout, int Cin, int Ck,
                                const uint32_t* maxabs, uint16_t* __restrict__ wp,
-                               uint16_t* __restrict__ wtp) {
+                               uint16_t* __restrict__ wtp, int* limbs_out) {
     const int L = limb_count(*maxabs);
+    if (blockIdx.x == 0 && threadIdx.x == 0) *limbs_out = L;
     const int64_t n = (int64_t)Cout * 9 * Cin;
     const int64_t nk = (int64_t)Cout * 9 * Ck;
     for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
@@ -771,12 +829,8 @@ cudaError_t tc_refresh_weights(TcLayer& t, const LayerGeom& g, const int32_t* W,
     {
         ProfScope ps(K_TC_PACK, s, 0.0, (double)n * 4 * 2);
         k_pack_weights<<<grid1d(n), 256, 0, s>>>(W, g.cout, g.cin, t.cin_k, maxabs_w, t.w_planes,
-                                                 t.wt_planes);
+                                                 t.wt_planes, t.limbs);
     }
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
-    ProfScope ps(K_TC_PACK, s, 0.0, 0.0);
-    k_set_limbs<<<1, 1, 0, s>>>(maxabs_w, t.limbs);
     return cudaGetLastError();
 }
 
@@ -793,10 +847,10 @@ cudaError_t tc_pack_input(TcLayer& t, const LayerGeom& g, const int8_t* x, int b
     }
     if (t.wgrad) {
         const int bp = round_up(batch, 8);
-        dim3 grid(hw, (g.cin + 31) / 32, (bp + 31) / 32);
+        dim3 grid(hw, (g.cin + 31) / 32, (bp + 63) / 64);
         ProfScope ps(K_TC_PACK, s, 0.0, (double)batch * hw * g.cin * 3);
         k_pack_transposed<int8_t><<<grid, dim3(32, 8), 0, s>>>(x, batch, hw, g.cin, bp, nullptr,
-                                                               t.act_t);
+                                                               t.act_t, nullptr);
         return cudaGetLastError();
     }
     return cudaSuccess;
@@ -826,7 +880,10 @@ cudaError_t tc_conv_forward(TcLayer& t, const LayerGeom& g, int batch, int64_t* 
     a.atomic_out = 0;
     if (fo && g.cout % 16 == 0) {
         a.fuse = 1;
-        a.sf = FloorDiv::make(256ull * 9ull * (uint64_t)g.cin);
+        const int64_t sf = 256LL * 9LL * g.cin;
+        a.sf32 = FloorDiv32::make(9u * (uint32_t)g.cin);
+        a.z_hi = 128 * sf;
+        a.z_lo = -127 * sf;
         a.alpha = FloorDiv::make((uint64_t)fo->alpha_inv);
         a.mu = fo->mu;
         a.pool = g.pool;
@@ -864,25 +921,23 @@ cudaError_t tc_conv_wgrad(TcLayer& t, const LayerGeom& g, const int32_t* delta,
     if (batch <= 0 || (!t.wgrad && !t.dgrad)) return cudaSuccess;
     const int hw = g.h * g.w;
     const int bp = round_up(batch, 8);
-    // limb planes of delta in the layouts the tensor-core passes read
+    // limb planes of delta in the layouts the tensor-core passes read; the
+    // first pack launch also records the limb count for the GEMMs
+    bool counted = false;
     if (t.dgrad) {
-        const int64_t n = (int64_t)batch * hw * g.cout;
+        const int64_t n = (int64_t)batch * hw * g.cout;   // cout % 8 == 0 for dgrad
         ProfScope ps(K_TC_PACK, s, 0.0, (double)n * 4 * 2);
-        k_pack_delta_nhwc<<<grid1d(n), 256, 0, s>>>(delta, n, maxabs_delta, t.d_nhwc);
+        k_pack_delta_nhwc<<<grid1d(n / 8), 256, 0, s>>>(delta, n, maxabs_delta, t.d_nhwc,
+                                                         t.limbs + 1);
         cudaError_t e = cudaGetLastError();
         if (e != cudaSuccess) return e;
+        counted = true;
     }
     if (t.wgrad) {
-        dim3 grid(hw, (g.cout + 31) / 32, (bp + 31) / 32);
+        dim3 grid(hw, (g.cout + 31) / 32, (bp + 63) / 64);
         ProfScope ps(K_TC_PACK, s, 0.0, (double)batch * hw * g.cout * 4 * 2);
-        k_pack_transposed<int32_t><<<grid, dim3(32, 8), 0, s>>>(delta, batch, hw, g.cout, bp,
-                                                                maxabs_delta, t.d_t);
-        cudaError_t e = cudaGetLastError();
-        if (e != cudaSuccess) return e;
-    }
-    {
-        ProfScope ps(K_TC_PACK, s, 0.0, 0.0);
-        k_set_limbs<<<1, 1, 0, s>>>(maxabs_delta, t.limbs + 1);
+        k_pack_transposed<int32_t><<<grid, dim3(32, 8), 0, s>>>(
+            delta, batch, hw, g.cout, bp, maxabs_delta, t.d_t, counted ? nullptr : t.limbs + 1);
         cudaError_t e = cudaGetLastError();
         if (e != cudaSuccess) return e;
     }
