@@ -208,12 +208,46 @@ __global__ void __launch_bounds__(256) k_learn_partial(const int8_t* __restrict_
     int8_t* as = reinterpret_cast<int8_t*>(ws + (size_t)G * wstride);
     const int j0 = blockIdx.x * slice, n = min(slice, d - j0);
     const int b0 = blockIdx.y * kLrSamples, nb = min(kLrSamples, B - b0);
-    for (int g = 0; g < G; ++g)
-        for (int j = threadIdx.x; j < n; j += blockDim.x)
-            ws[g * wstride + j] = wlr[(int64_t)g * d + j0 + j];
-    for (int u = 0; u < nb; ++u)
-        for (int j = threadIdx.x; j < n; j += blockDim.x)
-            as[u * astride + j] = a[(int64_t)(b0 + u) * d + j0 + j];
+    // eight independent loads in flight per thread before the stores
+    const int wtot = G * n, atot = nb * n;
+    for (int base = 0; base < wtot; base += 8 * 256) {
+        int32_t v[8];
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+            const int i = base + k * 256 + (int)threadIdx.x;
+            if (i < wtot) {
+                const int g = i / n, j = i - g * n;
+                v[k] = wlr[(int64_t)g * d + j0 + j];
+            }
+        }
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+            const int i = base + k * 256 + (int)threadIdx.x;
+            if (i < wtot) {
+                const int g = i / n, j = i - g * n;
+                ws[g * wstride + j] = v[k];
+            }
+        }
+    }
+    for (int base = 0; base < atot; base += 8 * 256) {
+        int8_t v[8];
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+            const int i = base + k * 256 + (int)threadIdx.x;
+            if (i < atot) {
+                const int u = i / n, j = i - u * n;
+                v[k] = a[(int64_t)(b0 + u) * d + j0 + j];
+            }
+        }
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+            const int i = base + k * 256 + (int)threadIdx.x;
+            if (i < atot) {
+                const int u = i / n, j = i - u * n;
+                as[u * astride + j] = v[k];
+            }
+        }
+    }
     __syncthreads();
     for (int p = threadIdx.x; p < nb * G; p += blockDim.x) {
         const int u = p / G, g = p - u * G;
@@ -280,6 +314,7 @@ __global__ void k_learn_dw(const int8_t* __restrict__ a, const int32_t* __restri
     const int g = blockIdx.y;
     if (j >= d) return;
     int64_t s = 0;
+#pragma unroll 8
     for (int b = 0; b < B; ++b) s += (int64_t)grad_l[(int64_t)b * G + g] * a[(int64_t)b * d + j];
     dwlr[(int64_t)g * d + j] = s;
 }
@@ -304,6 +339,7 @@ __global__ void k_grad_to_delta(DeltaSrc src, LayerGeom g, int B, int alpha_inv,
         int64_t gv;
         if (src.wlr) {
             uint64_t acc = 0;  // modulo 2^64, exact below the bound
+#pragma unroll 16
             for (int k = 0; k < src.G; ++k)
                 acc += (uint64_t)(int64_t)src.grad_l[b * src.G + k] *
                        (uint64_t)(int64_t)src.wlr[(int64_t)k * out_f + q];

@@ -339,12 +339,19 @@ nitro_status nitro_block_backward(nitro_block* b, const int8_t* a_in, const int3
         }
         if (i == 0) break;
         done = false;
-        NITRO_TRY(tc_conv_dgrad(ly.tc, g, batch, b->z64, w_status(b), s, &done));
+        bool fused = false;
+        Layer& lo = b->L[i - 1];
+        TcDgradOut fo{b->desc.alpha_inv, w_delta(b, i), w_w(b, i), lo.g.h, lo.g.w, lo.g.pool,
+                      lo.region, lo.argmax, lo.delta, w_delta(b, i - 1)};
+        // the fused epilogue needs the lower layer to be a conv on the same grid
+        const bool can_fuse = lo.g.kind == NITRO_CONV3X3 && lo.g.oh == g.h && lo.g.ow == g.w;
+        NITRO_TRY(tc_conv_dgrad(ly.tc, g, batch, b->z64, can_fuse ? &fo : nullptr, w_status(b), s,
+                                &done, &fused));
         if (!done) {
             const int mode = g.kind == NITRO_CONV3X3 ? GM_CONV_DGRAD : GM_LIN_DGRAD;
             NITRO_TRY(simt_gemm(mode, nullptr, ly.delta, ly.W, b->z64, batch, g.h, g.w, g.cin, g.cout, s));
         }
-        Layer& lo = b->L[i - 1];
+        if (fused) continue;
         DeltaSrc src{};
         src.g64 = b->z64;
         src.maxabs_a = w_delta(b, i); src.maxabs_b = w_w(b, i);

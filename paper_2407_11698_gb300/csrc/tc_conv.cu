@@ -190,6 +190,15 @@ struct TcArgs {
     int8_t* region;        // NITRO-ReLU piece per pre-pool output
     int8_t* argmax;        // window position per pooled output
     uint16_t* next_nhwc;   // bf16 copy of the output for the next layer's forward, or null
+    // dgrad with fused max-pool / NITRO-ReLU backward into the lower layer's delta
+    FloorDiv32 alpha32;
+    const uint32_t* bound_a;   // max|delta| and max|W| of this layer (int64 exactness bound)
+    const uint32_t* bound_b;
+    int low_h, low_w, low_pool;
+    const int8_t* low_region;
+    const int8_t* low_argmax;
+    int32_t* low_delta;
+    uint32_t* low_maxabs;
 };
 
 // 16 int8 values (4 packed words) -> one 16-byte store
@@ -271,6 +280,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         *abort_flag = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
+    // int32 x int32 contraction: flag when max|delta| max|W| 9 Cout >= 2^63
+    if (MODE == TC_DGRAD && args.fuse && blockIdx.x == 0 && threadIdx.x == 64 &&
+        int64_bound_exceeded(*args.bound_a, *args.bound_b, 9LL * args.Cout))
+        atomicOr(args.status, ST_OVERFLOW);
     // NITRO-ReLU value of every z* in [-127, 127] (fused forward epilogue)
     if (MODE == TC_FWD && args.fuse && threadIdx.x >= 64 && threadIdx.x < 64 + 255)
         relu_tab[threadIdx.x - 64] = (int8_t)relu_value((int64_t)threadIdx.x - 64 - 127, args.alpha, args.mu);
@@ -527,6 +540,69 @@ __global__ void __launch_bounds__(kThreads, 1)
                                 if (args.next_nhwc) st16_bf16(args.next_nhwc + o, opk + 4 * k);
                             }
                         }
+                    }
+                } else if (MODE == TC_DGRAD && args.fuse) {
+                    // gradient at the lower layer's (pooled) output -> int32 with
+                    // the OVERFLOW rule -> max-pool backward (to the recorded
+                    // window position) -> NITRO-ReLU backward -> lower delta.
+                    const int tx = T.mt % args.ntx, ty = (T.mt / args.ntx) % args.nty;
+                    const int tb = T.mt / (args.ntx * args.nty);
+                    const int xx = r % args.wb, yy = (r / args.wb) % args.hb;
+                    const int bbx = r / (args.wb * args.hb);
+                    const int x = tx * args.wb + xx, y = ty * args.hb + yy, b = tb * args.bb + bbx;
+                    const bool valid = x < args.W && y < args.H && b < args.B;
+                    const int Cl = args.Cin;
+                    bool ovf = false;
+                    uint32_t mx = 0;
+                    if (valid) {
+                        const int64_t opix = ((int64_t)b * args.H + y) * args.W + x;
+#pragma unroll
+                        for (int k16 = 0; k16 < NH / 16; ++k16) {
+                            const int c0 = col0 + 16 * k16;
+                            if (c0 >= Cl) break;
+                            int32_t gs[16];
+#pragma unroll
+                            for (int e = 0; e < 16; ++e) {
+                                const int64_t gv = (int64_t)acc[16 * k16 + e];
+                                ovf |= !fits_i32(gv);
+                                gs[e] = (int32_t)gv;
+                            }
+                            const uint4 amv = args.low_pool
+                                ? *reinterpret_cast<const uint4*>(args.low_argmax + opix * Cl + c0)
+                                : make_uint4(0, 0, 0, 0);
+                            const uint32_t amw[4] = {amv.x, amv.y, amv.z, amv.w};
+                            const int npos = args.low_pool ? 4 : 1;
+                            for (int k = 0; k < npos; ++k) {
+                                const int64_t ppix = args.low_pool
+                                    ? ((int64_t)b * args.low_h + 2 * y + (k >> 1)) * args.low_w + 2 * x + (k & 1)
+                                    : opix;
+                                const uint4 rgv = *reinterpret_cast<const uint4*>(args.low_region + ppix * Cl + c0);
+                                const uint32_t rgw[4] = {rgv.x, rgv.y, rgv.z, rgv.w};
+                                int32_t dv[16];
+#pragma unroll
+                                for (int e = 0; e < 16; ++e) {
+                                    const int reg = (int)((rgw[e >> 2] >> (8 * (e & 3))) & 255u);
+                                    const int am = (int)((amw[e >> 2] >> (8 * (e & 3))) & 255u);
+                                    int32_t v = 0;
+                                    if (am == k) {
+                                        v = reg == 1 ? args.alpha32.floor_div(gs[e]) : (reg == 2 ? gs[e] : 0);
+                                    }
+                                    dv[e] = v;
+                                    mx = max(mx, abs_u32(v));
+                                }
+                                int4* o = reinterpret_cast<int4*>(args.low_delta + ppix * Cl + c0);
+#pragma unroll
+                                for (int e = 0; e < 4; ++e)
+                                    o[e] = make_int4(dv[4 * e], dv[4 * e + 1], dv[4 * e + 2], dv[4 * e + 3]);
+                            }
+                        }
+                    }
+#pragma unroll
+                    for (int off = 16; off; off >>= 1) mx = max(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+                    ovf = __any_sync(0xffffffffu, ovf);
+                    if (lane == 0) {
+                        if (mx) atomicMax(args.low_maxabs, mx);
+                        if (ovf) atomicOr(args.status, ST_OVERFLOW);
                     }
                 } else {
                     const int tx = T.mt % args.ntx, ty = (T.mt / args.ntx) % args.nty;
@@ -987,8 +1063,10 @@ cudaError_t tc_conv_wgrad(TcLayer& t, const LayerGeom& g, const int32_t* delta,
 }
 
 cudaError_t tc_conv_dgrad(TcLayer& t, const LayerGeom& g, int batch, int64_t* g64,
-                          uint32_t* status, cudaStream_t s, bool* done) {
+                          const TcDgradOut* fo, uint32_t* status, cudaStream_t s, bool* done,
+                          bool* fused) {
     *done = false;
+    *fused = false;
     if (!t.dgrad || batch <= 0) return cudaSuccess;
     TcArgs a{};
     a.B = batch; a.H = g.h; a.W = g.w; a.Cin = g.cin; a.Cout = g.cout;
@@ -1006,6 +1084,24 @@ cudaError_t tc_conv_dgrad(TcLayer& t, const LayerGeom& g, int batch, int64_t* g6
     a.out = g64;
     a.status = status;
     a.atomic_out = 0;
+    if (fo && g.cin % 16 == 0) {
+        a.fuse = 1;
+        a.alpha32 = FloorDiv32::make((uint32_t)fo->alpha_inv);
+        a.bound_a = fo->maxabs_delta;
+        a.bound_b = fo->maxabs_w;
+        a.low_h = fo->low_h;
+        a.low_w = fo->low_w;
+        a.low_pool = fo->low_pool;
+        a.low_region = fo->low_region;
+        a.low_argmax = fo->low_argmax;
+        a.low_delta = fo->low_delta;
+        a.low_maxabs = fo->low_maxabs;
+        if (fo->low_pool && ((fo->low_h & 1) || (fo->low_w & 1))) {   // rows the pool dropped
+            cudaError_t e = cudaMemsetAsync(fo->low_delta, 0,
+                                            sizeof(int32_t) * (size_t)batch * fo->low_h * fo->low_w * g.cin, s);
+            if (e != cudaSuccess) return e;
+        }
+    }
     CUtensorMap ma, mb;
     const uint64_t da[5] = {(uint64_t)g.cout, (uint64_t)g.w, (uint64_t)g.h, (uint64_t)batch,
                             (uint64_t)kMaxLimbs};
@@ -1022,7 +1118,10 @@ cudaError_t tc_conv_dgrad(TcLayer& t, const LayerGeom& g, int batch, int64_t* g6
     const double ops = 2.0 * batch * g.h * g.w * g.cin * 9.0 * g.cout;
     ProfScope ps(K_TC_CONV_DGRAD, s, ops, 0.0);
     cudaError_t e = launch_gemm_n<TC_DGRAD>(n, ma, mb, a, s);
-    if (e == cudaSuccess) *done = true;
+    if (e == cudaSuccess) {
+        *done = true;
+        *fused = a.fuse != 0;
+    }
     return e;
 }
 

@@ -83,8 +83,25 @@ cudaError_t tc_conv_wgrad(TcLayer& t, const LayerGeom& g, const int32_t* delta,
                           const uint32_t* maxabs_delta, int batch, int64_t* dW,
                           uint32_t* status, cudaStream_t s, bool* done);
 
-// g[p][ci] (int64) = sum_(t,co) delta[p - tap t][co] W[co][t][ci].
+// Where the input gradient goes when the dgrad epilogue is fused: through the
+// lower layer's max-pool backward and NITRO-ReLU backward into its delta.
+struct TcDgradOut {
+    int alpha_inv;
+    const uint32_t* maxabs_delta;   // this layer's max|delta| and max|W|
+    const uint32_t* maxabs_w;
+    int low_h, low_w, low_pool;     // lower layer's pre-pool size and pool flag
+    const int8_t* low_region;
+    const int8_t* low_argmax;
+    int32_t* low_delta;             // [B][low_h][low_w][Cin] int32
+    uint32_t* low_maxabs;           // max|lower delta| (atomic max)
+};
+
+// g[p][ci] = sum_(t,co) delta[p - tap t][co] W[co][t][ci] on tcgen05
+// (*done = false if the layer does not run there).  With fo != null and
+// Cin % 16 == 0 the epilogue produces the lower layer's delta (*fused = true);
+// otherwise g is written as int64 to g64.
 cudaError_t tc_conv_dgrad(TcLayer& t, const LayerGeom& g, int batch, int64_t* g64,
-                          uint32_t* status, cudaStream_t s, bool* done);
+                          const TcDgradOut* fo, uint32_t* status, cudaStream_t s, bool* done,
+                          bool* fused);
 
 }  // namespace nitro

@@ -23,9 +23,10 @@ def _cuda():
     nb.lib()
 
 
-def _two_conv_block(B, h, w, c0, c1, c2, pool):
-    oh, ow = (h // 2, w // 2) if pool else (h, w)
-    return [{"layers": [(C, c0, c1, h, w, 0), (C, c1, c2, h, w, int(pool))],
+def _two_conv_block(B, h, w, c0, c1, c2, pool, pool_first=False):
+    h1, w1 = (h // 2, w // 2) if pool_first else (h, w)
+    oh, ow = (h1 // 2, w1 // 2) if pool else (h1, w1)
+    return [{"layers": [(C, c0, c1, h, w, int(pool_first)), (C, c1, c2, h1, w1, int(pool))],
              "in_features": h * w * c0},
             {"layers": [], "in_features": oh * ow * c2}]
 
@@ -50,7 +51,20 @@ def _widen(pair, scale):
     (130, 8, 16, 64, 64, 64, True, 1),         # batch over 128 (wgrad batch blocks)
 ])
 def test_two_conv_block_parity(B, h, w, c0, c1, c2, pool, scale):
-    blocks = _two_conv_block(B, h, w, c0, c1, c2, pool)
+    _run_two_conv(B, h, w, c0, c1, c2, pool, scale, False)
+
+
+@pytest.mark.parametrize("B,h,w,c0,c1,c2,pool,scale", [
+    (4, 16, 16, 64, 64, 64, False, 1),         # pooled lower layer: dgrad routes to argmax
+    (3, 17, 18, 64, 128, 64, True, 300),       # odd pooled lower layer (dropped row)
+    (5, 16, 32, 64, 64, 128, False, 70001),    # wide weights through the pooled path
+])
+def test_two_conv_block_pooled_lower_layer(B, h, w, c0, c1, c2, pool, scale):
+    _run_two_conv(B, h, w, c0, c1, c2, pool, scale, True)
+
+
+def _run_two_conv(B, h, w, c0, c1, c2, pool, scale, pool_first):
+    blocks = _two_conv_block(B, h, w, c0, c1, c2, pool, pool_first)
     pair = NetPair(blocks, B, seed=31)
     try:
         if scale != 1:
