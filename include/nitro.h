@@ -172,6 +172,37 @@ uint32_t nitro_block_status_bits(nitro_block* blk);
 /* Releases every device buffer of the block.  NULL is ignored. */
 void nitro_destroy_block(nitro_block* blk);
 
+/* ---- Kernel-level contractions ----------------------------------------------
+ * One contraction of a 3x3 conv layer (stride 1, zero padding 1; Sec. 3.2.1
+ * conv expression and its two adjoints) or one integer GEMM, on caller-owned
+ * device buffers, through the same operand split and kernels as the block
+ * step.  Outputs are the exact integer sums modulo 2^64, as int64:
+ *   NITRO_CONTRACT_FWD   x = int8 a [B][H][W][Cin],  y = int32 W [Cout][3][3][Cin]
+ *                        out = z [B][H][W][Cout],  z = sum_(ky,kx,ci) a[y+ky-1][x+kx-1][ci] W
+ *   NITRO_CONTRACT_WGRAD x = int8 a,                 y = int32 d [B][H][W][Cout]
+ *                        out = dW [Cout][3][3][Cin] = sum_(b,y,x) d[b,y,x,co] a[b,y+ky-1,x+kx-1,ci]
+ *   NITRO_CONTRACT_DGRAD x = int32 d [B][H][W][Cout], y = int32 W
+ *                        out = g [B][H][W][Cin] = sum_(ky,kx,co) d[b,y-ky+1,x-kx+1,co] W
+ * Asynchronous on `stream`; the handle owns its packing workspace (sized at
+ * create for max_batch) and must not be used by two streams at once. */
+typedef enum { NITRO_CONTRACT_FWD = 0, NITRO_CONTRACT_WGRAD = 1, NITRO_CONTRACT_DGRAD = 2 } nitro_contract_mode;
+typedef struct nitro_conv nitro_conv;
+nitro_status nitro_conv3x3_create(int max_batch, int h, int w, int cin, int cout, nitro_conv** out);
+nitro_status nitro_conv3x3_contract(nitro_conv* c, int mode, const void* x, const int32_t* y,
+                                    int batch, int64_t* out, void* stream);
+nitro_status nitro_conv3x3_status(nitro_conv* c);   /* synchronises; latched TIMEOUT */
+void nitro_conv3x3_destroy(nitro_conv* c);
+
+/* C[m][n] = sum_k A[m][k] B[n][k]: A int8 [M][K], B int32 [N][K], C int64
+ * [M][N], row-major.  The integer matrix product the linear layers reduce to
+ * (Sec. 3.2.1 linear expression). */
+typedef struct nitro_gemm nitro_gemm;
+nitro_status nitro_gemm_create(int max_m, int max_n, int max_k, nitro_gemm** out);
+nitro_status nitro_gemm_run(nitro_gemm* g, const int8_t* a, const int32_t* b, int m, int n, int k,
+                            int64_t* c, void* stream);
+nitro_status nitro_gemm_status(nitro_gemm* g);      /* synchronises; latched TIMEOUT */
+void nitro_gemm_destroy(nitro_gemm* g);
+
 /* ---- Allocation-free layer forward ----------------------------------------
  * The paper has no counterpart to this call: it exists for callers that
  * cannot allocate device memory once running - code inside a host program

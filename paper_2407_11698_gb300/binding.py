@@ -18,6 +18,7 @@ NITRO_OK, NITRO_ERR_ARG, NITRO_ERR_OVERFLOW, NITRO_ERR_TIMEOUT, NITRO_ERR_CUDA, 
 NITRO_CONV3X3, NITRO_LINEAR = 0, 1
 NITRO_ROUND_FLOOR, NITRO_ROUND_TRUNC = 0, 1
 STATUS_BIT_OVERFLOW, STATUS_BIT_BAD_LABEL, STATUS_BIT_TIMEOUT = 1, 2, 4
+NITRO_CONTRACT_FWD, NITRO_CONTRACT_WGRAD, NITRO_CONTRACT_DGRAD = 0, 1, 2
 (NITRO_T_W, NITRO_T_DW, NITRO_T_WLR, NITRO_T_DWLR, NITRO_T_ACT, NITRO_T_REGION,
  NITRO_T_ARGMAX, NITRO_T_DELTA, NITRO_T_GRAD_L, NITRO_T_SSE) = range(10)
 
@@ -91,6 +92,19 @@ def lib():
     L.nitro_profile_read.restype = ctypes.c_int
     L.nitro_conv3x3_forward_noalloc.argtypes = [_VP, _VP] + [ctypes.c_int] * 7 + [_VP, _VP, _VP, _VP]
     L.nitro_conv3x3_forward_noalloc.restype = ctypes.c_int
+    L.nitro_conv3x3_create.argtypes = [ctypes.c_int] * 5 + [ctypes.POINTER(_VP)]
+    L.nitro_conv3x3_contract.argtypes = [_VP, ctypes.c_int, _VP, _VP, ctypes.c_int, _VP, _VP]
+    L.nitro_conv3x3_status.argtypes = [_VP]
+    L.nitro_conv3x3_destroy.argtypes = [_VP]
+    L.nitro_conv3x3_destroy.restype = None
+    L.nitro_gemm_create.argtypes = [ctypes.c_int] * 3 + [ctypes.POINTER(_VP)]
+    L.nitro_gemm_run.argtypes = [_VP, _VP, _VP, ctypes.c_int, ctypes.c_int, ctypes.c_int, _VP, _VP]
+    L.nitro_gemm_status.argtypes = [_VP]
+    L.nitro_gemm_destroy.argtypes = [_VP]
+    L.nitro_gemm_destroy.restype = None
+    for name in ("nitro_conv3x3_create", "nitro_conv3x3_contract", "nitro_conv3x3_status",
+                 "nitro_gemm_create", "nitro_gemm_run", "nitro_gemm_status"):
+        getattr(L, name).restype = ctypes.c_int
     for name in ("nitro_init_block", "nitro_block_forward", "nitro_block_backward",
                  "nitro_integersgd_step", "nitro_block_tensor_bytes", "nitro_block_get_tensor",
                  "nitro_block_set_tensor", "nitro_block_status"):
@@ -250,6 +264,71 @@ class Block:
     def close(self):
         if getattr(self, "h", None):
             nitro_destroy_block(self.h)
+            self.h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+class Conv3x3:
+    """One 3x3 conv layer's contractions (kernel-level entry points)."""
+
+    def __init__(self, max_batch, h, w, cin, cout):
+        self.h = _VP()
+        st = lib().nitro_conv3x3_create(int(max_batch), int(h), int(w), int(cin), int(cout),
+                                        ctypes.byref(self.h))
+        if st != NITRO_OK:
+            raise NitroError(st, "nitro_conv3x3_create")
+
+    def contract(self, mode, x, y, out, stream=None):
+        st = lib().nitro_conv3x3_contract(self.h, int(mode), _ptr(x), _ptr(y), int(x.shape[0]),
+                                          _ptr(out), _stream_ptr(stream))
+        if st != NITRO_OK:
+            raise NitroError(st, "nitro_conv3x3_contract")
+        return out
+
+    def status(self):
+        return lib().nitro_conv3x3_status(self.h)
+
+    def close(self):
+        if getattr(self, "h", None):
+            lib().nitro_conv3x3_destroy(self.h)
+            self.h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+class IntGemm:
+    """C = A B^T with A int8 [M][K], B int32 [N][K], C int64 (kernel-level)."""
+
+    def __init__(self, max_m, max_n, max_k):
+        self.h = _VP()
+        st = lib().nitro_gemm_create(int(max_m), int(max_n), int(max_k), ctypes.byref(self.h))
+        if st != NITRO_OK:
+            raise NitroError(st, "nitro_gemm_create")
+
+    def run(self, a, b, c, stream=None):
+        m, k = a.shape
+        n = b.shape[0]
+        st = lib().nitro_gemm_run(self.h, _ptr(a), _ptr(b), int(m), int(n), int(k), _ptr(c),
+                                  _stream_ptr(stream))
+        if st != NITRO_OK:
+            raise NitroError(st, "nitro_gemm_run")
+        return c
+
+    def status(self):
+        return lib().nitro_gemm_status(self.h)
+
+    def close(self):
+        if getattr(self, "h", None):
+            lib().nitro_gemm_destroy(self.h)
             self.h = None
 
     def __del__(self):

@@ -29,6 +29,7 @@ enum KernelId : int {
     K_TC_CONV_DGRAD,
     K_TC_PACK,
     K_TC_FINISH,
+    K_TC_GEMM,
     K_COUNT
 };
 

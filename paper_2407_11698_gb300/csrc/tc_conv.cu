@@ -22,7 +22,7 @@
 namespace nitro {
 namespace {
 
-enum TcMode : int { TC_FWD = 0, TC_WGRAD = 1, TC_DGRAD = 2 };
+enum TcMode : int { TC_FWD = 0, TC_WGRAD = 1, TC_DGRAD = 2, TC_GEMM = 3 };
 
 constexpr int kBM = 128;              // rows per tile (TMEM lanes)
 constexpr int kBK = 64;               // K elements per block (one 128-byte row)
@@ -80,6 +80,14 @@ __device__ __noinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile i
     }
 }
 
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* m, uint32_t bar,
+                                            int c0, int c1) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%3, %4}], [%2];" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(m)), "r"(bar), "r"(c0), "r"(c1)
+        : "memory");
+}
 __device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap* m, uint32_t bar,
                                             int c0, int c1, int c2) {
     asm volatile(
@@ -325,7 +333,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                         const uint32_t a_dst = smem_u32(smem + s * C::STAGE);
                         const uint32_t b_dst = a_dst + C::A_BYTES;
                         mbar_expect_tx(fb, C::STAGE);
-                        if (MODE == TC_FWD) {
+                        if (MODE == TC_GEMM) {
+                            tma_load_2d(a_dst, &tmA, fb, kb * kBK, T.mt * kBM);
+                            tma_load_3d(b_dst, &tmB, fb, kb * kBK, n0, lb);
+                        } else if (MODE == TC_FWD) {
                             const int nc = args.cin_k / kBK;
                             const int t = kb / nc, cb = kb - t * nc, ky = t / 3, kx = t - 3 * ky;
                             tma_load_4d(a_dst, &tmA, fb, cb * kBK, x0 + kx - 1, y0 + ky - 1, b0);
@@ -430,7 +441,15 @@ __global__ void __launch_bounds__(kThreads, 1)
             {
                 const int r = 32 * q + lane;   // output row of this thread
                 const int col0 = T.nt * N + half * NH;
-                if (MODE == TC_WGRAD) {
+                if (MODE == TC_GEMM) {
+                    const int m = T.mt * kBM + r;      // C[m][n], M rows in args.B
+                    if (m < args.B) {
+                        int64_t* o = args.out + (int64_t)m * args.ncols + col0;
+#pragma unroll
+                        for (int i = 0; i < NH; ++i)
+                            if (col0 + i < args.ncols) o[i] = (int64_t)acc[i];
+                    }
+                } else if (MODE == TC_WGRAD) {
                     const int m = T.mt * kBM + r;
                     const int t = m / args.cin_k, ci = m - t * args.cin_k;
                     if (t < 9 && ci < args.Cin) {
@@ -990,10 +1009,8 @@ cudaError_t tc_conv_forward(TcLayer& t, const LayerGeom& g, int batch, int64_t* 
     return e;
 }
 
-cudaError_t tc_conv_wgrad(TcLayer& t, const LayerGeom& g, const int32_t* delta,
-                          const uint32_t* maxabs_delta, int batch, int64_t* dW,
-                          uint32_t* status, cudaStream_t s, bool* done) {
-    *done = false;
+cudaError_t tc_pack_delta(TcLayer& t, const LayerGeom& g, const int32_t* delta,
+                          const uint32_t* maxabs_delta, int batch, cudaStream_t s) {
     if (batch <= 0 || (!t.wgrad && !t.dgrad)) return cudaSuccess;
     const int hw = g.h * g.w;
     const int bp = round_up(batch, 8);
@@ -1017,7 +1034,19 @@ cudaError_t tc_conv_wgrad(TcLayer& t, const LayerGeom& g, const int32_t* delta,
         cudaError_t e = cudaGetLastError();
         if (e != cudaSuccess) return e;
     }
+    return cudaSuccess;
+}
+
+cudaError_t tc_conv_wgrad(TcLayer& t, const LayerGeom& g, const int32_t* delta,
+                          const uint32_t* maxabs_delta, int batch, int64_t* dW,
+                          uint32_t* status, cudaStream_t s, bool* done) {
+    *done = false;
+    if (batch <= 0 || (!t.wgrad && !t.dgrad)) return cudaSuccess;
+    cudaError_t pe = tc_pack_delta(t, g, delta, maxabs_delta, batch, s);
+    if (pe != cudaSuccess) return pe;
     if (!t.wgrad) return cudaSuccess;
+    const int hw = g.h * g.w;
+    const int bp = round_up(batch, 8);
     TcArgs a{};
     a.B = batch; a.H = g.h; a.W = g.w; a.Cin = g.cin; a.Cout = g.cout; a.Bp = bp;
     a.cin_k = t.cin_k;
@@ -1123,6 +1152,73 @@ cudaError_t tc_conv_dgrad(TcLayer& t, const LayerGeom& g, int batch, int64_t* g6
         *fused = a.fuse != 0;
     }
     return e;
+}
+
+// ------------------------------------------------------------------ plain GEMM
+namespace {
+__global__ void k_maxabs(const int32_t* __restrict__ x, int64_t n, uint32_t* out) {
+    uint32_t m = 0;
+    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
+         i += (int64_t)gridDim.x * blockDim.x)
+        m = max(m, abs_u32(x[i]));
+#pragma unroll
+    for (int off = 16; off; off >>= 1) m = max(m, __shfl_xor_sync(0xffffffffu, m, off));
+    if ((threadIdx.x & 31) == 0 && m) atomicMax(out, m);
+}
+}  // namespace
+
+cudaError_t tc_maxabs(const int32_t* x, int64_t n, uint32_t* out, cudaStream_t s) {
+    cudaError_t e = cudaMemsetAsync(out, 0, sizeof(uint32_t), s);
+    if (e != cudaSuccess || n <= 0) return e;
+    ProfScope ps(K_TC_PACK, s, 0.0, (double)n * 4);
+    k_maxabs<<<grid1d(n), 256, 0, s>>>(x, n, out);
+    return cudaGetLastError();
+}
+
+cudaError_t tc_pack_int8(const int8_t* x, int64_t rows, int cols, uint16_t* out, cudaStream_t s) {
+    if (rows <= 0) return cudaSuccess;
+    ProfScope ps(K_TC_PACK, s, 0.0, (double)rows * cols * 3);
+    k_pack_act_nhwc<<<grid1d(rows * cols), 256, 0, s>>>(x, rows, cols, cols, out);
+    return cudaGetLastError();
+}
+
+cudaError_t tc_pack_limbs(const int32_t* x, int64_t n, const uint32_t* maxabs, uint16_t* planes,
+                          int* limbs, cudaStream_t s) {
+    if (n <= 0) return cudaSuccess;
+    ProfScope ps(K_TC_PACK, s, 0.0, (double)n * 4 * 2);
+    k_pack_delta_nhwc<<<grid1d(n / 8), 256, 0, s>>>(x, n, maxabs, planes, limbs);
+    return cudaGetLastError();
+}
+
+cudaError_t tc_gemm_run(const uint16_t* a_bf16, const uint16_t* b_planes, int M, int N, int K,
+                        const int* limbs_b, int64_t* out, uint32_t* status, cudaStream_t s) {
+    if (M <= 0 || N <= 0) return cudaSuccess;
+    TcArgs a{};
+    a.B = M;
+    a.ncols = N;
+    a.ntx = a.nty = 1;
+    a.wb = a.hb = a.bb = 1;
+    const int n = pick_n(N);
+    a.tiles_m = (M + kBM - 1) / kBM;
+    a.tiles_n = (N + n - 1) / n;
+    a.total_tiles = a.tiles_m * a.tiles_n;
+    a.kb_total = (K + kBK - 1) / kBK;
+    a.kb_per_split = a.kb_total;
+    a.limbs_a = nullptr;
+    a.limbs_b = limbs_b;
+    a.out = out;
+    a.status = status;
+    CUtensorMap ma, mb;
+    const uint64_t da[2] = {(uint64_t)K, (uint64_t)M};
+    const uint64_t sa[1] = {(uint64_t)K};
+    const uint32_t ba[2] = {64, 128};
+    const uint64_t db[3] = {(uint64_t)K, (uint64_t)N, (uint64_t)kMaxLimbs};
+    const uint64_t sb[2] = {(uint64_t)K, (uint64_t)K * N};
+    const uint32_t bb[3] = {64, (uint32_t)n, 1};
+    if (!make_map(&ma, a_bf16, 2, da, sa, ba) || !make_map(&mb, b_planes, 3, db, sb, bb))
+        return cudaErrorInvalidValue;
+    ProfScope ps(K_TC_GEMM, s, 2.0 * M * N * (double)K, 0.0);
+    return launch_gemm_n<TC_GEMM>(n, ma, mb, a, s);
 }
 
 }  // namespace nitro

@@ -77,8 +77,13 @@ cudaError_t tc_conv_forward(TcLayer& t, const LayerGeom& g, int batch, int64_t* 
                             const TcFwdOut* fo, uint32_t* status, cudaStream_t s, bool* done,
                             bool* fused);
 
-// Splits delta into limb planes (both layouts as needed) and, if wgrad runs on
-// tcgen05, dW = sum_p delta (x) im2col(a).  Must precede tc_conv_dgrad.
+// Splits delta into limb planes in the layouts the wgrad and dgrad passes read
+// (limb count from *maxabs_delta, recorded on the device for the GEMMs).
+cudaError_t tc_pack_delta(TcLayer& t, const LayerGeom& g, const int32_t* delta,
+                          const uint32_t* maxabs_delta, int batch, cudaStream_t s);
+
+// tc_pack_delta, then, if wgrad runs on tcgen05, dW = sum_p delta (x)
+// im2col(a).  Must precede tc_conv_dgrad.
 cudaError_t tc_conv_wgrad(TcLayer& t, const LayerGeom& g, const int32_t* delta,
                           const uint32_t* maxabs_delta, int batch, int64_t* dW,
                           uint32_t* status, cudaStream_t s, bool* done);
@@ -103,5 +108,16 @@ struct TcDgradOut {
 cudaError_t tc_conv_dgrad(TcLayer& t, const LayerGeom& g, int batch, int64_t* g64,
                           const TcDgradOut* fo, uint32_t* status, cudaStream_t s, bool* done,
                           bool* fused);
+
+// Helpers of the kernel-level entry points (contract.cu).
+cudaError_t tc_maxabs(const int32_t* x, int64_t n, uint32_t* out, cudaStream_t s);
+cudaError_t tc_pack_int8(const int8_t* x, int64_t rows, int cols, uint16_t* out, cudaStream_t s);
+// n % 8 == 0; planes [4][n]; the limb count (from *maxabs) goes to *limbs
+cudaError_t tc_pack_limbs(const int32_t* x, int64_t n, const uint32_t* maxabs, uint16_t* planes,
+                          int* limbs, cudaStream_t s);
+// C[m][n] (int64) = sum_k A[m][k] B[n][k]; A bf16 [M][K] (int8 values), B limb
+// planes [4][N][K]; K % 8 == 0.
+cudaError_t tc_gemm_run(const uint16_t* a_bf16, const uint16_t* b_planes, int M, int N, int K,
+                        const int* limbs_b, int64_t* out, uint32_t* status, cudaStream_t s);
 
 }  // namespace nitro

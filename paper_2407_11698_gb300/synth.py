@@ -31,6 +31,6 @@ def gaussian_images(seed: int, step: int, batch: int, shape, sigma: float = 64.0
     return np.clip(x, -128, 127).astype(np.int8)
 
 
-def int_tensor(seed: int, shape, lo: int, hi: int, stream: int = 3) -> np.ndarray:
-    """int64 tensor uniform on [lo, hi] (inclusive), for kernel-level tests."""
-    return _rng(seed, 0, stream).integers(lo, hi + 1, size=shape, dtype=np.int64)
+def int_tensor(seed: int, shape, lo: int, hi: int, stream: int = 3, dtype=np.int64) -> np.ndarray:
+    """Integer tensor uniform on [lo, hi] (inclusive), for kernel-level tests."""
+    return _rng(seed, 0, stream).integers(lo, hi + 1, size=shape, dtype=dtype)

@@ -39,11 +39,12 @@ def test_cnn_32_64_b64_100_steps():
     run_workload(WL.WORKLOADS["cnn_32_64_b64"], steps=100, check_every=25)
 
 
-def test_vgg_64_128_256_b128_two_steps():
-    # Full-size VGG-style network: the first step drives the first conv of
-    # each block to multi-limb weights (|W| ~ 1e6) and deltas (~7e5), so
-    # step two exercises the wide-operand path.
-    run_workload(WL.WORKLOADS["vgg_64_128_256_b128"], steps=2)
+def test_vgg_64_128_256_b128_50_steps():
+    # Full-size VGG-style network for all 50 steps of the workload: the first
+    # step drives the first conv of each block to multi-limb weights (|W| ~
+    # 1e6) and deltas (~7e5); around step 4 deltas leave int32 (OVERFLOW on
+    # both sides, identical wrap), so later steps run with four-limb operands.
+    run_workload(WL.WORKLOADS["vgg_64_128_256_b128"], steps=50, check_every=5)
 
 
 # ---------------------------------------------------------------- edge cases
