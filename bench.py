@@ -38,7 +38,25 @@ def parse():
     p.add_argument("--no-graph", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--profile-steps", type=int, default=3)
+    p.add_argument("--sweep", action="store_true",
+                   help="time the kernel sweep (conv contractions and integer GEMM) instead")
     return p.parse_args()
+
+
+def ncu_traffic(kernel):
+    """Per-launch DRAM bytes of `kernel` from the committed ncu summary, or None
+    when the kernel source changed since the counters were taken."""
+    import hashlib
+    try:
+        src = open(os.path.join(ROOT, "paper_2407_11698_gb300", "csrc", "tc_conv.cu"), "rb").read()
+        sha = hashlib.sha1(src).hexdigest()[:12]
+        for line in open(os.path.join(ROOT, "profiles", "tc_conv_kernels_vgg_step.md")):
+            parts = line.split()
+            if len(parts) == 4 and parts[0] == "traffic" and parts[1] == kernel:
+                return int(parts[2]) if parts[3] == "sha1=" + sha else None
+    except OSError:
+        pass
+    return None
 
 
 def measured_peaks():
@@ -301,7 +319,7 @@ def run_ours(args, rank, world, local_rank):
         "gpu_launches": int(launches_per_step * args.steps),
         "roofline": {"bound": bound, "kernel": dom_name, "achieved": round(achieved, 3),
                      "peak": round(peak, 2), "unit": unit, "frac": round(achieved / peak, 4),
-                     "traffic": None, "peak_source": peak_note,
+                     "traffic": ncu_traffic(dom_name), "peak_source": peak_note,
                      "per_launch_ms": round(per_launch_ms, 5),
                      "share_of_kernel_time": round(dom["ms"] / total_k, 4)},
         "conv_tops": round(conv_ops / (conv_ms / 1e3) / 1e12, 3) if conv_ms else None,
@@ -333,8 +351,110 @@ def oracle_rate(wl_name, sample_batch, steps, warmup=0):
     return sample_batch * steps / dt, dt, O.num_threads()
 
 
+# ------------------------------------------------------------------ kernel sweep
+SWEEP_RANGES = {1: (-127, 127), 2: (-32768, 32639), 3: (-2**23, 2**23 - 1)}
+
+
+def run_sweep(args):
+    """One JSON line per (contraction, shape, operand limbs): device time of
+    the contraction kernel alone (library events) and of the whole call
+    (limb packing included), as algorithmic TOPS (2 x MACs of the integer
+    contraction) and as a fraction of the measured bf16 dense peak."""
+    import ctypes
+    import numpy as np
+    import torch
+    from paper_2407_11698_gb300 import binding as nb
+    from paper_2407_11698_gb300 import synth
+    from paper_2407_11698_gb300 import workloads as WL
+    nb.lib()
+    L = nb.lib()
+    peaks, src = measured_peaks()
+    peak = peaks["bf16_tflops"]
+    stream = torch.cuda.current_stream()
+
+    def timed(fn, reps):
+        fn()
+        torch.cuda.synchronize()
+        L.nitro_profile_reset()
+        L.nitro_profile_enable(1)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(reps):
+            fn()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        L.nitro_profile_enable(0)
+        prof = kernel_profile(nb)
+        L.nitro_profile_reset()
+        return e0.elapsed_time(e1) / reps, prof
+
+    def emit(kind, shape, limbs, ops, call_ms, prof, key):
+        k = prof.get(key, {"ms": float("nan"), "launches": 1})
+        kms = k["ms"] / max(1, k["launches"])
+        line = {"sweep": kind, "shape": shape, "limbs": limbs, "ops": ops,
+                "kernel": key, "kernel_ms": round(kms, 5), "call_ms": round(call_ms, 5),
+                "kernel_tops": round(ops / kms / 1e9, 2), "call_tops": round(ops / call_ms / 1e9, 2),
+                "kernel_frac_bf16": round(ops / kms / 1e9 / peak, 4), "peak": peak,
+                "peak_source": "bf16 dense, %s" % src}
+        print(json.dumps(line), flush=True)
+
+    for B, hw, c in WL.SWEEP_CONV:
+        a = torch.from_numpy(synth.images(51, 0, B, (hw, hw, c))).cuda()
+        conv = nb.Conv3x3(B, hw, hw, c, c)
+        out = torch.empty((B, hw, hw, c), dtype=torch.int64, device="cuda")
+        dw = torch.empty((c, 3, 3, c), dtype=torch.int64, device="cuda")
+        ops = 2.0 * B * hw * hw * c * 9 * c
+        for limbs in (1, 2, 3):
+            lo, hi = SWEEP_RANGES[limbs]
+            W = torch.from_numpy(synth.int_tensor(52, (c, 3, 3, c), lo, hi, dtype=np.int32)).cuda()
+            d = torch.from_numpy(synth.int_tensor(53, (B, hw, hw, c), lo, hi, dtype=np.int32)).cuda()
+            ms, prof = timed(lambda: conv.contract(nb.NITRO_CONTRACT_FWD, a, W, out), 5)
+            emit("conv_fwd", [B, hw, hw, c, c], {"W": limbs}, ops, ms, prof, "tc_conv_fwd")
+            ms, prof = timed(lambda: conv.contract(nb.NITRO_CONTRACT_WGRAD, a, d, dw), 5)
+            emit("conv_wgrad", [B, hw, hw, c, c], {"delta": limbs}, ops, ms, prof, "tc_conv_wgrad")
+            ms, prof = timed(lambda: conv.contract(nb.NITRO_CONTRACT_DGRAD, d, W, out), 5)
+            emit("conv_dgrad", [B, hw, hw, c, c], {"delta": limbs, "W": limbs}, ops, ms, prof,
+                 "tc_conv_dgrad")
+            del W, d
+        conv.close()
+        del a, out, dw
+        torch.cuda.empty_cache()
+    for n in WL.SWEEP_GEMM:
+        a = torch.from_numpy(synth.int_tensor(61, (n, n), -128, 127, dtype=np.int8)).cuda()
+        b8 = torch.from_numpy(synth.int_tensor(62, (n, n), -128, 127, dtype=np.int8)).cuda()
+        gm = nb.IntGemm(n, n, n)
+        c = torch.empty((n, n), dtype=torch.int64, device="cuda")
+        ops = 2.0 * n * n * n
+        for limbs in (1, 2):
+            lo, hi = SWEEP_RANGES[limbs]
+            b = torch.from_numpy(synth.int_tensor(63, (n, n), lo, hi, dtype=np.int32)).cuda()
+            ms, prof = timed(lambda: gm.run(a, b, c), 5)
+            emit("gemm", [n, n, n], {"B": limbs}, ops, ms, prof, "tc_gemm")
+        # library baseline: torch._int_mm (int8 x int8 -> int32, cuBLASLt)
+        bt = b8.t()
+        torch._int_mm(a, bt)
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(5):
+            torch._int_mm(a, bt)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        ms = e0.elapsed_time(e1) / 5
+        print(json.dumps({"sweep": "torch_int_mm", "shape": [n, n, n], "call_ms": round(ms, 5),
+                          "call_tops": round(ops / ms / 1e9, 2),
+                          "note": "int8 x int8 -> int32 library GEMM, context for the int8 tensor rate"}),
+              flush=True)
+        gm.close()
+        del a, b8, c
+        torch.cuda.empty_cache()
+    return 0
+
+
 def main():
     args = parse()
+    if args.sweep:
+        return run_sweep(args)
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))
