@@ -17,6 +17,7 @@ struct nitro_conv {
     int max_batch = 0;
     uint32_t* words = nullptr;   // [0] max|W| [1] max|delta| [2] status
     std::vector<void*> allocs;
+    std::vector<void*> host_allocs;
 };
 
 struct nitro_gemm {
@@ -41,6 +42,11 @@ bool dalloc(std::vector<void*>& allocs, T** p, size_t count) {
 
 void free_all(std::vector<void*>& allocs) {
     for (void* p : allocs) cudaFree(p);
+    allocs.clear();
+}
+
+void free_host(std::vector<void*>& allocs) {
+    for (void* p : allocs) cudaFreeHost(p);
     allocs.clear();
 }
 
@@ -71,10 +77,12 @@ nitro_status nitro_conv3x3_create(int max_batch, int h, int w, int cin, int cout
     if (!c) return NITRO_ERR_CUDA;
     c->g = LayerGeom{NITRO_CONV3X3, cin, cout, h, w, 0, h, w};
     c->max_batch = max_batch;
-    bool ok = tc_layer_init(c->t, c->g, max_batch, true, c->allocs) && dalloc(c->allocs, &c->words, 4);
+    bool ok = tc_layer_init(c->t, c->g, max_batch, true, c->allocs, c->host_allocs) &&
+              dalloc(c->allocs, &c->words, 4);
     if (ok) ok = cudaMemset(c->words, 0, 16) == cudaSuccess;
     if (!ok) {
         free_all(c->allocs);
+        free_host(c->host_allocs);
         delete c;
         return NITRO_ERR_CUDA;
     }
@@ -135,6 +143,7 @@ void nitro_conv3x3_destroy(nitro_conv* c) {
     if (!c) return;
     cudaDeviceSynchronize();
     free_all(c->allocs);
+    free_host(c->host_allocs);
     delete c;
 }
 

@@ -49,6 +49,7 @@ struct nitro_block {
     unsigned long long* sse = nullptr;
     int batch = 0;
     std::vector<void*> allocs;
+    std::vector<void*> host_allocs;
 };
 
 namespace {
@@ -72,7 +73,9 @@ bool dalloc(nitro_block* b, T** p, size_t count) {
 
 void free_all(nitro_block* b) {
     for (void* p : b->allocs) cudaFree(p);
+    for (void* p : b->host_allocs) cudaFreeHost(p);
     b->allocs.clear();
+    b->host_allocs.clear();
 }
 
 uint64_t splitmix64_at(uint64_t seed, uint64_t index) {
@@ -222,7 +225,7 @@ nitro_status nitro_init_block(const nitro_block_desc* desc, uint64_t seed, void*
          dalloc(b, &b->words, n_words(desc->n_layers)) && dalloc(b, &b->sse, 1);
     b->z64_elems = z_need;
     for (int i = 0; ok && i < desc->n_layers; ++i)
-        ok = tc_layer_init(b->L[i].tc, b->L[i].g, desc->max_batch, i > 0, b->allocs);
+        ok = tc_layer_init(b->L[i].tc, b->L[i].g, desc->max_batch, i > 0, b->allocs, b->host_allocs);
     if (!ok) {
         free_all(b);
         delete b;

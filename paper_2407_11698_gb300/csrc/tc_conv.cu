@@ -6,8 +6,8 @@
 // K-blocks (64 elements each).  Warp 0 issues TMA loads into an S-stage shared-memory ring,
 // warp 1 allocates TMEM and issues the MMAs, warps 2..17 drain the fp32 TMEM
 // accumulator every <= 16 K-blocks into int64 registers (four warps per TMEM
-// lane quadrant, each owning a quarter of the N columns).  Two TMEM accumulators
-// alternate so the MMAs of the next chunk overlap the drain of the last.
+// lane quadrant, each owning a quarter of the N columns).  Four TMEM accumulators
+// rotate so the MMAs run up to three chunks ahead of the drain.
 // Every wait on an mbarrier is bounded in time; on expiry the kernel raises
 // the TIMEOUT status bit, lets the other roles leave, frees TMEM and returns.
 #include <cuda.h>
@@ -227,13 +227,18 @@ __device__ __forceinline__ void st16_bf16(uint16_t* dst, const uint32_t* w) {
     reinterpret_cast<uint4*>(dst)[1] = make_uint4(o[4], o[5], o[6], o[7]);
 }
 
-template <int N>
+// PB = B-operand limbs carried per stage: one A tile feeds PB limb tiles of B
+// and PB accumulators, so wide B operands do not re-stream A once per limb.
+template <int N, int PB>
 struct TcCfg {
     static constexpr int A_BYTES = kBM * kBK * 2;
     static constexpr int B_BYTES = N * kBK * 2;
-    static constexpr int STAGE = A_BYTES + B_BYTES;
-    static constexpr int S = N >= 128 ? 6 : 8;
+    static constexpr int STAGE = A_BYTES + PB * B_BYTES;
+    static constexpr int S_FIT = (230912 - 1536) / STAGE;   // ~225 KB of shared memory
+    static constexpr int S = S_FIT > 9 ? 9 : S_FIT;
     static constexpr int SMEM = 1024 + S * STAGE + 512;
+    static constexpr int NBUF = (512 / (PB * N)) > 4 ? 4 : (512 / (PB * N));   // accumulator sets
+    static constexpr int TCOLS = NBUF * PB * N;                                  // 256 or 512
 };
 
 struct Tile {
@@ -253,19 +258,20 @@ __device__ __forceinline__ Tile decode_tile(const TcArgs& a, int tile) {
 // Persistent: CTA c handles tiles c, c + gridDim.x, ...; the TMA ring, the
 // MMA chunk sequence and the two TMEM accumulators run on across tiles, so
 // one tile's epilogue overlaps the next tile's loads and MMAs.
-template <int MODE, int N>
+template <int MODE, int N, int PB>
 __global__ void __launch_bounds__(kThreads, 1)
     k_tc_gemm(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
               const TcArgs args) {
-    using C = TcCfg<N>;
+    using C = TcCfg<N, PB>;
     constexpr int S = C::S;
     constexpr int NH = N / 4;            // columns per epilogue warp
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
     uint64_t* bars = reinterpret_cast<uint64_t*>(smem + S * C::STAGE);
-    // bars[0..S) full, [S..2S) empty, [2S..2S+2) tmem full, [2S+2..2S+4) tmem empty
-    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * S + 4);
+    // bars[0..S) full, [S..2S) empty, then NBUF tmem-full and NBUF tmem-empty
+    constexpr int NBUF = C::NBUF;
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * S + 2 * NBUF);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
     int8_t* relu_tab = reinterpret_cast<int8_t*>(smem + S * C::STAGE + 256);   // 255 entries
 
@@ -274,14 +280,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     auto full_bar = [&](int s) { return bar0 + 8u * s; };
     auto empty_bar = [&](int s) { return bar0 + 8u * (S + s); };
     auto tfull_bar = [&](int b) { return bar0 + 8u * (2 * S + b); };
-    auto tempty_bar = [&](int b) { return bar0 + 8u * (2 * S + 2 + b); };
+    auto tempty_bar = [&](int b) { return bar0 + 8u * (2 * S + NBUF + b); };
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < S; ++s) {
             mbar_init(full_bar(s), 1);
             mbar_init(empty_bar(s), 1);
         }
-        for (int b = 0; b < 2; ++b) {
+        for (int b = 0; b < NBUF; ++b) {
             mbar_init(tfull_bar(b), 1);
             mbar_init(tempty_bar(b), kEpiWarps);
         }
@@ -298,7 +304,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (warp == 1) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
                          smem_u32(tmem_slot)),
-                     "r"(2 * N)
+                     "r"(C::TCOLS)
                      : "memory");
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
     }
@@ -311,7 +317,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     int LB = args.limbs_b ? *args.limbs_b : 1;
     LA = LA < 1 ? 1 : (LA > kMaxLimbs ? kMaxLimbs : LA);
     LB = LB < 1 ? 1 : (LB > kMaxLimbs ? kMaxLimbs : LB);
-    const int passes = LA * LB;
+    const int NG = (LB + PB - 1) / PB;       // groups of B limbs per A limb
+    const int passes = LA * NG;
 
     if (warp == 0) {
         if (lane == 0) {
@@ -324,7 +331,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const int tb = T.mt / (args.ntx * args.nty);
                 const int x0 = tx * args.wb, y0 = ty * args.hb, b0 = tb * args.bb;
                 for (int p = 0; p < passes; ++p) {
-                    const int la = p / LB, lb = p % LB;
+                    const int la = p / NG, lb0 = (p % NG) * PB;
+                    const int nb = min(PB, LB - lb0);
                     for (int kb = T.kb0; kb < T.kb1; ++kb, ++it) {
                         const int s = it % S;
                         if (!mbar_wait(empty_bar(s), ((it / S) & 1) ^ 1, abort_flag, args.status))
@@ -332,20 +340,24 @@ __global__ void __launch_bounds__(kThreads, 1)
                         const uint32_t fb = full_bar(s);
                         const uint32_t a_dst = smem_u32(smem + s * C::STAGE);
                         const uint32_t b_dst = a_dst + C::A_BYTES;
-                        mbar_expect_tx(fb, C::STAGE);
+                        mbar_expect_tx(fb, C::A_BYTES + nb * C::B_BYTES);
                         if (MODE == TC_GEMM) {
                             tma_load_2d(a_dst, &tmA, fb, kb * kBK, T.mt * kBM);
-                            tma_load_3d(b_dst, &tmB, fb, kb * kBK, n0, lb);
+                            for (int j = 0; j < nb; ++j)
+                                tma_load_3d(b_dst + j * C::B_BYTES, &tmB, fb, kb * kBK, n0, lb0 + j);
                         } else if (MODE == TC_FWD) {
                             const int nc = args.cin_k / kBK;
                             const int t = kb / nc, cb = kb - t * nc, ky = t / 3, kx = t - 3 * ky;
                             tma_load_4d(a_dst, &tmA, fb, cb * kBK, x0 + kx - 1, y0 + ky - 1, b0);
-                            tma_load_3d(b_dst, &tmB, fb, t * args.cin_k + cb * kBK, n0, lb);
+                            for (int j = 0; j < nb; ++j)
+                                tma_load_3d(b_dst + j * C::B_BYTES, &tmB, fb, t * args.cin_k + cb * kBK,
+                                            n0, lb0 + j);
                         } else if (MODE == TC_DGRAD) {
                             const int nc = (args.Cout + kBK - 1) / kBK;
                             const int t = kb / nc, cb = kb - t * nc, ky = t / 3, kx = t - 3 * ky;
                             tma_load_5d(a_dst, &tmA, fb, cb * kBK, x0 - kx + 1, y0 - ky + 1, b0, la);
-                            tma_load_4d(b_dst, &tmB, fb, cb * kBK, n0, t, lb);
+                            for (int j = 0; j < nb; ++j)
+                                tma_load_4d(b_dst + j * C::B_BYTES, &tmB, fb, cb * kBK, n0, t, lb0 + j);
                         } else {  // TC_WGRAD: rows (tap, ci), K = (y, x, b)
                             const int nbb = (args.Bp + kBK - 1) / kBK;
                             const int pos = kb / nbb, bbk = kb - pos * nbb;
@@ -359,7 +371,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                                 tma_load_4d(a_dst + j * (64 * 128), &tmA, fb, bbk * kBK, x + kx - 1,
                                             y + ky - 1, ci0);
                             }
-                            tma_load_5d(b_dst, &tmB, fb, bbk * kBK, x, y, n0, lb);
+                            for (int j = 0; j < nb; ++j)
+                                tma_load_5d(b_dst + j * C::B_BYTES, &tmB, fb, bbk * kBK, x, y, n0, lb0 + j);
                         }
                     }
                 }
@@ -375,13 +388,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const Tile T = decode_tile(args, tile);
                 const int cpp = (T.kb1 - T.kb0 + kChunkBlocks - 1) / kChunkBlocks;
                 for (int p = 0; p < passes; ++p) {
+                    const int nb = min(PB, LB - (p % NG) * PB);
                     for (int c = 0; c < cpp; ++c, ++chunk) {
-                        const int buf = chunk & 1;
-                        if (!mbar_wait(tempty_bar(buf), ((chunk >> 1) & 1) ^ 1, abort_flag,
+                        const int buf = chunk % NBUF;
+                        if (!mbar_wait(tempty_bar(buf), ((chunk / NBUF) & 1) ^ 1, abort_flag,
                                        args.status))
                             goto mma_done;
                         tc_fence_after();
-                        const uint32_t d = tmem + (uint32_t)(buf * N);
+                        const uint32_t d = tmem + (uint32_t)(buf * PB * N);
                         const int c0 = T.kb0 + c * kChunkBlocks;
                         const int c1 = min(T.kb1, c0 + kChunkBlocks);
                         for (int kb = c0; kb < c1; ++kb, ++it) {
@@ -390,12 +404,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                                 goto mma_done;
                             tc_fence_after();
                             const uint32_t a_addr = smem_u32(smem + s * C::STAGE);
-                            const uint32_t b_addr = a_addr + C::A_BYTES;
+                            for (int j = 0; j < nb; ++j) {
+                                const uint32_t b_addr = a_addr + C::A_BYTES + j * C::B_BYTES;
 #pragma unroll
-                            for (int k = 0; k < kBK / 16; ++k)
-                                umma_bf16(d, desc_sw128(a_addr + 32 * k),
-                                          desc_sw128(b_addr + 32 * k), idesc,
-                                          (kb > c0 || k > 0) ? 1u : 0u);
+                                for (int k = 0; k < kBK / 16; ++k)
+                                    umma_bf16(d + (uint32_t)(j * N), desc_sw128(a_addr + 32 * k),
+                                              desc_sw128(b_addr + 32 * k), idesc,
+                                              (kb > c0 || k > 0) ? 1u : 0u);
+                            }
                             umma_commit(empty_bar(s));
                         }
                         umma_commit(tfull_bar(buf));
@@ -416,22 +432,27 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
             for (int i = 0; i < NH; ++i) acc[i] = 0;
             for (int p = 0; p < passes; ++p) {
-                const int shift = 8 * (p / LB + p % LB);
+                const int lb0 = (p % NG) * PB;
+                const int nb = min(PB, LB - lb0);
+                const int shift0 = 8 * (p / NG + lb0);
                 for (int c = 0; c < cpp; ++c, ++chunk) {
-                    const int buf = chunk & 1;
-                    if (!mbar_wait(tfull_bar(buf), (chunk >> 1) & 1, abort_flag, args.status))
+                    const int buf = chunk % NBUF;
+                    if (!mbar_wait(tfull_bar(buf), (chunk / NBUF) & 1, abort_flag, args.status))
                         goto epi_done;
                     tc_fence_after();
-                    const uint32_t base =
-                        tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(buf * N + half * NH);
-                    uint32_t r[NH];
+                    for (int jb = 0; jb < nb; ++jb) {
+                        const uint32_t base = tmem + ((uint32_t)(32 * q) << 16) +
+                                              (uint32_t)((buf * PB + jb) * N + half * NH);
+                        const int shift = shift0 + 8 * jb;
+                        uint32_t r[NH];
 #pragma unroll
-                    for (int j = 0; j < NH / 16; ++j) tmem_ld16_nowait(base + 16 * j, r + 16 * j);
-                    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+                        for (int j = 0; j < NH / 16; ++j) tmem_ld16_nowait(base + 16 * j, r + 16 * j);
+                        asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 #pragma unroll
-                    for (int i = 0; i < NH; ++i) {
-                        const int v = __float2int_rz(__uint_as_float(r[i]));   // exact integer
-                        acc[i] += (uint64_t)(int64_t)v << shift;
+                        for (int i = 0; i < NH; ++i) {
+                            const int v = __float2int_rz(__uint_as_float(r[i]));   // exact integer
+                            acc[i] += (uint64_t)(int64_t)v << shift;
+                        }
                     }
                     tc_fence_before();
                     __syncwarp();
@@ -654,7 +675,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncthreads();
     if (warp == 1) {
         tc_fence_after();
-        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(2 * N)
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(C::TCOLS)
                      : "memory");
     }
 }
@@ -838,26 +859,31 @@ int sm_count() {
     return n;
 }
 
-template <int MODE, int N>
+template <int MODE, int N, int PB>
 cudaError_t launch_gemm(const CUtensorMap& a, const CUtensorMap& b, const TcArgs& args,
                         cudaStream_t s) {
-    using C = TcCfg<N>;
+    using C = TcCfg<N, PB>;
     static bool attr_set = false;
     if (!attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(k_tc_gemm<MODE, N>,
+        cudaError_t e = cudaFuncSetAttribute(k_tc_gemm<MODE, N, PB>,
                                              cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
         if (e != cudaSuccess) return e;
         attr_set = true;
     }
     const int grid = args.total_tiles < sm_count() ? args.total_tiles : sm_count();
-    k_tc_gemm<MODE, N><<<grid, kThreads, C::SMEM, s>>>(a, b, args);
+    k_tc_gemm<MODE, N, PB><<<grid, kThreads, C::SMEM, s>>>(a, b, args);
     return cudaGetLastError();
 }
 
+// Tile width n and B limbs per stage: interleave when the (last seen) limb
+// count of B is above one.  Any choice is exact; it only changes speed.
 template <int MODE>
-cudaError_t launch_gemm_n(int n, const CUtensorMap& a, const CUtensorMap& b, const TcArgs& args,
-                          cudaStream_t s) {
-    return n == 128 ? launch_gemm<MODE, 128>(a, b, args, s) : launch_gemm<MODE, 64>(a, b, args, s);
+cudaError_t launch_gemm_n(int n, int limbs_hint, const CUtensorMap& a, const CUtensorMap& b,
+                          const TcArgs& args, cudaStream_t s) {
+    const bool wide = limbs_hint > 1;
+    if (n == 128)
+        return wide ? launch_gemm<MODE, 128, 2>(a, b, args, s) : launch_gemm<MODE, 128, 1>(a, b, args, s);
+    return wide ? launch_gemm<MODE, 64, 4>(a, b, args, s) : launch_gemm<MODE, 64, 1>(a, b, args, s);
 }
 
 int pick_n(int cols) { return cols % 128 == 0 ? 128 : 64; }
@@ -889,7 +915,7 @@ inline int round_up(int v, int m) { return (v + m - 1) / m * m; }
 }  // namespace
 
 bool tc_layer_init(TcLayer& t, const LayerGeom& g, int max_batch, bool has_dgrad,
-                   std::vector<void*>& allocs) {
+                   std::vector<void*>& allocs, std::vector<void*>& host_allocs) {
     t = TcLayer();
     if (g.kind != NITRO_CONV3X3 || max_batch < 1 || !encode_fn()) return true;
     // Narrow inputs (Cin < 32, e.g. image channels) stay on the CUDA-core
@@ -913,6 +939,15 @@ bool tc_layer_init(TcLayer& t, const LayerGeom& g, int max_batch, bool has_dgrad
     if (ok && t.fwd) ok = dalloc(allocs, &t.w_planes, (size_t)kMaxLimbs * nwk);
     if (ok && t.dgrad) ok = dalloc(allocs, &t.wt_planes, (size_t)kMaxLimbs * nw);
     if (ok) ok = cudaMemset(t.limbs, 0, 2 * sizeof(int)) == cudaSuccess;
+    if (ok) {
+        void* h = nullptr;
+        ok = cudaMallocHost(&h, 2 * sizeof(int)) == cudaSuccess;
+        if (ok) {
+            host_allocs.push_back(h);
+            t.limbs_host = static_cast<int*>(h);
+            t.limbs_host[0] = t.limbs_host[1] = 1;
+        }
+    }
     if (ok && t.fwd) ok = cudaMemset(t.w_planes, 0, (size_t)kMaxLimbs * nwk * 2) == cudaSuccess;
     return ok;
 }
@@ -926,7 +961,10 @@ cudaError_t tc_refresh_weights(TcLayer& t, const LayerGeom& g, const int32_t* W,
         k_pack_weights<<<grid1d(n), 256, 0, s>>>(W, g.cout, g.cin, t.cin_k, maxabs_w, t.w_planes,
                                                  t.wt_planes, t.limbs);
     }
-    return cudaGetLastError();
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    // host copy of the limb count, read later as a kernel-variant hint only
+    return cudaMemcpyAsync(t.limbs_host, t.limbs, sizeof(int), cudaMemcpyDeviceToHost, s);
 }
 
 cudaError_t tc_pack_input(TcLayer& t, const LayerGeom& g, const int8_t* x, int batch,
@@ -1001,7 +1039,7 @@ cudaError_t tc_conv_forward(TcLayer& t, const LayerGeom& g, int batch, int64_t* 
         return cudaErrorInvalidValue;
     const double ops = 2.0 * batch * g.h * g.w * g.cout * 9.0 * g.cin;
     ProfScope ps(K_TC_CONV_FWD, s, ops, 0.0);
-    cudaError_t e = launch_gemm_n<TC_FWD>(n, ma, mb, a, s);
+    cudaError_t e = launch_gemm_n<TC_FWD>(n, t.limbs_host[0], ma, mb, a, s);
     if (e == cudaSuccess) {
         *done = true;
         *fused = a.fuse != 0;
@@ -1034,7 +1072,7 @@ cudaError_t tc_pack_delta(TcLayer& t, const LayerGeom& g, const int32_t* delta,
         cudaError_t e = cudaGetLastError();
         if (e != cudaSuccess) return e;
     }
-    return cudaSuccess;
+    return cudaMemcpyAsync(t.limbs_host + 1, t.limbs + 1, sizeof(int), cudaMemcpyDeviceToHost, s);
 }
 
 cudaError_t tc_conv_wgrad(TcLayer& t, const LayerGeom& g, const int32_t* delta,
@@ -1086,7 +1124,7 @@ cudaError_t tc_conv_wgrad(TcLayer& t, const LayerGeom& g, const int32_t* delta,
     }
     const double ops = 2.0 * batch * hw * g.cout * 9.0 * g.cin;
     ProfScope ps(K_TC_CONV_WGRAD, s, ops, 0.0);
-    cudaError_t e = launch_gemm_n<TC_WGRAD>(n, ma, mb, a, s);
+    cudaError_t e = launch_gemm_n<TC_WGRAD>(n, t.limbs_host[1], ma, mb, a, s);
     if (e == cudaSuccess) *done = true;
     return e;
 }
@@ -1146,7 +1184,7 @@ cudaError_t tc_conv_dgrad(TcLayer& t, const LayerGeom& g, int batch, int64_t* g6
         return cudaErrorInvalidValue;
     const double ops = 2.0 * batch * g.h * g.w * g.cin * 9.0 * g.cout;
     ProfScope ps(K_TC_CONV_DGRAD, s, ops, 0.0);
-    cudaError_t e = launch_gemm_n<TC_DGRAD>(n, ma, mb, a, s);
+    cudaError_t e = launch_gemm_n<TC_DGRAD>(n, t.limbs_host[0], ma, mb, a, s);
     if (e == cudaSuccess) {
         *done = true;
         *fused = a.fuse != 0;
@@ -1218,7 +1256,7 @@ cudaError_t tc_gemm_run(const uint16_t* a_bf16, const uint16_t* b_planes, int M,
     if (!make_map(&ma, a_bf16, 2, da, sa, ba) || !make_map(&mb, b_planes, 3, db, sb, bb))
         return cudaErrorInvalidValue;
     ProfScope ps(K_TC_GEMM, s, 2.0 * M * N * (double)K, 0.0);
-    return launch_gemm_n<TC_GEMM>(n, ma, mb, a, s);
+    return launch_gemm_n<TC_GEMM>(n, 1, ma, mb, a, s);
 }
 
 }  // namespace nitro

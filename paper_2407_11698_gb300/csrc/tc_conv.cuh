@@ -41,13 +41,17 @@ struct TcLayer {
     uint16_t* w_planes = nullptr;
     uint16_t* wt_planes = nullptr;
     int* limbs = nullptr;   // device: [0] weight limbs, [1] delta limbs
+    // pinned host copy of `limbs`, refreshed asynchronously after each split;
+    // possibly stale, used only to pick a kernel variant (any choice is exact)
+    int* limbs_host = nullptr;
 };
 
 // Decides which passes of a layer run on tensor cores and allocates their
-// buffers (recorded in `allocs`).  `has_dgrad`: the layer is not the block's
-// first, so its input gradient is needed.
+// buffers (device memory recorded in `allocs`, pinned host memory in
+// `host_allocs`).  `has_dgrad`: the layer is not the block's first, so its
+// input gradient is needed.
 bool tc_layer_init(TcLayer& t, const LayerGeom& g, int max_batch, bool has_dgrad,
-                   std::vector<void*>& allocs);
+                   std::vector<void*>& allocs, std::vector<void*>& host_allocs);
 
 // Re-splits the layer's int32 weights into limb planes (after init, an update
 // or a checkpoint load); the limb count follows *maxabs_w.
