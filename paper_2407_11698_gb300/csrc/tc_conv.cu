@@ -133,10 +133,25 @@ __device__ __forceinline__ uint64_t desc_sw128(uint32_t saddr) {
     return d;
 }
 
-// Instruction descriptor: kind::f16, A = B = bf16, D = f32, both K-major.
-__host__ __device__ constexpr uint32_t idesc_bf16(int m, int n) {
-    return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(n >> 3) << 17) |
-           ((uint32_t)(m >> 4) << 24);
+// MN-major operand, 128-byte swizzle: rows of 128 bytes run along K, each
+// holding 64 consecutive M (or N) elements; 64-element blocks along M/N lie
+// `mn_stride` bytes apart (leading byte offset), 8-row groups along K 1024
+// bytes apart (stride byte offset).
+__device__ __forceinline__ uint64_t desc_sw128_mn(uint32_t saddr, uint32_t mn_stride) {
+    uint64_t d = 0;
+    d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);
+    d |= (uint64_t)((mn_stride >> 4) & 0x3FFFu) << 16;
+    d |= (uint64_t)(1024 >> 4) << 32;
+    d |= (uint64_t)1 << 46;
+    d |= (uint64_t)2 << 61;
+    return d;
+}
+
+// Instruction descriptor: kind::f16, A = B = bf16, D = f32; A and B K-major
+// unless mn (bits 15 and 16: MN-major).
+__host__ __device__ constexpr uint32_t idesc_bf16(int m, int n, bool mn = false) {
+    return (1u << 4) | (1u << 7) | (1u << 10) | (mn ? (3u << 15) : 0u) |
+           ((uint32_t)(n >> 3) << 17) | ((uint32_t)(m >> 4) << 24);
 }
 
 __device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc,
@@ -358,21 +373,26 @@ __global__ void __launch_bounds__(kThreads, 1)
                             tma_load_5d(a_dst, &tmA, fb, cb * kBK, x0 - kx + 1, y0 - ky + 1, b0, la);
                             for (int j = 0; j < nb; ++j)
                                 tma_load_4d(b_dst + j * C::B_BYTES, &tmB, fb, cb * kBK, n0, t, lb0 + j);
-                        } else {  // TC_WGRAD: rows (tap, ci), K = (y, x, b)
-                            const int nbb = (args.Bp + kBK - 1) / kBK;
-                            const int pos = kb / nbb, bbk = kb - pos * nbb;
-                            const int y = pos / args.W, x = pos - y * args.W;
+                        } else {  // TC_WGRAD: rows (tap, ci), K = a 64-pixel box (wb x hb)
+                            // of one image; both operands MN-major from the NHWC
+                            // copies (channels contiguous), the tap shift on x / y.
+                            const int xt = kb % args.ntx, yt = (kb / args.ntx) % args.nty;
+                            const int bk = kb / (args.ntx * args.nty);
+                            const int px = xt * args.wb, py = yt * args.hb;
 #pragma unroll
                             for (int j = 0; j < 2; ++j) {
                                 const int m = T.mt * kBM + j * 64;
                                 int t = m / args.cin_k, ci0 = m - t * args.cin_k;
                                 if (t >= 9) { t = 0; ci0 = args.cin_k; }   // past the last tap: zeros
                                 const int ky = t / 3, kx = t - 3 * ky;
-                                tma_load_4d(a_dst + j * (64 * 128), &tmA, fb, bbk * kBK, x + kx - 1,
-                                            y + ky - 1, ci0);
+                                tma_load_4d(a_dst + j * (64 * 128), &tmA, fb, ci0, px + kx - 1,
+                                            py + ky - 1, bk);
                             }
                             for (int j = 0; j < nb; ++j)
-                                tma_load_5d(b_dst + j * C::B_BYTES, &tmB, fb, bbk * kBK, x, y, n0, lb0 + j);
+#pragma unroll
+                                for (int h = 0; h < N / 64; ++h)
+                                    tma_load_5d(b_dst + j * C::B_BYTES + h * (64 * 128), &tmB, fb,
+                                                n0 + 64 * h, px, py, bk, lb0 + j);
                         }
                     }
                 }
@@ -382,7 +402,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     } else if (warp == 1) {
         if (lane == 0) {
             // ---------------- MMA issuer
-            constexpr uint32_t idesc = idesc_bf16(kBM, N);
+            constexpr uint32_t idesc = idesc_bf16(kBM, N, MODE == TC_WGRAD);
             int it = 0, chunk = 0;
             for (int tile = blockIdx.x; tile < args.total_tiles; tile += gridDim.x) {
                 const Tile T = decode_tile(args, tile);
@@ -407,10 +427,18 @@ __global__ void __launch_bounds__(kThreads, 1)
                             for (int j = 0; j < nb; ++j) {
                                 const uint32_t b_addr = a_addr + C::A_BYTES + j * C::B_BYTES;
 #pragma unroll
-                                for (int k = 0; k < kBK / 16; ++k)
-                                    umma_bf16(d + (uint32_t)(j * N), desc_sw128(a_addr + 32 * k),
-                                              desc_sw128(b_addr + 32 * k), idesc,
+                                for (int k = 0; k < kBK / 16; ++k) {
+                                    // K-major: a K-step of 16 is 32 bytes along each row;
+                                    // MN-major: 16 rows, two 1024-byte row groups
+                                    const uint64_t da = MODE == TC_WGRAD
+                                        ? desc_sw128_mn(a_addr + 2048 * k, 64 * 128)
+                                        : desc_sw128(a_addr + 32 * k);
+                                    const uint64_t db = MODE == TC_WGRAD
+                                        ? desc_sw128_mn(b_addr + 2048 * k, N > 64 ? 64 * 128 : 0)
+                                        : desc_sw128(b_addr + 32 * k);
+                                    umma_bf16(d + (uint32_t)(j * N), da, db, idesc,
                                               (kb > c0 || k > 0) ? 1u : 0u);
+                                }
                             }
                             umma_commit(empty_bar(s));
                         }
@@ -701,49 +729,6 @@ __global__ void k_pack_act_nhwc(const int8_t* __restrict__ x, int64_t P, int C, 
     }
 }
 
-// [B][HW][C] int (int8, or int32 split into limbs) -> [L][C][HW][Bp] bf16,
-// zero for b >= B.  Tile: one pixel, 32 channels x 64 batch entries; each
-// thread writes two consecutive batch entries per plane (128-byte warp rows).
-// Block (0,0,0) thread 0 records the limb count in *limbs_out if given.
-template <typename T>
-__global__ void __launch_bounds__(256) k_pack_transposed(const T* __restrict__ x, int B, int HW,
-                                                         int C, int Bp, const uint32_t* maxabs,
-                                                         uint16_t* __restrict__ out,
-                                                         int* limbs_out) {
-    __shared__ int tile[32][65];
-    const int pos = blockIdx.x;
-    const int c0 = blockIdx.y * 32, b0 = blockIdx.z * 64;
-    const int L = maxabs ? limb_count(*maxabs) : 1;
-    if (limbs_out && blockIdx.x == 0 && blockIdx.y == 0 && blockIdx.z == 0 && threadIdx.x == 0 &&
-        threadIdx.y == 0)
-        *limbs_out = L;
-    for (int k = threadIdx.y; k < 64; k += 8) {      // read: b = b0 + k, c = c0 + tx
-        const int b = b0 + k, c = c0 + threadIdx.x;
-        tile[threadIdx.x][k] = (b < B && c < C) ? (int)x[((int64_t)b * HW + pos) * C + c] : 0;
-    }
-    __syncthreads();
-    const int64_t plane = (int64_t)C * HW * Bp;
-    for (int k = threadIdx.y; k < 32; k += 8) {      // write: c = c0 + k, b = b0 + 2 tx (+1)
-        const int c = c0 + k, b = b0 + 2 * threadIdx.x;
-        if (c >= C || b >= Bp) continue;
-        int64_t v0 = tile[k][2 * threadIdx.x], v1 = tile[k][2 * threadIdx.x + 1];
-        uint32_t* o = reinterpret_cast<uint32_t*>(out + ((int64_t)c * HW + pos) * Bp + b);
-        for (int l = 0; l < L; ++l) {
-            int d0, d1;
-            if (l < L - 1) {
-                d0 = (int)(((v0 + 128) & 255) - 128);
-                d1 = (int)(((v1 + 128) & 255) - 128);
-                v0 = (v0 - d0) >> 8;
-                v1 = (v1 - d1) >> 8;
-            } else {
-                d0 = (int)v0;
-                d1 = (int)v1;
-            }
-            o[l * (plane / 2)] = (uint32_t)bf16_bits(d0) | ((uint32_t)bf16_bits(d1) << 16);
-        }
-    }
-}
-
 // int32 delta NHWC (n values, n % 8 == 0) -> limb planes [L][n], eight values
 // per thread and one 16-byte store per plane; records the limb count.
 __global__ void __launch_bounds__(256) k_pack_delta_nhwc(const int32_t* __restrict__ d, int64_t n,
@@ -923,19 +908,17 @@ bool tc_layer_init(TcLayer& t, const LayerGeom& g, int max_batch, bool has_dgrad
     const bool pix_ok = g.h >= 8 && g.w >= 8;
     const bool wide = g.cin >= 32;
     t.fwd = pix_ok && wide;
-    t.wgrad = wide;
+    t.wgrad = wide && g.cout % 8 == 0;
     t.dgrad = has_dgrad && pix_ok && g.cout % 8 == 0;
-    t.max_bp = round_up(max_batch, 8);
     t.cin8 = round_up(g.cin, 8);
     t.cin_k = round_up(g.cin, 64);
     const size_t hw = (size_t)g.h * g.w;
     const size_t nw = (size_t)g.cout * 9 * g.cin;
     const size_t nwk = (size_t)g.cout * 9 * t.cin_k;
     bool ok = dalloc(allocs, &t.limbs, 2);
-    if (ok && t.fwd) ok = dalloc(allocs, &t.act_nhwc, (size_t)max_batch * hw * t.cin8);
-    if (ok && t.wgrad) ok = dalloc(allocs, &t.act_t, (size_t)g.cin * hw * t.max_bp);
-    if (ok && t.wgrad) ok = dalloc(allocs, &t.d_t, (size_t)kMaxLimbs * g.cout * hw * t.max_bp);
-    if (ok && t.dgrad) ok = dalloc(allocs, &t.d_nhwc, (size_t)kMaxLimbs * max_batch * hw * g.cout);
+    if (ok && (t.fwd || t.wgrad)) ok = dalloc(allocs, &t.act_nhwc, (size_t)max_batch * hw * t.cin8);
+    if (ok && (t.wgrad || t.dgrad))
+        ok = dalloc(allocs, &t.d_nhwc, (size_t)kMaxLimbs * max_batch * hw * g.cout);
     if (ok && t.fwd) ok = dalloc(allocs, &t.w_planes, (size_t)kMaxLimbs * nwk);
     if (ok && t.dgrad) ok = dalloc(allocs, &t.wt_planes, (size_t)kMaxLimbs * nw);
     if (ok) ok = cudaMemset(t.limbs, 0, 2 * sizeof(int)) == cudaSuccess;
@@ -969,24 +952,11 @@ cudaError_t tc_refresh_weights(TcLayer& t, const LayerGeom& g, const int32_t* W,
 
 cudaError_t tc_pack_input(TcLayer& t, const LayerGeom& g, const int8_t* x, int batch,
                           bool nhwc_done, cudaStream_t s) {
-    if (batch <= 0 || (!t.fwd && !t.wgrad)) return cudaSuccess;
-    const int hw = g.h * g.w;
-    if (t.fwd && !nhwc_done) {
-        const int64_t P = (int64_t)batch * hw;
-        ProfScope ps(K_TC_PACK, s, 0.0, (double)P * (g.cin + 2 * t.cin8));
-        k_pack_act_nhwc<<<grid1d(P * t.cin8), 256, 0, s>>>(x, P, g.cin, t.cin8, t.act_nhwc);
-        cudaError_t e = cudaGetLastError();
-        if (e != cudaSuccess) return e;
-    }
-    if (t.wgrad) {
-        const int bp = round_up(batch, 8);
-        dim3 grid(hw, (g.cin + 31) / 32, (bp + 63) / 64);
-        ProfScope ps(K_TC_PACK, s, 0.0, (double)batch * hw * g.cin * 3);
-        k_pack_transposed<int8_t><<<grid, dim3(32, 8), 0, s>>>(x, batch, hw, g.cin, bp, nullptr,
-                                                               t.act_t, nullptr);
-        return cudaGetLastError();
-    }
-    return cudaSuccess;
+    if (batch <= 0 || !t.act_nhwc || nhwc_done) return cudaSuccess;
+    const int64_t P = (int64_t)batch * g.h * g.w;
+    ProfScope ps(K_TC_PACK, s, 0.0, (double)P * (g.cin + 2 * t.cin8));
+    k_pack_act_nhwc<<<grid1d(P * t.cin8), 256, 0, s>>>(x, P, g.cin, t.cin8, t.act_nhwc);
+    return cudaGetLastError();
 }
 
 cudaError_t tc_conv_forward(TcLayer& t, const LayerGeom& g, int batch, int64_t* z,
@@ -1050,28 +1020,15 @@ cudaError_t tc_conv_forward(TcLayer& t, const LayerGeom& g, int batch, int64_t* 
 cudaError_t tc_pack_delta(TcLayer& t, const LayerGeom& g, const int32_t* delta,
                           const uint32_t* maxabs_delta, int batch, cudaStream_t s) {
     if (batch <= 0 || (!t.wgrad && !t.dgrad)) return cudaSuccess;
-    const int hw = g.h * g.w;
-    const int bp = round_up(batch, 8);
-    // limb planes of delta in the layouts the tensor-core passes read; the
-    // first pack launch also records the limb count for the GEMMs
-    bool counted = false;
-    if (t.dgrad) {
-        const int64_t n = (int64_t)batch * hw * g.cout;   // cout % 8 == 0 for dgrad
+    // limb planes of delta (NHWC, read by the wgrad and dgrad passes); the
+    // launch also records the limb count for the GEMMs
+    const int64_t n = (int64_t)batch * g.h * g.w * g.cout;   // cout % 8 == 0
+    {
         ProfScope ps(K_TC_PACK, s, 0.0, (double)n * 4 * 2);
-        k_pack_delta_nhwc<<<grid1d(n / 8), 256, 0, s>>>(delta, n, maxabs_delta, t.d_nhwc,
-                                                         t.limbs + 1);
-        cudaError_t e = cudaGetLastError();
-        if (e != cudaSuccess) return e;
-        counted = true;
+        k_pack_delta_nhwc<<<grid1d(n / 8), 256, 0, s>>>(delta, n, maxabs_delta, t.d_nhwc, t.limbs + 1);
     }
-    if (t.wgrad) {
-        dim3 grid(hw, (g.cout + 31) / 32, (bp + 63) / 64);
-        ProfScope ps(K_TC_PACK, s, 0.0, (double)batch * hw * g.cout * 4 * 2);
-        k_pack_transposed<int32_t><<<grid, dim3(32, 8), 0, s>>>(
-            delta, batch, hw, g.cout, bp, maxabs_delta, t.d_t, counted ? nullptr : t.limbs + 1);
-        cudaError_t e = cudaGetLastError();
-        if (e != cudaSuccess) return e;
-    }
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
     return cudaMemcpyAsync(t.limbs_host + 1, t.limbs + 1, sizeof(int), cudaMemcpyDeviceToHost, s);
 }
 
@@ -1084,16 +1041,20 @@ cudaError_t tc_conv_wgrad(TcLayer& t, const LayerGeom& g, const int32_t* delta,
     if (pe != cudaSuccess) return pe;
     if (!t.wgrad) return cudaSuccess;
     const int hw = g.h * g.w;
-    const int bp = round_up(batch, 8);
     TcArgs a{};
-    a.B = batch; a.H = g.h; a.W = g.w; a.Cin = g.cin; a.Cout = g.cout; a.Bp = bp;
+    a.B = batch; a.H = g.h; a.W = g.w; a.Cin = g.cin; a.Cout = g.cout;
+    a.Bp = round_up(batch, 8);
     a.cin_k = t.cin_k;
-    a.ntx = a.nty = 1; a.wb = a.hb = a.bb = 1;
+    // K-blocks: 64-pixel boxes (wb x hb) of one image
+    a.wb = g.w <= 8 ? 8 : (g.w <= 16 ? 16 : (g.w <= 32 ? 32 : 64));
+    a.hb = 64 / a.wb;
+    a.bb = 1;
+    a.ntx = (g.w + a.wb - 1) / a.wb;
+    a.nty = (g.h + a.hb - 1) / a.hb;
     const int n = pick_n(g.cout);
     a.tiles_m = (9 * t.cin_k + kBM - 1) / kBM;
     a.tiles_n = (g.cout + n - 1) / n;
-    const int nbb = (bp + kBK - 1) / kBK;
-    a.kb_total = hw * nbb;
+    a.kb_total = batch * a.ntx * a.nty;
     // split K so that about one wave of CTAs runs, each with >= one exact chunk
     const int tiles = a.tiles_m * a.tiles_n;
     int splits = (sm_count() + tiles - 1) / tiles;
@@ -1109,14 +1070,15 @@ cudaError_t tc_conv_wgrad(TcLayer& t, const LayerGeom& g, const int32_t* delta,
     a.status = status;
     a.atomic_out = splits > 1;
     CUtensorMap ma, mb;
-    const uint64_t da[4] = {(uint64_t)bp, (uint64_t)g.w, (uint64_t)g.h, (uint64_t)g.cin};
-    const uint64_t sa[4] = {(uint64_t)bp, (uint64_t)g.w * bp, (uint64_t)hw * bp,
-                            (uint64_t)g.cout * hw * bp};
-    const uint32_t ba[4] = {64, 1, 1, 64};
-    const uint64_t db[5] = {(uint64_t)bp, (uint64_t)g.w, (uint64_t)g.h, (uint64_t)g.cout,
+    const uint64_t da[4] = {(uint64_t)t.cin8, (uint64_t)g.w, (uint64_t)g.h, (uint64_t)batch};
+    const uint64_t sa[3] = {(uint64_t)t.cin8, (uint64_t)g.w * t.cin8, (uint64_t)hw * t.cin8};
+    const uint32_t ba[4] = {64, (uint32_t)a.wb, (uint32_t)a.hb, 1};
+    const uint64_t db[5] = {(uint64_t)g.cout, (uint64_t)g.w, (uint64_t)g.h, (uint64_t)batch,
                             (uint64_t)kMaxLimbs};
-    const uint32_t bb[5] = {64, 1, 1, (uint32_t)n, 1};
-    if (!make_map(&ma, t.act_t, 4, da, sa, ba) || !make_map(&mb, t.d_t, 5, db, sa, bb))
+    const uint64_t sb[4] = {(uint64_t)g.cout, (uint64_t)g.w * g.cout, (uint64_t)hw * g.cout,
+                            (uint64_t)batch * hw * g.cout};
+    const uint32_t bb[5] = {64, (uint32_t)a.wb, (uint32_t)a.hb, 1, 1};
+    if (!make_map(&ma, t.act_nhwc, 4, da, sa, ba) || !make_map(&mb, t.d_nhwc, 5, db, sb, bb))
         return cudaErrorInvalidValue;
     if (a.atomic_out) {
         cudaError_t e = cudaMemsetAsync(dW, 0, sizeof(int64_t) * 9 * g.cin * g.cout, s);

@@ -9,15 +9,13 @@
 // are combined in int64 (modulo 2^64) with shifts 8 (la + lb).
 //
 // Layouts (bf16, limb planes outermost):
-//   act_nhwc  [B][H][W][Cin8]          forward A  (pixels x taps*channels)
-//   act_t     [Cin][H][W][Bp]          wgrad A    ((tap, ci) x (y, x, b))
-//   d_nhwc    [L][B][H][W][Cout]       dgrad A
-//   d_t       [L][Cout][H][W][Bp]      wgrad B
+//   act_nhwc  [B][H][W][Cin8]          forward A (K-major: pixels x taps*channels)
+//                                      and wgrad A (MN-major: (tap, ci) x pixels)
+//   d_nhwc    [L][B][H][W][Cout]       dgrad A (K-major) and wgrad B (MN-major)
 //   w_planes  [L][Cout][9][Cin64]      forward B
 //   wt_planes [L][9][Cin][Cout]        dgrad B
-// Bp = batch rounded up to 8 and Cin8 = Cin rounded up to 8 (TMA strides are
-// multiples of 16 bytes); Cin64 = Cin rounded up to 64 so that a K-block of
-// the forward never spans two taps.  Padding holds zeros; tiles that run past
+// Cin8 = Cin rounded up to 8 (TMA strides are multiples of 16 bytes); Cin64 =
+// Cin rounded up to 64 so that a K-block of the forward never spans two taps.  Padding holds zeros; tiles that run past
 // a tensor edge read zeros (TMA out-of-bounds fill) and skip their stores.
 #pragma once
 
@@ -31,13 +29,10 @@ constexpr int kMaxLimbs = 4;
 
 struct TcLayer {
     bool fwd = false, wgrad = false, dgrad = false;   // passes that run on tcgen05
-    int max_bp = 0;   // batch rounded up to 8
     int cin8 = 0;     // channels of the NHWC bf16 input copy (Cin rounded up to 8)
     int cin_k = 0;    // channels per tap in the forward K index (Cin rounded up to 64)
     uint16_t* act_nhwc = nullptr;
-    uint16_t* act_t = nullptr;
     uint16_t* d_nhwc = nullptr;
-    uint16_t* d_t = nullptr;
     uint16_t* w_planes = nullptr;
     uint16_t* wt_planes = nullptr;
     int* limbs = nullptr;   // device: [0] weight limbs, [1] delta limbs
@@ -58,8 +53,8 @@ bool tc_layer_init(TcLayer& t, const LayerGeom& g, int max_batch, bool has_dgrad
 cudaError_t tc_refresh_weights(TcLayer& t, const LayerGeom& g, const int32_t* W,
                                const uint32_t* maxabs_w, cudaStream_t s);
 
-// bf16 copies of the layer's int8 input for the forward and wgrad operands
-// (the forward copy is skipped when the previous layer's epilogue wrote it).
+// bf16 NHWC copy of the layer's int8 input for the forward and wgrad operands
+// (skipped when the previous layer's epilogue wrote it).
 cudaError_t tc_pack_input(TcLayer& t, const LayerGeom& g, const int8_t* x, int batch,
                           bool nhwc_done, cudaStream_t s);
 
@@ -81,8 +76,8 @@ cudaError_t tc_conv_forward(TcLayer& t, const LayerGeom& g, int batch, int64_t* 
                             const TcFwdOut* fo, uint32_t* status, cudaStream_t s, bool* done,
                             bool* fused);
 
-// Splits delta into limb planes in the layouts the wgrad and dgrad passes read
-// (limb count from *maxabs_delta, recorded on the device for the GEMMs).
+// Splits delta into NHWC limb planes for the wgrad and dgrad passes (limb
+// count from *maxabs_delta, recorded on the device for the GEMMs).
 cudaError_t tc_pack_delta(TcLayer& t, const LayerGeom& g, const int32_t* delta,
                           const uint32_t* maxabs_delta, int batch, cudaStream_t s);
 
