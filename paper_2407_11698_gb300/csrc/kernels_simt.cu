@@ -7,6 +7,8 @@
 // These serve the layers whose contraction is too narrow for the tensor-core
 // path (first layers with 1 or 3 input channels, MLP layers, learning layers
 // with G = 10 outputs) and are the exactness reference on the device.
+#include <cuda_bf16.h>
+
 #include "nitro_internal.cuh"
 #include "prof.cuh"
 
@@ -404,6 +406,158 @@ __global__ void k_integersgd(SgdBatch bt) {
     }
 }
 
+// ---------------------------------------------------------------------------
+// Narrow-input 3x3 conv (Cin <= 8, e.g. image channels): forward with the
+// NITRO-Scaling / NITRO-ReLU / max-pool epilogue fused, one thread per
+// (pooling window or pixel, 16 output channels).  The weights sit in shared
+// memory; sums are exact int64.
+// ---------------------------------------------------------------------------
+constexpr int kSmallCin = 8;
+constexpr int kSmallCo = 16;
+
+struct SmallFwdArgs {
+    const int8_t* x;       // [B][H][W][Cin]
+    const int32_t* w;      // [Cout][3][3][Cin]
+    int B, H, W, Cin, Cout, pool, oh, ow;
+    FloorDiv32 sf32;       // divide by 9 * Cin (after >> 8)
+    int64_t z_hi, z_lo;    // saturation thresholds 128 SF and -127 SF
+    FloorDiv alpha;
+    int mu;
+    int8_t* act;           // [B][oh][ow][Cout]
+    int8_t* out2;
+    int8_t* region;        // [B][H][W][Cout]
+    int8_t* argmax;
+    uint16_t* next_nhwc;   // bf16 copy of act, or null
+};
+
+__global__ void __launch_bounds__(256) k_conv_small_fwd(const SmallFwdArgs a) {
+    extern __shared__ int32_t wsm[];                 // Cout * 9 * Cin
+    __shared__ int8_t relu_tab[256];
+    const int nw = a.Cout * 9 * a.Cin;
+    for (int i = threadIdx.x; i < nw; i += blockDim.x) wsm[i] = a.w[i];
+    if (threadIdx.x < 255) relu_tab[threadIdx.x] = (int8_t)relu_value((int64_t)threadIdx.x - 127, a.alpha, a.mu);
+    __syncthreads();
+    const int step = a.pool ? 2 : 1;
+    const int wy_n = (a.H + step - 1) / step, wx_n = (a.W + step - 1) / step;
+    const int ngrp = a.Cout / kSmallCo;
+    const int64_t total = (int64_t)a.B * wy_n * wx_n * ngrp;
+    for (int64_t idx = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; idx < total;
+         idx += (int64_t)gridDim.x * blockDim.x) {
+        const int grp = (int)(idx % ngrp);
+        int64_t r = idx / ngrp;
+        const int wx = (int)(r % wx_n);
+        r /= wx_n;
+        const int wy = (int)(r % wy_n);
+        const int b = (int)(r / wy_n);
+        const int co0 = grp * kSmallCo;
+        int8_t vals[4][kSmallCo];
+        bool valid[4];
+        for (int k = 0; k < step * step; ++k) {
+            const int y = wy * step + (k >> 1), x = wx * step + (k & 1);
+            valid[k] = y < a.H && x < a.W;
+            if (!valid[k]) continue;
+            // 3x3 x Cin input patch, zero outside the image
+            int32_t patch[9 * kSmallCin];
+            for (int t = 0; t < 9; ++t) {
+                const int iy = y + t / 3 - 1, ix = x + t % 3 - 1;
+                const bool in = iy >= 0 && iy < a.H && ix >= 0 && ix < a.W;
+                const int8_t* src = a.x + (((int64_t)b * a.H + iy) * a.W + ix) * a.Cin;
+                for (int c = 0; c < a.Cin; ++c) patch[t * a.Cin + c] = in ? (int32_t)src[c] : 0;
+            }
+            const int K = 9 * a.Cin;
+            uint32_t rg[kSmallCo / 4] = {0, 0, 0, 0};
+            for (int j = 0; j < kSmallCo; ++j) {
+                const int32_t* wr = wsm + (co0 + j) * K;
+                int64_t z = 0;
+                for (int q = 0; q < K; ++q) z += (int64_t)wr[q] * patch[q];
+                int reg, val;
+                if (z >= a.z_hi) { reg = 3; val = relu_tab[254]; }
+                else if (z < a.z_lo) { reg = 0; val = relu_tab[0]; }
+                else {
+                    const int zq = a.sf32.floor_div((int32_t)(z >> 8));
+                    reg = zq < 0 ? 1 : 2;
+                    val = relu_tab[zq + 127];
+                }
+                vals[k][j] = (int8_t)val;
+                rg[j >> 2] |= (uint32_t)reg << (8 * (j & 3));
+            }
+            const int64_t pix = ((int64_t)b * a.H + y) * a.W + x;
+            *reinterpret_cast<uint4*>(a.region + pix * a.Cout + co0) = make_uint4(rg[0], rg[1], rg[2], rg[3]);
+        }
+        int64_t o;
+        int8_t outv[kSmallCo];
+        uint32_t am[kSmallCo / 4] = {0, 0, 0, 0};
+        if (a.pool) {
+            if (!(valid[0] && valid[1] && valid[2] && valid[3])) continue;   // floor-sized pool
+            for (int j = 0; j < kSmallCo; ++j) {
+                int best = vals[0][j], kb = 0;                 // first maximum wins
+                for (int k = 1; k < 4; ++k)
+                    if (vals[k][j] > best) { best = vals[k][j]; kb = k; }
+                outv[j] = (int8_t)best;
+                am[j >> 2] |= (uint32_t)kb << (8 * (j & 3));
+            }
+            o = (((int64_t)b * a.oh + wy) * a.ow + wx) * a.Cout + co0;
+            *reinterpret_cast<uint4*>(a.argmax + o) = make_uint4(am[0], am[1], am[2], am[3]);
+        } else {
+            for (int j = 0; j < kSmallCo; ++j) outv[j] = vals[0][j];
+            o = (((int64_t)b * a.H + wy) * a.W + wx) * a.Cout + co0;
+        }
+        uint32_t pk[4];
+        for (int q = 0; q < 4; ++q)
+            pk[q] = (uint32_t)(uint8_t)outv[4 * q] | ((uint32_t)(uint8_t)outv[4 * q + 1] << 8) |
+                    ((uint32_t)(uint8_t)outv[4 * q + 2] << 16) | ((uint32_t)(uint8_t)outv[4 * q + 3] << 24);
+        *reinterpret_cast<uint4*>(a.act + o) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+        if (a.out2) *reinterpret_cast<uint4*>(a.out2 + o) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+        if (a.next_nhwc) {
+            uint32_t bw[8];
+            for (int q = 0; q < 8; ++q)
+                bw[q] = (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn((float)outv[2 * q])) |
+                        ((uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn((float)outv[2 * q + 1])) << 16);
+            reinterpret_cast<uint4*>(a.next_nhwc + o)[0] = make_uint4(bw[0], bw[1], bw[2], bw[3]);
+            reinterpret_cast<uint4*>(a.next_nhwc + o)[1] = make_uint4(bw[4], bw[5], bw[6], bw[7]);
+        }
+    }
+}
+
+// Narrow-input weight gradient: CTA = a chunk of kWgRows image rows of one
+// image; delta rows and the input rows with their halo are staged in shared
+// memory; each thread owns a few (co, tap, ci) entries, sums them over the
+// chunk in int64 and adds them into dW with 64-bit atomics.
+constexpr int kWgRows = 8;
+
+__global__ void __launch_bounds__(256) k_conv_small_wgrad(const int8_t* __restrict__ x,
+                                                          const int32_t* __restrict__ d, int B,
+                                                          int H, int W, int Cin, int Cout,
+                                                          unsigned long long* __restrict__ dw) {
+    extern __shared__ int32_t sm[];
+    const int rows = min(kWgRows, H - blockIdx.x * kWgRows);
+    const int y0 = blockIdx.x * kWgRows, b = blockIdx.y;
+    int32_t* dsm = sm;                                   // [rows][W][Cout]
+    int8_t* xsm = reinterpret_cast<int8_t*>(sm + kWgRows * W * Cout);   // [rows+2][W+2][Cin]
+    const int nd = rows * W * Cout;
+    for (int i = threadIdx.x; i < nd; i += blockDim.x)
+        dsm[i] = d[((int64_t)b * H + y0) * W * Cout + i];
+    const int hx = (rows + 2) * (W + 2) * Cin;
+    for (int i = threadIdx.x; i < hx; i += blockDim.x) {
+        const int c = i % Cin, rest = i / Cin, xx = rest % (W + 2), yy = rest / (W + 2);
+        const int iy = y0 + yy - 1, ix = xx - 1;
+        xsm[i] = (iy >= 0 && iy < H && ix >= 0 && ix < W) ? x[(((int64_t)b * H + iy) * W + ix) * Cin + c] : 0;
+    }
+    __syncthreads();
+    const int nout = Cout * 9 * Cin;
+    for (int e = threadIdx.x; e < nout; e += blockDim.x) {
+        const int ci = e % Cin, t = (e / Cin) % 9, co = e / (9 * Cin);
+        const int ky = t / 3, kx = t % 3;
+        int64_t acc = 0;
+        for (int yy = 0; yy < rows; ++yy) {
+            const int32_t* drow = dsm + (yy * W) * Cout + co;
+            const int8_t* xrow = xsm + ((yy + ky) * (W + 2) + kx) * Cin + ci;
+            for (int xx = 0; xx < W; ++xx) acc += (int64_t)drow[xx * Cout] * xrow[xx * Cin];
+        }
+        atomicAdd(&dw[e], (unsigned long long)acc);
+    }
+}
+
 inline int grid_for(int64_t n, int threads, int cap = 152 * 16) {
     int64_t g = (n + threads - 1) / threads;
     return (int)(g < 1 ? 1 : (g > cap ? cap : g));
@@ -530,5 +684,54 @@ cudaError_t simt_integersgd(const SgdBatch& b, cudaStream_t s) {
     return cudaGetLastError();
 }
 
+
+bool simt_small_conv_ok(const LayerGeom& g) {
+    if (g.kind != NITRO_CONV3X3 || g.cin > kSmallCin || g.cout % kSmallCo != 0) return false;
+    // weights of the forward and a row chunk of delta for the weight gradient
+    // must fit in shared memory
+    const int64_t fwd_smem = 4LL * g.cout * 9 * g.cin;
+    const int64_t wg_smem = 4LL * kWgRows * g.w * g.cout + (int64_t)(kWgRows + 2) * (g.w + 2) * g.cin;
+    return fwd_smem <= 48 * 1024 && wg_smem <= 200 * 1024;
+}
+
+cudaError_t simt_conv_small_fwd(const int8_t* x, const int32_t* w, const LayerGeom& g, int B,
+                                int alpha_inv, int mu, int8_t* act, int8_t* out2, int8_t* region,
+                                int8_t* argmax, uint16_t* next_nhwc, cudaStream_t s) {
+    if (B <= 0) return cudaSuccess;
+    SmallFwdArgs a{};
+    a.x = x; a.w = w; a.B = B; a.H = g.h; a.W = g.w; a.Cin = g.cin; a.Cout = g.cout;
+    a.pool = g.pool; a.oh = g.oh; a.ow = g.ow;
+    a.sf32 = FloorDiv32::make(9u * (uint32_t)g.cin);
+    const int64_t sf = 256LL * 9 * g.cin;
+    a.z_hi = 128 * sf;
+    a.z_lo = -127 * sf;
+    a.alpha = FloorDiv::make((uint64_t)alpha_inv);
+    a.mu = mu;
+    a.act = act; a.out2 = out2; a.region = region; a.argmax = argmax; a.next_nhwc = next_nhwc;
+    const int step = g.pool ? 2 : 1;
+    const int64_t n = (int64_t)B * ((g.h + step - 1) / step) * ((g.w + step - 1) / step) * (g.cout / kSmallCo);
+    const size_t smem = sizeof(int32_t) * (size_t)g.cout * 9 * g.cin;
+    ProfScope ps(K_SIMT_CONV_FWD, s, 2.0 * B * g.h * g.w * g.cout * 9.0 * g.cin, 0.0);
+    k_conv_small_fwd<<<grid_for(n, 256, 152 * 32), 256, smem, s>>>(a);
+    return cudaGetLastError();
+}
+
+cudaError_t simt_conv_small_wgrad(const int8_t* x, const int32_t* d, const LayerGeom& g, int B,
+                                  int64_t* dw, cudaStream_t s) {
+    cudaError_t e = cudaMemsetAsync(dw, 0, sizeof(int64_t) * 9 * g.cin * g.cout, s);
+    if (e != cudaSuccess || B <= 0) return e;
+    dim3 grid((g.h + kWgRows - 1) / kWgRows, B);
+    const size_t smem = sizeof(int32_t) * (size_t)kWgRows * g.w * g.cout +
+                        (size_t)(kWgRows + 2) * (g.w + 2) * g.cin + 16;
+    if (smem > 200 * 1024) return cudaErrorInvalidValue;
+    if (smem > 48 * 1024) {
+        e = cudaFuncSetAttribute(k_conv_small_wgrad, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e != cudaSuccess) return e;
+    }
+    ProfScope ps(K_SIMT_CONV_WGRAD, s, 2.0 * B * g.h * g.w * g.cout * 9.0 * g.cin, 0.0);
+    k_conv_small_wgrad<<<grid, 256, smem, s>>>(x, d, B, g.h, g.w, g.cin, g.cout,
+                                               reinterpret_cast<unsigned long long*>(dw));
+    return cudaGetLastError();
+}
 
 }  // namespace nitro

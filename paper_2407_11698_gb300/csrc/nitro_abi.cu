@@ -285,6 +285,12 @@ nitro_status nitro_block_forward(nitro_block* b, const int8_t* a_in, int batch, 
             next_nhwc = b->L[i + 1].tc.act_nhwc;
         TcFwdOut fo{b->desc.alpha_inv, b->mu, ly.act, out2, ly.region, ly.argmax, next_nhwc};
         NITRO_TRY(tc_conv_forward(ly.tc, g, batch, b->z64, &fo, w_status(b), s, &done, &fused));
+        if (!done && simt_small_conv_ok(g)) {
+            // narrow input (image channels): fused CUDA-core forward
+            NITRO_TRY(simt_conv_small_fwd(x, ly.W, g, batch, b->desc.alpha_inv, b->mu, ly.act, out2,
+                                          ly.region, ly.argmax, next_nhwc, s));
+            done = fused = true;
+        }
         if (!done) {
             const int mode = g.kind == NITRO_CONV3X3 ? GM_CONV_FWD : GM_LIN_FWD;
             NITRO_TRY(simt_gemm(mode, x, nullptr, ly.W, b->z64, batch, g.h, g.w, g.cin, g.cout, s));
@@ -336,6 +342,10 @@ nitro_status nitro_block_backward(nitro_block* b, const int8_t* a_in, const int3
         const int8_t* x = i ? b->L[i - 1].act : a_in;
         bool done = false;
         NITRO_TRY(tc_conv_wgrad(ly.tc, g, ly.delta, w_delta(b, i), batch, ly.dW, w_status(b), s, &done));
+        if (!done && simt_small_conv_ok(g)) {
+            NITRO_TRY(simt_conv_small_wgrad(x, ly.delta, g, batch, ly.dW, s));
+            done = true;
+        }
         if (!done) {
             const int mode = g.kind == NITRO_CONV3X3 ? GM_CONV_WGRAD : GM_LIN_WGRAD;
             NITRO_TRY(simt_gemm(mode, x, ly.delta, nullptr, ly.dW, batch, g.h, g.w, g.cin, g.cout, s));

@@ -196,6 +196,16 @@ cudaError_t simt_grad_to_delta(const DeltaSrc& src, const LayerGeom& g, int B, i
                                const int8_t* region, const int8_t* argmax, int32_t* delta,
                                uint32_t* maxabs_delta, uint32_t* status, cudaStream_t s);
 
+// Narrow-input conv (Cin <= 8, Cout % 16 == 0): fused forward (writes act,
+// out2, region, argmax and, if next_nhwc != null, a bf16 copy of act) and
+// weight gradient (dw overwritten).
+bool simt_small_conv_ok(const LayerGeom& g);
+cudaError_t simt_conv_small_fwd(const int8_t* x, const int32_t* w, const LayerGeom& g, int B,
+                                int alpha_inv, int mu, int8_t* act, int8_t* out2, int8_t* region,
+                                int8_t* argmax, uint16_t* next_nhwc, cudaStream_t s);
+cudaError_t simt_conv_small_wgrad(const int8_t* x, const int32_t* d, const LayerGeom& g, int B,
+                                  int64_t* dw, cudaStream_t s);
+
 // IntegerSGD (Algorithm 1) over up to kMaxSgdTensors tensors in one launch.
 constexpr int kMaxSgdTensors = 16;
 struct SgdTensor {
