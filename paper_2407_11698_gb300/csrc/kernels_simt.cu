@@ -558,6 +558,95 @@ __global__ void __launch_bounds__(256) k_conv_small_wgrad(const int8_t* __restri
     }
 }
 
+// ---------------------------------------------------------------------------
+// Learning-layer backward, fused: for feature q of the block output and a
+// group of kLbSamples samples, delta_fw[b][q] = sum_g grad_L[b][g] W_lr[g][q]
+// (int32 storage rule, then max-pool backward and NITRO-ReLU backward into
+// the last layer's delta) and the learning-weight gradient
+// dW_lr[g][q] += sum_b grad_L[b][g] a[b][q] (64-bit atomics into a zeroed
+// dW_lr).  G <= 16; the W_lr column lives in registers.
+// ---------------------------------------------------------------------------
+constexpr int kLbSamples = 16;
+constexpr int kLbMaxG = 16;
+
+__global__ void __launch_bounds__(256) k_lr_backward(const int8_t* __restrict__ a,
+                                                     const int32_t* __restrict__ gl,
+                                                     const int32_t* __restrict__ wlr, int B, int G,
+                                                     LayerGeom lg, int alpha_inv,
+                                                     const int8_t* __restrict__ region,
+                                                     const int8_t* __restrict__ argmax,
+                                                     int32_t* __restrict__ delta,
+                                                     unsigned long long* __restrict__ dwlr,
+                                                     const uint32_t* maxabs_gl,
+                                                     const uint32_t* maxabs_wlr,
+                                                     uint32_t* maxabs_delta, uint32_t* status) {
+    __shared__ int32_t gls[kLbSamples][kLbMaxG];
+    const int d = lg.oh * lg.ow * lg.cout;               // features of the block output
+    const int q = blockIdx.x * blockDim.x + threadIdx.x;
+    const int b0 = blockIdx.y * kLbSamples;
+    const int nb = min(kLbSamples, B - b0);
+    for (int i = threadIdx.x; i < kLbSamples * kLbMaxG; i += blockDim.x) {
+        const int u = i / kLbMaxG, g = i % kLbMaxG;
+        gls[u][g] = (u < nb && g < G) ? gl[(int64_t)(b0 + u) * G + g] : 0;
+    }
+    if (blockIdx.x == 0 && blockIdx.y == 0 && threadIdx.x == 0 &&
+        int64_bound_exceeded(*maxabs_gl, *maxabs_wlr, G))
+        atomicOr(status, ST_OVERFLOW);
+    __syncthreads();
+    uint32_t mx = 0;
+    bool ovf = false;
+    if (q < d) {
+        int32_t w[kLbMaxG];
+        int64_t dw[kLbMaxG];
+#pragma unroll
+        for (int g = 0; g < kLbMaxG; ++g) {
+            w[g] = g < G ? wlr[(int64_t)g * d + q] : 0;
+            dw[g] = 0;
+        }
+        // position of feature q in the (pooled) output grid
+        const int c = q % lg.cout;
+        const int r = q / lg.cout;
+        const int ox = r % lg.ow, oy = r / lg.ow;
+        for (int u = 0; u < nb; ++u) {
+            const int64_t b = b0 + u;
+            uint64_t acc = 0;     // modulo 2^64, exact below the bound
+#pragma unroll
+            for (int g = 0; g < kLbMaxG; ++g) acc += (uint64_t)((int64_t)gls[u][g] * w[g]);
+            const int32_t av = a[b * d + q];
+#pragma unroll
+            for (int g = 0; g < kLbMaxG; ++g) dw[g] += (int64_t)gls[u][g] * av;
+            const int64_t gv = (int64_t)acc;
+            ovf |= !fits_i32(gv);
+            const int32_t gs = (int32_t)gv;
+            if (lg.pool) {
+                const int am = argmax[b * d + q];
+#pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                    const int64_t pi = ((b * lg.h + 2 * oy + (k >> 1)) * lg.w + 2 * ox + (k & 1)) * lg.cout + c;
+                    const int32_t dv = (k == am) ? relu_backward(gs, region[pi], alpha_inv) : 0;
+                    delta[pi] = dv;
+                    mx = max(mx, abs_u32(dv));
+                }
+            } else {
+                const int64_t pi = b * d + q;
+                const int32_t dv = relu_backward(gs, region[pi], alpha_inv);
+                delta[pi] = dv;
+                mx = max(mx, abs_u32(dv));
+            }
+        }
+#pragma unroll
+        for (int g = 0; g < kLbMaxG; ++g)
+            if (g < G && dw[g] != 0) atomicAdd(&dwlr[(int64_t)g * d + q], (unsigned long long)dw[g]);
+    }
+#pragma unroll
+    for (int off = 16; off; off >>= 1) mx = max(mx, __shfl_xor_sync(kFull, mx, off));
+    ovf = __any_sync(kFull, ovf);
+    if ((threadIdx.x & 31) == 0) {
+        if (mx) atomicMax(maxabs_delta, mx);
+        if (ovf) atomicOr(status, ST_OVERFLOW);
+    }
+}
+
 inline int grid_for(int64_t n, int threads, int cap = 152 * 16) {
     int64_t g = (n + threads - 1) / threads;
     return (int)(g < 1 ? 1 : (g > cap ? cap : g));
@@ -633,7 +722,7 @@ cudaError_t simt_learn_fwd(const int8_t* a, const int32_t* wlr, const int32_t* l
     {
         // slice sized so the staged tiles fit 48 KB of shared memory
         int slice = (48 * 1024 - 64) / (4 * G + kLrSamples + 8);
-        slice = slice > 1024 ? 1024 : (slice / 32) * 32;
+        slice = slice > 256 ? 256 : (slice / 32) * 32;
         if (slice < 32) slice = 32;
         const size_t smem = (size_t)G * (slice + 1) * 4 + (size_t)kLrSamples * (slice + 4);
         dim3 grid((d + slice - 1) / slice, (B + kLrSamples - 1) / kLrSamples);
@@ -731,6 +820,28 @@ cudaError_t simt_conv_small_wgrad(const int8_t* x, const int32_t* d, const Layer
     ProfScope ps(K_SIMT_CONV_WGRAD, s, 2.0 * B * g.h * g.w * g.cout * 9.0 * g.cin, 0.0);
     k_conv_small_wgrad<<<grid, 256, smem, s>>>(x, d, B, g.h, g.w, g.cin, g.cout,
                                                reinterpret_cast<unsigned long long*>(dw));
+    return cudaGetLastError();
+}
+
+bool simt_lr_backward_ok(int G) { return G <= kLbMaxG; }
+
+cudaError_t simt_lr_backward(const int8_t* a, const int32_t* gl, const int32_t* wlr, int B, int G,
+                             const LayerGeom& lg, int alpha_inv, const int8_t* region,
+                             const int8_t* argmax, int32_t* delta, int64_t* dwlr,
+                             const uint32_t* maxabs_gl, const uint32_t* maxabs_wlr,
+                             uint32_t* maxabs_delta, uint32_t* status, cudaStream_t s) {
+    const int d = lg.oh * lg.ow * lg.cout;
+    cudaError_t e = cudaMemsetAsync(dwlr, 0, sizeof(int64_t) * (size_t)G * d, s);
+    if (e != cudaSuccess || B <= 0) return e;
+    if (lg.pool && ((lg.h & 1) || (lg.w & 1))) {   // rows / columns the pool dropped
+        e = cudaMemsetAsync(delta, 0, sizeof(int32_t) * (size_t)B * lg.h * lg.w * lg.cout, s);
+        if (e != cudaSuccess) return e;
+    }
+    dim3 grid((d + 255) / 256, (B + kLbSamples - 1) / kLbSamples);
+    ProfScope ps(K_LR_BACKWARD, s, 4.0 * B * d * G, 0.0);
+    k_lr_backward<<<grid, 256, 0, s>>>(a, gl, wlr, B, G, lg, alpha_inv, region, argmax, delta,
+                                       reinterpret_cast<unsigned long long*>(dwlr), maxabs_gl,
+                                       maxabs_wlr, maxabs_delta, status);
     return cudaGetLastError();
 }
 

@@ -325,10 +325,18 @@ nitro_status nitro_block_backward(nitro_block* b, const int8_t* a_in, const int3
     const int8_t* a_last = n ? b->L[n - 1].act : a_in;
     NITRO_TRY(simt_learn_fwd(a_last, b->Wlr, labels, batch, (int)d, G, b->zsum, b->grad_l, b->sse,
                              loss_dev, w_gl(b), w_status(b), s));
-    NITRO_TRY(simt_learn_dw(a_last, b->grad_l, batch, (int)d, G, b->dWlr, s));
+    if (n > 0 && simt_lr_backward_ok(G)) {
+        // learning-weight gradient and delta_fw -> last layer's delta in one pass
+        Layer& ly = b->L[n - 1];
+        NITRO_TRY(simt_lr_backward(a_last, b->grad_l, b->Wlr, batch, G, ly.g, b->desc.alpha_inv,
+                                   ly.region, ly.argmax, ly.delta, b->dWlr, w_gl(b), w_wlr(b),
+                                   w_delta(b, n - 1), w_status(b), s));
+    } else {
+        NITRO_TRY(simt_learn_dw(a_last, b->grad_l, batch, (int)d, G, b->dWlr, s));
+    }
     if (n == 0) return NITRO_OK;
     // delta_fw = grad_L W_lr (pre-update), into the last layer
-    {
+    if (!simt_lr_backward_ok(G)) {
         Layer& ly = b->L[n - 1];
         DeltaSrc src{};
         src.grad_l = b->grad_l; src.wlr = b->Wlr; src.G = G;

@@ -206,6 +206,17 @@ cudaError_t simt_conv_small_fwd(const int8_t* x, const int32_t* w, const LayerGe
 cudaError_t simt_conv_small_wgrad(const int8_t* x, const int32_t* d, const LayerGeom& g, int B,
                                   int64_t* dw, cudaStream_t s);
 
+// Learning-layer backward for G <= 16, fused: dW_lr (overwritten) and the
+// last forward layer's delta from delta_fw = grad_L W_lr (pre-update), with
+// the int32 storage rule, the int64 bound check, max-pool and NITRO-ReLU
+// backward.  lg: geometry of the block's last forward layer.
+bool simt_lr_backward_ok(int G);
+cudaError_t simt_lr_backward(const int8_t* a, const int32_t* gl, const int32_t* wlr, int B, int G,
+                             const LayerGeom& lg, int alpha_inv, const int8_t* region,
+                             const int8_t* argmax, int32_t* delta, int64_t* dwlr,
+                             const uint32_t* maxabs_gl, const uint32_t* maxabs_wlr,
+                             uint32_t* maxabs_delta, uint32_t* status, cudaStream_t s);
+
 // IntegerSGD (Algorithm 1) over up to kMaxSgdTensors tensors in one launch.
 constexpr int kMaxSgdTensors = 16;
 struct SgdTensor {

@@ -39,7 +39,7 @@ const char* const kNames[K_COUNT] = {
     "simt_conv_fwd", "simt_conv_dgrad", "simt_conv_wgrad", "simt_linear_fwd",
     "simt_linear_dgrad", "simt_linear_wgrad", "fwd_epilogue", "learn_partial",
     "learn_dw", "grad_to_delta", "integersgd", "learn_finish_loss", "tc_conv_fwd",
-    "tc_conv_wgrad", "tc_conv_dgrad", "tc_pack_limbs", "tc_finish", "tc_gemm"};
+    "tc_conv_wgrad", "tc_conv_dgrad", "tc_pack_limbs", "tc_finish", "tc_gemm", "lr_backward"};
 
 }  // namespace
 

@@ -30,6 +30,7 @@ enum KernelId : int {
     K_TC_PACK,
     K_TC_FINISH,
     K_TC_GEMM,
+    K_LR_BACKWARD,
     K_COUNT
 };
 
