@@ -281,7 +281,8 @@ nitro_status nitro_block_forward(nitro_block* b, const int8_t* a_in, int batch, 
         NITRO_TRY(tc_pack_input(ly.tc, g, x, batch, nhwc_done, s));
         // the epilogue also writes the next layer's bf16 forward operand
         uint16_t* next_nhwc = nullptr;
-        if (i + 1 < n && b->L[i + 1].tc.act_nhwc && b->L[i + 1].tc.cin8 == g.cout)
+        if (i + 1 < n && b->L[i + 1].tc.act_nhwc && !b->L[i + 1].tc.im2col &&
+            b->L[i + 1].tc.cin8 == g.cout)
             next_nhwc = b->L[i + 1].tc.act_nhwc;
         TcFwdOut fo{b->desc.alpha_inv, b->mu, ly.act, out2, ly.region, ly.argmax, next_nhwc};
         NITRO_TRY(tc_conv_forward(ly.tc, g, batch, b->z64, &fo, w_status(b), s, &done, &fused));

@@ -192,6 +192,7 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
 struct TcArgs {
     int B, H, W, Cin, Cout, Bp;
     int cin_k;             // channels per tap in the K index (Cin rounded up to 64)
+    int taps;              // 9, or 1 for im2col input (forward / wgrad: no tap shift)
     int ntx, nty;          // pixel tiles along x and y (forward / dgrad)
     int wb, hb, bb;        // pixel box (forward / dgrad): wb * hb * bb = 128
     int tiles_m, tiles_n, total_tiles;
@@ -362,7 +363,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                                 tma_load_3d(b_dst + j * C::B_BYTES, &tmB, fb, kb * kBK, n0, lb0 + j);
                         } else if (MODE == TC_FWD) {
                             const int nc = args.cin_k / kBK;
-                            const int t = kb / nc, cb = kb - t * nc, ky = t / 3, kx = t - 3 * ky;
+                            const int t = kb / nc, cb = kb - t * nc;
+                            const int tc = args.taps == 1 ? 4 : t;   // im2col rows: centre tap
+                            const int ky = tc / 3, kx = tc - 3 * ky;
                             tma_load_4d(a_dst, &tmA, fb, cb * kBK, x0 + kx - 1, y0 + ky - 1, b0);
                             for (int j = 0; j < nb; ++j)
                                 tma_load_3d(b_dst + j * C::B_BYTES, &tmB, fb, t * args.cin_k + cb * kBK,
@@ -383,7 +386,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                             for (int j = 0; j < 2; ++j) {
                                 const int m = T.mt * kBM + j * 64;
                                 int t = m / args.cin_k, ci0 = m - t * args.cin_k;
-                                if (t >= 9) { t = 0; ci0 = args.cin_k; }   // past the last tap: zeros
+                                if (t >= args.taps) { t = 0; ci0 = args.cin_k; }   // past the last tap: zeros
+                                if (args.taps == 1) t = 4;                         // im2col rows: centre tap
                                 const int ky = t / 3, kx = t - 3 * ky;
                                 tma_load_4d(a_dst + j * (64 * 128), &tmA, fb, ci0, px + kx - 1,
                                             py + ky - 1, bk);
@@ -501,8 +505,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                 } else if (MODE == TC_WGRAD) {
                     const int m = T.mt * kBM + r;
                     const int t = m / args.cin_k, ci = m - t * args.cin_k;
-                    if (t < 9 && ci < args.Cin) {
-                        int64_t* o = args.out + (int64_t)t * args.Cin + ci;
+                    // im2col rows: row m is already the (tap, ci) index t Cin + ci
+                    const bool ok = args.taps == 1 ? m < 9 * args.Cin : (t < 9 && ci < args.Cin);
+                    if (ok) {
+                        int64_t* o = args.out + (args.taps == 1 ? (int64_t)m : (int64_t)t * args.Cin + ci);
                         const int64_t cstride = 9LL * args.Cin;
 #pragma unroll
                         for (int i = 0; i < NH; ++i) {
@@ -729,6 +735,43 @@ __global__ void k_pack_act_nhwc(const int8_t* __restrict__ x, int64_t P, int C, 
     }
 }
 
+// int8 NHWC x [B][H][W][Cin] (9 Cin <= 64) -> bf16 im2col rows [B][H][W][64]:
+// entry k = t Cin + ci holds x at (y + ky - 1, x + kx - 1) for tap t = 3 ky + kx,
+// zero outside the image and for k >= 9 Cin.  Eight entries per thread.
+__global__ void k_pack_im2col(const int8_t* __restrict__ x, int B, int H, int W, int Cin,
+                              uint16_t* __restrict__ out) {
+    const int64_t n = (int64_t)B * H * W * (kBK / 8);
+    const int kmax = 9 * Cin;
+    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t p = i / (kBK / 8);
+        const int k0 = (int)(i - p * (kBK / 8)) * 8;
+        const int px = (int)(p % W);
+        const int64_t r = p / W;
+        const int py = (int)(r % H);
+        const int64_t b = r / H;
+        uint32_t w[4];
+#pragma unroll
+        for (int j = 0; j < 8; j += 2) {
+            uint32_t h[2];
+#pragma unroll
+            for (int u = 0; u < 2; ++u) {
+                const int k = k0 + j + u;
+                int v = 0;
+                if (k < kmax) {
+                    const int t = k / Cin, ci = k - t * Cin;
+                    const int iy = py + t / 3 - 1, ix = px + t % 3 - 1;
+                    if (iy >= 0 && iy < H && ix >= 0 && ix < W)
+                        v = x[((b * H + iy) * W + ix) * Cin + ci];
+                }
+                h[u] = bf16_bits(v);
+            }
+            w[j / 2] = h[0] | (h[1] << 16);
+        }
+        reinterpret_cast<uint4*>(out)[i] = make_uint4(w[0], w[1], w[2], w[3]);
+    }
+}
+
 // int32 delta NHWC (n values, n % 8 == 0) -> limb planes [L][n], eight values
 // per thread and one 16-byte store per plane; records the limb count.
 __global__ void __launch_bounds__(256) k_pack_delta_nhwc(const int32_t* __restrict__ d, int64_t n,
@@ -765,15 +808,17 @@ __global__ void __launch_bounds__(256) k_pack_delta_nhwc(const int32_t* __restri
 }
 
 
-// W [Cout][9][Cin] -> w_planes [L][Cout][9][Ck] (Ck = Cin rounded up to 64,
-// padding left zero) and wt_planes [L][9][Cin][Cout]
-__global__ void k_pack_weights(const int32_t* __restrict__ W, int Cout, int Cin, int Ck,
-                               const uint32_t* maxabs, uint16_t* __restrict__ wp,
+// W [Cout][9][Cin] -> w_planes [L][Cout][row_k] with entry (t, ci) at
+// t tap_k + ci (padding left zero; row_k = 9 Ck, tap_k = Ck with Ck = Cin
+// rounded up to 64, or row_k = 64, tap_k = Cin for im2col rows) and
+// wt_planes [L][9][Cin][Cout]
+__global__ void k_pack_weights(const int32_t* __restrict__ W, int Cout, int Cin, int row_k,
+                               int tap_k, const uint32_t* maxabs, uint16_t* __restrict__ wp,
                                uint16_t* __restrict__ wtp, int* limbs_out) {
     const int L = limb_count(*maxabs);
     if (blockIdx.x == 0 && threadIdx.x == 0) *limbs_out = L;
     const int64_t n = (int64_t)Cout * 9 * Cin;
-    const int64_t nk = (int64_t)Cout * 9 * Ck;
+    const int64_t nk = (int64_t)Cout * row_k;
     for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
          i += (int64_t)gridDim.x * blockDim.x) {
         const int ci = (int)(i % Cin);
@@ -781,7 +826,7 @@ __global__ void k_pack_weights(const int32_t* __restrict__ W, int Cout, int Cin,
         const int co = (int)(i / (9LL * Cin));
         int64_t x = W[i];
         const int64_t it = ((int64_t)t * Cin + ci) * Cout + co;
-        const int64_t ik = ((int64_t)co * 9 + t) * Ck + ci;
+        const int64_t ik = (int64_t)co * row_k + t * tap_k + ci;
         for (int l = 0; l < L; ++l) {
             int v;
             if (l < L - 1) {
@@ -905,16 +950,18 @@ bool tc_layer_init(TcLayer& t, const LayerGeom& g, int max_batch, bool has_dgrad
     if (g.kind != NITRO_CONV3X3 || max_batch < 1 || !encode_fn()) return true;
     // Narrow inputs (Cin < 32, e.g. image channels) stay on the CUDA-core
     // kernels: zero-padding them to a 64-wide K-block wastes most MMA work.
+    // Inputs with 9 Cin <= 64 run as one 64-wide K-block of im2col rows.
     const bool pix_ok = g.h >= 8 && g.w >= 8;
     const bool wide = g.cin >= 32;
-    t.fwd = pix_ok && wide;
-    t.wgrad = wide && g.cout % 8 == 0;
+    t.im2col = pix_ok && 9 * g.cin <= kBK;
+    t.fwd = pix_ok && (wide || t.im2col);
+    t.wgrad = (wide || t.im2col) && g.cout % 8 == 0;
     t.dgrad = has_dgrad && pix_ok && g.cout % 8 == 0;
-    t.cin8 = round_up(g.cin, 8);
+    t.cin8 = t.im2col ? kBK : round_up(g.cin, 8);
     t.cin_k = round_up(g.cin, 64);
     const size_t hw = (size_t)g.h * g.w;
     const size_t nw = (size_t)g.cout * 9 * g.cin;
-    const size_t nwk = (size_t)g.cout * 9 * t.cin_k;
+    const size_t nwk = (size_t)g.cout * (t.im2col ? kBK : 9 * t.cin_k);
     bool ok = dalloc(allocs, &t.limbs, 2);
     if (ok && (t.fwd || t.wgrad)) ok = dalloc(allocs, &t.act_nhwc, (size_t)max_batch * hw * t.cin8);
     if (ok && (t.wgrad || t.dgrad))
@@ -941,8 +988,9 @@ cudaError_t tc_refresh_weights(TcLayer& t, const LayerGeom& g, const int32_t* W,
     const int64_t n = (int64_t)g.cout * 9 * g.cin;
     {
         ProfScope ps(K_TC_PACK, s, 0.0, (double)n * 4 * 2);
-        k_pack_weights<<<grid1d(n), 256, 0, s>>>(W, g.cout, g.cin, t.cin_k, maxabs_w, t.w_planes,
-                                                 t.wt_planes, t.limbs);
+        const int row_k = t.im2col ? kBK : 9 * t.cin_k, tap_k = t.im2col ? g.cin : t.cin_k;
+        k_pack_weights<<<grid1d(n), 256, 0, s>>>(W, g.cout, g.cin, row_k, tap_k, maxabs_w,
+                                                 t.w_planes, t.wt_planes, t.limbs);
     }
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
@@ -954,6 +1002,11 @@ cudaError_t tc_pack_input(TcLayer& t, const LayerGeom& g, const int8_t* x, int b
                           bool nhwc_done, cudaStream_t s) {
     if (batch <= 0 || !t.act_nhwc || nhwc_done) return cudaSuccess;
     const int64_t P = (int64_t)batch * g.h * g.w;
+    if (t.im2col) {
+        ProfScope ps(K_TC_PACK, s, 0.0, (double)P * (g.cin + 2 * kBK));
+        k_pack_im2col<<<grid1d(P * (kBK / 8)), 256, 0, s>>>(x, batch, g.h, g.w, g.cin, t.act_nhwc);
+        return cudaGetLastError();
+    }
     ProfScope ps(K_TC_PACK, s, 0.0, (double)P * (g.cin + 2 * t.cin8));
     k_pack_act_nhwc<<<grid1d(P * t.cin8), 256, 0, s>>>(x, P, g.cin, t.cin8, t.act_nhwc);
     return cudaGetLastError();
@@ -969,11 +1022,12 @@ cudaError_t tc_conv_forward(TcLayer& t, const LayerGeom& g, int batch, int64_t* 
     a.B = batch; a.H = g.h; a.W = g.w; a.Cin = g.cin; a.Cout = g.cout;
     a.Bp = round_up(batch, 8);
     a.cin_k = t.cin_k;
+    a.taps = t.im2col ? 1 : 9;
     pixel_tiling(g, batch, a);
     const int n = pick_n(g.cout);
     a.tiles_n = (g.cout + n - 1) / n;
     a.total_tiles = a.tiles_m * a.tiles_n;
-    a.kb_total = 9 * (t.cin_k / kBK);
+    a.kb_total = a.taps * (t.cin_k / kBK);
     a.kb_per_split = a.kb_total;
     a.ncols = g.cout;
     a.limbs_a = nullptr;
@@ -1002,8 +1056,9 @@ cudaError_t tc_conv_forward(TcLayer& t, const LayerGeom& g, int batch, int64_t* 
     const uint64_t da[4] = {(uint64_t)t.cin8, (uint64_t)g.w, (uint64_t)g.h, (uint64_t)batch};
     const uint64_t sa[3] = {(uint64_t)t.cin8, (uint64_t)g.w * t.cin8, (uint64_t)g.h * g.w * t.cin8};
     const uint32_t ba[4] = {64, (uint32_t)a.wb, (uint32_t)a.hb, (uint32_t)a.bb};
-    const uint64_t db[3] = {(uint64_t)9 * t.cin_k, (uint64_t)g.cout, (uint64_t)kMaxLimbs};
-    const uint64_t sb[2] = {(uint64_t)9 * t.cin_k, (uint64_t)9 * t.cin_k * g.cout};
+    const uint64_t kw = (uint64_t)a.taps * t.cin_k;   // w_planes row length
+    const uint64_t db[3] = {kw, (uint64_t)g.cout, (uint64_t)kMaxLimbs};
+    const uint64_t sb[2] = {kw, kw * g.cout};
     const uint32_t bb[3] = {64, (uint32_t)n, 1};
     if (!make_map(&ma, t.act_nhwc, 4, da, sa, ba) || !make_map(&mb, t.w_planes, 3, db, sb, bb))
         return cudaErrorInvalidValue;
@@ -1045,6 +1100,7 @@ cudaError_t tc_conv_wgrad(TcLayer& t, const LayerGeom& g, const int32_t* delta,
     a.B = batch; a.H = g.h; a.W = g.w; a.Cin = g.cin; a.Cout = g.cout;
     a.Bp = round_up(batch, 8);
     a.cin_k = t.cin_k;
+    a.taps = t.im2col ? 1 : 9;
     // K-blocks: 64-pixel boxes (wb x hb) of one image
     a.wb = g.w <= 8 ? 8 : (g.w <= 16 ? 16 : (g.w <= 32 ? 32 : 64));
     a.hb = 64 / a.wb;
@@ -1052,7 +1108,7 @@ cudaError_t tc_conv_wgrad(TcLayer& t, const LayerGeom& g, const int32_t* delta,
     a.ntx = (g.w + a.wb - 1) / a.wb;
     a.nty = (g.h + a.hb - 1) / a.hb;
     const int n = pick_n(g.cout);
-    a.tiles_m = (9 * t.cin_k + kBM - 1) / kBM;
+    a.tiles_m = (a.taps * t.cin_k + kBM - 1) / kBM;
     a.tiles_n = (g.cout + n - 1) / n;
     a.kb_total = batch * a.ntx * a.nty;
     // split K so that about one wave of CTAs runs, each with >= one exact chunk
@@ -1101,6 +1157,7 @@ cudaError_t tc_conv_dgrad(TcLayer& t, const LayerGeom& g, int batch, int64_t* g6
     a.B = batch; a.H = g.h; a.W = g.w; a.Cin = g.cin; a.Cout = g.cout;
     a.Bp = round_up(batch, 8);
     a.cin_k = t.cin_k;
+    a.taps = 9;
     pixel_tiling(g, batch, a);
     const int n = pick_n(g.cin);
     a.tiles_n = (g.cin + n - 1) / n;

@@ -14,6 +14,7 @@
 //   d_nhwc    [L][B][H][W][Cout]       dgrad A (K-major) and wgrad B (MN-major)
 //   w_planes  [L][Cout][9][Cin64]      forward B
 //   wt_planes [L][9][Cin][Cout]        dgrad B
+// Narrow inputs (9 Cin <= 64) use im2col rows instead, see TcLayer::im2col.
 // Cin8 = Cin rounded up to 8 (TMA strides are multiples of 16 bytes); Cin64 =
 // Cin rounded up to 64 so that a K-block of the forward never spans two taps.  Padding holds zeros; tiles that run past
 // a tensor edge read zeros (TMA out-of-bounds fill) and skip their stores.
@@ -29,7 +30,11 @@ constexpr int kMaxLimbs = 4;
 
 struct TcLayer {
     bool fwd = false, wgrad = false, dgrad = false;   // passes that run on tcgen05
-    int cin8 = 0;     // channels of the NHWC bf16 input copy (Cin rounded up to 8)
+    // narrow input (9 Cin <= 64, e.g. image channels): act_nhwc holds im2col
+    // rows [B][H][W][64] (entry t Cin + ci = input at tap t, zero past 9 Cin)
+    // and w_planes is [L][Cout][64]; forward and wgrad see one centred tap.
+    bool im2col = false;
+    int cin8 = 0;     // channels of the NHWC bf16 input copy (Cin rounded up to 8; 64 for im2col)
     int cin_k = 0;    // channels per tap in the forward K index (Cin rounded up to 64)
     uint16_t* act_nhwc = nullptr;
     uint16_t* d_nhwc = nullptr;

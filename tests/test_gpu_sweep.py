@@ -42,6 +42,9 @@ def _wrap64(x):
     (2, 7, 7, 64, 64, 4, 3),       # 7x7: forward / dgrad on CUDA cores, wgrad on tcgen05
     (4, 8, 8, 32, 64, 2, 2),       # 32 input channels (padded to a 64-wide K-block)
     (9, 10, 11, 64, 48, 1, 1),     # 48 output channels: masked columns
+    (3, 12, 9, 3, 64, 3, 4),       # 3 input channels: im2col rows (27 of 64 K entries)
+    (2, 8, 10, 7, 16, 4, 2),       # 7 input channels (63 entries), 16 output channels
+    (2, 9, 8, 1, 128, 2, 3),       # single input channel, N = 128 tiles
 ])
 def test_conv_contractions_full(torch, B, h, w, cin, cout, lw, ld):
     a = synth.images(21, 0, B, (h, w, cin)).astype(np.int64)

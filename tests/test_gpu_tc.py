@@ -1,6 +1,6 @@
 """Tensor-core (tcgen05) conv path: bit-exact against the oracle through the
-C-ABI on shapes that exercise ragged tiles, batch padding and 1..4 limb
-operands.  Every block has two conv layers, so fwd, wgrad and dgrad of the
+C-ABI on shapes that exercise ragged tiles, batch padding, 1..4 limb operands
+and narrow (image-channel) inputs that run as im2col rows.  Every block has two conv layers, so fwd, wgrad and dgrad of the
 second layer and the fwd of the first all run on tensor cores when the
 channel counts are multiples of 64."""
 import numpy as np
@@ -63,6 +63,17 @@ def test_two_conv_block_pooled_lower_layer(B, h, w, c0, c1, c2, pool, scale):
     _run_two_conv(B, h, w, c0, c1, c2, pool, scale, True)
 
 
+@pytest.mark.parametrize("B,h,w,c0,c1,c2,pool,scale", [
+    (8, 8, 8, 3, 64, 64, True, 1),             # image channels: im2col rows on tcgen05
+    (3, 12, 9, 1, 16, 64, False, 1),           # one input channel, 16 outputs (ragged N tile)
+    (5, 16, 16, 7, 128, 64, True, 300),        # 63 of the 64 im2col entries, two-limb weights
+    (4, 10, 12, 5, 48, 64, False, 70001),      # 48 outputs, three-limb weights
+    (130, 8, 16, 3, 64, 64, True, 2**22),      # batch over 128, four-limb weights
+])
+def test_narrow_input_first_layer(B, h, w, c0, c1, c2, pool, scale):
+    _run_two_conv(B, h, w, c0, c1, c2, pool, scale, False)
+
+
 def _run_two_conv(B, h, w, c0, c1, c2, pool, scale, pool_first):
     blocks = _two_conv_block(B, h, w, c0, c1, c2, pool, pool_first)
     pair = NetPair(blocks, B, seed=31)
@@ -79,17 +90,19 @@ def _run_two_conv(B, h, w, c0, c1, c2, pool, scale, pool_first):
         pair.close()
 
 
-def test_tensor_core_kernels_ran():
-    """The tc kernels are the ones launched for a 64-channel layer."""
+@pytest.mark.parametrize("c0", [64, 3])
+def test_tensor_core_kernels_ran(c0):
+    """The tc kernels are the ones launched for a 64-channel layer and for a
+    3-channel (image) layer."""
     torch = pytest.importorskip("torch")
     import ctypes
     L = nb.lib()
-    blocks = _two_conv_block(8, 8, 8, 64, 64, 64, True)
+    blocks = _two_conv_block(8, 8, 8, c0, 64, 64, True)
     pair = NetPair(blocks, 8, seed=2)
     try:
         L.nitro_profile_reset()
         L.nitro_profile_enable(1)
-        pair.step_gpu(synth.images(1, 0, 8, (8, 8, 64)), synth.labels(1, 0, 8))
+        pair.step_gpu(synth.images(1, 0, 8, (8, 8, c0)), synth.labels(1, 0, 8))
         L.nitro_profile_enable(0)
         names = {}
         for k in range(L.nitro_profile_kernel_count()):
