@@ -184,7 +184,8 @@ void nitro_destroy_block(nitro_block* blk);
  *   NITRO_CONTRACT_DGRAD x = int32 d [B][H][W][Cout], y = int32 W
  *                        out = g [B][H][W][Cin] = sum_(ky,kx,co) d[b,y-ky+1,x-kx+1,co] W
  * Asynchronous on `stream`; the handle owns its packing workspace (sized at
- * create for max_batch) and must not be used by two streams at once. */
+ * create for max_batch) and must not be used by two streams at once.  Buffers
+ * need only the alignment of their element type (here and in the block calls). */
 typedef enum { NITRO_CONTRACT_FWD = 0, NITRO_CONTRACT_WGRAD = 1, NITRO_CONTRACT_DGRAD = 2 } nitro_contract_mode;
 typedef struct nitro_conv nitro_conv;
 nitro_status nitro_conv3x3_create(int max_batch, int h, int w, int cin, int cout, nitro_conv** out);
@@ -244,6 +245,11 @@ const char* nitro_profile_kernel_name(int id);   /* static string            */
  * summed device time (ms) and summed algorithmic ops and bytes. */
 nitro_status nitro_profile_read(int id, uint64_t* launches, double* ms, double* ops,
                                 double* bytes);
+/* Launches recorded since the last reset, and launch i (0-based, in launch
+ * order): its kernel class, device time (ms), algorithmic ops and bytes.
+ * Synchronises on that launch's events; NITRO_ERR_ARG for i out of range. */
+int nitro_profile_record_count(void);
+nitro_status nitro_profile_record(int i, int* kernel, double* ms, double* ops, double* bytes);
 
 /* Static, human-readable name of a status code. */
 const char* nitro_status_str(nitro_status s);

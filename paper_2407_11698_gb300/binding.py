@@ -90,6 +90,10 @@ def lib():
     _PD = ctypes.POINTER(ctypes.c_double)
     L.nitro_profile_read.argtypes = [ctypes.c_int, ctypes.POINTER(ctypes.c_uint64), _PD, _PD, _PD]
     L.nitro_profile_read.restype = ctypes.c_int
+    L.nitro_profile_record_count.argtypes = []
+    L.nitro_profile_record_count.restype = ctypes.c_int
+    L.nitro_profile_record.argtypes = [ctypes.c_int, ctypes.POINTER(ctypes.c_int), _PD, _PD, _PD]
+    L.nitro_profile_record.restype = ctypes.c_int
     L.nitro_conv3x3_forward_noalloc.argtypes = [_VP, _VP] + [ctypes.c_int] * 7 + [_VP, _VP, _VP, _VP]
     L.nitro_conv3x3_forward_noalloc.restype = ctypes.c_int
     L.nitro_conv3x3_create.argtypes = [ctypes.c_int] * 5 + [ctypes.POINTER(_VP)]

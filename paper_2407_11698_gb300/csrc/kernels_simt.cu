@@ -389,8 +389,9 @@ __global__ void k_integersgd(SgdBatch bt) {
     for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < t.n;
          i += (int64_t)gridDim.x * blockDim.x) {
         const int64_t w = t.w[i];
-        int64_t d = bt.round_trunc ? tdiv64(t.dw[i], t.gamma_inv) : fdiv64(t.dw[i], t.gamma_inv);
-        if (t.eta_inv != 0) d += bt.round_trunc ? tdiv64(w, t.eta_inv) : fdiv64(w, t.eta_inv);
+        const int64_t g = t.dw[i];
+        int64_t d = bt.round_trunc ? t.gdiv.trunc_div(g) : t.gdiv.floor_div(g);
+        if (t.eta_inv != 0) d += bt.round_trunc ? t.ediv.trunc_div(w) : t.ediv.floor_div(w);
         const int64_t nw = w - d;
         ovf |= !fits_i32(nw);
         const int32_t s = (int32_t)nw;
@@ -761,10 +762,16 @@ cudaError_t simt_grad_to_delta(const DeltaSrc& src, const LayerGeom& g, int B, i
     return cudaGetLastError();
 }
 
-cudaError_t simt_integersgd(const SgdBatch& b, cudaStream_t s) {
-    if (b.count <= 0) return cudaSuccess;
+cudaError_t simt_integersgd(const SgdBatch& b_in, cudaStream_t s) {
+    if (b_in.count <= 0) return cudaSuccess;
+    SgdBatch b = b_in;
     int64_t nmax = 0;
-    for (int i = 0; i < b.count; ++i) nmax = b.t[i].n > nmax ? b.t[i].n : nmax;
+    for (int i = 0; i < b.count; ++i) {
+        nmax = b.t[i].n > nmax ? b.t[i].n : nmax;
+        if (b.t[i].gamma_inv <= 0 || b.t[i].eta_inv < 0) return cudaErrorInvalidValue;
+        b.t[i].gdiv = FloorDiv::make((uint64_t)b.t[i].gamma_inv);
+        b.t[i].ediv = FloorDiv::make(b.t[i].eta_inv > 0 ? (uint64_t)b.t[i].eta_inv : 1);
+    }
     dim3 grid(grid_for(nmax, 256, 152 * 4), b.count);
     double bytes = 0;
     for (int i = 0; i < b.count; ++i) bytes += 16.0 * b.t[i].n;   // W r+w, dW r

@@ -276,7 +276,9 @@ nitro_status nitro_block_forward(nitro_block* b, const int8_t* a_in, int batch, 
     for (int i = 0; i < n; ++i) {
         Layer& ly = b->L[i];
         const LayerGeom& g = ly.g;
-        int8_t* out2 = (i == n - 1) ? a_out : nullptr;
+        // the fused epilogues store 16 bytes at a time: an unaligned a_out
+        // is filled by a copy after the last layer instead
+        int8_t* out2 = (i == n - 1 && ((uintptr_t)a_out & 15) == 0) ? a_out : nullptr;
         bool done = false, fused = false;
         NITRO_TRY(tc_pack_input(ly.tc, g, x, batch, nhwc_done, s));
         // the epilogue also writes the next layer's bf16 forward operand
@@ -302,6 +304,9 @@ nitro_status nitro_block_forward(nitro_block* b, const int8_t* a_in, int batch, 
         nhwc_done = fused && next_nhwc != nullptr;
         x = ly.act;
     }
+    if (n > 0 && a_out && ((uintptr_t)a_out & 15) != 0)
+        NITRO_TRY(cudaMemcpyAsync(a_out, b->L[n - 1].act, (size_t)batch * b->d,
+                                  cudaMemcpyDeviceToDevice, s));
     return NITRO_OK;
 }
 
@@ -395,9 +400,9 @@ nitro_status nitro_integersgd_step(nitro_block* b, void* stream) {
     bt.status = w_status(b);
     for (int i = 0; i < n; ++i)
         bt.t[bt.count++] = SgdTensor{b->L[i].W, b->L[i].dW, b->L[i].wcount, gamma_fw,
-                                     b->desc.eta_inv_fw, w_w(b, i)};
+                                     b->desc.eta_inv_fw, w_w(b, i), {}, {}};
     bt.t[bt.count++] = SgdTensor{b->Wlr, b->dWlr, (int64_t)b->G * b->d, b->desc.gamma_inv_lr,
-                                 b->desc.eta_inv_lr, w_wlr(b)};
+                                 b->desc.eta_inv_lr, w_wlr(b), {}, {}};
     NITRO_TRY(cudaMemsetAsync(w_wlr(b), 0, 4, s));
     if (n) NITRO_TRY(cudaMemsetAsync(w_w(b, 0), 0, 4 * n, s));
     NITRO_TRY(simt_integersgd(bt, s));

@@ -225,6 +225,7 @@ struct SgdTensor {
     int64_t n;
     int64_t gamma_inv, eta_inv;
     uint32_t* maxabs_w;
+    FloorDiv gdiv, ediv;   // dividers for gamma_inv and eta_inv (filled by simt_integersgd)
 };
 struct SgdBatch {
     SgdTensor t[kMaxSgdTensors];

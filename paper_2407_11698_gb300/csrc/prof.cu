@@ -39,7 +39,8 @@ const char* const kNames[K_COUNT] = {
     "simt_conv_fwd", "simt_conv_dgrad", "simt_conv_wgrad", "simt_linear_fwd",
     "simt_linear_dgrad", "simt_linear_wgrad", "fwd_epilogue", "learn_partial",
     "learn_dw", "grad_to_delta", "integersgd", "learn_finish_loss", "tc_conv_fwd",
-    "tc_conv_wgrad", "tc_conv_dgrad", "tc_pack_limbs", "tc_finish", "tc_gemm", "lr_backward"};
+    "tc_conv_wgrad", "tc_conv_dgrad", "tc_pack_limbs", "tc_finish", "tc_gemm", "lr_backward",
+    "tc_pack_weights", "tc_pack_input", "tc_pack_delta"};
 
 }  // namespace
 
@@ -102,6 +103,26 @@ nitro_status nitro_profile_read(int id, uint64_t* launches, double* ms, double* 
         *ops += r.ops;
         *bytes += r.bytes;
     }
+    return NITRO_OK;
+}
+
+int nitro_profile_record_count(void) {
+    std::lock_guard<std::mutex> lk(g_mu);
+    return (int)g_records.size();
+}
+
+nitro_status nitro_profile_record(int i, int* kernel, double* ms, double* ops, double* bytes) {
+    if (!kernel || !ms || !ops || !bytes) return NITRO_ERR_ARG;
+    std::lock_guard<std::mutex> lk(g_mu);
+    if (i < 0 || i >= (int)g_records.size()) return NITRO_ERR_ARG;
+    Record& r = g_records[i];
+    if (cudaEventSynchronize(r.b) != cudaSuccess) return NITRO_ERR_CUDA;
+    float t = 0.f;
+    if (cudaEventElapsedTime(&t, r.a, r.b) != cudaSuccess) return NITRO_ERR_CUDA;
+    *kernel = r.id;
+    *ms = t;
+    *ops = r.ops;
+    *bytes = r.bytes;
     return NITRO_OK;
 }
 

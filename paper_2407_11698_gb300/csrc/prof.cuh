@@ -31,6 +31,9 @@ enum KernelId : int {
     K_TC_FINISH,
     K_TC_GEMM,
     K_LR_BACKWARD,
+    K_TC_PACK_W,
+    K_TC_PACK_X,
+    K_TC_PACK_D,
     K_COUNT
 };
 

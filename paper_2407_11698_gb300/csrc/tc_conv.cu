@@ -203,6 +203,7 @@ struct TcArgs {
     int64_t* out;
     uint32_t* status;
     int atomic_out;
+    int out_vec;           // out is 16-byte aligned: pairs of int64 stored together
     // forward with fused NITRO-Scaling / NITRO-ReLU / max-pool epilogue
     int fuse;
     FloorDiv alpha;        // divide by alpha_inv
@@ -406,7 +407,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     } else if (warp == 1) {
         if (lane == 0) {
             // ---------------- MMA issuer
-            constexpr uint32_t idesc = idesc_bf16(kBM, N, MODE == TC_WGRAD);
+            // the nb limb tiles of B lie back to back in shared memory and their
+            // accumulators side by side in TMEM: one MMA of width nb * N covers them
+            uint32_t idesc_nb[PB + 1];
+#pragma unroll
+            for (int j = 1; j <= PB; ++j) idesc_nb[j] = idesc_bf16(kBM, j * N, MODE == TC_WGRAD);
             int it = 0, chunk = 0;
             for (int tile = blockIdx.x; tile < args.total_tiles; tile += gridDim.x) {
                 const Tile T = decode_tile(args, tile);
@@ -428,21 +433,20 @@ __global__ void __launch_bounds__(kThreads, 1)
                                 goto mma_done;
                             tc_fence_after();
                             const uint32_t a_addr = smem_u32(smem + s * C::STAGE);
-                            for (int j = 0; j < nb; ++j) {
-                                const uint32_t b_addr = a_addr + C::A_BYTES + j * C::B_BYTES;
+                            const uint32_t b_addr = a_addr + C::A_BYTES;
+                            const uint32_t idesc = idesc_nb[nb];
 #pragma unroll
-                                for (int k = 0; k < kBK / 16; ++k) {
-                                    // K-major: a K-step of 16 is 32 bytes along each row;
-                                    // MN-major: 16 rows, two 1024-byte row groups
-                                    const uint64_t da = MODE == TC_WGRAD
-                                        ? desc_sw128_mn(a_addr + 2048 * k, 64 * 128)
-                                        : desc_sw128(a_addr + 32 * k);
-                                    const uint64_t db = MODE == TC_WGRAD
-                                        ? desc_sw128_mn(b_addr + 2048 * k, N > 64 ? 64 * 128 : 0)
-                                        : desc_sw128(b_addr + 32 * k);
-                                    umma_bf16(d + (uint32_t)(j * N), da, db, idesc,
-                                              (kb > c0 || k > 0) ? 1u : 0u);
-                                }
+                            for (int k = 0; k < kBK / 16; ++k) {
+                                // K-major: a K-step of 16 is 32 bytes along each row;
+                                // MN-major: 16 rows, two 1024-byte row groups, and
+                                // 64-wide blocks along M / N 8 KB apart
+                                const uint64_t da = MODE == TC_WGRAD
+                                    ? desc_sw128_mn(a_addr + 2048 * k, 64 * 128)
+                                    : desc_sw128(a_addr + 32 * k);
+                                const uint64_t db = MODE == TC_WGRAD
+                                    ? desc_sw128_mn(b_addr + 2048 * k, 64 * 128)
+                                    : desc_sw128(b_addr + 32 * k);
+                                umma_bf16(d, da, db, idesc, (kb > c0 || k > 0) ? 1u : 0u);
                             }
                             umma_commit(empty_bar(s));
                         }
@@ -686,7 +690,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const int x = tx * args.wb + xx, y = ty * args.hb + yy, b = tb * args.bb + bbx;
                     if (x < args.W && y < args.H && b < args.B) {
                         int64_t* o = args.out + (((int64_t)b * args.H + y) * args.W + x) * args.ncols + col0;
-                        if (col0 + NH <= args.ncols && (args.ncols & 1) == 0) {
+                        if (args.out_vec && col0 + NH <= args.ncols && (args.ncols & 1) == 0) {
 #pragma unroll
                             for (int i = 0; i < NH; i += 2) {
                                 longlong2 v;
@@ -737,45 +741,80 @@ __global__ void k_pack_act_nhwc(const int8_t* __restrict__ x, int64_t P, int C, 
 
 // int8 NHWC x [B][H][W][Cin] (9 Cin <= 64) -> bf16 im2col rows [B][H][W][64]:
 // entry k = t Cin + ci holds x at (y + ky - 1, x + kx - 1) for tap t = 3 ky + kx,
-// zero outside the image and for k >= 9 Cin.  Eight entries per thread.
-__global__ void k_pack_im2col(const int8_t* __restrict__ x, int B, int H, int W, int Cin,
-                              uint16_t* __restrict__ out) {
-    const int64_t n = (int64_t)B * H * W * (kBK / 8);
-    const int kmax = 9 * Cin;
-    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
+// zero outside the image and for k >= 9 Cin.  A CTA takes one image row at a
+// time: the three input rows around it (with a zero pixel on either side) are
+// staged in shared memory, then each thread writes 8 entries (16 bytes).
+__global__ void __launch_bounds__(256) k_pack_im2col(const int8_t* __restrict__ x, int B, int H,
+                                                     int W, int Cin,
+                                                     uint16_t* __restrict__ out) {
+    extern __shared__ int8_t win[];            // [3][W + 2][Cin]
+    __shared__ int tab[kBK];                   // window offset of entry k, or -1
+    const int rowlen = (W + 2) * Cin;
+    for (int k = threadIdx.x; k < kBK; k += blockDim.x) {
+        int off = -1;
+        if (k < 9 * Cin) {
+            const int t = k / Cin, ci = k - t * Cin;
+            off = (t / 3) * rowlen + (t % 3) * Cin + ci;
+        }
+        tab[k] = off;
+    }
+    for (int64_t row = blockIdx.x; row < (int64_t)B * H; row += gridDim.x) {
+        const int y = (int)(row % H);
+        const int64_t b = row / H;
+        __syncthreads();                       // readers of the previous row are done
+        for (int i = threadIdx.x; i < 3 * rowlen; i += blockDim.x) {
+            const int r = i / rowlen, rem = i - r * rowlen;
+            const int px = rem / Cin - 1, ci = rem - (rem / Cin) * Cin;
+            const int iy = y + r - 1;
+            win[i] = (iy >= 0 && iy < H && px >= 0 && px < W)
+                         ? x[((b * H + iy) * W + px) * Cin + ci]
+                         : (int8_t)0;
+        }
+        __syncthreads();
+        uint4* orow = reinterpret_cast<uint4*>(out + row * W * kBK);
+        for (int i = threadIdx.x; i < W * (kBK / 8); i += blockDim.x) {
+            const int px = i / (kBK / 8), k0 = (i - px * (kBK / 8)) * 8;
+            const int8_t* wp = win + px * Cin;
+            uint32_t w[4];
+#pragma unroll
+            for (int j = 0; j < 8; j += 2) {
+                const int o0 = tab[k0 + j], o1 = tab[k0 + j + 1];
+                const uint32_t h0 = bf16_bits(o0 >= 0 ? wp[o0] : 0);
+                const uint32_t h1 = bf16_bits(o1 >= 0 ? wp[o1] : 0);
+                w[j / 2] = h0 | (h1 << 16);
+            }
+            orow[i] = make_uint4(w[0], w[1], w[2], w[3]);
+        }
+    }
+}
+
+// shared memory of k_pack_im2col's row window
+inline size_t im2col_smem(int W, int Cin) { return (size_t)3 * (W + 2) * Cin; }
+
+// int8 NHWC [P][C] -> bf16 NHWC [P][C] for C % 8 == 0: eight channels per
+// thread (one 8-byte load, one 16-byte store)
+__global__ void k_pack_act_nhwc8(const int8_t* __restrict__ x, int64_t n8,
+                                 uint16_t* __restrict__ out) {
+    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n8;
          i += (int64_t)gridDim.x * blockDim.x) {
-        const int64_t p = i / (kBK / 8);
-        const int k0 = (int)(i - p * (kBK / 8)) * 8;
-        const int px = (int)(p % W);
-        const int64_t r = p / W;
-        const int py = (int)(r % H);
-        const int64_t b = r / H;
+        const uint2 v = reinterpret_cast<const uint2*>(x)[i];
+        const uint32_t in[2] = {v.x, v.y};
         uint32_t w[4];
 #pragma unroll
-        for (int j = 0; j < 8; j += 2) {
-            uint32_t h[2];
-#pragma unroll
-            for (int u = 0; u < 2; ++u) {
-                const int k = k0 + j + u;
-                int v = 0;
-                if (k < kmax) {
-                    const int t = k / Cin, ci = k - t * Cin;
-                    const int iy = py + t / 3 - 1, ix = px + t % 3 - 1;
-                    if (iy >= 0 && iy < H && ix >= 0 && ix < W)
-                        v = x[((b * H + iy) * W + ix) * Cin + ci];
-                }
-                h[u] = bf16_bits(v);
-            }
-            w[j / 2] = h[0] | (h[1] << 16);
+        for (int k = 0; k < 4; ++k) {
+            const uint32_t word = in[k >> 1] >> (16 * (k & 1));
+            w[k] = (uint32_t)bf16_bits((int8_t)(word & 255u)) |
+                   ((uint32_t)bf16_bits((int8_t)((word >> 8) & 255u)) << 16);
         }
         reinterpret_cast<uint4*>(out)[i] = make_uint4(w[0], w[1], w[2], w[3]);
     }
 }
 
 // int32 delta NHWC (n values, n % 8 == 0) -> limb planes [L][n], eight values
-// per thread and one 16-byte store per plane; records the limb count.
+// per thread and one 16-byte store per plane; records the limb count.  The
+// input is read as 16-byte words when `d` is 16-byte aligned (vec != 0).
 __global__ void __launch_bounds__(256) k_pack_delta_nhwc(const int32_t* __restrict__ d, int64_t n,
-                                                         const uint32_t* maxabs,
+                                                         int vec, const uint32_t* maxabs,
                                                          uint16_t* __restrict__ out,
                                                          int* limbs_out) {
     const int L = limb_count(*maxabs);
@@ -783,9 +822,16 @@ __global__ void __launch_bounds__(256) k_pack_delta_nhwc(const int32_t* __restri
     const int64_t n8 = n / 8;
     for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n8;
          i += (int64_t)gridDim.x * blockDim.x) {
-        const int4 a0 = reinterpret_cast<const int4*>(d)[2 * i];
-        const int4 a1 = reinterpret_cast<const int4*>(d)[2 * i + 1];
-        int64_t v[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
+        int64_t v[8];
+        if (vec) {
+            const int4 a0 = reinterpret_cast<const int4*>(d)[2 * i];
+            const int4 a1 = reinterpret_cast<const int4*>(d)[2 * i + 1];
+            v[0] = a0.x; v[1] = a0.y; v[2] = a0.z; v[3] = a0.w;
+            v[4] = a1.x; v[5] = a1.y; v[6] = a1.z; v[7] = a1.w;
+        } else {
+#pragma unroll
+            for (int k = 0; k < 8; ++k) v[k] = d[8 * i + k];
+        }
         for (int l = 0; l < L; ++l) {
             uint32_t w[4];
 #pragma unroll
@@ -819,14 +865,7 @@ __global__ void k_pack_weights(const int32_t* __restrict__ W, int Cout, int Cin,
     if (blockIdx.x == 0 && threadIdx.x == 0) *limbs_out = L;
     const int64_t n = (int64_t)Cout * 9 * Cin;
     const int64_t nk = (int64_t)Cout * row_k;
-    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
-         i += (int64_t)gridDim.x * blockDim.x) {
-        const int ci = (int)(i % Cin);
-        const int t = (int)((i / Cin) % 9);
-        const int co = (int)(i / (9LL * Cin));
-        int64_t x = W[i];
-        const int64_t it = ((int64_t)t * Cin + ci) * Cout + co;
-        const int64_t ik = (int64_t)co * row_k + t * tap_k + ci;
+    auto split = [L](int64_t x, uint16_t* dst, int64_t plane) {
         for (int l = 0; l < L; ++l) {
             int v;
             if (l < L - 1) {
@@ -836,9 +875,27 @@ __global__ void k_pack_weights(const int32_t* __restrict__ W, int Cout, int Cin,
             } else {
                 v = (int)x;
             }
-            const uint16_t bits = bf16_bits(v);
-            if (wp) wp[l * nk + ik] = bits;
-            if (wtp) wtp[l * n + it] = bits;
+            dst[l * plane] = bf16_bits(v);
+        }
+    };
+    // each layout in its own pass, in its own element order, so that the
+    // 2-byte stores of a warp are contiguous
+    if (wp) {
+        for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
+             i += (int64_t)gridDim.x * blockDim.x) {
+            const int ci = (int)(i % Cin);
+            const int t = (int)((i / Cin) % 9);
+            const int co = (int)(i / (9LL * Cin));
+            split(W[i], wp + (int64_t)co * row_k + t * tap_k + ci, nk);
+        }
+    }
+    if (wtp) {
+        for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
+             i += (int64_t)gridDim.x * blockDim.x) {
+            // i = (t Cin + ci) Cout + co
+            const int co = (int)(i % Cout);
+            const int64_t r = i / Cout;
+            split(W[(int64_t)co * 9 * Cin + r], wtp + i, n);
         }
     }
 }
@@ -905,15 +962,18 @@ cudaError_t launch_gemm(const CUtensorMap& a, const CUtensorMap& b, const TcArgs
     return cudaGetLastError();
 }
 
-// Tile width n and B limbs per stage: interleave when the (last seen) limb
-// count of B is above one.  Any choice is exact; it only changes speed.
+// Tile width n and B limbs per stage from the (last seen) limb count of B:
+// as many limbs per stage as the operand has, up to the TMEM budget (PB N <=
+// 256).  Any choice is exact; it only changes speed.
 template <int MODE>
 cudaError_t launch_gemm_n(int n, int limbs_hint, const CUtensorMap& a, const CUtensorMap& b,
                           const TcArgs& args, cudaStream_t s) {
-    const bool wide = limbs_hint > 1;
     if (n == 128)
-        return wide ? launch_gemm<MODE, 128, 2>(a, b, args, s) : launch_gemm<MODE, 128, 1>(a, b, args, s);
-    return wide ? launch_gemm<MODE, 64, 4>(a, b, args, s) : launch_gemm<MODE, 64, 1>(a, b, args, s);
+        return limbs_hint > 1 ? launch_gemm<MODE, 128, 2>(a, b, args, s)
+                              : launch_gemm<MODE, 128, 1>(a, b, args, s);
+    if (limbs_hint > 2) return launch_gemm<MODE, 64, 4>(a, b, args, s);
+    return limbs_hint == 2 ? launch_gemm<MODE, 64, 2>(a, b, args, s)
+                           : launch_gemm<MODE, 64, 1>(a, b, args, s);
 }
 
 int pick_n(int cols) { return cols % 128 == 0 ? 128 : 64; }
@@ -953,7 +1013,7 @@ bool tc_layer_init(TcLayer& t, const LayerGeom& g, int max_batch, bool has_dgrad
     // Inputs with 9 Cin <= 64 run as one 64-wide K-block of im2col rows.
     const bool pix_ok = g.h >= 8 && g.w >= 8;
     const bool wide = g.cin >= 32;
-    t.im2col = pix_ok && 9 * g.cin <= kBK;
+    t.im2col = pix_ok && 9 * g.cin <= kBK && im2col_smem(g.w, g.cin) <= 48 * 1024;
     t.fwd = pix_ok && (wide || t.im2col);
     t.wgrad = (wide || t.im2col) && g.cout % 8 == 0;
     t.dgrad = has_dgrad && pix_ok && g.cout % 8 == 0;
@@ -987,7 +1047,7 @@ cudaError_t tc_refresh_weights(TcLayer& t, const LayerGeom& g, const int32_t* W,
     if (!t.fwd && !t.dgrad) return cudaSuccess;
     const int64_t n = (int64_t)g.cout * 9 * g.cin;
     {
-        ProfScope ps(K_TC_PACK, s, 0.0, (double)n * 4 * 2);
+        ProfScope ps(K_TC_PACK_W, s, 0.0, (double)n * 4 * 2);
         const int row_k = t.im2col ? kBK : 9 * t.cin_k, tap_k = t.im2col ? g.cin : t.cin_k;
         k_pack_weights<<<grid1d(n), 256, 0, s>>>(W, g.cout, g.cin, row_k, tap_k, maxabs_w,
                                                  t.w_planes, t.wt_planes, t.limbs);
@@ -1003,11 +1063,18 @@ cudaError_t tc_pack_input(TcLayer& t, const LayerGeom& g, const int8_t* x, int b
     if (batch <= 0 || !t.act_nhwc || nhwc_done) return cudaSuccess;
     const int64_t P = (int64_t)batch * g.h * g.w;
     if (t.im2col) {
-        ProfScope ps(K_TC_PACK, s, 0.0, (double)P * (g.cin + 2 * kBK));
-        k_pack_im2col<<<grid1d(P * (kBK / 8)), 256, 0, s>>>(x, batch, g.h, g.w, g.cin, t.act_nhwc);
+        ProfScope ps(K_TC_PACK_X, s, 0.0, (double)P * (g.cin + 2 * kBK));
+        const int64_t rows = (int64_t)batch * g.h;
+        const int grid = (int)(rows < 152 * 8 ? rows : 152 * 8);
+        k_pack_im2col<<<grid, 256, im2col_smem(g.w, g.cin), s>>>(x, batch, g.h, g.w, g.cin,
+                                                                 t.act_nhwc);
         return cudaGetLastError();
     }
-    ProfScope ps(K_TC_PACK, s, 0.0, (double)P * (g.cin + 2 * t.cin8));
+    ProfScope ps(K_TC_PACK_X, s, 0.0, (double)P * (g.cin + 2 * t.cin8));
+    if (g.cin == t.cin8 && g.cin % 8 == 0 && ((uintptr_t)x & 7) == 0) {
+        k_pack_act_nhwc8<<<grid1d(P * g.cin / 8), 256, 0, s>>>(x, P * g.cin / 8, t.act_nhwc);
+        return cudaGetLastError();
+    }
     k_pack_act_nhwc<<<grid1d(P * t.cin8), 256, 0, s>>>(x, P, g.cin, t.cin8, t.act_nhwc);
     return cudaGetLastError();
 }
@@ -1033,6 +1100,7 @@ cudaError_t tc_conv_forward(TcLayer& t, const LayerGeom& g, int batch, int64_t* 
     a.limbs_a = nullptr;
     a.limbs_b = t.limbs;
     a.out = z;
+    a.out_vec = ((uintptr_t)z & 15) == 0;
     a.status = status;
     a.atomic_out = 0;
     if (fo && g.cout % 16 == 0) {
@@ -1079,8 +1147,9 @@ cudaError_t tc_pack_delta(TcLayer& t, const LayerGeom& g, const int32_t* delta,
     // launch also records the limb count for the GEMMs
     const int64_t n = (int64_t)batch * g.h * g.w * g.cout;   // cout % 8 == 0
     {
-        ProfScope ps(K_TC_PACK, s, 0.0, (double)n * 4 * 2);
-        k_pack_delta_nhwc<<<grid1d(n / 8), 256, 0, s>>>(delta, n, maxabs_delta, t.d_nhwc, t.limbs + 1);
+        ProfScope ps(K_TC_PACK_D, s, 0.0, (double)n * 4 * 2);
+        k_pack_delta_nhwc<<<grid1d(n / 8), 256, 0, s>>>(delta, n, ((uintptr_t)delta & 15) == 0,
+                                                       maxabs_delta, t.d_nhwc, t.limbs + 1);
     }
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
@@ -1111,9 +1180,10 @@ cudaError_t tc_conv_wgrad(TcLayer& t, const LayerGeom& g, const int32_t* delta,
     a.tiles_m = (a.taps * t.cin_k + kBM - 1) / kBM;
     a.tiles_n = (g.cout + n - 1) / n;
     a.kb_total = batch * a.ntx * a.nty;
-    // split K so that about one wave of CTAs runs, each with >= one exact chunk
+    // split K so that at most one wave of CTAs runs (every CTA one work unit),
+    // each with >= one exact chunk
     const int tiles = a.tiles_m * a.tiles_n;
-    int splits = (sm_count() + tiles - 1) / tiles;
+    int splits = sm_count() / tiles;
     const int max_splits = (a.kb_total + kChunkBlocks - 1) / kChunkBlocks;
     splits = splits < 1 ? 1 : (splits > max_splits ? max_splits : splits);
     a.kb_per_split = (a.kb_total + splits - 1) / splits;
@@ -1168,6 +1238,7 @@ cudaError_t tc_conv_dgrad(TcLayer& t, const LayerGeom& g, int batch, int64_t* g6
     a.limbs_a = t.limbs + 1;
     a.limbs_b = t.limbs;
     a.out = g64;
+    a.out_vec = ((uintptr_t)g64 & 15) == 0;
     a.status = status;
     a.atomic_out = 0;
     if (fo && g.cin % 16 == 0) {
@@ -1243,7 +1314,8 @@ cudaError_t tc_pack_limbs(const int32_t* x, int64_t n, const uint32_t* maxabs, u
                           int* limbs, cudaStream_t s) {
     if (n <= 0) return cudaSuccess;
     ProfScope ps(K_TC_PACK, s, 0.0, (double)n * 4 * 2);
-    k_pack_delta_nhwc<<<grid1d(n / 8), 256, 0, s>>>(x, n, maxabs, planes, limbs);
+    k_pack_delta_nhwc<<<grid1d(n / 8), 256, 0, s>>>(x, n, ((uintptr_t)x & 15) == 0, maxabs, planes,
+                                                   limbs);
     return cudaGetLastError();
 }
 
