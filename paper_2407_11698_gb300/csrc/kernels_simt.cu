@@ -187,105 +187,77 @@ __global__ void k_fwd_epilogue(const int64_t* __restrict__ z, LayerGeom g, int B
 }
 
 // ---------------------------------------------------------------------------
-// Learning layer forward + RSS loss, in two kernels.
-// k_learn_partial: CTA (d-slice, group of kLrSamples samples) adds its partial
-// sums of z[b][g] = sum_j a[b][j] W_lr[g][j] into zsum with int64 atomics
-// (exact, order independent).  k_learn_finish: one CTA turns zsum into
-// y_hat = floor(z / (256 d)), grad_L = y_hat - 32 onehot, SSE and the loss.
+// Learning layer forward + RSS loss, in one kernel.  A CTA (128-feature
+// slice, 16 samples) adds its partial sums of z[b][g] = sum_j a[b][j] W_lr[g][j]
+// into zsum with int64 atomics (exact, order independent).  The last CTA of
+// a sample group (per-group ticket) turns that group's z into
+// y_hat = floor(z / (256 d)) and grad_L = y_hat - 32 onehot and adds its part
+// of the SSE; the last of those (final ticket) writes the loss.
+// Tickets live behind zsum: zsum[B G + y] per group, zsum[B G + groups].
 // ---------------------------------------------------------------------------
 constexpr int kLrSamples = 16;   // samples per CTA
+constexpr int kLpSlice = 128;    // features per CTA
 
-// CTA (feature slice, group of kLrSamples samples): the slice of a and of
-// every row of W_lr is staged in shared memory with coalesced loads (rows
-// padded so that concurrent rows fall in distinct banks), then each thread
-// forms whole dot products for (sample, class) pairs and adds them into zsum.
 __global__ void __launch_bounds__(256) k_learn_partial(const int8_t* __restrict__ a,
                                                        const int32_t* __restrict__ wlr, int B,
-                                                       int d, int G, int slice,
-                                                       unsigned long long* __restrict__ zsum) {
-    extern __shared__ int32_t lr_smem[];
-    const int wstride = slice + 1;                    // int32 row stride of the W tile
-    const int astride = slice + 4;                    // byte row stride of the a tile
-    int32_t* ws = lr_smem;
-    int8_t* as = reinterpret_cast<int8_t*>(ws + (size_t)G * wstride);
-    const int j0 = blockIdx.x * slice, n = min(slice, d - j0);
-    const int b0 = blockIdx.y * kLrSamples, nb = min(kLrSamples, B - b0);
-    // eight independent loads in flight per thread before the stores
-    const int wtot = G * n, atot = nb * n;
-    for (int base = 0; base < wtot; base += 8 * 256) {
-        int32_t v[8];
-#pragma unroll
-        for (int k = 0; k < 8; ++k) {
-            const int i = base + k * 256 + (int)threadIdx.x;
-            if (i < wtot) {
-                const int g = i / n, j = i - g * n;
-                v[k] = wlr[(int64_t)g * d + j0 + j];
-            }
-        }
-#pragma unroll
-        for (int k = 0; k < 8; ++k) {
-            const int i = base + k * 256 + (int)threadIdx.x;
-            if (i < wtot) {
-                const int g = i / n, j = i - g * n;
-                ws[g * wstride + j] = v[k];
-            }
-        }
-    }
-    for (int base = 0; base < atot; base += 8 * 256) {
-        int8_t v[8];
-#pragma unroll
-        for (int k = 0; k < 8; ++k) {
-            const int i = base + k * 256 + (int)threadIdx.x;
-            if (i < atot) {
-                const int u = i / n, j = i - u * n;
-                v[k] = a[(int64_t)(b0 + u) * d + j0 + j];
-            }
-        }
-#pragma unroll
-        for (int k = 0; k < 8; ++k) {
-            const int i = base + k * 256 + (int)threadIdx.x;
-            if (i < atot) {
-                const int u = i / n, j = i - u * n;
-                as[u * astride + j] = v[k];
-            }
-        }
-    }
-    __syncthreads();
-    for (int p = threadIdx.x; p < nb * G; p += blockDim.x) {
-        const int u = p / G, g = p - u * G;
-        const int32_t* wr = ws + g * wstride;
-        const int8_t* ar = as + u * astride;
-        int64_t acc = 0;
-#pragma unroll 8
-        for (int j = 0; j < n; ++j) acc += (int64_t)wr[j] * ar[j];
-        atomicAdd(&zsum[(int64_t)(b0 + u) * G + g], (unsigned long long)acc);
-    }
-}
-
-__global__ void __launch_bounds__(1024) k_learn_finish(const unsigned long long* __restrict__ zsum,
-                                                       const int32_t* __restrict__ labels, int B,
-                                                       int d, int G, int32_t* __restrict__ grad_l,
+                                                       int d, int G,
+                                                       unsigned long long* __restrict__ zsum,
+                                                       FloorDiv dv, const int32_t* __restrict__ labels,
+                                                       int32_t* __restrict__ grad_l,
                                                        unsigned long long* sse, int64_t* loss,
                                                        uint32_t* maxabs_gl, uint32_t* status) {
-    __shared__ unsigned long long red_s[32];
-    __shared__ uint32_t red_m[32];
+    // thread (u, k): sample u of the group, features k, k + 16, ... of the slice
+    const int u = threadIdx.x >> 4, k = threadIdx.x & 15;
+    const int b = blockIdx.y * kLrSamples + u;
+    const int j0 = blockIdx.x * kLpSlice;
+    int av[kLpSlice / 16];
+#pragma unroll
+    for (int m = 0; m < kLpSlice / 16; ++m) {
+        const int j = j0 + k + 16 * m;
+        av[m] = (b < B && j < d) ? a[(int64_t)b * d + j] : 0;
+    }
+    for (int g = 0; g < G; ++g) {
+        const int32_t* wr = wlr + (int64_t)g * d;
+        long long t = 0;
+#pragma unroll
+        for (int m = 0; m < kLpSlice / 16; ++m) {
+            const int j = j0 + k + 16 * m;
+            if (j < d) t += (long long)__ldg(wr + j) * av[m];
+        }
+#pragma unroll
+        for (int off = 8; off; off >>= 1) t += __shfl_xor_sync(kFull, t, off);
+        if (k == 0 && b < B && t != 0) atomicAdd(&zsum[(int64_t)b * G + g], (unsigned long long)t);
+    }
+    __shared__ int last;
+    __shared__ unsigned long long red_s[8];
+    __shared__ uint32_t red_m[8];
     __shared__ int flags;
-    if (threadIdx.x == 0) flags = 0;
+    unsigned long long* tickets = zsum + (int64_t)B * G;
+    __threadfence();
     __syncthreads();
+    if (threadIdx.x == 0) {
+        flags = 0;
+        last = atomicAdd(&tickets[blockIdx.y], 1ull) == (unsigned long long)gridDim.x - 1;
+    }
+    __syncthreads();
+    if (!last) return;
+    __threadfence();
+    // this sample group's z is complete: y_hat, grad_L, its share of the SSE
     unsigned long long ss = 0;
     uint32_t mx = 0;
     int fl = 0;
-    const int64_t n = (int64_t)B * G;
-    for (int64_t i = threadIdx.x; i < n; i += blockDim.x) {
-        const int b = (int)(i / G), g = (int)(i - (int64_t)b * G);
-        const int lab = labels[b];
+    const int nb = min(kLrSamples, B - (int)blockIdx.y * kLrSamples);
+    for (int i = threadIdx.x; i < nb * G; i += blockDim.x) {
+        const int bb = blockIdx.y * kLrSamples + i / G, g = i % G;
+        const int lab = labels[bb];
         const bool bad = lab < 0 || lab >= G;
         if (bad && g == 0) fl |= ST_BAD_LABEL;
-        const int64_t yhat = scale_floor((int64_t)zsum[i], d);     // NITRO-Scaling, SF = 2^8 d
+        // NITRO-Scaling, SF = 2^8 d: floor(floor(z / 256) / d)
+        const int64_t yhat = dv.floor_div((int64_t)__ldcg(zsum + (int64_t)bb * G + g) >> 8);
         const int64_t v = yhat - ((!bad && g == lab) ? 32 : 0);
         if (!fits_i32(v)) fl |= ST_OVERFLOW;
         const int32_t sv = (int32_t)v;
-        grad_l[i] = sv;
+        grad_l[(int64_t)bb * G + g] = sv;
         ss += (unsigned long long)((int64_t)sv * sv);
         mx = max(mx, abs_u32(sv));
     }
@@ -301,11 +273,16 @@ __global__ void __launch_bounds__(1024) k_learn_finish(const unsigned long long*
     if (threadIdx.x == 0) {
         unsigned long long t = 0;
         uint32_t m = 0;
-        for (int w = 0; w < (int)(blockDim.x >> 5); ++w) { t += red_s[w]; m = max(m, red_m[w]); }
-        *sse = t;                                            // modulo 2^64
-        if (loss) *loss = fdiv64((int64_t)t, 2);
-        atomicMax(maxabs_gl, m);
+        for (int w = 0; w < 8; ++w) { t += red_s[w]; m = max(m, red_m[w]); }
+        atomicAdd(sse, t);                                   // modulo 2^64
+        if (m) atomicMax(maxabs_gl, m);
         if (flags) atomicOr(status, (uint32_t)flags);
+        __threadfence();
+        if (atomicAdd(&tickets[gridDim.y], 1ull) == (unsigned long long)gridDim.y - 1) {
+            __threadfence();
+            const unsigned long long tot = atomicAdd(sse, 0ull);
+            if (loss) *loss = fdiv64((int64_t)tot, 2);
+        }
     }
 }
 
@@ -382,22 +359,40 @@ __global__ void k_grad_to_delta(DeltaSrc src, LayerGeom g, int B, int alpha_inv,
 // ---------------------------------------------------------------------------
 // IntegerSGD (Algorithm 1); blockIdx.y selects the tensor.
 // ---------------------------------------------------------------------------
+__device__ __forceinline__ int32_t sgd_one(const SgdTensor& t, int round_trunc, int32_t w32,
+                                           int64_t g, uint32_t& mx, bool& ovf) {
+    const int64_t w = w32;
+    int64_t d = round_trunc ? t.gdiv.trunc_div(g) : t.gdiv.floor_div(g);
+    if (t.eta_inv != 0) d += round_trunc ? t.ediv.trunc_div(w) : t.ediv.floor_div(w);
+    const int64_t nw = w - d;
+    ovf |= !fits_i32(nw);
+    const int32_t s = (int32_t)nw;
+    mx = max(mx, abs_u32(s));
+    return s;
+}
+
+// Four consecutive weights per thread (16-byte loads of W, two of dW; the
+// tensors are this library's own 256-byte aligned buffers), the tail singly.
 __global__ void k_integersgd(SgdBatch bt) {
     const SgdTensor t = bt.t[blockIdx.y];
     uint32_t mx = 0;
     bool ovf = false;
-    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < t.n;
+    const int64_t n4 = t.n / 4;
+    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n4;
          i += (int64_t)gridDim.x * blockDim.x) {
-        const int64_t w = t.w[i];
-        const int64_t g = t.dw[i];
-        int64_t d = bt.round_trunc ? t.gdiv.trunc_div(g) : t.gdiv.floor_div(g);
-        if (t.eta_inv != 0) d += bt.round_trunc ? t.ediv.trunc_div(w) : t.ediv.floor_div(w);
-        const int64_t nw = w - d;
-        ovf |= !fits_i32(nw);
-        const int32_t s = (int32_t)nw;
-        t.w[i] = s;
-        mx = max(mx, abs_u32(s));
+        const int4 w = reinterpret_cast<const int4*>(t.w)[i];
+        const longlong2 g0 = reinterpret_cast<const longlong2*>(t.dw)[2 * i];
+        const longlong2 g1 = reinterpret_cast<const longlong2*>(t.dw)[2 * i + 1];
+        int4 o;
+        o.x = sgd_one(t, bt.round_trunc, w.x, g0.x, mx, ovf);
+        o.y = sgd_one(t, bt.round_trunc, w.y, g0.y, mx, ovf);
+        o.z = sgd_one(t, bt.round_trunc, w.z, g1.x, mx, ovf);
+        o.w = sgd_one(t, bt.round_trunc, w.w, g1.y, mx, ovf);
+        reinterpret_cast<int4*>(t.w)[i] = o;
     }
+    for (int64_t i = 4 * n4 + blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < t.n;
+         i += (int64_t)gridDim.x * blockDim.x)
+        t.w[i] = sgd_one(t, bt.round_trunc, t.w[i], t.dw[i], mx, ovf);
 #pragma unroll
     for (int off = 16; off; off >>= 1) mx = max(mx, __shfl_xor_sync(kFull, mx, off));
     ovf = __any_sync(kFull, ovf);
@@ -560,20 +555,28 @@ __global__ void __launch_bounds__(256) k_conv_small_wgrad(const int8_t* __restri
 }
 
 // ---------------------------------------------------------------------------
-// Learning-layer backward, fused: for feature q of the block output and a
-// group of kLbSamples samples, delta_fw[b][q] = sum_g grad_L[b][g] W_lr[g][q]
-// (int32 storage rule, then max-pool backward and NITRO-ReLU backward into
-// the last layer's delta) and the learning-weight gradient
-// dW_lr[g][q] += sum_b grad_L[b][g] a[b][q] (64-bit atomics into a zeroed
-// dW_lr).  G <= 16; the W_lr column lives in registers.
+// Learning-layer backward, fused, for G <= 16.  CTA: 64 features q of the
+// block output x 16 samples; grad_L and the 16 x 64 slice of a are staged in
+// shared memory.  dW_lr[g][q] partials over the 16 samples are dot products
+// out of shared memory, added to a zeroed dW_lr with 64-bit atomics.  With a
+// forward layer below (has_delta): thread (q, lane) forms delta_fw[b][q] =
+// sum_g grad_L[b][g] W_lr[g][q] (int32 storage rule) for samples lane,
+// lane + 4, ... and routes it through max-pool backward and NITRO-ReLU
+// backward into that layer's delta; the region bytes of its four samples are
+// loaded before any is used.
 // ---------------------------------------------------------------------------
-constexpr int kLbSamples = 16;
+constexpr int kLbQ = 64;                         // features per CTA
+constexpr int kLbLanes = 4;                      // sample lanes per feature
+constexpr int kLbPer = 4;                        // samples per lane
+constexpr int kLbSamples = kLbLanes * kLbPer;    // samples per CTA
 constexpr int kLbMaxG = 16;
 
+template <int GM>   // classes held in registers: G <= GM
 __global__ void __launch_bounds__(256) k_lr_backward(const int8_t* __restrict__ a,
                                                      const int32_t* __restrict__ gl,
                                                      const int32_t* __restrict__ wlr, int B, int G,
-                                                     LayerGeom lg, int alpha_inv,
+                                                     int d, int has_delta, LayerGeom lg,
+                                                     FloorDiv32 alpha,
                                                      const int8_t* __restrict__ region,
                                                      const int8_t* __restrict__ argmax,
                                                      int32_t* __restrict__ delta,
@@ -581,63 +584,88 @@ __global__ void __launch_bounds__(256) k_lr_backward(const int8_t* __restrict__ 
                                                      const uint32_t* maxabs_gl,
                                                      const uint32_t* maxabs_wlr,
                                                      uint32_t* maxabs_delta, uint32_t* status) {
-    __shared__ int32_t gls[kLbSamples][kLbMaxG];
-    const int d = lg.oh * lg.ow * lg.cout;               // features of the block output
-    const int q = blockIdx.x * blockDim.x + threadIdx.x;
+    __shared__ int32_t gls[kLbSamples][GM];
+    __shared__ int8_t as[kLbSamples][kLbQ];
+    const int ql = threadIdx.x % kLbQ, sl = threadIdx.x / kLbQ;
+    const int q0 = blockIdx.x * kLbQ, q = q0 + ql;
     const int b0 = blockIdx.y * kLbSamples;
     const int nb = min(kLbSamples, B - b0);
-    for (int i = threadIdx.x; i < kLbSamples * kLbMaxG; i += blockDim.x) {
-        const int u = i / kLbMaxG, g = i % kLbMaxG;
+    for (int i = threadIdx.x; i < kLbSamples * GM; i += blockDim.x) {
+        const int u = i / GM, g = i % GM;
         gls[u][g] = (u < nb && g < G) ? gl[(int64_t)(b0 + u) * G + g] : 0;
     }
-    if (blockIdx.x == 0 && blockIdx.y == 0 && threadIdx.x == 0 &&
+#pragma unroll
+    for (int i = 0; i < kLbPer; ++i) {
+        const int u = sl + kLbLanes * i;
+        as[u][ql] = (u < nb && q < d) ? a[(int64_t)(b0 + u) * d + q] : (int8_t)0;
+    }
+    if (has_delta && blockIdx.x == 0 && blockIdx.y == 0 && threadIdx.x == 0 &&
         int64_bound_exceeded(*maxabs_gl, *maxabs_wlr, G))
         atomicOr(status, ST_OVERFLOW);
     __syncthreads();
+    // dW_lr partials: (g, q) pairs over the CTA's samples
+    for (int i = threadIdx.x; i < G * kLbQ; i += blockDim.x) {
+        const int g = i / kLbQ, qq = i - g * kLbQ;
+        if (q0 + qq >= d) continue;
+        long long t = 0;
+#pragma unroll
+        for (int u = 0; u < kLbSamples; ++u) t += (long long)gls[u][g] * as[u][qq];
+        if (t != 0) atomicAdd(&dwlr[(int64_t)g * d + q0 + qq], (unsigned long long)t);
+    }
+    if (!has_delta) return;
     uint32_t mx = 0;
     bool ovf = false;
     if (q < d) {
-        int32_t w[kLbMaxG];
-        int64_t dw[kLbMaxG];
+        int32_t w[GM];
 #pragma unroll
-        for (int g = 0; g < kLbMaxG; ++g) {
-            w[g] = g < G ? wlr[(int64_t)g * d + q] : 0;
-            dw[g] = 0;
-        }
+        for (int g = 0; g < GM; ++g) w[g] = g < G ? wlr[(int64_t)g * d + q] : 0;
         // position of feature q in the (pooled) output grid
         const int c = q % lg.cout;
         const int r = q / lg.cout;
         const int ox = r % lg.ow, oy = r / lg.ow;
-        for (int u = 0; u < nb; ++u) {
-            const int64_t b = b0 + u;
-            uint64_t acc = 0;     // modulo 2^64, exact below the bound
+        // element offsets of the (up to) four pre-pool positions within one image
+        const int64_t img = lg.pool ? (int64_t)lg.h * lg.w * lg.cout : (int64_t)d;
+        const int64_t p00 = lg.pool ? ((int64_t)(2 * oy) * lg.w + 2 * ox) * lg.cout + c : q;
+        const int64_t dx = lg.cout, dy = (int64_t)lg.w * lg.cout;
+        int rgv[kLbPer], am[kLbPer];
 #pragma unroll
-            for (int g = 0; g < kLbMaxG; ++g) acc += (uint64_t)((int64_t)gls[u][g] * w[g]);
-            const int32_t av = a[b * d + q];
-#pragma unroll
-            for (int g = 0; g < kLbMaxG; ++g) dw[g] += (int64_t)gls[u][g] * av;
-            const int64_t gv = (int64_t)acc;
-            ovf |= !fits_i32(gv);
-            const int32_t gs = (int32_t)gv;
-            if (lg.pool) {
-                const int am = argmax[b * d + q];
-#pragma unroll
-                for (int k = 0; k < 4; ++k) {
-                    const int64_t pi = ((b * lg.h + 2 * oy + (k >> 1)) * lg.w + 2 * ox + (k & 1)) * lg.cout + c;
-                    const int32_t dv = (k == am) ? relu_backward(gs, region[pi], alpha_inv) : 0;
-                    delta[pi] = dv;
-                    mx = max(mx, abs_u32(dv));
+        for (int i = 0; i < kLbPer; ++i) {
+            const int u = sl + kLbLanes * i;
+            rgv[i] = 0;
+            am[i] = 0;
+            if (u < nb) {
+                const int64_t base = (b0 + u) * img + p00;
+                if (lg.pool) {
+                    // only the recorded window position receives the gradient
+                    am[i] = argmax[(int64_t)(b0 + u) * d + q];
+                    rgv[i] = region[base + (am[i] & 1) * dx + (am[i] >> 1) * dy];
+                } else {
+                    rgv[i] = region[base];
                 }
-            } else {
-                const int64_t pi = b * d + q;
-                const int32_t dv = relu_backward(gs, region[pi], alpha_inv);
-                delta[pi] = dv;
-                mx = max(mx, abs_u32(dv));
             }
         }
 #pragma unroll
-        for (int g = 0; g < kLbMaxG; ++g)
-            if (g < G && dw[g] != 0) atomicAdd(&dwlr[(int64_t)g * d + q], (unsigned long long)dw[g]);
+        for (int i = 0; i < kLbPer; ++i) {
+            const int u = sl + kLbLanes * i;
+            if (u >= nb) break;
+            uint64_t acc = 0;     // modulo 2^64, exact below the bound
+#pragma unroll
+            for (int g = 0; g < GM; ++g) acc += (uint64_t)((int64_t)gls[u][g] * w[g]);
+            const int64_t gv = (int64_t)acc;
+            ovf |= !fits_i32(gv);
+            const int32_t gs = (int32_t)gv;
+            // NITRO-ReLU backward: piece 1 -> floor(g / alpha_inv), piece 2 -> g, else 0
+            const int32_t dvv = rgv[i] == 1 ? alpha.floor_div(gs) : (rgv[i] == 2 ? gs : 0);
+            mx = max(mx, abs_u32(dvv));
+            const int64_t base = (b0 + u) * img + p00;
+            if (lg.pool) {
+#pragma unroll
+                for (int k = 0; k < 4; ++k)
+                    delta[base + (k & 1) * dx + (k >> 1) * dy] = k == am[i] ? dvv : 0;
+            } else {
+                delta[base] = dvv;
+            }
+        }
     }
 #pragma unroll
     for (int off = 16; off; off >>= 1) mx = max(mx, __shfl_xor_sync(kFull, mx, off));
@@ -718,24 +746,15 @@ cudaError_t simt_learn_fwd(const int8_t* a, const int32_t* wlr, const int32_t* l
                            int d, int G, int64_t* zsum, int32_t* grad_l, unsigned long long* sse,
                            int64_t* loss, uint32_t* maxabs_gl, uint32_t* status, cudaStream_t s) {
     if (B <= 0) return cudaSuccess;
-    cudaError_t e = cudaMemsetAsync(zsum, 0, sizeof(int64_t) * (size_t)B * G, s);
+    const int groups = (B + kLrSamples - 1) / kLrSamples;
+    // partial sums, then the per-group tickets and the final ticket
+    cudaError_t e = cudaMemsetAsync(zsum, 0, sizeof(int64_t) * ((size_t)B * G + groups + 1), s);
     if (e != cudaSuccess) return e;
-    {
-        // slice sized so the staged tiles fit 48 KB of shared memory
-        int slice = (48 * 1024 - 64) / (4 * G + kLrSamples + 8);
-        slice = slice > 256 ? 256 : (slice / 32) * 32;
-        if (slice < 32) slice = 32;
-        const size_t smem = (size_t)G * (slice + 1) * 4 + (size_t)kLrSamples * (slice + 4);
-        dim3 grid((d + slice - 1) / slice, (B + kLrSamples - 1) / kLrSamples);
-        ProfScope ps(K_LEARN_FWD, s, 2.0 * B * d * G, 0.0);
-        k_learn_partial<<<grid, 256, smem, s>>>(a, wlr, B, d, G, slice,
-                                                reinterpret_cast<unsigned long long*>(zsum));
-        e = cudaGetLastError();
-        if (e != cudaSuccess) return e;
-    }
-    ProfScope ps(K_FINISH_LOSS, s, 0.0, 0.0);
-    k_learn_finish<<<1, 1024, 0, s>>>(reinterpret_cast<const unsigned long long*>(zsum), labels, B,
-                                      d, G, grad_l, sse, loss, maxabs_gl, status);
+    dim3 grid((d + kLpSlice - 1) / kLpSlice, groups);
+    ProfScope ps(K_LEARN_FWD, s, 2.0 * B * d * G, 0.0);
+    k_learn_partial<<<grid, 256, 0, s>>>(a, wlr, B, d, G, reinterpret_cast<unsigned long long*>(zsum),
+                                         FloorDiv::make((uint64_t)d), labels, grad_l, sse, loss,
+                                         maxabs_gl, status);
     return cudaGetLastError();
 }
 
@@ -772,7 +791,7 @@ cudaError_t simt_integersgd(const SgdBatch& b_in, cudaStream_t s) {
         b.t[i].gdiv = FloorDiv::make((uint64_t)b.t[i].gamma_inv);
         b.t[i].ediv = FloorDiv::make(b.t[i].eta_inv > 0 ? (uint64_t)b.t[i].eta_inv : 1);
     }
-    dim3 grid(grid_for(nmax, 256, 152 * 4), b.count);
+    dim3 grid(grid_for((nmax + 3) / 4, 256, 152 * 4), b.count);
     double bytes = 0;
     for (int i = 0; i < b.count; ++i) bytes += 16.0 * b.t[i].n;   // W r+w, dW r
     ProfScope ps(K_INTEGERSGD, s, 0.0, bytes);
@@ -833,22 +852,29 @@ cudaError_t simt_conv_small_wgrad(const int8_t* x, const int32_t* d, const Layer
 bool simt_lr_backward_ok(int G) { return G <= kLbMaxG; }
 
 cudaError_t simt_lr_backward(const int8_t* a, const int32_t* gl, const int32_t* wlr, int B, int G,
-                             const LayerGeom& lg, int alpha_inv, const int8_t* region,
+                             int d, const LayerGeom* lg, int alpha_inv, const int8_t* region,
                              const int8_t* argmax, int32_t* delta, int64_t* dwlr,
                              const uint32_t* maxabs_gl, const uint32_t* maxabs_wlr,
                              uint32_t* maxabs_delta, uint32_t* status, cudaStream_t s) {
-    const int d = lg.oh * lg.ow * lg.cout;
     cudaError_t e = cudaMemsetAsync(dwlr, 0, sizeof(int64_t) * (size_t)G * d, s);
     if (e != cudaSuccess || B <= 0) return e;
-    if (lg.pool && ((lg.h & 1) || (lg.w & 1))) {   // rows / columns the pool dropped
-        e = cudaMemsetAsync(delta, 0, sizeof(int32_t) * (size_t)B * lg.h * lg.w * lg.cout, s);
+    if (lg && lg->pool && ((lg->h & 1) || (lg->w & 1))) {   // rows / columns the pool dropped
+        e = cudaMemsetAsync(delta, 0, sizeof(int32_t) * (size_t)B * lg->h * lg->w * lg->cout, s);
         if (e != cudaSuccess) return e;
     }
-    dim3 grid((d + 255) / 256, (B + kLbSamples - 1) / kLbSamples);
-    ProfScope ps(K_LR_BACKWARD, s, 4.0 * B * d * G, 0.0);
-    k_lr_backward<<<grid, 256, 0, s>>>(a, gl, wlr, B, G, lg, alpha_inv, region, argmax, delta,
-                                       reinterpret_cast<unsigned long long*>(dwlr), maxabs_gl,
-                                       maxabs_wlr, maxabs_delta, status);
+    dim3 grid((d + kLbQ - 1) / kLbQ, (B + kLbSamples - 1) / kLbSamples);
+    ProfScope ps(K_LR_BACKWARD, s, (lg ? 4.0 : 2.0) * B * d * G, 0.0);
+    const FloorDiv32 al = FloorDiv32::make((uint32_t)(alpha_inv > 0 ? alpha_inv : 1));
+    auto* dw64 = reinterpret_cast<unsigned long long*>(dwlr);
+    const LayerGeom g0 = lg ? *lg : LayerGeom{};
+    if (G <= 10)
+        k_lr_backward<10><<<grid, 256, 0, s>>>(a, gl, wlr, B, G, d, lg != nullptr, g0, al, region,
+                                               argmax, delta, dw64, maxabs_gl, maxabs_wlr,
+                                               maxabs_delta, status);
+    else
+        k_lr_backward<kLbMaxG><<<grid, 256, 0, s>>>(a, gl, wlr, B, G, d, lg != nullptr, g0, al,
+                                                    region, argmax, delta, dw64, maxabs_gl,
+                                                    maxabs_wlr, maxabs_delta, status);
     return cudaGetLastError();
 }
 

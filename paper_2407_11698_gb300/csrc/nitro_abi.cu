@@ -41,7 +41,7 @@ struct nitro_block {
     int32_t* Wlr = nullptr;
     int64_t* dWlr = nullptr;
     int32_t* grad_l = nullptr;      // [max_batch x G]
-    int64_t* zsum = nullptr;        // [max_batch x G] learning-layer pre-activations
+    int64_t* zsum = nullptr;        // [max_batch x G] learning-layer pre-activations, then a ticket
     int64_t* z64 = nullptr;         // scratch, int64 pre-activations / dgrad outputs
     size_t z64_elems = 0;
     uint32_t* words = nullptr;      // [0] status [1] max|grad_l| [2] max|W_lr|
@@ -221,7 +221,7 @@ nitro_status nitro_init_block(const nitro_block_desc* desc, uint64_t seed, void*
     }
     b->d = desc->n_layers ? b->L.back().out_f : desc->in_features;
     ok = ok && dalloc(b, &b->Wlr, (size_t)b->G * b->d) && dalloc(b, &b->dWlr, (size_t)b->G * b->d) &&
-         dalloc(b, &b->grad_l, (size_t)MB * b->G) && dalloc(b, &b->zsum, (size_t)MB * b->G) && dalloc(b, &b->z64, z_need) &&
+         dalloc(b, &b->grad_l, (size_t)MB * b->G) && dalloc(b, &b->zsum, (size_t)MB * b->G + (MB + 15) / 16 + 1) && dalloc(b, &b->z64, z_need) &&
          dalloc(b, &b->words, n_words(desc->n_layers)) && dalloc(b, &b->sse, 1);
     b->z64_elems = z_need;
     for (int i = 0; ok && i < desc->n_layers; ++i)
@@ -331,12 +331,14 @@ nitro_status nitro_block_backward(nitro_block* b, const int8_t* a_in, const int3
     const int8_t* a_last = n ? b->L[n - 1].act : a_in;
     NITRO_TRY(simt_learn_fwd(a_last, b->Wlr, labels, batch, (int)d, G, b->zsum, b->grad_l, b->sse,
                              loss_dev, w_gl(b), w_status(b), s));
-    if (n > 0 && simt_lr_backward_ok(G)) {
-        // learning-weight gradient and delta_fw -> last layer's delta in one pass
-        Layer& ly = b->L[n - 1];
-        NITRO_TRY(simt_lr_backward(a_last, b->grad_l, b->Wlr, batch, G, ly.g, b->desc.alpha_inv,
-                                   ly.region, ly.argmax, ly.delta, b->dWlr, w_gl(b), w_wlr(b),
-                                   w_delta(b, n - 1), w_status(b), s));
+    if (simt_lr_backward_ok(G)) {
+        // learning-weight gradient and (below a forward layer) delta_fw -> that
+        // layer's delta in one pass
+        Layer* ly = n ? &b->L[n - 1] : nullptr;
+        NITRO_TRY(simt_lr_backward(a_last, b->grad_l, b->Wlr, batch, G, (int)d, ly ? &ly->g : nullptr,
+                                   b->desc.alpha_inv, ly ? ly->region : nullptr,
+                                   ly ? ly->argmax : nullptr, ly ? ly->delta : nullptr, b->dWlr,
+                                   w_gl(b), w_wlr(b), n ? w_delta(b, n - 1) : nullptr, w_status(b), s));
     } else {
         NITRO_TRY(simt_learn_dw(a_last, b->grad_l, batch, (int)d, G, b->dWlr, s));
     }

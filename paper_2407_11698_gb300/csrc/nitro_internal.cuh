@@ -171,7 +171,8 @@ cudaError_t simt_fwd_epilogue(const int64_t* z, const LayerGeom& g, int B, int a
 
 // Learning layer forward + loss: grad_l = floor(a W^T / (256 d)) - 32 onehot,
 // sse = sum grad_l^2 (mod 2^64), loss = floor(sse / 2) (if loss != NULL),
-// max|grad_l| into *maxabs_gl, status bits.  zsum: int64 scratch [B x G].
+// max|grad_l| into *maxabs_gl, status bits.  zsum: int64 scratch of
+// B x G + ceil(B / 16) + 1 words; *sse must be zero on entry.
 cudaError_t simt_learn_fwd(const int8_t* a, const int32_t* wlr, const int32_t* labels, int B,
                            int d, int G, int64_t* zsum, int32_t* grad_l, unsigned long long* sse,
                            int64_t* loss, uint32_t* maxabs_gl, uint32_t* status, cudaStream_t s);
@@ -206,13 +207,14 @@ cudaError_t simt_conv_small_fwd(const int8_t* x, const int32_t* w, const LayerGe
 cudaError_t simt_conv_small_wgrad(const int8_t* x, const int32_t* d, const LayerGeom& g, int B,
                                   int64_t* dw, cudaStream_t s);
 
-// Learning-layer backward for G <= 16, fused: dW_lr (overwritten) and the
-// last forward layer's delta from delta_fw = grad_L W_lr (pre-update), with
-// the int32 storage rule, the int64 bound check, max-pool and NITRO-ReLU
-// backward.  lg: geometry of the block's last forward layer.
+// Learning-layer backward for G <= 16, fused: dW_lr (overwritten) and, when
+// lg (geometry of the block's last forward layer) is not null, that layer's
+// delta from delta_fw = grad_L W_lr (pre-update), with the int32 storage
+// rule, the int64 bound check, max-pool and NITRO-ReLU backward.  d: features
+// of the block output.
 bool simt_lr_backward_ok(int G);
 cudaError_t simt_lr_backward(const int8_t* a, const int32_t* gl, const int32_t* wlr, int B, int G,
-                             const LayerGeom& lg, int alpha_inv, const int8_t* region,
+                             int d, const LayerGeom* lg, int alpha_inv, const int8_t* region,
                              const int8_t* argmax, int32_t* delta, int64_t* dwlr,
                              const uint32_t* maxabs_gl, const uint32_t* maxabs_wlr,
                              uint32_t* maxabs_delta, uint32_t* status, cudaStream_t s);
