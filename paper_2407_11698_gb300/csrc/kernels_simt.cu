@@ -206,7 +206,10 @@ __global__ void __launch_bounds__(256) k_learn_partial(const int8_t* __restrict_
                                                        int32_t* __restrict__ grad_l,
                                                        unsigned long long* sse, int64_t* loss,
                                                        uint32_t* maxabs_gl, uint32_t* status) {
-    // thread (u, k): sample u of the group, features k, k + 16, ... of the slice
+    // thread (u, k): sample u of the group, features k, k + 16, ... of the slice;
+    // the slice of W_lr is staged in shared memory, classes in chunks of kLpG
+    constexpr int kLpG = 16;
+    __shared__ int32_t ws[kLpG][kLpSlice + 1];
     const int u = threadIdx.x >> 4, k = threadIdx.x & 15;
     const int b = blockIdx.y * kLrSamples + u;
     const int j0 = blockIdx.x * kLpSlice;
@@ -216,17 +219,23 @@ __global__ void __launch_bounds__(256) k_learn_partial(const int8_t* __restrict_
         const int j = j0 + k + 16 * m;
         av[m] = (b < B && j < d) ? a[(int64_t)b * d + j] : 0;
     }
-    for (int g = 0; g < G; ++g) {
-        const int32_t* wr = wlr + (int64_t)g * d;
-        long long t = 0;
-#pragma unroll
-        for (int m = 0; m < kLpSlice / 16; ++m) {
-            const int j = j0 + k + 16 * m;
-            if (j < d) t += (long long)__ldg(wr + j) * av[m];
+    for (int gc = 0; gc < G; gc += kLpG) {
+        const int ng = min(kLpG, G - gc);
+        if (gc) __syncthreads();
+        for (int i = threadIdx.x; i < ng * kLpSlice; i += blockDim.x) {
+            const int g = i / kLpSlice, j = i - g * kLpSlice;
+            ws[g][j] = j0 + j < d ? wlr[(int64_t)(gc + g) * d + j0 + j] : 0;
         }
+        __syncthreads();
+        for (int g = 0; g < ng; ++g) {
+            long long t = 0;
 #pragma unroll
-        for (int off = 8; off; off >>= 1) t += __shfl_xor_sync(kFull, t, off);
-        if (k == 0 && b < B && t != 0) atomicAdd(&zsum[(int64_t)b * G + g], (unsigned long long)t);
+            for (int m = 0; m < kLpSlice / 16; ++m) t += (long long)ws[g][k + 16 * m] * av[m];
+#pragma unroll
+            for (int off = 8; off; off >>= 1) t += __shfl_xor_sync(kFull, t, off);
+            if (k == 0 && b < B && t != 0)
+                atomicAdd(&zsum[(int64_t)b * G + gc + g], (unsigned long long)t);
+        }
     }
     __shared__ int last;
     __shared__ unsigned long long red_s[8];
@@ -636,9 +645,12 @@ __global__ void __launch_bounds__(256) k_lr_backward(const int8_t* __restrict__ 
             if (u < nb) {
                 const int64_t base = (b0 + u) * img + p00;
                 if (lg.pool) {
-                    // only the recorded window position receives the gradient
+                    // only the recorded window position receives the gradient; the
+                    // four region bytes load alongside the argmax, not after it
                     am[i] = argmax[(int64_t)(b0 + u) * d + q];
-                    rgv[i] = region[base + (am[i] & 1) * dx + (am[i] >> 1) * dy];
+                    const int r0 = region[base], r1 = region[base + dx];
+                    const int r2 = region[base + dy], r3 = region[base + dy + dx];
+                    rgv[i] = am[i] == 0 ? r0 : (am[i] == 1 ? r1 : (am[i] == 2 ? r2 : r3));
                 } else {
                     rgv[i] = region[base];
                 }

@@ -85,9 +85,11 @@ struct FloorDiv32 {
 #endif
         return (t + ((n - t) >> sh1)) >> sh2;
     }
+    // branch-free: for x < 0, ~x = -(x + 1) and ~q = -q - 1
     __host__ __device__ __forceinline__ int32_t floor_div(int32_t x) const {
-        if (x >= 0) return (int32_t)udiv((uint32_t)x);
-        return -(int32_t)udiv((uint32_t)(-(x + 1))) - 1;
+        const uint32_t ux = x >= 0 ? (uint32_t)x : ~(uint32_t)x;
+        const uint32_t q = udiv(ux);
+        return x >= 0 ? (int32_t)q : (int32_t)~q;
     }
 };
 

@@ -230,15 +230,15 @@ struct TcArgs {
 __device__ __forceinline__ void st16(int8_t* dst, const uint32_t* w) {
     *reinterpret_cast<uint4*>(dst) = make_uint4(w[0], w[1], w[2], w[3]);
 }
-// 16 int8 values (4 packed words) -> 16 bf16 values (two 16-byte stores)
-__device__ __forceinline__ void st16_bf16(uint16_t* dst, const uint32_t* w) {
+// 16 int8 values (4 packed words) -> 16 bf16 values (two 16-byte stores),
+// through the 256-entry table of bf16 bits indexed by byte ^ 0x80
+__device__ __forceinline__ void st16_bf16(uint16_t* dst, const uint32_t* w, const uint16_t* tab) {
     uint32_t o[8];
 #pragma unroll
     for (int k = 0; k < 8; ++k) {
-        const int lo = (int8_t)(w[k >> 1] >> (16 * (k & 1)));
-        const int hi = (int8_t)(w[k >> 1] >> (16 * (k & 1) + 8));
-        o[k] = (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn((float)lo)) |
-               ((uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn((float)hi)) << 16);
+        const uint32_t lo = (w[k >> 1] >> (16 * (k & 1))) & 255u;
+        const uint32_t hi = (w[k >> 1] >> (16 * (k & 1) + 8)) & 255u;
+        o[k] = (uint32_t)tab[lo ^ 0x80u] | ((uint32_t)tab[hi ^ 0x80u] << 16);
     }
     reinterpret_cast<uint4*>(dst)[0] = make_uint4(o[0], o[1], o[2], o[3]);
     reinterpret_cast<uint4*>(dst)[1] = make_uint4(o[4], o[5], o[6], o[7]);
@@ -253,7 +253,7 @@ struct TcCfg {
     static constexpr int STAGE = A_BYTES + PB * B_BYTES;
     static constexpr int S_FIT = (230912 - 1536) / STAGE;   // ~225 KB of shared memory
     static constexpr int S = S_FIT > 9 ? 9 : S_FIT;
-    static constexpr int SMEM = 1024 + S * STAGE + 512;
+    static constexpr int SMEM = 1024 + S * STAGE + 1024;
     static constexpr int NBUF = (512 / (PB * N)) > 4 ? 4 : (512 / (PB * N));   // accumulator sets
     static constexpr int TCOLS = NBUF * PB * N;                                  // 256 or 512
 };
@@ -291,6 +291,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * S + 2 * NBUF);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
     int8_t* relu_tab = reinterpret_cast<int8_t*>(smem + S * C::STAGE + 256);   // 255 entries
+    // bf16 bits of every int8 value v, at index (v + 128) = byte ^ 0x80
+    uint16_t* bf16_tab = reinterpret_cast<uint16_t*>(smem + S * C::STAGE + 512);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const uint32_t bar0 = smem_u32(bars);
@@ -318,6 +320,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     // NITRO-ReLU value of every z* in [-127, 127] (fused forward epilogue)
     if (MODE == TC_FWD && args.fuse && threadIdx.x >= 64 && threadIdx.x < 64 + 255)
         relu_tab[threadIdx.x - 64] = (int8_t)relu_value((int64_t)threadIdx.x - 64 - 127, args.alpha, args.mu);
+    if (MODE == TC_FWD && args.fuse && threadIdx.x >= 320 && threadIdx.x < 320 + 256)
+        bf16_tab[threadIdx.x - 320] = __bfloat16_as_ushort(__float2bfloat16_rn((float)((int)threadIdx.x - 320 - 128)));
     if (warp == 1) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
                          smem_u32(tmem_slot)),
@@ -480,14 +484,27 @@ __global__ void __launch_bounds__(kThreads, 1)
                         const uint32_t base = tmem + ((uint32_t)(32 * q) << 16) +
                                               (uint32_t)((buf * PB + jb) * N + half * NH);
                         const int shift = shift0 + 8 * jb;
-                        uint32_t r[NH];
+                        // 16 columns at a time; acc += v 2^shift as one 32 x 32 -> 64
+                        // multiply-add below 2^32, an add to the high word above
+                        // (shift is a multiple of 8)
 #pragma unroll
-                        for (int j = 0; j < NH / 16; ++j) tmem_ld16_nowait(base + 16 * j, r + 16 * j);
-                        asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+                        for (int j = 0; j < NH / 16; ++j) {
+                            uint32_t r[16];
+                            tmem_ld16(base + 16 * j, r);
+                            if (shift < 32) {
+                                const int m = 1 << shift;
 #pragma unroll
-                        for (int i = 0; i < NH; ++i) {
-                            const int v = __float2int_rz(__uint_as_float(r[i]));   // exact integer
-                            acc[i] += (uint64_t)(int64_t)v << shift;
+                                for (int i = 0; i < 16; ++i) {
+                                    const int v = __float2int_rz(__uint_as_float(r[i]));   // exact integer
+                                    acc[16 * j + i] += (uint64_t)((long long)v * (long long)m);
+                                }
+                            } else {
+#pragma unroll
+                                for (int i = 0; i < 16; ++i) {
+                                    const int v = __float2int_rz(__uint_as_float(r[i]));
+                                    acc[16 * j + i] += (uint64_t)((uint32_t)v << (shift - 32)) << 32;
+                                }
+                            }
                         }
                     }
                     tc_fence_before();
@@ -535,30 +552,23 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const int x = tx * args.wb + xx, y = ty * args.hb + yy, b = tb * args.bb + bbx;
                     const bool valid = x < args.W && y < args.H && b < args.B;
                     const int C = args.Cout;
+                    const int64_t zlo = args.z_lo, zhi = args.z_hi;
+                    const FloorDiv32 sf32 = args.sf32;
                     uint32_t vpk[NH / 4], rpk[NH / 4];
 #pragma unroll
                     for (int g4 = 0; g4 < NH / 4; ++g4) {
                         uint32_t vp = 0, rp = 0;
 #pragma unroll
                         for (int u = 0; u < 4; ++u) {
-                            // z* = floor(z / SF): outside [-127, 127] only the
-                            // saturated piece matters; inside, floor((z >> 8) / 9Cin)
-                            // fits 32 bits.
+                            // z* = floor(z / SF) clamped to [-127, 127] (the NITRO-ReLU
+                            // value is flat outside): floor((z >> 8) / 9Cin) of the
+                            // clamped z fits 32 bits.  The piece comes from z itself.
                             const int64_t z = (int64_t)acc[4 * g4 + u];
-                            int reg, val;
-                            if (z >= args.z_hi) {
-                                reg = 3;
-                                val = relu_tab[254];
-                            } else if (z < args.z_lo) {
-                                reg = 0;
-                                val = relu_tab[0];
-                            } else {
-                                const int zq = args.sf32.floor_div((int32_t)(z >> 8));
-                                reg = zq < 0 ? 1 : 2;
-                                val = relu_tab[zq + 127];
-                            }
+                            const int64_t zc = z < zlo ? zlo : (z >= zhi ? zhi - 1 : z);
+                            const int zq = sf32.floor_div((int32_t)(zc >> 8));
+                            const int reg = z >= zhi ? 3 : (z < zlo ? 0 : (z < 0 ? 1 : 2));
                             rp |= (uint32_t)reg << (8 * u);
-                            vp |= (uint32_t)(uint8_t)(int8_t)val << (8 * u);
+                            vp |= (uint32_t)(uint8_t)relu_tab[zq + 127] << (8 * u);
                         }
                         vpk[g4] = vp;
                         rpk[g4] = rp;
@@ -577,7 +587,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                                 const int64_t o = pix * C + col0 + 16 * k;
                                 st16(args.act + o, vpk + 4 * k);
                                 if (args.out2) st16(args.out2 + o, vpk + 4 * k);
-                                if (args.next_nhwc) st16_bf16(args.next_nhwc + o, vpk + 4 * k);
+                                if (args.next_nhwc) st16_bf16(args.next_nhwc + o, vpk + 4 * k, bf16_tab);
                             }
                         }
                     } else {
@@ -589,21 +599,18 @@ __global__ void __launch_bounds__(kThreads, 1)
                             const uint32_t v01 = __shfl_xor_sync(0xffffffffu, v00, 1);
                             const uint32_t v10 = __shfl_xor_sync(0xffffffffu, v00, dys);
                             const uint32_t v11 = __shfl_xor_sync(0xffffffffu, v00, dys ^ 1);
-                            uint32_t op = 0, ap = 0;
-#pragma unroll
-                            for (int u = 0; u < 4; ++u) {
-                                // window order (0,0), (0,1), (1,0), (1,1); first maximum wins
-                                int best = (int8_t)(v00 >> (8 * u)), k = 0;
-                                const int c1 = (int8_t)(v01 >> (8 * u));
-                                const int c2 = (int8_t)(v10 >> (8 * u));
-                                const int c3 = (int8_t)(v11 >> (8 * u));
-                                if (c1 > best) { best = c1; k = 1; }
-                                if (c2 > best) { best = c2; k = 2; }
-                                if (c3 > best) { best = c3; k = 3; }
-                                op |= (uint32_t)(uint8_t)best << (8 * u);
-                                ap |= (uint32_t)k << (8 * u);
-                            }
-                            opk[g4] = op;
+                            // four windows at once, a byte each: signed maxima, then
+                            // the first position (order (0,0), (0,1), (1,0), (1,1))
+                            // that holds the maximum
+                            const uint32_t best = __vmaxs4(__vmaxs4(v00, v01), __vmaxs4(v10, v11));
+                            const uint32_t e0 = __vcmpeq4(v00, best);
+                            const uint32_t e1 = __vcmpeq4(v01, best);
+                            const uint32_t e2 = __vcmpeq4(v10, best);
+                            uint32_t ap = 0x03030303u;
+                            ap = (ap & ~e2) | (0x02020202u & e2);
+                            ap = (ap & ~e1) | (0x01010101u & e1);
+                            ap &= ~e0;
+                            opk[g4] = best;
                             apk[g4] = ap;
                         }
                         if (valid && !(x & 1) && !(y & 1) && x + 1 < args.W && y + 1 < args.H) {
@@ -615,7 +622,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                                 st16(args.act + o, opk + 4 * k);
                                 if (args.out2) st16(args.out2 + o, opk + 4 * k);
                                 st16(args.argmax + o, apk + 4 * k);
-                                if (args.next_nhwc) st16_bf16(args.next_nhwc + o, opk + 4 * k);
+                                if (args.next_nhwc) st16_bf16(args.next_nhwc + o, opk + 4 * k, bf16_tab);
                             }
                         }
                     }
@@ -634,44 +641,40 @@ __global__ void __launch_bounds__(kThreads, 1)
                     uint32_t mx = 0;
                     if (valid) {
                         const int64_t opix = ((int64_t)b * args.H + y) * args.W + x;
+                        const int npos = args.low_pool ? 4 : 1;
+                        // four channels at a time: gradient, its floor quotient by
+                        // alpha_inv, then each window position's region byte
 #pragma unroll
-                        for (int k16 = 0; k16 < NH / 16; ++k16) {
-                            const int c0 = col0 + 16 * k16;
+                        for (int e4 = 0; e4 < NH / 4; ++e4) {
+                            const int c0 = col0 + 4 * e4;
                             if (c0 >= Cl) break;
-                            int32_t gs[16];
+                            int32_t gs[4], gq[4];
 #pragma unroll
-                            for (int e = 0; e < 16; ++e) {
-                                const int64_t gv = (int64_t)acc[16 * k16 + e];
+                            for (int e = 0; e < 4; ++e) {
+                                const int64_t gv = (int64_t)acc[4 * e4 + e];
                                 ovf |= !fits_i32(gv);
                                 gs[e] = (int32_t)gv;
+                                gq[e] = args.alpha32.floor_div(gs[e]);
                             }
-                            const uint4 amv = args.low_pool
-                                ? *reinterpret_cast<const uint4*>(args.low_argmax + opix * Cl + c0)
-                                : make_uint4(0, 0, 0, 0);
-                            const uint32_t amw[4] = {amv.x, amv.y, amv.z, amv.w};
-                            const int npos = args.low_pool ? 4 : 1;
+                            const uint32_t amw = args.low_pool
+                                ? *reinterpret_cast<const uint32_t*>(args.low_argmax + opix * Cl + c0)
+                                : 0u;
                             for (int k = 0; k < npos; ++k) {
                                 const int64_t ppix = args.low_pool
                                     ? ((int64_t)b * args.low_h + 2 * y + (k >> 1)) * args.low_w + 2 * x + (k & 1)
                                     : opix;
-                                const uint4 rgv = *reinterpret_cast<const uint4*>(args.low_region + ppix * Cl + c0);
-                                const uint32_t rgw[4] = {rgv.x, rgv.y, rgv.z, rgv.w};
-                                int32_t dv[16];
+                                const uint32_t rgw = *reinterpret_cast<const uint32_t*>(args.low_region + ppix * Cl + c0);
+                                int32_t dv[4];
 #pragma unroll
-                                for (int e = 0; e < 16; ++e) {
-                                    const int reg = (int)((rgw[e >> 2] >> (8 * (e & 3))) & 255u);
-                                    const int am = (int)((amw[e >> 2] >> (8 * (e & 3))) & 255u);
-                                    int32_t v = 0;
-                                    if (am == k) {
-                                        v = reg == 1 ? args.alpha32.floor_div(gs[e]) : (reg == 2 ? gs[e] : 0);
-                                    }
+                                for (int e = 0; e < 4; ++e) {
+                                    const int reg = (int)((rgw >> (8 * e)) & 255u);
+                                    const int am = (int)((amw >> (8 * e)) & 255u);
+                                    const int32_t v = am != k ? 0 : (reg == 1 ? gq[e] : (reg == 2 ? gs[e] : 0));
                                     dv[e] = v;
                                     mx = max(mx, abs_u32(v));
                                 }
-                                int4* o = reinterpret_cast<int4*>(args.low_delta + ppix * Cl + c0);
-#pragma unroll
-                                for (int e = 0; e < 4; ++e)
-                                    o[e] = make_int4(dv[4 * e], dv[4 * e + 1], dv[4 * e + 2], dv[4 * e + 3]);
+                                *reinterpret_cast<int4*>(args.low_delta + ppix * Cl + c0) =
+                                    make_int4(dv[0], dv[1], dv[2], dv[3]);
                             }
                         }
                     }
