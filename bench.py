@@ -169,6 +169,69 @@ def kernel_profile(nb):
     return out
 
 
+def _limbs(m):
+    """Signed 8-bit limbs the kernels use for a tensor with max |x| = m."""
+    m = int(m)
+    return 1 if m <= 127 else 2 if m <= 32639 else 3 if m <= 8355711 else 4
+
+
+def issued_profile(nb, net, flush, steps, torch):
+    """Issued tensor work of the tcgen05 contractions over `steps` eager steps:
+    each launch's algorithmic ops times the product of its operands' limb
+    counts (activations 1; W and delta from the layers' max |.|, W read before
+    the step, delta after it).  Launches map to layers by order: every conv's
+    forward in network order, then per block, last layer first, its weight
+    gradient and (above the block's first layer) its input gradient.  Returns
+    {kernel: {"issued_ops", "ms"}} or None when the launches do not match."""
+    import ctypes
+    import numpy as np
+    L = nb.lib()
+    convs = [(bi, i) for bi, g in enumerate(net.blocks) for i, l in enumerate(g.layers)
+             if l[0] == nb.NITRO_CONV3X3]
+    bwd = []
+    for bi, g in enumerate(net.blocks):
+        for i in reversed(range(len(g.layers))):
+            if g.layers[i][0] != nb.NITRO_CONV3X3:
+                continue
+            bwd.append(("tc_conv_wgrad", bi, i))
+            if i > 0:
+                bwd.append(("tc_conv_dgrad", bi, i))
+
+    def maxabs(bi, which, i):
+        return np.abs(net.blocks[bi].get(which, i, check=False).astype(np.int64)).max()
+
+    out = {}
+    for _ in range(steps):
+        wl = {c: _limbs(maxabs(c[0], nb.NITRO_T_W, c[1])) for c in convs}
+        L.nitro_profile_reset()
+        L.nitro_profile_enable(1)
+        flush.zero_()
+        net.step()
+        torch.cuda.synchronize()
+        L.nitro_profile_enable(0)
+        dl = {c: _limbs(maxabs(c[0], nb.NITRO_T_DELTA, c[1])) for c in convs}
+        recs = []
+        for r in range(L.nitro_profile_record_count()):
+            k, ms, ops, by = ctypes.c_int(), ctypes.c_double(), ctypes.c_double(), ctypes.c_double()
+            L.nitro_profile_record(r, ctypes.byref(k), ctypes.byref(ms), ctypes.byref(ops), ctypes.byref(by))
+            recs.append((L.nitro_profile_kernel_name(k.value).decode(), ms.value, ops.value))
+        L.nitro_profile_reset()
+        fwd = [r for r in recs if r[0] == "tc_conv_fwd"]
+        back = [r for r in recs if r[0] in ("tc_conv_wgrad", "tc_conv_dgrad")]
+        if len(fwd) != len(convs) or [r[0] for r in back] != [b[0] for b in bwd]:
+            return None
+        for r, c in zip(fwd, convs):
+            o = out.setdefault("tc_conv_fwd", {"issued_ops": 0.0, "ms": 0.0})
+            o["issued_ops"] += r[2] * wl[c]
+            o["ms"] += r[1]
+        for r, (name, bi, i) in zip(back, bwd):
+            o = out.setdefault(name, {"issued_ops": 0.0, "ms": 0.0})
+            f = dl[(bi, i)] * (wl[(bi, i)] if name == "tc_conv_dgrad" else 1)
+            o["issued_ops"] += r[2] * f
+            o["ms"] += r[1]
+    return out
+
+
 def run_ours(args, rank, world, local_rank):
     import torch
     import torch.distributed as dist
@@ -273,6 +336,7 @@ def run_ours(args, rank, world, local_rank):
     L.nitro_profile_enable(0)
     prof = kernel_profile(nb)
     L.nitro_profile_reset()
+    issued = issued_profile(nb, net, flush, 1, torch) if rank == 0 else None
 
     if rank != 0:
         return None
@@ -293,6 +357,12 @@ def run_ours(args, rank, world, local_rank):
         bound, peak, unit = "hbm", peaks["hbm_gbs"], "GB/s"
         peak_note = "HBM copy, %s" % peak_src
         achieved = dom["bytes"] / dom["launches"] / (per_launch_ms / 1e3) / 1e9
+    issued_line = None
+    if issued and dom_name in issued and bound == "tensor":
+        it = issued[dom_name]
+        iss = it["issued_ops"] / (it["ms"] / 1e3) / 1e12
+        issued_line = {"kernel": dom_name, "tflops": round(iss, 2), "frac": round(iss / peak, 4),
+                       "note": "bf16 MMA work actually issued: algorithmic ops x (A limbs x B limbs)"}
     conv_ops = sum(v["ops"] for k, v in prof.items() if "conv" in k)
     conv_ms = sum(v["ms"] for k, v in prof.items() if "conv" in k)
     line = {
@@ -321,7 +391,10 @@ def run_ours(args, rank, world, local_rank):
                      "peak": round(peak, 2), "unit": unit, "frac": round(achieved / peak, 4),
                      "traffic": ncu_traffic(dom_name), "peak_source": peak_note,
                      "per_launch_ms": round(per_launch_ms, 5),
-                     "share_of_kernel_time": round(dom["ms"] / total_k, 4)},
+                     "share_of_kernel_time": round(dom["ms"] / total_k, 4),
+                     "issued": issued_line},
+        "issued_tflops": ({k: round(v["issued_ops"] / (v["ms"] / 1e3) / 1e12, 2)
+                           for k, v in sorted(issued.items())} if issued else None),
         "conv_tops": round(conv_ops / (conv_ms / 1e3) / 1e12, 3) if conv_ms else None,
         "kernels": {k: {"launches": v["launches"], "ms": round(v["ms"], 4),
                         "share": round(v["ms"] / total_k, 4)} for k, v in sorted(prof.items())},
@@ -352,7 +425,7 @@ def oracle_rate(wl_name, sample_batch, steps, warmup=0):
 
 
 # ------------------------------------------------------------------ kernel sweep
-SWEEP_RANGES = {1: (-127, 127), 2: (-32768, 32639), 3: (-2**23, 2**23 - 1)}
+SWEEP_RANGES = {1: (-127, 127), 2: (-32639, 32639), 3: (-8355711, 8355711)}
 
 
 def run_sweep(args):
@@ -391,10 +464,15 @@ def run_sweep(args):
     def emit(kind, shape, limbs, ops, call_ms, prof, key):
         k = prof.get(key, {"ms": float("nan"), "launches": 1})
         kms = k["ms"] / max(1, k["launches"])
+        passes = 1
+        for v in limbs.values():
+            passes *= v
         line = {"sweep": kind, "shape": shape, "limbs": limbs, "ops": ops,
                 "kernel": key, "kernel_ms": round(kms, 5), "call_ms": round(call_ms, 5),
                 "kernel_tops": round(ops / kms / 1e9, 2), "call_tops": round(ops / call_ms / 1e9, 2),
-                "kernel_frac_bf16": round(ops / kms / 1e9 / peak, 4), "peak": peak,
+                "kernel_frac_bf16": round(ops / kms / 1e9 / peak, 4),
+                "issued_tflops": round(ops * passes / kms / 1e9, 2),
+                "issued_frac_bf16": round(ops * passes / kms / 1e9 / peak, 4), "peak": peak,
                 "peak_source": "bf16 dense, %s" % src}
         print(json.dumps(line), flush=True)
 
@@ -447,6 +525,23 @@ def run_sweep(args):
               flush=True)
         gm.close()
         del a, b8, c
+        torch.cuda.empty_cache()
+    # IntegerSGD alone: one linear layer of n x n weights, 16 bytes per weight
+    # (W read + write, dW read), against the measured HBM copy bandwidth
+    hbm = peaks["hbm_gbs"]
+    for n in (4096, 16384):
+        blk = nb.Block([(nb.NITRO_LINEAR, n, n, 1, 1, 0)], n, seed=1, max_batch=1)
+        ms, prof = timed(lambda: blk.sgd(), 5)
+        k = prof.get("integersgd", {"ms": float("nan"), "launches": 1})
+        kms = k["ms"] / max(1, k["launches"])
+        params = n * n + 10 * n
+        byts = 16.0 * params
+        print(json.dumps({"sweep": "integersgd", "params": params, "bytes": byts,
+                          "kernel_ms": round(kms, 5), "call_ms": round(ms, 5),
+                          "kernel_gbs": round(byts / kms / 1e6, 1),
+                          "kernel_frac_hbm": round(byts / kms / 1e6 / hbm, 4), "peak": hbm,
+                          "peak_source": "HBM copy, %s" % src}), flush=True)
+        blk.close()
         torch.cuda.empty_cache()
     return 0
 

@@ -24,7 +24,6 @@ struct nitro_gemm {
     int max_m = 0, max_n = 0, max_k = 0;
     uint16_t* a = nullptr;       // bf16 [M][K]
     uint16_t* b = nullptr;       // bf16 limb planes [4][N][K]
-    int* limbs = nullptr;
     uint32_t* words = nullptr;   // [0] max|B| [1] status
     std::vector<void*> allocs;
 };
@@ -77,8 +76,9 @@ nitro_status nitro_conv3x3_create(int max_batch, int h, int w, int cin, int cout
     if (!c) return NITRO_ERR_CUDA;
     c->g = LayerGeom{NITRO_CONV3X3, cin, cout, h, w, 0, h, w};
     c->max_batch = max_batch;
-    bool ok = tc_layer_init(c->t, c->g, max_batch, true, c->allocs, c->host_allocs) &&
-              dalloc(c->allocs, &c->words, 4);
+    bool ok = dalloc(c->allocs, &c->words, 4) &&
+              tc_layer_init(c->t, c->g, max_batch, true, c->words, c->words + 1, c->allocs,
+                            c->host_allocs);
     if (ok) ok = cudaMemset(c->words, 0, 16) == cudaSuccess;
     if (!ok) {
         free_all(c->allocs);
@@ -161,7 +161,7 @@ nitro_status nitro_gemm_create(int max_m, int max_n, int max_k, nitro_gemm** out
     g->max_k = max_k;
     bool ok = dalloc(g->allocs, &g->a, (size_t)max_m * max_k) &&
               dalloc(g->allocs, &g->b, (size_t)kMaxLimbs * max_n * max_k) &&
-              dalloc(g->allocs, &g->limbs, 1) && dalloc(g->allocs, &g->words, 2);
+              dalloc(g->allocs, &g->words, 2);
     if (ok) ok = cudaMemset(g->words, 0, 8) == cudaSuccess;
     if (!ok) {
         free_all(g->allocs);
@@ -190,8 +190,8 @@ nitro_status nitro_gemm_run(nitro_gemm* g, const int8_t* a, const int32_t* b, in
     }
     TRY(tc_pack_int8(a, m, k, g->a, s));
     TRY(tc_maxabs(b, (int64_t)n * k, g->words, s));
-    TRY(tc_pack_limbs(b, (int64_t)n * k, g->words, g->b, g->limbs, s));
-    TRY(tc_gemm_run(g->a, g->b, m, n, k, g->limbs, c, g->words + 1, s));
+    TRY(tc_pack_limbs(b, (int64_t)n * k, g->words, g->b, s));
+    TRY(tc_gemm_run(g->a, g->b, m, n, k, g->words, c, g->words + 1, s));
     return NITRO_OK;
 }
 

@@ -242,7 +242,7 @@ __global__ void __launch_bounds__(256) k_learn_partial(const int8_t* __restrict_
     __shared__ uint32_t red_m[8];
     __shared__ int flags;
     unsigned long long* tickets = zsum + (int64_t)B * G;
-    __threadfence();
+    if (k == 0) __threadfence();     // the lanes that added into zsum
     __syncthreads();
     if (threadIdx.x == 0) {
         flags = 0;
@@ -380,6 +380,29 @@ __device__ __forceinline__ int32_t sgd_one(const SgdTensor& t, int round_trunc, 
     return s;
 }
 
+// The updated weight w (element i of [Cout][9][cin]) into its four bf16 limb
+// planes: limbs 0..2 the digits ((x + 128) & 255) - 128 of successive base-256
+// remainders, limb 3 the rest; each limb is an integer of at most 8 bits, so
+// the top half of its fp32 bits is its exact bf16.
+__device__ __forceinline__ void sgd_planes(const SgdTensor& t, int64_t i, int32_t w) {
+    const uint32_t q = t.cin_div.udiv((uint32_t)i);
+    const int ci = (int)(i - (int64_t)q * t.cin);
+    const int tap = (int)(q % 9u), co = (int)(q / 9u);
+    uint16_t* p = t.planes + (int64_t)co * t.row_k + tap * t.tap_k + ci;
+    int64_t x = w;
+#pragma unroll
+    for (int l = 0; l < 4; ++l) {
+        int v;
+        if (l < 3) {
+            v = (int)(((x + 128) & 255) - 128);
+            x = (x - v) >> 8;
+        } else {
+            v = (int)x;
+        }
+        p[l * t.plane] = (uint16_t)(__float_as_uint((float)v) >> 16);
+    }
+}
+
 // Four consecutive weights per thread (16-byte loads of W, two of dW; the
 // tensors are this library's own 256-byte aligned buffers), the tail singly.
 __global__ void k_integersgd(SgdBatch bt) {
@@ -398,10 +421,19 @@ __global__ void k_integersgd(SgdBatch bt) {
         o.z = sgd_one(t, bt.round_trunc, w.z, g1.x, mx, ovf);
         o.w = sgd_one(t, bt.round_trunc, w.w, g1.y, mx, ovf);
         reinterpret_cast<int4*>(t.w)[i] = o;
+        if (t.planes) {
+            sgd_planes(t, 4 * i, o.x);
+            sgd_planes(t, 4 * i + 1, o.y);
+            sgd_planes(t, 4 * i + 2, o.z);
+            sgd_planes(t, 4 * i + 3, o.w);
+        }
     }
     for (int64_t i = 4 * n4 + blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < t.n;
-         i += (int64_t)gridDim.x * blockDim.x)
-        t.w[i] = sgd_one(t, bt.round_trunc, t.w[i], t.dw[i], mx, ovf);
+         i += (int64_t)gridDim.x * blockDim.x) {
+        const int32_t nw = sgd_one(t, bt.round_trunc, t.w[i], t.dw[i], mx, ovf);
+        t.w[i] = nw;
+        if (t.planes) sgd_planes(t, i, nw);
+    }
 #pragma unroll
     for (int off = 16; off; off >>= 1) mx = max(mx, __shfl_xor_sync(kFull, mx, off));
     ovf = __any_sync(kFull, ovf);
@@ -611,6 +643,43 @@ __global__ void __launch_bounds__(256) k_lr_backward(const int8_t* __restrict__ 
     if (has_delta && blockIdx.x == 0 && blockIdx.y == 0 && threadIdx.x == 0 &&
         int64_bound_exceeded(*maxabs_gl, *maxabs_wlr, G))
         atomicOr(status, ST_OVERFLOW);
+    // loads of the delta path (W_lr column, argmax, region bytes) go out with
+    // the staging loads, before the barrier
+    const bool act = has_delta && q < d;
+    int32_t w[GM];
+    int rgv[kLbPer], am[kLbPer];
+    int64_t img = 0, p00 = 0, dx = 0, dy = 0;
+#pragma unroll
+    for (int g = 0; g < GM; ++g) w[g] = (act && g < G) ? wlr[(int64_t)g * d + q] : 0;
+    if (act) {
+        // position of feature q in the (pooled) output grid
+        const int c = q % lg.cout;
+        const int r = q / lg.cout;
+        const int ox = r % lg.ow, oy = r / lg.ow;
+        // element offsets of the (up to) four pre-pool positions within one image
+        img = lg.pool ? (int64_t)lg.h * lg.w * lg.cout : (int64_t)d;
+        p00 = lg.pool ? ((int64_t)(2 * oy) * lg.w + 2 * ox) * lg.cout + c : q;
+        dx = lg.cout;
+        dy = (int64_t)lg.w * lg.cout;
+    }
+#pragma unroll
+    for (int i = 0; i < kLbPer; ++i) {
+        const int u = sl + kLbLanes * i;
+        rgv[i] = 0;
+        am[i] = 0;
+        if (act && u < nb) {
+            const int64_t base = (b0 + u) * img + p00;
+            if (lg.pool) {
+                // only the recorded window position receives the gradient
+                am[i] = argmax[(int64_t)(b0 + u) * d + q];
+                const int r0 = region[base], r1 = region[base + dx];
+                const int r2 = region[base + dy], r3 = region[base + dy + dx];
+                rgv[i] = am[i] == 0 ? r0 : (am[i] == 1 ? r1 : (am[i] == 2 ? r2 : r3));
+            } else {
+                rgv[i] = region[base];
+            }
+        }
+    }
     __syncthreads();
     // dW_lr partials: (g, q) pairs over the CTA's samples
     for (int i = threadIdx.x; i < G * kLbQ; i += blockDim.x) {
@@ -625,37 +694,6 @@ __global__ void __launch_bounds__(256) k_lr_backward(const int8_t* __restrict__ 
     uint32_t mx = 0;
     bool ovf = false;
     if (q < d) {
-        int32_t w[GM];
-#pragma unroll
-        for (int g = 0; g < GM; ++g) w[g] = g < G ? wlr[(int64_t)g * d + q] : 0;
-        // position of feature q in the (pooled) output grid
-        const int c = q % lg.cout;
-        const int r = q / lg.cout;
-        const int ox = r % lg.ow, oy = r / lg.ow;
-        // element offsets of the (up to) four pre-pool positions within one image
-        const int64_t img = lg.pool ? (int64_t)lg.h * lg.w * lg.cout : (int64_t)d;
-        const int64_t p00 = lg.pool ? ((int64_t)(2 * oy) * lg.w + 2 * ox) * lg.cout + c : q;
-        const int64_t dx = lg.cout, dy = (int64_t)lg.w * lg.cout;
-        int rgv[kLbPer], am[kLbPer];
-#pragma unroll
-        for (int i = 0; i < kLbPer; ++i) {
-            const int u = sl + kLbLanes * i;
-            rgv[i] = 0;
-            am[i] = 0;
-            if (u < nb) {
-                const int64_t base = (b0 + u) * img + p00;
-                if (lg.pool) {
-                    // only the recorded window position receives the gradient; the
-                    // four region bytes load alongside the argmax, not after it
-                    am[i] = argmax[(int64_t)(b0 + u) * d + q];
-                    const int r0 = region[base], r1 = region[base + dx];
-                    const int r2 = region[base + dy], r3 = region[base + dy + dx];
-                    rgv[i] = am[i] == 0 ? r0 : (am[i] == 1 ? r1 : (am[i] == 2 ? r2 : r3));
-                } else {
-                    rgv[i] = region[base];
-                }
-            }
-        }
 #pragma unroll
         for (int i = 0; i < kLbPer; ++i) {
             const int u = sl + kLbLanes * i;
@@ -802,10 +840,15 @@ cudaError_t simt_integersgd(const SgdBatch& b_in, cudaStream_t s) {
         if (b.t[i].gamma_inv <= 0 || b.t[i].eta_inv < 0) return cudaErrorInvalidValue;
         b.t[i].gdiv = FloorDiv::make((uint64_t)b.t[i].gamma_inv);
         b.t[i].ediv = FloorDiv::make(b.t[i].eta_inv > 0 ? (uint64_t)b.t[i].eta_inv : 1);
+        if (b.t[i].planes) {
+            if (b.t[i].cin < 1 || b.t[i].n >= ((int64_t)1 << 31)) return cudaErrorInvalidValue;
+            b.t[i].cin_div = FloorDiv32::make((uint32_t)b.t[i].cin);
+        }
     }
     dim3 grid(grid_for((nmax + 3) / 4, 256, 152 * 4), b.count);
     double bytes = 0;
-    for (int i = 0; i < b.count; ++i) bytes += 16.0 * b.t[i].n;   // W r+w, dW r
+    for (int i = 0; i < b.count; ++i)
+        bytes += (b.t[i].planes ? 24.0 : 16.0) * b.t[i].n;   // W r+w, dW r (+ 4 bf16 planes)
     ProfScope ps(K_INTEGERSGD, s, 0.0, bytes);
     k_integersgd<<<grid, 256, 0, s>>>(b);
     return cudaGetLastError();

@@ -225,7 +225,8 @@ nitro_status nitro_init_block(const nitro_block_desc* desc, uint64_t seed, void*
          dalloc(b, &b->words, n_words(desc->n_layers)) && dalloc(b, &b->sse, 1);
     b->z64_elems = z_need;
     for (int i = 0; ok && i < desc->n_layers; ++i)
-        ok = tc_layer_init(b->L[i].tc, b->L[i].g, desc->max_batch, i > 0, b->allocs, b->host_allocs);
+        ok = tc_layer_init(b->L[i].tc, b->L[i].g, desc->max_batch, i > 0, w_w(b, i), w_delta(b, i),
+                           b->allocs, b->host_allocs);
     if (!ok) {
         free_all(b);
         delete b;
@@ -400,16 +401,20 @@ nitro_status nitro_integersgd_step(nitro_block* b, void* stream) {
     SgdBatch bt{};
     bt.round_trunc = b->desc.sgd_round == NITRO_ROUND_TRUNC;
     bt.status = w_status(b);
-    for (int i = 0; i < n; ++i)
-        bt.t[bt.count++] = SgdTensor{b->L[i].W, b->L[i].dW, b->L[i].wcount, gamma_fw,
-                                     b->desc.eta_inv_fw, w_w(b, i), {}, {}};
+    for (int i = 0; i < n; ++i) {
+        // the update also writes the tensor-core weight planes of the layer
+        SgdTensor st{b->L[i].W, b->L[i].dW, b->L[i].wcount, gamma_fw, b->desc.eta_inv_fw,
+                     w_w(b, i), {}, {}, nullptr, 0, 0, 0, 0, {}};
+        tc_weight_planes(b->L[i].tc, b->L[i].g, &st.planes, &st.plane, &st.row_k, &st.tap_k);
+        st.cin = b->L[i].g.cin;
+        bt.t[bt.count++] = st;
+    }
     bt.t[bt.count++] = SgdTensor{b->Wlr, b->dWlr, (int64_t)b->G * b->d, b->desc.gamma_inv_lr,
-                                 b->desc.eta_inv_lr, w_wlr(b), {}, {}};
+                                 b->desc.eta_inv_lr, w_wlr(b), {}, {}, nullptr, 0, 0, 0, 0, {}};
     NITRO_TRY(cudaMemsetAsync(w_wlr(b), 0, 4, s));
     if (n) NITRO_TRY(cudaMemsetAsync(w_w(b, 0), 0, 4 * n, s));
     NITRO_TRY(simt_integersgd(bt, s));
-    for (int i = 0; i < n; ++i)
-        NITRO_TRY(tc_refresh_weights(b->L[i].tc, b->L[i].g, b->L[i].W, w_w(b, i), s));
+    for (int i = 0; i < n; ++i) NITRO_TRY(tc_weights_hint(b->L[i].tc, s));
     return NITRO_OK;
 }
 

@@ -230,6 +230,12 @@ struct SgdTensor {
     int64_t gamma_inv, eta_inv;
     uint32_t* maxabs_w;
     FloorDiv gdiv, ediv;   // dividers for gamma_inv and eta_inv (filled by simt_integersgd)
+    // optional bf16 limb planes of a conv weight [Cout][9][cin] that the update
+    // writes itself: planes[l plane + co row_k + t tap_k + ci], all four limbs
+    uint16_t* planes;
+    int64_t plane;
+    int row_k, tap_k, cin;
+    FloorDiv32 cin_div;    // filled by simt_integersgd
 };
 struct SgdBatch {
     SgdTensor t[kMaxSgdTensors];

@@ -147,10 +147,10 @@ __device__ __forceinline__ uint64_t desc_sw128_mn(uint32_t saddr, uint32_t mn_st
     return d;
 }
 
-// Instruction descriptor: kind::f16, A = B = bf16, D = f32; A and B K-major
-// unless mn (bits 15 and 16: MN-major).
-__host__ __device__ constexpr uint32_t idesc_bf16(int m, int n, bool mn = false) {
-    return (1u << 4) | (1u << 7) | (1u << 10) | (mn ? (3u << 15) : 0u) |
+// Instruction descriptor: kind::f16, A = B = bf16, D = f32; A (bit 15) and B
+// (bit 16) K-major unless marked MN-major.
+__host__ __device__ constexpr uint32_t idesc_bf16(int m, int n, bool a_mn = false, bool b_mn = false) {
+    return (1u << 4) | (1u << 7) | (1u << 10) | (a_mn ? (1u << 15) : 0u) | (b_mn ? (1u << 16) : 0u) |
            ((uint32_t)(n >> 3) << 17) | ((uint32_t)(m >> 4) << 24);
 }
 
@@ -188,6 +188,15 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
     asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
 
+// Limbs of a tensor with max |x| = m.  The split is canonical: limbs 0..2 are
+// the digits ((x + 128) & 255) - 128 of successive base-256 remainders and
+// limb 3 takes the rest (in [-128, 128] for int32).  With the thresholds below
+// every limb at index >= L is zero, so the first L planes of the 4-limb split
+// are exact and producers may write all four without knowing L.
+__host__ __device__ __forceinline__ int limb_count(uint32_t m) {
+    return m <= 127u ? 1 : (m <= 32639u ? 2 : (m <= 8355711u ? 3 : 4));
+}
+
 // ------------------------------------------------------------------ kernel
 struct TcArgs {
     int B, H, W, Cin, Cout, Bp;
@@ -198,8 +207,8 @@ struct TcArgs {
     int tiles_m, tiles_n, total_tiles;
     int kb_total, kb_per_split;
     int ncols;             // valid output columns (Cout for fwd/wgrad, Cin for dgrad)
-    const int* limbs_a;    // limb counts (nullptr = 1)
-    const int* limbs_b;
+    const uint32_t* max_a;  // max |operand| words setting the limb counts (nullptr = 1 limb)
+    const uint32_t* max_b;
     int64_t* out;
     uint32_t* status;
     int atomic_out;
@@ -334,10 +343,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
 
-    int LA = args.limbs_a ? *args.limbs_a : 1;
-    int LB = args.limbs_b ? *args.limbs_b : 1;
-    LA = LA < 1 ? 1 : (LA > kMaxLimbs ? kMaxLimbs : LA);
-    LB = LB < 1 ? 1 : (LB > kMaxLimbs ? kMaxLimbs : LB);
+    const int LA = args.max_a ? limb_count(*args.max_a) : 1;
+    const int LB = args.max_b ? limb_count(*args.max_b) : 1;
     const int NG = (LB + PB - 1) / PB;       // groups of B limbs per A limb
     const int passes = LA * NG;
 
@@ -379,8 +386,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                             const int nc = (args.Cout + kBK - 1) / kBK;
                             const int t = kb / nc, cb = kb - t * nc, ky = t / 3, kx = t - 3 * ky;
                             tma_load_5d(a_dst, &tmA, fb, cb * kBK, x0 - kx + 1, y0 - ky + 1, b0, la);
+                            // B MN-major from the forward planes [L][Cout][9][Cin64]:
+                            // rows co (K) of 64 consecutive ci (N) for tap t
                             for (int j = 0; j < nb; ++j)
-                                tma_load_4d(b_dst + j * C::B_BYTES, &tmB, fb, cb * kBK, n0, t, lb0 + j);
+#pragma unroll
+                                for (int h = 0; h < N / 64; ++h)
+                                    tma_load_4d(b_dst + j * C::B_BYTES + h * (64 * 128), &tmB, fb,
+                                                n0 + 64 * h, t, cb * kBK, lb0 + j);
                         } else {  // TC_WGRAD: rows (tap, ci), K = a 64-pixel box (wb x hb)
                             // of one image; both operands MN-major from the NHWC
                             // copies (channels contiguous), the tap shift on x / y.
@@ -415,7 +427,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             // accumulators side by side in TMEM: one MMA of width nb * N covers them
             uint32_t idesc_nb[PB + 1];
 #pragma unroll
-            for (int j = 1; j <= PB; ++j) idesc_nb[j] = idesc_bf16(kBM, j * N, MODE == TC_WGRAD);
+            for (int j = 1; j <= PB; ++j)
+                idesc_nb[j] = idesc_bf16(kBM, j * N, MODE == TC_WGRAD, MODE == TC_WGRAD || MODE == TC_DGRAD);
             int it = 0, chunk = 0;
             for (int tile = blockIdx.x; tile < args.total_tiles; tile += gridDim.x) {
                 const Tile T = decode_tile(args, tile);
@@ -447,7 +460,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                                 const uint64_t da = MODE == TC_WGRAD
                                     ? desc_sw128_mn(a_addr + 2048 * k, 64 * 128)
                                     : desc_sw128(a_addr + 32 * k);
-                                const uint64_t db = MODE == TC_WGRAD
+                                const uint64_t db = (MODE == TC_WGRAD || MODE == TC_DGRAD)
                                     ? desc_sw128_mn(b_addr + 2048 * k, 64 * 128)
                                     : desc_sw128(b_addr + 32 * k);
                                 umma_bf16(d, da, db, idesc, (kb > c0 || k > 0) ? 1u : 0u);
@@ -722,10 +735,6 @@ __global__ void __launch_bounds__(kThreads, 1)
 }
 
 // ------------------------------------------------------------------ limb packing
-__device__ __forceinline__ int limb_count(uint32_t m) {
-    // top limb in [-128, 128]: ranges of 1..4 signed-digit limbs
-    return m <= 128u ? 1 : (m <= 32895u ? 2 : (m <= 8421375u ? 3 : 4));
-}
 __device__ __forceinline__ uint16_t bf16_bits(int v) {
     return __bfloat16_as_ushort(__float2bfloat16_rn((float)v));   // exact for |v| <= 256
 }
@@ -814,14 +823,12 @@ __global__ void k_pack_act_nhwc8(const int8_t* __restrict__ x, int64_t n8,
 }
 
 // int32 delta NHWC (n values, n % 8 == 0) -> limb planes [L][n], eight values
-// per thread and one 16-byte store per plane; records the limb count.  The
+// per thread and one 16-byte store per plane (L from *maxabs).  The
 // input is read as 16-byte words when `d` is 16-byte aligned (vec != 0).
 __global__ void __launch_bounds__(256) k_pack_delta_nhwc(const int32_t* __restrict__ d, int64_t n,
                                                          int vec, const uint32_t* maxabs,
-                                                         uint16_t* __restrict__ out,
-                                                         int* limbs_out) {
+                                                         uint16_t* __restrict__ out) {
     const int L = limb_count(*maxabs);
-    if (limbs_out && blockIdx.x == 0 && threadIdx.x == 0) *limbs_out = L;
     const int64_t n8 = n / 8;
     for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n8;
          i += (int64_t)gridDim.x * blockDim.x) {
@@ -859,13 +866,10 @@ __global__ void __launch_bounds__(256) k_pack_delta_nhwc(const int32_t* __restri
 
 // W [Cout][9][Cin] -> w_planes [L][Cout][row_k] with entry (t, ci) at
 // t tap_k + ci (padding left zero; row_k = 9 Ck, tap_k = Ck with Ck = Cin
-// rounded up to 64, or row_k = 64, tap_k = Cin for im2col rows) and
-// wt_planes [L][9][Cin][Cout]
+// rounded up to 64, or row_k = 64, tap_k = Cin for im2col rows)
 __global__ void k_pack_weights(const int32_t* __restrict__ W, int Cout, int Cin, int row_k,
-                               int tap_k, const uint32_t* maxabs, uint16_t* __restrict__ wp,
-                               uint16_t* __restrict__ wtp, int* limbs_out) {
+                               int tap_k, const uint32_t* maxabs, uint16_t* __restrict__ wp) {
     const int L = limb_count(*maxabs);
-    if (blockIdx.x == 0 && threadIdx.x == 0) *limbs_out = L;
     const int64_t n = (int64_t)Cout * 9 * Cin;
     const int64_t nk = (int64_t)Cout * row_k;
     auto split = [L](int64_t x, uint16_t* dst, int64_t plane) {
@@ -881,8 +885,6 @@ __global__ void k_pack_weights(const int32_t* __restrict__ W, int Cout, int Cin,
             dst[l * plane] = bf16_bits(v);
         }
     };
-    // each layout in its own pass, in its own element order, so that the
-    // 2-byte stores of a warp are contiguous
     if (wp) {
         for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
              i += (int64_t)gridDim.x * blockDim.x) {
@@ -892,15 +894,7 @@ __global__ void k_pack_weights(const int32_t* __restrict__ W, int Cout, int Cin,
             split(W[i], wp + (int64_t)co * row_k + t * tap_k + ci, nk);
         }
     }
-    if (wtp) {
-        for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
-             i += (int64_t)gridDim.x * blockDim.x) {
-            // i = (t Cin + ci) Cout + co
-            const int co = (int)(i % Cout);
-            const int64_t r = i / Cout;
-            split(W[(int64_t)co * 9 * Cin + r], wtp + i, n);
-        }
-    }
+
 }
 
 // ------------------------------------------------------------------ host side
@@ -1008,8 +1002,11 @@ inline int round_up(int v, int m) { return (v + m - 1) / m * m; }
 }  // namespace
 
 bool tc_layer_init(TcLayer& t, const LayerGeom& g, int max_batch, bool has_dgrad,
+                   const uint32_t* maxabs_w, const uint32_t* maxabs_d,
                    std::vector<void*>& allocs, std::vector<void*>& host_allocs) {
     t = TcLayer();
+    t.maxabs_w = maxabs_w;
+    t.maxabs_d = maxabs_d;
     if (g.kind != NITRO_CONV3X3 || max_batch < 1 || !encode_fn()) return true;
     // Narrow inputs (Cin < 32, e.g. image channels) stay on the CUDA-core
     // kernels: zero-padding them to a 64-wide K-block wastes most MMA work.
@@ -1019,46 +1016,62 @@ bool tc_layer_init(TcLayer& t, const LayerGeom& g, int max_batch, bool has_dgrad
     t.im2col = pix_ok && 9 * g.cin <= kBK && im2col_smem(g.w, g.cin) <= 48 * 1024;
     t.fwd = pix_ok && (wide || t.im2col);
     t.wgrad = (wide || t.im2col) && g.cout % 8 == 0;
-    t.dgrad = has_dgrad && pix_ok && g.cout % 8 == 0;
+    // the input gradient reads the forward planes, which im2col layers lay out
+    // without taps
+    t.dgrad = has_dgrad && pix_ok && g.cout % 8 == 0 && !t.im2col;
     t.cin8 = t.im2col ? kBK : round_up(g.cin, 8);
     t.cin_k = round_up(g.cin, 64);
     const size_t hw = (size_t)g.h * g.w;
-    const size_t nw = (size_t)g.cout * 9 * g.cin;
     const size_t nwk = (size_t)g.cout * (t.im2col ? kBK : 9 * t.cin_k);
-    bool ok = dalloc(allocs, &t.limbs, 2);
+    bool ok = true;
     if (ok && (t.fwd || t.wgrad)) ok = dalloc(allocs, &t.act_nhwc, (size_t)max_batch * hw * t.cin8);
     if (ok && (t.wgrad || t.dgrad))
         ok = dalloc(allocs, &t.d_nhwc, (size_t)kMaxLimbs * max_batch * hw * g.cout);
-    if (ok && t.fwd) ok = dalloc(allocs, &t.w_planes, (size_t)kMaxLimbs * nwk);
-    if (ok && t.dgrad) ok = dalloc(allocs, &t.wt_planes, (size_t)kMaxLimbs * nw);
-    if (ok) ok = cudaMemset(t.limbs, 0, 2 * sizeof(int)) == cudaSuccess;
+    if (ok && (t.fwd || t.dgrad)) ok = dalloc(allocs, &t.w_planes, (size_t)kMaxLimbs * nwk);
     if (ok) {
         void* h = nullptr;
-        ok = cudaMallocHost(&h, 2 * sizeof(int)) == cudaSuccess;
+        ok = cudaMallocHost(&h, 2 * sizeof(uint32_t)) == cudaSuccess;
         if (ok) {
             host_allocs.push_back(h);
-            t.limbs_host = static_cast<int*>(h);
-            t.limbs_host[0] = t.limbs_host[1] = 1;
+            t.max_host = static_cast<uint32_t*>(h);
+            t.max_host[0] = t.max_host[1] = 0;
         }
     }
-    if (ok && t.fwd) ok = cudaMemset(t.w_planes, 0, (size_t)kMaxLimbs * nwk * 2) == cudaSuccess;
+    if (ok && t.w_planes) ok = cudaMemset(t.w_planes, 0, (size_t)kMaxLimbs * nwk * 2) == cudaSuccess;
     return ok;
+}
+
+int tc_limb_hint(const TcLayer& t, int which) {
+    return t.max_host ? limb_count(t.max_host[which]) : 1;
+}
+
+cudaError_t tc_weights_hint(TcLayer& t, cudaStream_t s) {
+    if (!t.w_planes || !t.maxabs_w) return cudaSuccess;
+    // host copy of max |W|, read later as a kernel-variant hint only
+    return cudaMemcpyAsync(t.max_host, t.maxabs_w, sizeof(uint32_t), cudaMemcpyDeviceToHost, s);
+}
+
+void tc_weight_planes(const TcLayer& t, const LayerGeom& g, uint16_t** planes, int64_t* plane,
+                      int* row_k, int* tap_k) {
+    *planes = t.w_planes;
+    *row_k = t.im2col ? kBK : 9 * t.cin_k;
+    *tap_k = t.im2col ? g.cin : t.cin_k;
+    *plane = (int64_t)g.cout * *row_k;
 }
 
 cudaError_t tc_refresh_weights(TcLayer& t, const LayerGeom& g, const int32_t* W,
                                const uint32_t* maxabs_w, cudaStream_t s) {
-    if (!t.fwd && !t.dgrad) return cudaSuccess;
+    if (!t.w_planes) return cudaSuccess;
     const int64_t n = (int64_t)g.cout * 9 * g.cin;
     {
         ProfScope ps(K_TC_PACK_W, s, 0.0, (double)n * 4 * 2);
         const int row_k = t.im2col ? kBK : 9 * t.cin_k, tap_k = t.im2col ? g.cin : t.cin_k;
         k_pack_weights<<<grid1d(n), 256, 0, s>>>(W, g.cout, g.cin, row_k, tap_k, maxabs_w,
-                                                 t.w_planes, t.wt_planes, t.limbs);
+                                                 t.w_planes);
     }
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    // host copy of the limb count, read later as a kernel-variant hint only
-    return cudaMemcpyAsync(t.limbs_host, t.limbs, sizeof(int), cudaMemcpyDeviceToHost, s);
+    return cudaMemcpyAsync(t.max_host, maxabs_w, sizeof(uint32_t), cudaMemcpyDeviceToHost, s);
 }
 
 cudaError_t tc_pack_input(TcLayer& t, const LayerGeom& g, const int8_t* x, int batch,
@@ -1100,8 +1113,8 @@ cudaError_t tc_conv_forward(TcLayer& t, const LayerGeom& g, int batch, int64_t* 
     a.kb_total = a.taps * (t.cin_k / kBK);
     a.kb_per_split = a.kb_total;
     a.ncols = g.cout;
-    a.limbs_a = nullptr;
-    a.limbs_b = t.limbs;
+    a.max_a = nullptr;
+    a.max_b = t.maxabs_w;
     a.out = z;
     a.out_vec = ((uintptr_t)z & 15) == 0;
     a.status = status;
@@ -1135,7 +1148,7 @@ cudaError_t tc_conv_forward(TcLayer& t, const LayerGeom& g, int batch, int64_t* 
         return cudaErrorInvalidValue;
     const double ops = 2.0 * batch * g.h * g.w * g.cout * 9.0 * g.cin;
     ProfScope ps(K_TC_CONV_FWD, s, ops, 0.0);
-    cudaError_t e = launch_gemm_n<TC_FWD>(n, t.limbs_host[0], ma, mb, a, s);
+    cudaError_t e = launch_gemm_n<TC_FWD>(n, tc_limb_hint(t, 0), ma, mb, a, s);
     if (e == cudaSuccess) {
         *done = true;
         *fused = a.fuse != 0;
@@ -1152,11 +1165,11 @@ cudaError_t tc_pack_delta(TcLayer& t, const LayerGeom& g, const int32_t* delta,
     {
         ProfScope ps(K_TC_PACK_D, s, 0.0, (double)n * 4 * 2);
         k_pack_delta_nhwc<<<grid1d(n / 8), 256, 0, s>>>(delta, n, ((uintptr_t)delta & 15) == 0,
-                                                       maxabs_delta, t.d_nhwc, t.limbs + 1);
+                                                       maxabs_delta, t.d_nhwc);
     }
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    return cudaMemcpyAsync(t.limbs_host + 1, t.limbs + 1, sizeof(int), cudaMemcpyDeviceToHost, s);
+    return cudaMemcpyAsync(t.max_host + 1, maxabs_delta, sizeof(uint32_t), cudaMemcpyDeviceToHost, s);
 }
 
 cudaError_t tc_conv_wgrad(TcLayer& t, const LayerGeom& g, const int32_t* delta,
@@ -1193,8 +1206,8 @@ cudaError_t tc_conv_wgrad(TcLayer& t, const LayerGeom& g, const int32_t* delta,
     splits = (a.kb_total + a.kb_per_split - 1) / a.kb_per_split;
     a.total_tiles = tiles * splits;
     a.ncols = g.cout;
-    a.limbs_a = nullptr;
-    a.limbs_b = t.limbs + 1;
+    a.max_a = nullptr;
+    a.max_b = maxabs_delta;
     a.out = dW;
     a.status = status;
     a.atomic_out = splits > 1;
@@ -1215,7 +1228,7 @@ cudaError_t tc_conv_wgrad(TcLayer& t, const LayerGeom& g, const int32_t* delta,
     }
     const double ops = 2.0 * batch * hw * g.cout * 9.0 * g.cin;
     ProfScope ps(K_TC_CONV_WGRAD, s, ops, 0.0);
-    cudaError_t e = launch_gemm_n<TC_WGRAD>(n, t.limbs_host[1], ma, mb, a, s);
+    cudaError_t e = launch_gemm_n<TC_WGRAD>(n, tc_limb_hint(t, 1), ma, mb, a, s);
     if (e == cudaSuccess) *done = true;
     return e;
 }
@@ -1238,8 +1251,8 @@ cudaError_t tc_conv_dgrad(TcLayer& t, const LayerGeom& g, int batch, int64_t* g6
     a.kb_total = 9 * ((g.cout + kBK - 1) / kBK);
     a.kb_per_split = a.kb_total;
     a.ncols = g.cin;
-    a.limbs_a = t.limbs + 1;
-    a.limbs_b = t.limbs;
+    a.max_a = t.maxabs_d;
+    a.max_b = t.maxabs_w;
     a.out = g64;
     a.out_vec = ((uintptr_t)g64 & 15) == 0;
     a.status = status;
@@ -1270,14 +1283,15 @@ cudaError_t tc_conv_dgrad(TcLayer& t, const LayerGeom& g, int batch, int64_t* g6
     const uint64_t sa[4] = {(uint64_t)g.cout, (uint64_t)g.w * g.cout, (uint64_t)g.h * g.w * g.cout,
                             plane};
     const uint32_t ba[5] = {64, (uint32_t)a.wb, (uint32_t)a.hb, (uint32_t)a.bb, 1};
-    const uint64_t db[4] = {(uint64_t)g.cout, (uint64_t)g.cin, 9, (uint64_t)kMaxLimbs};
-    const uint64_t sb[3] = {(uint64_t)g.cout, (uint64_t)g.cin * g.cout, (uint64_t)9 * g.cin * g.cout};
-    const uint32_t bb[4] = {64, (uint32_t)n, 1, 1};
-    if (!make_map(&ma, t.d_nhwc, 5, da, sa, ba) || !make_map(&mb, t.wt_planes, 4, db, sb, bb))
+    // forward planes [L][Cout][9][Cin64], read MN-major: boxes of 64 ci x 64 co
+    const uint64_t db[4] = {(uint64_t)t.cin_k, 9, (uint64_t)g.cout, (uint64_t)kMaxLimbs};
+    const uint64_t sb[3] = {(uint64_t)t.cin_k, (uint64_t)9 * t.cin_k, (uint64_t)9 * t.cin_k * g.cout};
+    const uint32_t bb[4] = {64, 1, 64, 1};
+    if (!make_map(&ma, t.d_nhwc, 5, da, sa, ba) || !make_map(&mb, t.w_planes, 4, db, sb, bb))
         return cudaErrorInvalidValue;
     const double ops = 2.0 * batch * g.h * g.w * g.cin * 9.0 * g.cout;
     ProfScope ps(K_TC_CONV_DGRAD, s, ops, 0.0);
-    cudaError_t e = launch_gemm_n<TC_DGRAD>(n, t.limbs_host[0], ma, mb, a, s);
+    cudaError_t e = launch_gemm_n<TC_DGRAD>(n, tc_limb_hint(t, 0), ma, mb, a, s);
     if (e == cudaSuccess) {
         *done = true;
         *fused = a.fuse != 0;
@@ -1314,16 +1328,15 @@ cudaError_t tc_pack_int8(const int8_t* x, int64_t rows, int cols, uint16_t* out,
 }
 
 cudaError_t tc_pack_limbs(const int32_t* x, int64_t n, const uint32_t* maxabs, uint16_t* planes,
-                          int* limbs, cudaStream_t s) {
+                          cudaStream_t s) {
     if (n <= 0) return cudaSuccess;
     ProfScope ps(K_TC_PACK, s, 0.0, (double)n * 4 * 2);
-    k_pack_delta_nhwc<<<grid1d(n / 8), 256, 0, s>>>(x, n, ((uintptr_t)x & 15) == 0, maxabs, planes,
-                                                   limbs);
+    k_pack_delta_nhwc<<<grid1d(n / 8), 256, 0, s>>>(x, n, ((uintptr_t)x & 15) == 0, maxabs, planes);
     return cudaGetLastError();
 }
 
 cudaError_t tc_gemm_run(const uint16_t* a_bf16, const uint16_t* b_planes, int M, int N, int K,
-                        const int* limbs_b, int64_t* out, uint32_t* status, cudaStream_t s) {
+                        const uint32_t* max_b, int64_t* out, uint32_t* status, cudaStream_t s) {
     if (M <= 0 || N <= 0) return cudaSuccess;
     TcArgs a{};
     a.B = M;
@@ -1336,8 +1349,8 @@ cudaError_t tc_gemm_run(const uint16_t* a_bf16, const uint16_t* b_planes, int M,
     a.total_tiles = a.tiles_m * a.tiles_n;
     a.kb_total = (K + kBK - 1) / kBK;
     a.kb_per_split = a.kb_total;
-    a.limbs_a = nullptr;
-    a.limbs_b = limbs_b;
+    a.max_a = nullptr;
+    a.max_b = max_b;
     a.out = out;
     a.status = status;
     CUtensorMap ma, mb;

@@ -1,8 +1,10 @@
 // Tensor-core (tcgen05) path of the 3x3 conv contractions.
 //
-// Every operand is split exactly into signed 8-bit limbs, x = sum_l 2^(8l) x_l
-// with x_l in [-128, 127] and the top limb in [-128, 128], each held as a
-// bf16 value (exact).  A contraction runs one pass per (A limb, B limb) pair
+// Every operand is split exactly into signed 8-bit limbs, x = sum_l 2^(8l) x_l:
+// limbs 0..2 are digits in [-128, 127], limb 3 the remainder in [-128, 128];
+// a tensor with max |x| <= 127 / 32639 / 8355711 has zero limbs from index
+// 1 / 2 / 3 on, so its first L planes are exact.  Each limb is held as a bf16
+// value (exact).  A contraction runs one pass per (A limb, B limb) pair
 // on the bf16 tensor pipe with fp32 accumulation in TMEM; every partial sum
 // over at most 1024 products of magnitude <= 2^14 is an integer below 2^24 and
 // therefore exact, so chunks of 1024 are drained to integers and the passes
@@ -12,8 +14,8 @@
 //   act_nhwc  [B][H][W][Cin8]          forward A (K-major: pixels x taps*channels)
 //                                      and wgrad A (MN-major: (tap, ci) x pixels)
 //   d_nhwc    [L][B][H][W][Cout]       dgrad A (K-major) and wgrad B (MN-major)
-//   w_planes  [L][Cout][9][Cin64]      forward B
-//   wt_planes [L][9][Cin][Cout]        dgrad B
+//   w_planes  [L][Cout][9][Cin64]      forward B (K-major) and dgrad B (MN-major:
+//                                      rows co, 64 consecutive ci)
 // Narrow inputs (9 Cin <= 64) use im2col rows instead, see TcLayer::im2col.
 // Cin8 = Cin rounded up to 8 (TMA strides are multiples of 16 bytes); Cin64 =
 // Cin rounded up to 64 so that a K-block of the forward never spans two taps.  Padding holds zeros; tiles that run past
@@ -39,19 +41,32 @@ struct TcLayer {
     uint16_t* act_nhwc = nullptr;
     uint16_t* d_nhwc = nullptr;
     uint16_t* w_planes = nullptr;
-    uint16_t* wt_planes = nullptr;
-    int* limbs = nullptr;   // device: [0] weight limbs, [1] delta limbs
-    // pinned host copy of `limbs`, refreshed asynchronously after each split;
-    // possibly stale, used only to pick a kernel variant (any choice is exact)
-    int* limbs_host = nullptr;
+    // device words holding max |W| and max |delta| of the layer: the kernels
+    // take their limb counts from them
+    const uint32_t* maxabs_w = nullptr;
+    const uint32_t* maxabs_d = nullptr;
+    // pinned host copies of the two words, refreshed asynchronously; possibly
+    // stale, used only to pick a kernel variant (any choice is exact)
+    uint32_t* max_host = nullptr;
 };
 
 // Decides which passes of a layer run on tensor cores and allocates their
 // buffers (device memory recorded in `allocs`, pinned host memory in
 // `host_allocs`).  `has_dgrad`: the layer is not the block's first, so its
-// input gradient is needed.
+// input gradient is needed.  maxabs_w / maxabs_d: device words that will hold
+// max |W| and max |delta| of the layer.
 bool tc_layer_init(TcLayer& t, const LayerGeom& g, int max_batch, bool has_dgrad,
+                   const uint32_t* maxabs_w, const uint32_t* maxabs_d,
                    std::vector<void*>& allocs, std::vector<void*>& host_allocs);
+
+// Where IntegerSGD writes the layer's weight planes when it splits the updated
+// weights itself: planes [4][Cout][row_k], plane stride, entry (t, ci) of row
+// co at co row_k + t tap_k + ci.  *planes = null when the layer has none.
+void tc_weight_planes(const TcLayer& t, const LayerGeom& g, uint16_t** planes, int64_t* plane,
+                      int* row_k, int* tap_k);
+
+// After such an update: refresh the host hint of max |W|.
+cudaError_t tc_weights_hint(TcLayer& t, cudaStream_t s);
 
 // Re-splits the layer's int32 weights into limb planes (after init, an update
 // or a checkpoint load); the limb count follows *maxabs_w.
@@ -116,12 +131,12 @@ cudaError_t tc_conv_dgrad(TcLayer& t, const LayerGeom& g, int batch, int64_t* g6
 // Helpers of the kernel-level entry points (contract.cu).
 cudaError_t tc_maxabs(const int32_t* x, int64_t n, uint32_t* out, cudaStream_t s);
 cudaError_t tc_pack_int8(const int8_t* x, int64_t rows, int cols, uint16_t* out, cudaStream_t s);
-// n % 8 == 0; planes [4][n]; the limb count (from *maxabs) goes to *limbs
+// n % 8 == 0; planes [4][n], limb count from *maxabs
 cudaError_t tc_pack_limbs(const int32_t* x, int64_t n, const uint32_t* maxabs, uint16_t* planes,
-                          int* limbs, cudaStream_t s);
+                          cudaStream_t s);
 // C[m][n] (int64) = sum_k A[m][k] B[n][k]; A bf16 [M][K] (int8 values), B limb
-// planes [4][N][K]; K % 8 == 0.
+// planes [4][N][K] (limb count from *max_b); K % 8 == 0.
 cudaError_t tc_gemm_run(const uint16_t* a_bf16, const uint16_t* b_planes, int M, int N, int K,
-                        const int* limbs_b, int64_t* out, uint32_t* status, cudaStream_t s);
+                        const uint32_t* max_b, int64_t* out, uint32_t* status, cudaStream_t s);
 
 }  // namespace nitro

@@ -14,8 +14,8 @@ from paper_2407_11698_gb300 import workloads as WL
 
 pytestmark = pytest.mark.gpu
 
-# value ranges that need 1, 2, 3 and 4 signed 8-bit limbs
-RANGES = {1: (-127, 127), 2: (-32768, 32639), 3: (-2**23, 2**23 - 1), 4: (-2**31, 2**31 - 1)}
+# value ranges whose max |x| needs exactly 1, 2, 3 and 4 limbs
+RANGES = {1: (-127, 127), 2: (-32639, 32639), 3: (-8355711, 8355711), 4: (-2**31, 2**31 - 1)}
 
 
 @pytest.fixture(scope="module")
