@@ -361,9 +361,32 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const int tx = T.mt % args.ntx, ty = (T.mt / args.ntx) % args.nty;
                 const int tb = T.mt / (args.ntx * args.nty);
                 const int x0 = tx * args.wb, y0 = ty * args.hb, b0 = tb * args.bb;
+                // weight gradient: the tile's two 64-row blocks of (tap, ci) rows
+                // are fixed for the tile (channel start, tap offsets)
+                int wa_ci[2] = {0, 0}, wa_dx[2] = {0, 0}, wa_dy[2] = {0, 0};
+                if (MODE == TC_WGRAD) {
+#pragma unroll
+                    for (int j = 0; j < 2; ++j) {
+                        const int m = T.mt * kBM + j * 64;
+                        int t = m / args.cin_k, ci0 = m - t * args.cin_k;
+                        if (t >= args.taps) { t = 0; ci0 = args.cin_k; }   // past the last tap: zeros
+                        if (args.taps == 1) t = 4;                         // im2col rows: centre tap
+                        wa_ci[j] = ci0;
+                        wa_dx[j] = t % 3 - 1;
+                        wa_dy[j] = t / 3 - 1;
+                    }
+                }
                 for (int p = 0; p < passes; ++p) {
                     const int la = p / NG, lb0 = (p % NG) * PB;
                     const int nb = min(PB, LB - lb0);
+                    // weight gradient: K-block kb = pixel box (xt, yt) of image bk,
+                    // walked incrementally
+                    int wxt = 0, wyt = 0, wbk = 0;
+                    if (MODE == TC_WGRAD) {
+                        wxt = T.kb0 % args.ntx;
+                        wyt = (T.kb0 / args.ntx) % args.nty;
+                        wbk = T.kb0 / (args.ntx * args.nty);
+                    }
                     for (int kb = T.kb0; kb < T.kb1; ++kb, ++it) {
                         const int s = it % S;
                         if (!mbar_wait(empty_bar(s), ((it / S) & 1) ^ 1, abort_flag, args.status))
@@ -399,24 +422,23 @@ __global__ void __launch_bounds__(kThreads, 1)
                         } else {  // TC_WGRAD: rows (tap, ci), K = a 64-pixel box (wb x hb)
                             // of one image; both operands MN-major from the NHWC
                             // copies (channels contiguous), the tap shift on x / y.
-                            const int xt = kb % args.ntx, yt = (kb / args.ntx) % args.nty;
-                            const int bk = kb / (args.ntx * args.nty);
-                            const int px = xt * args.wb, py = yt * args.hb;
+                            const int px = wxt * args.wb, py = wyt * args.hb, bk = wbk;
 #pragma unroll
-                            for (int j = 0; j < 2; ++j) {
-                                const int m = T.mt * kBM + j * 64;
-                                int t = m / args.cin_k, ci0 = m - t * args.cin_k;
-                                if (t >= args.taps) { t = 0; ci0 = args.cin_k; }   // past the last tap: zeros
-                                if (args.taps == 1) t = 4;                         // im2col rows: centre tap
-                                const int ky = t / 3, kx = t - 3 * ky;
-                                tma_load_4d(a_dst + j * (64 * 128), &tmA, fb, ci0, px + kx - 1,
-                                            py + ky - 1, bk);
-                            }
+                            for (int j = 0; j < 2; ++j)
+                                tma_load_4d(a_dst + j * (64 * 128), &tmA, fb, wa_ci[j], px + wa_dx[j],
+                                            py + wa_dy[j], bk);
                             for (int j = 0; j < nb; ++j)
 #pragma unroll
                                 for (int h = 0; h < N / 64; ++h)
                                     tma_load_5d(b_dst + j * C::B_BYTES + h * (64 * 128), &tmB, fb,
                                                 n0 + 64 * h, px, py, bk, lb0 + j);
+                            if (++wxt == args.ntx) {
+                                wxt = 0;
+                                if (++wyt == args.nty) {
+                                    wyt = 0;
+                                    ++wbk;
+                                }
+                            }
                         }
                     }
                 }
