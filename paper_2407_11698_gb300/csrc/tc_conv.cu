@@ -387,6 +387,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                         wyt = (T.kb0 / args.ntx) % args.nty;
                         wbk = T.kb0 / (args.ntx * args.nty);
                     }
+                    // forward / input gradient: K-block kb = (tap t, 64-channel block cb),
+                    // cb fastest, walked incrementally
+                    const int knc = MODE == TC_FWD ? args.cin_k / kBK : (args.Cout + kBK - 1) / kBK;
+                    int kt = 0, kcb = 0;
+                    if (MODE == TC_FWD || MODE == TC_DGRAD) {
+                        kt = T.kb0 / knc;
+                        kcb = T.kb0 - kt * knc;
+                    }
                     for (int kb = T.kb0; kb < T.kb1; ++kb, ++it) {
                         const int s = it % S;
                         if (!mbar_wait(empty_bar(s), ((it / S) & 1) ^ 1, abort_flag, args.status))
@@ -400,17 +408,17 @@ __global__ void __launch_bounds__(kThreads, 1)
                             for (int j = 0; j < nb; ++j)
                                 tma_load_3d(b_dst + j * C::B_BYTES, &tmB, fb, kb * kBK, n0, lb0 + j);
                         } else if (MODE == TC_FWD) {
-                            const int nc = args.cin_k / kBK;
-                            const int t = kb / nc, cb = kb - t * nc;
+                            const int t = kt, cb = kcb;
                             const int tc = args.taps == 1 ? 4 : t;   // im2col rows: centre tap
                             const int ky = tc / 3, kx = tc - 3 * ky;
                             tma_load_4d(a_dst, &tmA, fb, cb * kBK, x0 + kx - 1, y0 + ky - 1, b0);
                             for (int j = 0; j < nb; ++j)
                                 tma_load_3d(b_dst + j * C::B_BYTES, &tmB, fb, t * args.cin_k + cb * kBK,
                                             n0, lb0 + j);
+                            if (++kcb == knc) { kcb = 0; ++kt; }
                         } else if (MODE == TC_DGRAD) {
-                            const int nc = (args.Cout + kBK - 1) / kBK;
-                            const int t = kb / nc, cb = kb - t * nc, ky = t / 3, kx = t - 3 * ky;
+                            const int t = kt, cb = kcb, ky = t / 3, kx = t - 3 * ky;
+                            if (++kcb == knc) { kcb = 0; ++kt; }
                             tma_load_5d(a_dst, &tmA, fb, cb * kBK, x0 - kx + 1, y0 - ky + 1, b0, la);
                             // B MN-major from the forward planes [L][Cout][9][Cin64]:
                             // rows co (K) of 64 consecutive ci (N) for tap t
@@ -460,6 +468,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const int cpp = (T.kb1 - T.kb0 + kChunkBlocks - 1) / kChunkBlocks;
                 for (int p = 0; p < passes; ++p) {
                     const int nb = min(PB, LB - (p % NG) * PB);
+                    const uint32_t idesc = idesc_nb[nb];
                     for (int c = 0; c < cpp; ++c, ++chunk) {
                         const int buf = chunk % NBUF;
                         if (!mbar_wait(tempty_bar(buf), ((chunk / NBUF) & 1) ^ 1, abort_flag,
@@ -476,7 +485,6 @@ __global__ void __launch_bounds__(kThreads, 1)
                             tc_fence_after();
                             const uint32_t a_addr = smem_u32(smem + s * C::STAGE);
                             const uint32_t b_addr = a_addr + C::A_BYTES;
-                            const uint32_t idesc = idesc_nb[nb];
 #pragma unroll
                             for (int k = 0; k < kBK / 16; ++k) {
                                 // K-major: a K-step of 16 is 32 bytes along each row;
