@@ -62,10 +62,9 @@ __device__ __forceinline__ uint64_t global_ns() {
 }
 
 // Bounded wait: false when the time limit passed (TIMEOUT raised) or another
-// role of this CTA gave up.
-__device__ __noinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag,
-                                       uint32_t* status) {
-    if (mbar_try_wait(bar, parity)) return true;
+// role of this CTA gave up.  The first test is inline; the polling loop is not.
+__device__ __noinline__ bool mbar_wait_slow(uint32_t bar, uint32_t parity, volatile int* abort_flag,
+                                            uint32_t* status) {
     const uint64_t t0 = global_ns();
     for (uint32_t i = 1;; ++i) {
         if (mbar_try_wait(bar, parity)) return true;
@@ -78,6 +77,10 @@ __device__ __noinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile i
             }
         }
     }
+}
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag,
+                                          uint32_t* status) {
+    return mbar_try_wait(bar, parity) || mbar_wait_slow(bar, parity, abort_flag, status);
 }
 
 __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* m, uint32_t bar,
@@ -205,6 +208,10 @@ struct TcArgs {
     int ntx, nty;          // pixel tiles along x and y (forward / dgrad)
     int wb, hb, bb;        // pixel box (forward / dgrad): wb * hb * bb = 128
     int tiles_m, tiles_n, total_tiles;
+    // dividers for the tile decode (filled at launch): tiles_n, tiles_m, ntx, nty;
+    // pixel-box sides are powers of two: log2 wb, log2 hb
+    FloorDiv32 dv_tn, dv_tm, dv_ntx, dv_nty;
+    int lg_wb, lg_hb;
     int kb_total, kb_per_split;
     int ncols;             // valid output columns (Cout for fwd/wgrad, Cin for dgrad)
     const uint32_t* max_a;  // max |operand| words setting the limb counts (nullptr = 1 limb)
@@ -273,12 +280,14 @@ struct TcCfg {
 struct Tile {
     int mt, nt, kb0, kb1;
 };
+__device__ __forceinline__ int udiv32(const FloorDiv32& f, int x) { return (int)f.udiv((uint32_t)x); }
+
 __device__ __forceinline__ Tile decode_tile(const TcArgs& a, int tile) {
     Tile t;
-    t.nt = tile % a.tiles_n;
-    const int r = tile / a.tiles_n;
-    t.mt = r % a.tiles_m;
-    const int split = r / a.tiles_m;
+    const int r = udiv32(a.dv_tn, tile);
+    t.nt = tile - r * a.tiles_n;
+    const int split = udiv32(a.dv_tm, r);
+    t.mt = r - split * a.tiles_m;
     t.kb0 = split * a.kb_per_split;
     t.kb1 = min(a.kb_total, t.kb0 + a.kb_per_split);
     return t;
@@ -358,8 +367,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int tile = blockIdx.x; tile < args.total_tiles; tile += gridDim.x) {
                 const Tile T = decode_tile(args, tile);
                 const int n0 = T.nt * N;
-                const int tx = T.mt % args.ntx, ty = (T.mt / args.ntx) % args.nty;
-                const int tb = T.mt / (args.ntx * args.nty);
+                const int mq = udiv32(args.dv_ntx, T.mt), tb = udiv32(args.dv_nty, mq);
+                const int tx = T.mt - mq * args.ntx, ty = mq - tb * args.nty;
                 const int x0 = tx * args.wb, y0 = ty * args.hb, b0 = tb * args.bb;
                 // weight gradient: the tile's two 64-row blocks of (tap, ci) rows
                 // are fixed for the tile (channel start, tap offsets)
@@ -591,10 +600,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                     // 2x2 max-pool across lanes; int8 outputs straight from
                     // registers (the 2x2 windows of a tile lie inside one warp:
                     // x partner lane ^ 1, y partner lane ^ wb).
-                    const int tx = T.mt % args.ntx, ty = (T.mt / args.ntx) % args.nty;
-                    const int tb = T.mt / (args.ntx * args.nty);
-                    const int xx = r % args.wb, yy = (r / args.wb) % args.hb;
-                    const int bbx = r / (args.wb * args.hb);
+                    const int mq = udiv32(args.dv_ntx, T.mt), tb = udiv32(args.dv_nty, mq);
+                    const int tx = T.mt - mq * args.ntx, ty = mq - tb * args.nty;
+                    const int xx = r & ((1 << args.lg_wb) - 1);
+                    const int yy = (r >> args.lg_wb) & ((1 << args.lg_hb) - 1);
+                    const int bbx = r >> (args.lg_wb + args.lg_hb);
                     const int x = tx * args.wb + xx, y = ty * args.hb + yy, b = tb * args.bb + bbx;
                     const bool valid = x < args.W && y < args.H && b < args.B;
                     const int C = args.Cout;
@@ -676,10 +686,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                     // gradient at the lower layer's (pooled) output -> int32 with
                     // the OVERFLOW rule -> max-pool backward (to the recorded
                     // window position) -> NITRO-ReLU backward -> lower delta.
-                    const int tx = T.mt % args.ntx, ty = (T.mt / args.ntx) % args.nty;
-                    const int tb = T.mt / (args.ntx * args.nty);
-                    const int xx = r % args.wb, yy = (r / args.wb) % args.hb;
-                    const int bbx = r / (args.wb * args.hb);
+                    const int mq = udiv32(args.dv_ntx, T.mt), tb = udiv32(args.dv_nty, mq);
+                    const int tx = T.mt - mq * args.ntx, ty = mq - tb * args.nty;
+                    const int xx = r & ((1 << args.lg_wb) - 1);
+                    const int yy = (r >> args.lg_wb) & ((1 << args.lg_hb) - 1);
+                    const int bbx = r >> (args.lg_wb + args.lg_hb);
                     const int x = tx * args.wb + xx, y = ty * args.hb + yy, b = tb * args.bb + bbx;
                     const bool valid = x < args.W && y < args.H && b < args.B;
                     const int Cl = args.Cin;
@@ -732,10 +743,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                         if (ovf) atomicOr(args.status, ST_OVERFLOW);
                     }
                 } else {
-                    const int tx = T.mt % args.ntx, ty = (T.mt / args.ntx) % args.nty;
-                    const int tb = T.mt / (args.ntx * args.nty);
-                    const int xx = r % args.wb, yy = (r / args.wb) % args.hb;
-                    const int bbx = r / (args.wb * args.hb);
+                    const int mq = udiv32(args.dv_ntx, T.mt), tb = udiv32(args.dv_nty, mq);
+                    const int tx = T.mt - mq * args.ntx, ty = mq - tb * args.nty;
+                    const int xx = r & ((1 << args.lg_wb) - 1);
+                    const int yy = (r >> args.lg_wb) & ((1 << args.lg_hb) - 1);
+                    const int bbx = r >> (args.lg_wb + args.lg_hb);
                     const int x = tx * args.wb + xx, y = ty * args.hb + yy, b = tb * args.bb + bbx;
                     if (x < args.W && y < args.H && b < args.B) {
                         int64_t* o = args.out + (((int64_t)b * args.H + y) * args.W + x) * args.ncols + col0;
@@ -976,10 +988,26 @@ int sm_count() {
     return n;
 }
 
+inline int log2_exact(int v) {
+    int l = 0;
+    while ((1 << l) < v) ++l;
+    return (1 << l) == v ? l : -1;
+}
+
 template <int MODE, int N, int PB>
-cudaError_t launch_gemm(const CUtensorMap& a, const CUtensorMap& b, const TcArgs& args,
+cudaError_t launch_gemm(const CUtensorMap& a, const CUtensorMap& b, const TcArgs& args_in,
                         cudaStream_t s) {
     using C = TcCfg<N, PB>;
+    TcArgs args = args_in;
+    args.dv_tn = FloorDiv32::make((uint32_t)args.tiles_n);
+    args.dv_tm = FloorDiv32::make((uint32_t)args.tiles_m);
+    args.dv_ntx = FloorDiv32::make((uint32_t)args.ntx);
+    args.dv_nty = FloorDiv32::make((uint32_t)args.nty);
+    args.lg_wb = log2_exact(args.wb);
+    args.lg_hb = log2_exact(args.hb);
+    if (args.tiles_n < 1 || args.tiles_m < 1 || args.ntx < 1 || args.nty < 1 || args.lg_wb < 0 ||
+        args.lg_hb < 0)
+        return cudaErrorInvalidValue;
     static bool attr_set = false;
     if (!attr_set) {
         cudaError_t e = cudaFuncSetAttribute(k_tc_gemm<MODE, N, PB>,
