@@ -494,19 +494,19 @@ __global__ void __launch_bounds__(kThreads, 1)
                             tc_fence_after();
                             const uint32_t a_addr = smem_u32(smem + s * C::STAGE);
                             const uint32_t b_addr = a_addr + C::A_BYTES;
+                            // K-major: a K-step of 16 is 32 bytes along each row;
+                            // MN-major: 16 rows, two 1024-byte row groups, and
+                            // 64-wide blocks along M / N 8 KB apart.  Only the
+                            // address field (bytes / 16, below 2^14) moves per step.
+                            constexpr bool a_mn = MODE == TC_WGRAD;
+                            constexpr bool b_mn = MODE == TC_WGRAD || MODE == TC_DGRAD;
+                            const uint64_t da0 = a_mn ? desc_sw128_mn(a_addr, 64 * 128) : desc_sw128(a_addr);
+                            const uint64_t db0 = b_mn ? desc_sw128_mn(b_addr, 64 * 128) : desc_sw128(b_addr);
 #pragma unroll
-                            for (int k = 0; k < kBK / 16; ++k) {
-                                // K-major: a K-step of 16 is 32 bytes along each row;
-                                // MN-major: 16 rows, two 1024-byte row groups, and
-                                // 64-wide blocks along M / N 8 KB apart
-                                const uint64_t da = MODE == TC_WGRAD
-                                    ? desc_sw128_mn(a_addr + 2048 * k, 64 * 128)
-                                    : desc_sw128(a_addr + 32 * k);
-                                const uint64_t db = (MODE == TC_WGRAD || MODE == TC_DGRAD)
-                                    ? desc_sw128_mn(b_addr + 2048 * k, 64 * 128)
-                                    : desc_sw128(b_addr + 32 * k);
-                                umma_bf16(d, da, db, idesc, (kb > c0 || k > 0) ? 1u : 0u);
-                            }
+                            for (int k = 0; k < kBK / 16; ++k)
+                                umma_bf16(d, da0 + (uint64_t)k * (a_mn ? 2048 / 16 : 32 / 16),
+                                          db0 + (uint64_t)k * (b_mn ? 2048 / 16 : 32 / 16), idesc,
+                                          (kb > c0 || k > 0) ? 1u : 0u);
                             umma_commit(empty_bar(s));
                         }
                         umma_commit(tfull_bar(buf));
