@@ -37,6 +37,8 @@ def parse():
     p.add_argument("--workload", default=WORKLOAD)
     p.add_argument("--no-graph", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--sequential-blocks", action="store_true",
+                   help="run all blocks on one stream (default: a stream per block)")
     p.add_argument("--profile-steps", type=int, default=3)
     p.add_argument("--sweep", action="store_true",
                    help="time the kernel sweep (conv contractions and integer GEMM) instead")
@@ -125,7 +127,12 @@ class ClockSampler:
 
 # ------------------------------------------------------------------ our step
 class GpuNet:
-    def __init__(self, wl, seed, torch, nb):
+    """A chain of block handles driven through the public calls.  With
+    `concurrent`, every block runs on its own stream: block i+1's forward waits
+    only for block i's forward, so block i's backward and update overlap the
+    blocks after it (blocks exchange no gradients, Sec. 3.3)."""
+
+    def __init__(self, wl, seed, torch, nb, concurrent=True):
         self.torch, self.nb = torch, nb
         B = wl["batch"]
         self.B = B
@@ -142,18 +149,33 @@ class GpuNet:
                              if g.layers else self.acts[-1])
         self.loss = torch.zeros((len(self.blocks),), dtype=torch.int64, device="cuda")
         self.in_bytes = self.x.numel() + 4 * self.y.numel()
+        self.streams = [torch.cuda.Stream() for _ in self.blocks] if concurrent else None
+        self.fwd_done = [torch.cuda.Event() for _ in self.blocks] if concurrent else None
 
-    def step(self, x=None, y=None, loss=None):
+    def step(self, x=None, y=None, loss=None, sequential=False):
         x = self.x if x is None else x
         y = self.y if y is None else y
         loss = self.loss if loss is None else loss
         acts = [x] + self.acts[1:]
-        for i, g in enumerate(self.blocks):
-            g.forward(acts[i], acts[i + 1] if g.layers else None)
-        for i, g in enumerate(self.blocks):
-            g.backward(acts[i], y, loss[i:i + 1])
-        for g in self.blocks:
-            g.sgd()
+        if not self.streams or sequential:
+            for i, g in enumerate(self.blocks):
+                g.forward(acts[i], acts[i + 1] if g.layers else None)
+            for i, g in enumerate(self.blocks):
+                g.backward(acts[i], y, loss[i:i + 1])
+            for g in self.blocks:
+                g.sgd()
+            return
+        main = self.torch.cuda.current_stream()
+        for i, (g, s) in enumerate(zip(self.blocks, self.streams)):
+            s.wait_stream(main)                      # inputs, labels
+            if i:
+                s.wait_event(self.fwd_done[i - 1])   # the block's input activations
+            g.forward(acts[i], acts[i + 1] if g.layers else None, stream=s)
+            self.fwd_done[i].record(s)
+            g.backward(acts[i], y, loss[i:i + 1], stream=s)
+            g.sgd(stream=s)
+        for s in self.streams:
+            main.wait_stream(s)
 
 
 def kernel_profile(nb):
@@ -206,7 +228,7 @@ def issued_profile(nb, net, flush, steps, torch):
         L.nitro_profile_reset()
         L.nitro_profile_enable(1)
         flush.zero_()
-        net.step()
+        net.step(sequential=True)
         torch.cuda.synchronize()
         L.nitro_profile_enable(0)
         dl = {c: _limbs(maxabs(c[0], nb.NITRO_T_DELTA, c[1])) for c in convs}
@@ -241,7 +263,7 @@ def run_ours(args, rank, world, local_rank):
     torch.cuda.set_device(local_rank)
     nb.lib()
     wl = WL.WORKLOADS[args.workload]
-    net = GpuNet(wl, 20240716 + 7 * rank, torch, nb)
+    net = GpuNet(wl, 20240716 + 7 * rank, torch, nb, concurrent=not args.sequential_blocks)
     stream = torch.cuda.current_stream()
     flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device="cuda")
 
@@ -326,12 +348,13 @@ def run_ours(args, rank, world, local_rank):
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
     e2e_value = world * net.B * args.steps / (float(t.item()) / 1e3)
 
-    # ---------------- per-kernel device time inside eager steps (roofline)
+    # ---------------- per-kernel device time inside eager steps (roofline); the
+    # blocks run one after another here so that no kernel shares the GPU
     L.nitro_profile_reset()
     L.nitro_profile_enable(1)
     for _ in range(args.profile_steps):
         flush.zero_()
-        net.step()
+        net.step(sequential=True)
     torch.cuda.synchronize()
     L.nitro_profile_enable(0)
     prof = kernel_profile(nb)
@@ -381,6 +404,7 @@ def run_ours(args, rank, world, local_rank):
         "config": {"workload": args.workload, "batch": net.B,
                    "input": "x".join(str(v) for v in wl["input_shape"]) + " int8 uniform [-128,127]",
                    "blocks": len(wl["blocks"]), "cuda_graph": graph is not None,
+                   "block_streams": "one" if args.sequential_blocks else "one per block",
                    "l2": "flushed (512 MiB write) between timed steps",
                    "parallelism": "replicas" if world > 1 else "single"},
         "e2e": {"value": round(e2e_value, 2), "unit": "images/s",

@@ -13,9 +13,10 @@ def _torch():
 
 
 class NetPair:
-    def __init__(self, blocks, batch, seed=1000, **hyper):
+    def __init__(self, blocks, batch, seed=1000, concurrent=False, **hyper):
         self.batch = batch
         self.spec = blocks
+        self.concurrent = concurrent   # a stream per block, as bench.py drives them
         self.ob = [O.OracleBlock([O.LayerDesc(*l) for l in b["layers"]],
                                  in_features=b["in_features"], seed=seed + i, **hyper)
                    for i, b in enumerate(blocks)]
@@ -35,15 +36,31 @@ class NetPair:
         for g in self.gb:
             out = torch.empty((B, max(1, g.out_features)), dtype=torch.int8, device="cuda") \
                 if g.layers else None
-            g.forward(acts[-1], out)
             acts.append(out if out is not None else acts[-1])
-        losses = []
-        for i, g in enumerate(self.gb):
-            loss = torch.full((1,), -7, dtype=torch.int64, device="cuda")
-            g.backward(acts[i], ys, loss)
-            losses.append(loss)
-        for g in self.gb:
-            g.sgd()
+        losses = [torch.full((1,), -7, dtype=torch.int64, device="cuda") for _ in self.gb]
+        if self.concurrent:
+            # block i+1's forward waits only for block i's forward; each block's
+            # backward and update run on its own stream alongside the others
+            main = torch.cuda.current_stream()
+            streams = [torch.cuda.Stream() for _ in self.gb]
+            done = [torch.cuda.Event() for _ in self.gb]
+            for i, (g, s) in enumerate(zip(self.gb, streams)):
+                s.wait_stream(main)
+                if i:
+                    s.wait_event(done[i - 1])
+                g.forward(acts[i], acts[i + 1] if g.layers else None, stream=s)
+                done[i].record(s)
+                g.backward(acts[i], ys, losses[i], stream=s)
+                g.sgd(stream=s)
+            for s in streams:
+                main.wait_stream(s)
+        else:
+            for i, g in enumerate(self.gb):
+                g.forward(acts[i], acts[i + 1] if g.layers else None)
+            for i, g in enumerate(self.gb):
+                g.backward(acts[i], ys, losses[i])
+            for g in self.gb:
+                g.sgd()
         torch.cuda.synchronize()
         return [int(l.item()) for l in losses]
 
@@ -84,8 +101,8 @@ def _eq(got, want, what):
             what, bad.size, want.size, bad[0], got[bad[0]], want[bad[0]]))
 
 
-def run_workload(wl, steps, seed=20240716, check_every=1, data_seed=7):
-    pair = NetPair(wl["blocks"], wl["batch"], seed=seed)
+def run_workload(wl, steps, seed=20240716, check_every=1, data_seed=7, concurrent=False):
+    pair = NetPair(wl["blocks"], wl["batch"], seed=seed, concurrent=concurrent)
     try:
         for s in range(steps):
             x = synth.images(data_seed, s, wl["batch"], wl["input_shape"])

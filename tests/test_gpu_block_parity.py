@@ -47,6 +47,15 @@ def test_vgg_64_128_256_b128_50_steps():
     run_workload(WL.WORKLOADS["vgg_64_128_256_b128"], steps=50, check_every=5)
 
 
+def test_blocks_on_their_own_streams():
+    # blocks share no gradients (Sec. 3.3): with a stream per block, block i's
+    # backward and update overlap the forward of the blocks after it; the
+    # results stay bit-identical to the oracle, through the first steps of limb
+    # growth and into the int32 overflow regime of the VGG-style network
+    run_workload(WL.WORKLOADS["cnn_32_64_b64"], steps=20, check_every=5, concurrent=True)
+    run_workload(WL.WORKLOADS["vgg_64_128_256_b128"], steps=8, check_every=2, concurrent=True)
+
+
 # ---------------------------------------------------------------- edge cases
 def _run(blocks, batch, steps=2, input_shape=None, **hyper):
     pair = NetPair(blocks, batch, **hyper)
