@@ -411,7 +411,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                         const uint32_t fb = full_bar(s);
                         const uint32_t a_dst = smem_u32(smem + s * C::STAGE);
                         const uint32_t b_dst = a_dst + C::A_BYTES;
-                        mbar_expect_tx(fb, C::A_BYTES + nb * C::B_BYTES);
+                        // the B box spans PB limb planes (past the last limb: zeros or
+                        // planes the MMA does not read)
+                        mbar_expect_tx(fb, C::A_BYTES + (MODE == TC_GEMM ? nb : PB) * C::B_BYTES);
                         if (MODE == TC_GEMM) {
                             tma_load_2d(a_dst, &tmA, fb, kb * kBK, T.mt * kBM);
                             for (int j = 0; j < nb; ++j)
@@ -421,21 +423,20 @@ __global__ void __launch_bounds__(kThreads, 1)
                             const int tc = args.taps == 1 ? 4 : t;   // im2col rows: centre tap
                             const int ky = tc / 3, kx = tc - 3 * ky;
                             tma_load_4d(a_dst, &tmA, fb, cb * kBK, x0 + kx - 1, y0 + ky - 1, b0);
-                            for (int j = 0; j < nb; ++j)
-                                tma_load_3d(b_dst + j * C::B_BYTES, &tmB, fb, t * args.cin_k + cb * kBK,
-                                            n0, lb0 + j);
+                            // PB limb tiles [limb][N rows][64 k], one box
+                            tma_load_3d(b_dst, &tmB, fb, t * args.cin_k + cb * kBK, n0, lb0);
                             if (++kcb == knc) { kcb = 0; ++kt; }
                         } else if (MODE == TC_DGRAD) {
                             const int t = kt, cb = kcb, ky = t / 3, kx = t - 3 * ky;
                             if (++kcb == knc) { kcb = 0; ++kt; }
                             tma_load_5d(a_dst, &tmA, fb, cb * kBK, x0 - kx + 1, y0 - ky + 1, b0, la);
                             // B MN-major from the forward planes [L][Cout][9][Cin64]:
-                            // rows co (K) of 64 consecutive ci (N) for tap t
-                            for (int j = 0; j < nb; ++j)
+                            // rows co (K) of 64 consecutive ci (N) for tap t; one box per
+                            // 64-channel block h brings PB limbs, stored [h][limb]
 #pragma unroll
-                                for (int h = 0; h < N / 64; ++h)
-                                    tma_load_4d(b_dst + j * C::B_BYTES + h * (64 * 128), &tmB, fb,
-                                                n0 + 64 * h, t, cb * kBK, lb0 + j);
+                            for (int h = 0; h < N / 64; ++h)
+                                tma_load_4d(b_dst + h * (PB * 64 * 128), &tmB, fb, n0 + 64 * h, t,
+                                            cb * kBK, lb0);
                         } else {  // TC_WGRAD: rows (tap, ci), K = a 64-pixel box (wb x hb)
                             // of one image; both operands MN-major from the NHWC
                             // copies (channels contiguous), the tap shift on x / y.
@@ -444,11 +445,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                             for (int j = 0; j < 2; ++j)
                                 tma_load_4d(a_dst + j * (64 * 128), &tmA, fb, wa_ci[j], px + wa_dx[j],
                                             py + wa_dy[j], bk);
-                            for (int j = 0; j < nb; ++j)
+                            // one box per 64-channel block h brings PB limbs, stored [h][limb]
 #pragma unroll
-                                for (int h = 0; h < N / 64; ++h)
-                                    tma_load_5d(b_dst + j * C::B_BYTES + h * (64 * 128), &tmB, fb,
-                                                n0 + 64 * h, px, py, bk, lb0 + j);
+                            for (int h = 0; h < N / 64; ++h)
+                                tma_load_5d(b_dst + h * (PB * 64 * 128), &tmB, fb, n0 + 64 * h, px,
+                                            py, bk, lb0);
                             if (++wxt == args.ntx) {
                                 wxt = 0;
                                 if (++wyt == args.nty) {
@@ -477,7 +478,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const int cpp = (T.kb1 - T.kb0 + kChunkBlocks - 1) / kChunkBlocks;
                 for (int p = 0; p < passes; ++p) {
                     const int nb = min(PB, LB - (p % NG) * PB);
-                    const uint32_t idesc = idesc_nb[nb];
+                    // MN-major B holds [64-channel block][PB limbs]: the MMA spans all
+                    // of them (unused limbs cost MMA time, not correctness)
+                    const uint32_t idesc = (MODE == TC_WGRAD || MODE == TC_DGRAD) ? idesc_nb[PB] : idesc_nb[nb];
                     for (int c = 0; c < cpp; ++c, ++chunk) {
                         const int buf = chunk % NBUF;
                         if (!mbar_wait(tempty_bar(buf), ((chunk / NBUF) & 1) ^ 1, abort_flag,
@@ -536,8 +539,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                         goto epi_done;
                     tc_fence_after();
                     for (int jb = 0; jb < nb; ++jb) {
+                        // K-major B: limb-major columns; MN-major B: 64-column blocks
+                        // ordered [channel block][limb]
+                        const int hb = (half * NH) / 64;
+                        const int colj = (MODE == TC_WGRAD || MODE == TC_DGRAD)
+                            ? (hb * PB + jb) * 64 + (half * NH - hb * 64)
+                            : jb * N + half * NH;
                         const uint32_t base = tmem + ((uint32_t)(32 * q) << 16) +
-                                              (uint32_t)((buf * PB + jb) * N + half * NH);
+                                              (uint32_t)(buf * PB * N + colj);
                         const int shift = shift0 + 8 * jb;
                         // 16 columns at a time; acc += v 2^shift as one 32 x 32 -> 64
                         // multiply-add below 2^32, an add to the high word above
@@ -1020,18 +1029,23 @@ cudaError_t launch_gemm(const CUtensorMap& a, const CUtensorMap& b, const TcArgs
     return cudaGetLastError();
 }
 
-// Tile width n and B limbs per stage from the (last seen) limb count of B:
-// as many limbs per stage as the operand has, up to the TMEM budget (PB N <=
-// 256).  Any choice is exact; it only changes speed.
+// Tile width n and B limbs per stage (pb) from the (last seen) limb count of
+// B: as many limbs per stage as the operand has, up to the TMEM budget
+// (pb n <= 256).  Any choice is exact; it only changes speed.
+int pick_pb(int n, int limbs_hint) {
+    if (n == 128) return limbs_hint > 1 ? 2 : 1;
+    return limbs_hint > 2 ? 4 : (limbs_hint == 2 ? 2 : 1);
+}
+
+// The B tensor map's box spans pb limb planes (one TMA load per stage and
+// 64-channel block brings all of them), so pb must match the variant.
 template <int MODE>
-cudaError_t launch_gemm_n(int n, int limbs_hint, const CUtensorMap& a, const CUtensorMap& b,
-                          const TcArgs& args, cudaStream_t s) {
+cudaError_t launch_gemm_pb(int n, int pb, const CUtensorMap& a, const CUtensorMap& b,
+                           const TcArgs& args, cudaStream_t s) {
     if (n == 128)
-        return limbs_hint > 1 ? launch_gemm<MODE, 128, 2>(a, b, args, s)
-                              : launch_gemm<MODE, 128, 1>(a, b, args, s);
-    if (limbs_hint > 2) return launch_gemm<MODE, 64, 4>(a, b, args, s);
-    return limbs_hint == 2 ? launch_gemm<MODE, 64, 2>(a, b, args, s)
-                           : launch_gemm<MODE, 64, 1>(a, b, args, s);
+        return pb == 2 ? launch_gemm<MODE, 128, 2>(a, b, args, s) : launch_gemm<MODE, 128, 1>(a, b, args, s);
+    if (pb == 4) return launch_gemm<MODE, 64, 4>(a, b, args, s);
+    return pb == 2 ? launch_gemm<MODE, 64, 2>(a, b, args, s) : launch_gemm<MODE, 64, 1>(a, b, args, s);
 }
 
 int pick_n(int cols) { return cols % 128 == 0 ? 128 : 64; }
@@ -1202,14 +1216,15 @@ cudaError_t tc_conv_forward(TcLayer& t, const LayerGeom& g, int batch, int64_t* 
     const uint64_t sa[3] = {(uint64_t)t.cin8, (uint64_t)g.w * t.cin8, (uint64_t)g.h * g.w * t.cin8};
     const uint32_t ba[4] = {64, (uint32_t)a.wb, (uint32_t)a.hb, (uint32_t)a.bb};
     const uint64_t kw = (uint64_t)a.taps * t.cin_k;   // w_planes row length
+    const int pb = pick_pb(n, tc_limb_hint(t, 0));
     const uint64_t db[3] = {kw, (uint64_t)g.cout, (uint64_t)kMaxLimbs};
     const uint64_t sb[2] = {kw, kw * g.cout};
-    const uint32_t bb[3] = {64, (uint32_t)n, 1};
+    const uint32_t bb[3] = {64, (uint32_t)n, (uint32_t)pb};
     if (!make_map(&ma, t.act_nhwc, 4, da, sa, ba) || !make_map(&mb, t.w_planes, 3, db, sb, bb))
         return cudaErrorInvalidValue;
     const double ops = 2.0 * batch * g.h * g.w * g.cout * 9.0 * g.cin;
     ProfScope ps(K_TC_CONV_FWD, s, ops, 0.0);
-    cudaError_t e = launch_gemm_n<TC_FWD>(n, tc_limb_hint(t, 0), ma, mb, a, s);
+    cudaError_t e = launch_gemm_pb<TC_FWD>(n, pb, ma, mb, a, s);
     if (e == cudaSuccess) {
         *done = true;
         *fused = a.fuse != 0;
@@ -1280,7 +1295,8 @@ cudaError_t tc_conv_wgrad(TcLayer& t, const LayerGeom& g, const int32_t* delta,
                             (uint64_t)kMaxLimbs};
     const uint64_t sb[4] = {(uint64_t)g.cout, (uint64_t)g.w * g.cout, (uint64_t)hw * g.cout,
                             (uint64_t)batch * hw * g.cout};
-    const uint32_t bb[5] = {64, (uint32_t)a.wb, (uint32_t)a.hb, 1, 1};
+    const int pb = pick_pb(n, tc_limb_hint(t, 1));
+    const uint32_t bb[5] = {64, (uint32_t)a.wb, (uint32_t)a.hb, 1, (uint32_t)pb};
     if (!make_map(&ma, t.act_nhwc, 4, da, sa, ba) || !make_map(&mb, t.d_nhwc, 5, db, sb, bb))
         return cudaErrorInvalidValue;
     if (a.atomic_out) {
@@ -1289,7 +1305,7 @@ cudaError_t tc_conv_wgrad(TcLayer& t, const LayerGeom& g, const int32_t* delta,
     }
     const double ops = 2.0 * batch * hw * g.cout * 9.0 * g.cin;
     ProfScope ps(K_TC_CONV_WGRAD, s, ops, 0.0);
-    cudaError_t e = launch_gemm_n<TC_WGRAD>(n, tc_limb_hint(t, 1), ma, mb, a, s);
+    cudaError_t e = launch_gemm_pb<TC_WGRAD>(n, pb, ma, mb, a, s);
     if (e == cudaSuccess) *done = true;
     return e;
 }
@@ -1347,12 +1363,13 @@ cudaError_t tc_conv_dgrad(TcLayer& t, const LayerGeom& g, int batch, int64_t* g6
     // forward planes [L][Cout][9][Cin64], read MN-major: boxes of 64 ci x 64 co
     const uint64_t db[4] = {(uint64_t)t.cin_k, 9, (uint64_t)g.cout, (uint64_t)kMaxLimbs};
     const uint64_t sb[3] = {(uint64_t)t.cin_k, (uint64_t)9 * t.cin_k, (uint64_t)9 * t.cin_k * g.cout};
-    const uint32_t bb[4] = {64, 1, 64, 1};
+    const int pb = pick_pb(n, tc_limb_hint(t, 0));
+    const uint32_t bb[4] = {64, 1, 64, (uint32_t)pb};
     if (!make_map(&ma, t.d_nhwc, 5, da, sa, ba) || !make_map(&mb, t.w_planes, 4, db, sb, bb))
         return cudaErrorInvalidValue;
     const double ops = 2.0 * batch * g.h * g.w * g.cin * 9.0 * g.cout;
     ProfScope ps(K_TC_CONV_DGRAD, s, ops, 0.0);
-    cudaError_t e = launch_gemm_n<TC_DGRAD>(n, tc_limb_hint(t, 0), ma, mb, a, s);
+    cudaError_t e = launch_gemm_pb<TC_DGRAD>(n, pb, ma, mb, a, s);
     if (e == cudaSuccess) {
         *done = true;
         *fused = a.fuse != 0;
@@ -1424,7 +1441,7 @@ cudaError_t tc_gemm_run(const uint16_t* a_bf16, const uint16_t* b_planes, int M,
     if (!make_map(&ma, a_bf16, 2, da, sa, ba) || !make_map(&mb, b_planes, 3, db, sb, bb))
         return cudaErrorInvalidValue;
     ProfScope ps(K_TC_GEMM, s, 2.0 * M * N * (double)K, 0.0);
-    return launch_gemm_n<TC_GEMM>(n, 1, ma, mb, a, s);
+    return launch_gemm_pb<TC_GEMM>(n, 1, ma, mb, a, s);
 }
 
 }  // namespace nitro
