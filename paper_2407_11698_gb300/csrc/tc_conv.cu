@@ -538,36 +538,51 @@ __global__ void __launch_bounds__(kThreads, 1)
                     if (!mbar_wait(tfull_bar(buf), (chunk / NBUF) & 1, abort_flag, args.status))
                         goto epi_done;
                     tc_fence_after();
-                    for (int jb = 0; jb < nb; ++jb) {
-                        // K-major B: limb-major columns; MN-major B: 64-column blocks
-                        // ordered [channel block][limb]
+                    // K-major B: limb-major columns; MN-major B: 64-column blocks
+                    // ordered [channel block][limb]
+                    auto limb_base = [&](int jb) -> uint32_t {
                         const int hb = (half * NH) / 64;
                         const int colj = (MODE == TC_WGRAD || MODE == TC_DGRAD)
                             ? (hb * PB + jb) * 64 + (half * NH - hb * 64)
                             : jb * N + half * NH;
-                        const uint32_t base = tmem + ((uint32_t)(32 * q) << 16) +
-                                              (uint32_t)(buf * PB * N + colj);
-                        const int shift = shift0 + 8 * jb;
-                        // 16 columns at a time; acc += v 2^shift as one 32 x 32 -> 64
-                        // multiply-add below 2^32, an add to the high word above
-                        // (shift is a multiple of 8)
+                        return tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(buf * PB * N + colj);
+                    };
+                    // acc += v 2^shift: one 32 x 32 -> 64 multiply-add below 2^32, an
+                    // add to the high word above (shift is a multiple of 8)
+                    auto accumulate = [&](const uint32_t* r, int j, int shift) {
+                        if (shift < 32) {
+                            const int m = 1 << shift;
 #pragma unroll
-                        for (int j = 0; j < NH / 16; ++j) {
-                            uint32_t r[16];
-                            tmem_ld16(base + 16 * j, r);
-                            if (shift < 32) {
-                                const int m = 1 << shift;
+                            for (int i = 0; i < 16; ++i) {
+                                const int v = __float2int_rz(__uint_as_float(r[i]));   // exact integer
+                                acc[16 * j + i] += (uint64_t)((long long)v * (long long)m);
+                            }
+                        } else {
 #pragma unroll
-                                for (int i = 0; i < 16; ++i) {
-                                    const int v = __float2int_rz(__uint_as_float(r[i]));   // exact integer
-                                    acc[16 * j + i] += (uint64_t)((long long)v * (long long)m);
-                                }
-                            } else {
+                            for (int i = 0; i < 16; ++i) {
+                                const int v = __float2int_rz(__uint_as_float(r[i]));
+                                acc[16 * j + i] += (uint64_t)((uint32_t)v << (shift - 32)) << 32;
+                            }
+                        }
+                    };
+                    if (NH == 16) {
+                        // 16 columns per limb: two limbs per TMEM round trip
+                        for (int jb = 0; jb < nb; jb += 2) {
+                            uint32_t r0[16], r1[16];
+                            tmem_ld16_nowait(limb_base(jb), r0);
+                            if (jb + 1 < nb) tmem_ld16_nowait(limb_base(jb + 1), r1);
+                            asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+                            accumulate(r0, 0, shift0 + 8 * jb);
+                            if (jb + 1 < nb) accumulate(r1, 0, shift0 + 8 * (jb + 1));
+                        }
+                    } else {
+                        for (int jb = 0; jb < nb; ++jb) {
+                            const uint32_t base = limb_base(jb);
 #pragma unroll
-                                for (int i = 0; i < 16; ++i) {
-                                    const int v = __float2int_rz(__uint_as_float(r[i]));
-                                    acc[16 * j + i] += (uint64_t)((uint32_t)v << (shift - 32)) << 32;
-                                }
+                            for (int j = 0; j < NH / 16; ++j) {
+                                uint32_t r[16];
+                                tmem_ld16(base + 16 * j, r);
+                                accumulate(r, j, shift0 + 8 * jb);
                             }
                         }
                     }
@@ -617,7 +632,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const int x = tx * args.wb + xx, y = ty * args.hb + yy, b = tb * args.bb + bbx;
                     const bool valid = x < args.W && y < args.H && b < args.B;
                     const int C = args.Cout;
-                    const int64_t zlo = args.z_lo, zhi = args.z_hi;
+                    const int64_t zlo = args.z_lo;
+                    const uint64_t zrange = (uint64_t)(args.z_hi - args.z_lo);
                     const FloorDiv32 sf32 = args.sf32;
                     uint32_t vpk[NH / 4], rpk[NH / 4];
 #pragma unroll
@@ -625,15 +641,18 @@ __global__ void __launch_bounds__(kThreads, 1)
                         uint32_t vp = 0, rp = 0;
 #pragma unroll
                         for (int u = 0; u < 4; ++u) {
-                            // z* = floor(z / SF) clamped to [-127, 127] (the NITRO-ReLU
-                            // value is flat outside): floor((z >> 8) / 9Cin) of the
-                            // clamped z fits 32 bits.  The piece comes from z itself.
-                            const int64_t z = (int64_t)acc[4 * g4 + u];
-                            const int64_t zc = z < zlo ? zlo : (z >= zhi ? zhi - 1 : z);
-                            const int zq = sf32.floor_div((int32_t)(zc >> 8));
-                            const int reg = z >= zhi ? 3 : (z < zlo ? 0 : (z < 0 ? 1 : 2));
+                            // z* = floor(z / SF) = floor((z >> 8) / 9Cin).  Inside
+                            // [-127 SF, 128 SF) it fits 32 bits and indexes the NITRO-ReLU
+                            // table; outside, the value is flat (table ends) and only the
+                            // sign picks the piece.
+                            const uint64_t z = acc[4 * g4 + u];
+                            const bool inside = z - (uint64_t)zlo < zrange;
+                            const bool neg = (int32_t)(z >> 32) < 0;
+                            const int zq = sf32.floor_div((int32_t)((int64_t)z >> 8));
+                            const int idx = inside ? zq + 127 : (neg ? 0 : 254);
+                            const int reg = inside ? (neg ? 1 : 2) : (neg ? 0 : 3);
                             rp |= (uint32_t)reg << (8 * u);
-                            vp |= (uint32_t)(uint8_t)relu_tab[zq + 127] << (8 * u);
+                            vp |= (uint32_t)(uint8_t)relu_tab[idx] << (8 * u);
                         }
                         vpk[g4] = vp;
                         rpk[g4] = rp;
