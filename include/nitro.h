@@ -9,7 +9,9 @@
  * trained on the RSS loss).  A block with zero forward layers is the network's
  * output block.  A network is a chain of handles; the caller runs every
  * block's forward, then every block's backward (they are independent, Sec.
- * 3.3), then every block's IntegerSGD step.
+ * 3.3), then every block's IntegerSGD step.  Handles share no state, so each
+ * block may run on its own stream: block i+1's forward needs only block i's
+ * output, and block i's backward and update may overlap the blocks after it.
  *
  * Conventions
  *   activations   int8, NHWC  a[((b*H + y)*W + x)*C + c]; linear: a[b*In + i]
