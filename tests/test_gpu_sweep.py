@@ -67,6 +67,34 @@ def test_conv_contractions_full(torch, B, h, w, cin, cout, lw, ld):
         conv.close()
 
 
+@pytest.mark.parametrize("edge", [127, 128, 32639, 32640, 8355711, 8355712, 2**31 - 1, -2**31])
+def test_limb_count_boundaries(torch, edge):
+    # operands whose max |x| sits exactly at (or one past) a limb-count boundary
+    # of the canonical split; every contraction must stay exact
+    B, h, w, c = 2, 8, 8, 64
+    a = synth.images(71, 0, B, (h, w, c)).astype(np.int64)
+    W = synth.int_tensor(72, (c, 3, 3, c), -100, 100)
+    d = synth.int_tensor(73, (B, h, w, c), -100, 100)
+    W.flat[5] = edge
+    W.flat[-3] = -edge if edge > -2**31 else 2**31 - 1
+    d.flat[7] = edge
+    conv = nb.Conv3x3(B, h, w, c, c)
+    try:
+        ad, Wd, dd = _dev(torch, a, np.int8), _dev(torch, W, np.int32), _dev(torch, d, np.int32)
+        z = torch.empty((B, h, w, c), dtype=torch.int64, device="cuda")
+        conv.contract(nb.NITRO_CONTRACT_FWD, ad, Wd, z)
+        assert np.array_equal(z.cpu().numpy(), O.conv3x3_fwd(a, W))
+        dw = torch.empty((c, 3, 3, c), dtype=torch.int64, device="cuda")
+        conv.contract(nb.NITRO_CONTRACT_WGRAD, ad, dd, dw)
+        assert np.array_equal(dw.cpu().numpy(), O.conv3x3_wgrad(a, d))
+        g = torch.empty((B, h, w, c), dtype=torch.int64, device="cuda")
+        conv.contract(nb.NITRO_CONTRACT_DGRAD, dd, Wd, g)
+        # the int64 wrap of an int32 x int32 contraction is the oracle's too
+        assert np.array_equal(g.cpu().numpy(), O.conv3x3_dgrad(d, W))
+    finally:
+        conv.close()
+
+
 def _patch(x, b, y, xx):
     """3x3 neighbourhood of pixel (y, xx) of image b, zero outside the image."""
     B, H, W, C = x.shape

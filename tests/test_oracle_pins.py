@@ -137,6 +137,69 @@ def test_conv_fwd_matches_scipy_correlate2d():
             assert np.array_equal(z[b, :, :, co], ref)
 
 
+def _brute_conv(a, w):
+    """Direct definition in Python integers: z[b,y,x,co] = sum over taps (ky, kx)
+    and ci of a[b, y+ky-1, x+kx-1, ci] w[co, ky, kx, ci], zero outside."""
+    B, H, W, Cin = a.shape
+    Cout = w.shape[0]
+    z = [[[[0] * Cout for _ in range(W)] for _ in range(H)] for _ in range(B)]
+    for b in range(B):
+        for y in range(H):
+            for x in range(W):
+                for co in range(Cout):
+                    t = 0
+                    for ky in range(3):
+                        for kx in range(3):
+                            iy, ix = y + ky - 1, x + kx - 1
+                            if 0 <= iy < H and 0 <= ix < W:
+                                for ci in range(Cin):
+                                    t += int(a[b, iy, ix, ci]) * int(w[co, ky, kx, ci])
+                    z[b][y][x][co] = t
+    return z
+
+
+def test_conv_contractions_match_brute_force():
+    # forward, weight gradient and input gradient of the oracle against the
+    # direct sums in Python integers; |w|, |d| < 2^27 keep every sum inside
+    # int64 while the products are far beyond int32, so a 32-bit truncation
+    # anywhere in the oracle would show
+    B, H, W, Cin, Cout = 2, 4, 3, 2, 3
+    a = RNG.integers(-128, 128, size=(B, H, W, Cin))
+    w = RNG.integers(-2**27, 2**27, size=(Cout, 3, 3, Cin))
+    d = RNG.integers(-2**27, 2**27, size=(B, H, W, Cout))
+    assert O.conv3x3_fwd(a, w).tolist() == _brute_conv(a, w)
+    # dW[co,ky,kx,ci] = sum_(b,y,x) d[b,y,x,co] a[b,y+ky-1,x+kx-1,ci]
+    dw = [[[[0] * Cin for _ in range(3)] for _ in range(3)] for _ in range(Cout)]
+    for co in range(Cout):
+        for ky in range(3):
+            for kx in range(3):
+                for ci in range(Cin):
+                    t = 0
+                    for b in range(B):
+                        for y in range(H):
+                            for x in range(W):
+                                iy, ix = y + ky - 1, x + kx - 1
+                                if 0 <= iy < H and 0 <= ix < W:
+                                    t += int(d[b, y, x, co]) * int(a[b, iy, ix, ci])
+                    dw[co][ky][kx][ci] = t
+    assert O.conv3x3_wgrad(a, d).tolist() == dw
+    # g[b,y,x,ci] = sum_(ky,kx,co) d[b,y-ky+1,x-kx+1,co] w[co,ky,kx,ci]
+    g = [[[[0] * Cin for _ in range(W)] for _ in range(H)] for _ in range(B)]
+    for b in range(B):
+        for y in range(H):
+            for x in range(W):
+                for ci in range(Cin):
+                    t = 0
+                    for ky in range(3):
+                        for kx in range(3):
+                            oy, ox = y - ky + 1, x - kx + 1
+                            if 0 <= oy < H and 0 <= ox < W:
+                                for co in range(Cout):
+                                    t += int(d[b, oy, ox, co]) * int(w[co, ky, kx, ci])
+                    g[b][y][x][ci] = t
+    assert O.conv3x3_dgrad(d, w).tolist() == g
+
+
 def test_conv_one_hot_reproduces_flipped_kernel():
     H = W = 5
     w = RNG.integers(-50, 50, size=(2, 3, 3, 3))
