@@ -727,39 +727,58 @@ __global__ void __launch_bounds__(kThreads, 1)
                     if (valid) {
                         const int64_t opix = ((int64_t)b * args.H + y) * args.W + x;
                         const int npos = args.low_pool ? 4 : 1;
-                        // four channels at a time: gradient, its floor quotient by
-                        // alpha_inv, then each window position's region byte
+                        int64_t ppix[4];
 #pragma unroll
-                        for (int e4 = 0; e4 < NH / 4; ++e4) {
-                            const int c0 = col0 + 4 * e4;
-                            if (c0 >= Cl) break;
-                            int32_t gs[4], gq[4];
+                        for (int k = 0; k < 4; ++k)
+                            ppix[k] = args.low_pool
+                                ? ((int64_t)b * args.low_h + 2 * y + (k >> 1)) * args.low_w + 2 * x + (k & 1)
+                                : opix;
+                        // per 16 channels: the argmax and region words of every window
+                        // position are loaded first (16-byte loads), then the gradient,
+                        // its floor quotient by alpha_inv and the stores, 4 channels at
+                        // a time
 #pragma unroll
-                            for (int e = 0; e < 4; ++e) {
-                                const int64_t gv = (int64_t)acc[4 * e4 + e];
-                                ovf |= !fits_i32(gv);
-                                gs[e] = (int32_t)gv;
-                                gq[e] = args.alpha32.floor_div(gs[e]);
-                            }
-                            const uint32_t amw = args.low_pool
-                                ? *reinterpret_cast<const uint32_t*>(args.low_argmax + opix * Cl + c0)
-                                : 0u;
-                            for (int k = 0; k < npos; ++k) {
-                                const int64_t ppix = args.low_pool
-                                    ? ((int64_t)b * args.low_h + 2 * y + (k >> 1)) * args.low_w + 2 * x + (k & 1)
-                                    : opix;
-                                const uint32_t rgw = *reinterpret_cast<const uint32_t*>(args.low_region + ppix * Cl + c0);
-                                int32_t dv[4];
+                        for (int k16 = 0; k16 < NH / 16; ++k16) {
+                            const int c16 = col0 + 16 * k16;
+                            if (c16 >= Cl) break;
+                            const uint4 amv = args.low_pool
+                                ? *reinterpret_cast<const uint4*>(args.low_argmax + opix * Cl + c16)
+                                : make_uint4(0, 0, 0, 0);
+                            uint4 rgv[4];
+#pragma unroll
+                            for (int k = 0; k < 4; ++k)
+                                rgv[k] = k < npos ? *reinterpret_cast<const uint4*>(args.low_region + ppix[k] * Cl + c16)
+                                                  : make_uint4(0, 0, 0, 0);
+                            const uint32_t amw4[4] = {amv.x, amv.y, amv.z, amv.w};
+#pragma unroll
+                            for (int e4 = 0; e4 < 4; ++e4) {
+                                const int c0 = c16 + 4 * e4;
+                                int32_t gs[4], gq[4];   // gradient and floor(gradient / alpha_inv)
 #pragma unroll
                                 for (int e = 0; e < 4; ++e) {
-                                    const int reg = (int)((rgw >> (8 * e)) & 255u);
-                                    const int am = (int)((amw >> (8 * e)) & 255u);
-                                    const int32_t v = am != k ? 0 : (reg == 1 ? gq[e] : (reg == 2 ? gs[e] : 0));
-                                    dv[e] = v;
-                                    mx = max(mx, abs_u32(v));
+                                    const int64_t gv = (int64_t)acc[16 * k16 + 4 * e4 + e];
+                                    ovf |= !fits_i32(gv);
+                                    gs[e] = (int32_t)gv;
+                                    gq[e] = args.alpha32.floor_div(gs[e]);
                                 }
-                                *reinterpret_cast<int4*>(args.low_delta + ppix * Cl + c0) =
-                                    make_int4(dv[0], dv[1], dv[2], dv[3]);
+                                const uint32_t amw = amw4[e4];
+#pragma unroll
+                                for (int k = 0; k < 4; ++k) {
+                                    if (k >= npos) break;
+                                    const uint32_t rw[4] = {rgv[k].x, rgv[k].y, rgv[k].z, rgv[k].w};
+                                    const uint32_t rgw = rw[e4];
+                                    int32_t dv[4];
+#pragma unroll
+                                    for (int e = 0; e < 4; ++e) {
+                                        const int reg = (int)((rgw >> (8 * e)) & 255u);
+                                        const int am = (int)((amw >> (8 * e)) & 255u);
+                                        const int32_t v = am != k ? 0 : (reg == 1 ? gq[e] : (reg == 2 ? gs[e] : 0));
+                                        dv[e] = v;
+                                        mx = max(mx, abs_u32(v));
+                                    }
+                                    *reinterpret_cast<int4*>(args.low_delta + ppix[k] * Cl + c0) =
+                                        make_int4(dv[0], dv[1], dv[2], dv[3]);
+                                }
                             }
                         }
                     }
@@ -905,7 +924,7 @@ __global__ void __launch_bounds__(256) k_pack_delta_nhwc(const int32_t* __restri
     const int64_t n8 = n / 8;
     for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n8;
          i += (int64_t)gridDim.x * blockDim.x) {
-        int64_t v[8];
+        int32_t v[8];
         if (vec) {
             const int4 a0 = reinterpret_cast<const int4*>(d)[2 * i];
             const int4 a1 = reinterpret_cast<const int4*>(d)[2 * i + 1];
@@ -919,17 +938,21 @@ __global__ void __launch_bounds__(256) k_pack_delta_nhwc(const int32_t* __restri
             uint32_t w[4];
 #pragma unroll
             for (int k = 0; k < 8; k += 2) {
-                int dg[2];
+                uint32_t hb[2];
 #pragma unroll
                 for (int u = 0; u < 2; ++u) {
+                    int dg;
                     if (l < L - 1) {
-                        dg[u] = (int)(((v[k + u] + 128) & 255) - 128);
-                        v[k + u] = (v[k + u] - dg[u]) >> 8;
+                        // v = 256 q + r: digit r or r - 256, remainder q or q + 1
+                        const int r = v[k + u] & 255;
+                        dg = r - ((r >> 7) << 8);
+                        v[k + u] = (v[k + u] >> 8) + (r >> 7);
                     } else {
-                        dg[u] = (int)v[k + u];
+                        dg = v[k + u];
                     }
+                    hb[u] = __float_as_uint((float)dg) >> 16;   // exact: |dg| <= 128
                 }
-                w[k / 2] = (uint32_t)bf16_bits(dg[0]) | ((uint32_t)bf16_bits(dg[1]) << 16);
+                w[k / 2] = hb[0] | (hb[1] << 16);
             }
             reinterpret_cast<uint4*>(out + (int64_t)l * n)[i] = make_uint4(w[0], w[1], w[2], w[3]);
         }
