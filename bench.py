@@ -41,7 +41,10 @@ def parse():
                    help="run all blocks on one stream (default: a stream per block)")
     p.add_argument("--profile-steps", type=int, default=3)
     p.add_argument("--sweep", action="store_true",
-                   help="time the kernel sweep (conv contractions and integer GEMM) instead")
+                   help="time the kernel sweep (conv contractions, integer GEMM, IntegerSGD, "
+                        "pre-processing) instead")
+    p.add_argument("--sweep-parts", default="conv,gemm,sgd,prep",
+                   help="comma-separated subset of the sweep to run")
     return p.parse_args()
 
 
@@ -500,7 +503,8 @@ def run_sweep(args):
                 "peak_source": "bf16 dense, %s" % src}
         print(json.dumps(line), flush=True)
 
-    for B, hw, c in WL.SWEEP_CONV:
+    parts = set(args.sweep_parts.split(","))
+    for B, hw, c in (WL.SWEEP_CONV if "conv" in parts else ()):
         a = torch.from_numpy(synth.images(51, 0, B, (hw, hw, c))).cuda()
         conv = nb.Conv3x3(B, hw, hw, c, c)
         out = torch.empty((B, hw, hw, c), dtype=torch.int64, device="cuda")
@@ -521,7 +525,7 @@ def run_sweep(args):
         conv.close()
         del a, out, dw
         torch.cuda.empty_cache()
-    for n in WL.SWEEP_GEMM:
+    for n in (WL.SWEEP_GEMM if "gemm" in parts else ()):
         a = torch.from_numpy(synth.int_tensor(61, (n, n), -128, 127, dtype=np.int8)).cuda()
         b8 = torch.from_numpy(synth.int_tensor(62, (n, n), -128, 127, dtype=np.int8)).cuda()
         gm = nb.IntGemm(n, n, n)
@@ -553,7 +557,7 @@ def run_sweep(args):
     # IntegerSGD alone: one linear layer of n x n weights, 16 bytes per weight
     # (W read + write, dW read), against the measured HBM copy bandwidth
     hbm = peaks["hbm_gbs"]
-    for n in (4096, 16384):
+    for n in ((4096, 16384) if "sgd" in parts else ()):
         blk = nb.Block([(nb.NITRO_LINEAR, n, n, 1, 1, 0)], n, seed=1, max_batch=1)
         ms, prof = timed(lambda: blk.sgd(), 5)
         k = prof.get("integersgd", {"ms": float("nan"), "launches": 1})
@@ -567,6 +571,38 @@ def run_sweep(args):
                           "peak_source": "HBM copy, %s" % src}), flush=True)
         blk.close()
         torch.cuda.empty_cache()
+    # integer data pre-processing (App. A) at the raw dataset shapes: fit
+    # (byte sum, then the sum of |x - mu|: n bytes read each) and apply (n bytes
+    # read, n written), against the measured HBM copy bandwidth.  The MNIST
+    # set (47 MB) stays in the 129 MB L2 between repetitions; CIFAR-10 does not.
+    prep = nb.IntPrep() if "prep" in parts else None
+    for name, shape, kind in ((("mnist_train", (60000, 28, 28), "digits"),
+                               ("cifar10_train", (50000, 32, 32, 3), "natural"))
+                              if prep else ()):
+        n = int(np.prod(shape))
+        x = torch.from_numpy(synth.raw_pixels(3, n, kind)).cuda()
+        out = torch.empty(n, dtype=torch.int8, device="cuda")
+        ms_fit, prof_fit = timed(lambda: prep.fit(x), 10)
+        ms_app, prof_app = timed(lambda: prep.apply(x, out), 10)
+        kern = {}
+        for key, prof, byts in (("prep_sum", prof_fit, n), ("prep_mad", prof_fit, n),
+                                ("prep_apply", prof_app, 2 * n)):
+            k = prof.get(key, {"ms": float("nan"), "launches": 1})
+            kms = k["ms"] / max(1, k["launches"])
+            kern[key] = {"kernel_ms": round(kms, 5), "bytes": byts,
+                         "kernel_gbs": round(byts / kms / 1e6, 1),
+                         "kernel_frac_hbm": round(byts / kms / 1e6 / hbm, 4)}
+        print(json.dumps({"sweep": "preprocess", "dataset": name, "shape": list(shape),
+                          "values": kind, "n": n, "fit_ms": round(ms_fit, 5),
+                          "apply_ms": round(ms_app, 5),
+                          "fit_gbs": round(2 * n / ms_fit / 1e6, 1),
+                          "apply_gbs": round(2 * n / ms_app / 1e6, 1), "kernels": kern,
+                          "l2_resident": n < 129e6, "peak": hbm,
+                          "peak_source": "HBM copy, %s" % src}), flush=True)
+        del x, out
+    if prep:
+        prep.close()
+    torch.cuda.empty_cache()
     return 0
 
 

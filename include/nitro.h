@@ -133,6 +133,18 @@ nitro_status nitro_block_backward(nitro_block* blk, const int8_t* a_in, const in
  * learning layer gamma_inv_lr and eta_inv_lr. */
 nitro_status nitro_integersgd_step(nitro_block* blk, void* stream);
 
+/* Replaces the IntegerSGD hyper-parameters of a block (Algorithm 1):
+ * gamma_inv_lr (the forward layers use 2^6*G*gamma_inv_lr, Sec. 3.3.5),
+ * eta_inv_fw and eta_inv_lr.  App. B multiplies the inverse learning rate by 3
+ * each time the test accuracy reaches a plateau; this is the call that applies
+ * such a change.  Host-only: it takes effect at the next nitro_integersgd_step
+ * call, while a CUDA graph that captured an earlier step keeps the values it
+ * was captured with until it is captured again.  Range checks as in
+ * nitro_init_block (1 <= gamma_inv_lr <= 2^48, eta >= 0); on NITRO_ERR_ARG
+ * nothing changes. */
+nitro_status nitro_block_set_hyper(nitro_block* blk, int64_t gamma_inv_lr, int64_t eta_inv_fw,
+                                   int64_t eta_inv_lr);
+
 /* Tensors readable / writable through get/set_tensor.  Batch-shaped tensors
  * hold the last forward/backward batch. */
 typedef enum {
@@ -231,6 +243,36 @@ nitro_status nitro_conv3x3_forward_noalloc(const int8_t* a_in, const int32_t* we
                                            int h, int w, int cin, int cout, int pool2x2,
                                            int alpha_inv, int8_t* a_out, int8_t* region,
                                            int8_t* argmax, void* stream);
+
+/* ---- Integer data pre-processing (App. A) ---------------------------------
+ * Maps a dataset of n 8-bit values x (every element of every sample, e.g.
+ * image bytes) to int8 values centred on 0 with a spread of about 64:
+ *   mu    = floor(sum x / n)
+ *   omega = floor(sum |x - mu| / n)          (mean absolute deviation)
+ *   x_hat = floor((x - mu) * 51 / omega), clamped to [-127, 127]
+ * 51 = floor(64 * 0.8), since the MAD of Gaussian data is ~0.8 sigma.  The
+ * appendix leaves omega = 0 undefined: it is read as a divisor of 1.
+ *
+ * nitro_prep_fit computes mu and omega of one device buffer x [n] (two
+ * passes over it) and keeps them in the handle with the 256-entry map they
+ * define; nitro_prep_apply maps any device buffer x [n] to out [n] (int8) with
+ * the statistics of the last fit, so a test set can be mapped with the
+ * training set's.  out may equal x (in place) but must not overlap it
+ * otherwise.  Both calls are asynchronous on `stream` and may be captured into
+ * a CUDA graph; the handle must not be used by two streams at once.
+ * nitro_prep_stats synchronises the device and returns the statistics of the
+ * last fit.  Buffers need no alignment; x and out at the same offset from a
+ * 16-byte boundary take 16-byte vector accesses.
+ * Errors: NITRO_ERR_ARG for a null handle or pointer, n < 1 in fit (n < 0 in
+ * apply, where 0 queues nothing), n > 2^48, or apply / stats before a fit;
+ * NITRO_ERR_CUDA for a failed allocation or launch. */
+typedef struct nitro_prep nitro_prep;
+nitro_status nitro_prep_create(nitro_prep** out);
+nitro_status nitro_prep_fit(nitro_prep* p, const uint8_t* x, int64_t n, void* stream);
+nitro_status nitro_prep_apply(nitro_prep* p, const uint8_t* x, int64_t n, int8_t* out,
+                              void* stream);
+nitro_status nitro_prep_stats(nitro_prep* p, int64_t* mu, int64_t* omega);
+void nitro_prep_destroy(nitro_prep* p);
 
 /* ---- Diagnostics (not part of the training step) -------------------------
  * Every kernel launch of the library is counted.  With profiling on, each

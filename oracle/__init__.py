@@ -13,5 +13,5 @@ from .nitro import (  # noqa: F401
     LayerDesc, OracleBlock, train_step, lib, fdiv, tdiv, relu_mu, relu, relu_region,
     relu_bwd, isqrt, init_bound, splitmix64_at, conv3x3_fwd, conv3x3_dgrad,
     conv3x3_wgrad, linear_fwd, linear_dgrad, linear_wgrad, maxpool_fwd, maxpool_bwd,
-    integersgd, amplification_factor, num_threads,
+    integersgd, amplification_factor, num_threads, prep_stats, prep_apply,
 )

@@ -71,6 +71,8 @@ def lib():
         getattr(L, name).argtypes = [_I64] * 4 + [_P64, _P64, _P64]
     L.nor_maxpool_bwd.argtypes = [_I64] * 4 + [_P64, _P64, _P64]
     L.nor_integersgd.argtypes = [_I64, _P64, _P64, _I64, _I64, _I64]
+    L.nor_prep_stats.argtypes = [_I64, ctypes.c_void_p, _P64, _P64]
+    L.nor_prep_apply.argtypes = [_I64, ctypes.c_void_p, _I64, _I64, ctypes.c_void_p]
     _lib = L
     return L
 
@@ -125,6 +127,24 @@ def splitmix64_at(seed, index):
 
 def num_threads():
     return lib().nor_num_threads()
+
+
+def prep_stats(x):
+    """(mu_int, omega_int) of the 8-bit values ``x`` (App. A)."""
+    x = np.ascontiguousarray(x, dtype=np.uint8).reshape(-1)
+    if x.size == 0:
+        raise ValueError("pre-processing needs at least one value")
+    mu, om = ctypes.c_int64(), ctypes.c_int64()
+    lib().nor_prep_stats(x.size, x.ctypes.data, ctypes.byref(mu), ctypes.byref(om))
+    return mu.value, om.value
+
+
+def prep_apply(x, mu, omega):
+    """x_hat = floor((x - mu) 51 / omega) as int8 in [-127, 127] (App. A)."""
+    x = np.ascontiguousarray(x, dtype=np.uint8)
+    out = np.empty(x.shape, dtype=np.int8)
+    lib().nor_prep_apply(x.size, x.ctypes.data, int(mu), int(omega), out.ctypes.data)
+    return out
 
 
 def amplification_factor(num_classes):

@@ -325,3 +325,36 @@ void nor_integersgd(int64_t n, int64_t* w, const int64_t* dw, int64_t gamma_inv,
         w[i] = w[i] - d;
     }
 }
+
+/* ---------------------------------------------------------------------- */
+/* Integer data pre-processing, App. A.  Over the n 8-bit values x of a    */
+/* dataset (every element of every sample counts once):                    */
+/*   mu    = floor(sum_i x_i / n)                                          */
+/*   omega = floor(sum_i |x_i - mu| / n)     (mean absolute deviation)     */
+/*   x_hat = floor((x_i - mu) * 51 / omega)  (51 = floor(64 * 0.8))        */
+/* Readings where the appendix is silent: omega = 0 divides by 1, and      */
+/* x_hat is stored as int8 clamped to [-127, 127], the interval the        */
+/* appendix names as the int8 range the output is meant to fill.           */
+/* ---------------------------------------------------------------------- */
+void nor_prep_stats(int64_t n, const uint8_t* x, int64_t* mu, int64_t* omega) {
+    int64_t s = 0;
+    for (int64_t i = 0; i < n; ++i) s += x[i];
+    const int64_t m = nor_fdiv(s, n);
+    int64_t a = 0;
+    for (int64_t i = 0; i < n; ++i) {
+        const int64_t dv = (int64_t)x[i] - m;
+        a += dv < 0 ? -dv : dv;
+    }
+    *mu = m;
+    *omega = nor_fdiv(a, n);
+}
+
+void nor_prep_apply(int64_t n, const uint8_t* x, int64_t mu, int64_t omega, int8_t* out) {
+    const int64_t div = omega > 0 ? omega : 1;
+    for (int64_t i = 0; i < n; ++i) {
+        int64_t v = nor_fdiv(((int64_t)x[i] - mu) * 51, div);
+        if (v < -127) v = -127;
+        if (v > 127) v = 127;
+        out[i] = (int8_t)v;
+    }
+}

@@ -106,8 +106,17 @@ def lib():
     L.nitro_gemm_status.argtypes = [_VP]
     L.nitro_gemm_destroy.argtypes = [_VP]
     L.nitro_gemm_destroy.restype = None
+    L.nitro_block_set_hyper.argtypes = [_VP, ctypes.c_int64, ctypes.c_int64, ctypes.c_int64]
+    L.nitro_block_set_hyper.restype = ctypes.c_int
+    L.nitro_prep_create.argtypes = [ctypes.POINTER(_VP)]
+    L.nitro_prep_fit.argtypes = [_VP, _VP, ctypes.c_int64, _VP]
+    L.nitro_prep_apply.argtypes = [_VP, _VP, ctypes.c_int64, _VP, _VP]
+    L.nitro_prep_stats.argtypes = [_VP, ctypes.POINTER(ctypes.c_int64), ctypes.POINTER(ctypes.c_int64)]
+    L.nitro_prep_destroy.argtypes = [_VP]
+    L.nitro_prep_destroy.restype = None
     for name in ("nitro_conv3x3_create", "nitro_conv3x3_contract", "nitro_conv3x3_status",
-                 "nitro_gemm_create", "nitro_gemm_run", "nitro_gemm_status"):
+                 "nitro_gemm_create", "nitro_gemm_run", "nitro_gemm_status",
+                 "nitro_prep_create", "nitro_prep_fit", "nitro_prep_apply", "nitro_prep_stats"):
         getattr(L, name).restype = ctypes.c_int
     for name in ("nitro_init_block", "nitro_block_forward", "nitro_block_backward",
                  "nitro_integersgd_step", "nitro_block_tensor_bytes", "nitro_block_get_tensor",
@@ -240,6 +249,12 @@ class Block:
         if st != NITRO_OK:
             raise NitroError(st, "nitro_integersgd_step")
 
+    def set_hyper(self, gamma_inv_lr, eta_inv_fw=0, eta_inv_lr=0):
+        st = lib().nitro_block_set_hyper(self.h, int(gamma_inv_lr), int(eta_inv_fw),
+                                         int(eta_inv_lr))
+        if st != NITRO_OK:
+            raise NitroError(st, "nitro_block_set_hyper")
+
     def get(self, which, layer=0, check=True):
         """Host copy of a tensor as a flat numpy array (synchronises)."""
         st, n = nitro_block_tensor_bytes(self.h, which, layer)
@@ -333,6 +348,48 @@ class IntGemm:
     def close(self):
         if getattr(self, "h", None):
             lib().nitro_gemm_destroy(self.h)
+            self.h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+class IntPrep:
+    """Integer data pre-processing (App. A): fit mu / omega on a uint8 device
+    tensor, then map uint8 tensors to int8 x_hat with them."""
+
+    def __init__(self):
+        self.h = _VP()
+        st = lib().nitro_prep_create(ctypes.byref(self.h))
+        if st != NITRO_OK:
+            raise NitroError(st, "nitro_prep_create")
+
+    def fit(self, x, stream=None):
+        st = lib().nitro_prep_fit(self.h, _ptr(x), int(x.numel()), _stream_ptr(stream))
+        if st != NITRO_OK:
+            raise NitroError(st, "nitro_prep_fit")
+
+    def apply(self, x, out, stream=None):
+        if out.numel() != x.numel():
+            raise ValueError("out must have as many elements as x")
+        st = lib().nitro_prep_apply(self.h, _ptr(x), int(x.numel()), _ptr(out), _stream_ptr(stream))
+        if st != NITRO_OK:
+            raise NitroError(st, "nitro_prep_apply")
+        return out
+
+    def stats(self):
+        mu, om = ctypes.c_int64(), ctypes.c_int64()
+        st = lib().nitro_prep_stats(self.h, ctypes.byref(mu), ctypes.byref(om))
+        if st != NITRO_OK:
+            raise NitroError(st, "nitro_prep_stats")
+        return mu.value, om.value
+
+    def close(self):
+        if getattr(self, "h", None):
+            lib().nitro_prep_destroy(self.h)
             self.h = None
 
     def __del__(self):

@@ -392,6 +392,20 @@ nitro_status nitro_block_backward(nitro_block* b, const int8_t* a_in, const int3
     return NITRO_OK;
 }
 
+nitro_status nitro_block_set_hyper(nitro_block* b, int64_t gamma_inv_lr, int64_t eta_inv_fw,
+                                   int64_t eta_inv_lr) {
+    if (!b) return NITRO_ERR_ARG;
+    nitro_block_desc d = b->desc;
+    d.gamma_inv_lr = gamma_inv_lr;
+    d.eta_inv_fw = eta_inv_fw;
+    d.eta_inv_lr = eta_inv_lr;
+    if (d.gamma_inv_lr < 1 || d.gamma_inv_lr > ((int64_t)1 << 48) || d.eta_inv_fw < 0 ||
+        d.eta_inv_lr < 0)
+        return NITRO_ERR_ARG;
+    b->desc = d;
+    return NITRO_OK;
+}
+
 nitro_status nitro_integersgd_step(nitro_block* b, void* stream) {
     if (!b) return NITRO_ERR_ARG;
     cudaStream_t s = (cudaStream_t)stream;

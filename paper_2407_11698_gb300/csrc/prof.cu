@@ -40,7 +40,8 @@ const char* const kNames[K_COUNT] = {
     "simt_linear_dgrad", "simt_linear_wgrad", "fwd_epilogue", "learn_partial",
     "learn_dw", "grad_to_delta", "integersgd", "learn_finish_loss", "tc_conv_fwd",
     "tc_conv_wgrad", "tc_conv_dgrad", "tc_pack_limbs", "tc_finish", "tc_gemm", "lr_backward",
-    "tc_pack_weights", "tc_pack_input", "tc_pack_delta"};
+    "tc_pack_weights", "tc_pack_input", "tc_pack_delta", "prep_sum", "prep_mad",
+    "prep_apply"};
 
 }  // namespace
 

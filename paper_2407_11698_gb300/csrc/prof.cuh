@@ -34,6 +34,9 @@ enum KernelId : int {
     K_TC_PACK_W,
     K_TC_PACK_X,
     K_TC_PACK_D,
+    K_PREP_SUM,
+    K_PREP_MAD,
+    K_PREP_APPLY,
     K_COUNT
 };
 

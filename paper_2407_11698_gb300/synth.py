@@ -34,3 +34,26 @@ def gaussian_images(seed: int, step: int, batch: int, shape, sigma: float = 64.0
 def int_tensor(seed: int, shape, lo: int, hi: int, stream: int = 3, dtype=np.int64) -> np.ndarray:
     """Integer tensor uniform on [lo, hi] (inclusive), for kernel-level tests."""
     return _rng(seed, 0, stream).integers(lo, hi + 1, size=shape, dtype=dtype)
+
+
+def raw_pixels(seed: int, n: int, kind: str = "natural") -> np.ndarray:
+    """uint8 pixel values standing in for a raw 8-bit image dataset before
+    pre-processing (App. A), flattened to n values:
+      "natural"  round(N(120, 64^2)) clamped to [0, 255]: a broad, mid-grey
+                 centred spread like CIFAR-10 photographs;
+      "digits"   80% background zeros, the rest uniform on [1, 255]: mostly
+                 empty strokes on black like MNIST / FashionMNIST;
+      "uniform"  uniform on [0, 255];
+      "constant" every value 77 (mean absolute deviation 0)."""
+    r = _rng(seed, 0, 4)
+    if kind == "natural":
+        return np.clip(np.rint(r.normal(120.0, 64.0, size=n)), 0, 255).astype(np.uint8)
+    if kind == "digits":
+        x = r.integers(1, 256, size=n, dtype=np.int64)
+        x[r.random(n) < 0.8] = 0
+        return x.astype(np.uint8)
+    if kind == "uniform":
+        return r.integers(0, 256, size=n, dtype=np.uint8)
+    if kind == "constant":
+        return np.full(n, 77, dtype=np.uint8)
+    raise ValueError(kind)

@@ -90,10 +90,21 @@ def test_null_handle_calls_are_rejected(lib):
     assert nb.nitro_block_forward(None, None, 0, None) == nb.NITRO_ERR_ARG
     assert nb.nitro_block_backward(None, None, None, 0, None) == nb.NITRO_ERR_ARG
     assert nb.nitro_integersgd_step(None) == nb.NITRO_ERR_ARG
+    assert lib.nitro_block_set_hyper(None, 512, 0, 0) == nb.NITRO_ERR_ARG
     assert nb.nitro_block_status(None) == nb.NITRO_ERR_ARG
     nb.nitro_destroy_block(None)
     st, _ = nb.nitro_block_tensor_bytes(None, nb.NITRO_T_W, 0)
     assert st == nb.NITRO_ERR_ARG
+
+
+def test_prep_null_handle_and_bad_sizes_are_rejected(lib):
+    mu, om = ctypes.c_int64(), ctypes.c_int64()
+    x = ctypes.c_void_p(16)            # never dereferenced: the checks come first
+    assert lib.nitro_prep_fit(None, x, 10, None) == nb.NITRO_ERR_ARG
+    assert lib.nitro_prep_apply(None, x, 10, x, None) == nb.NITRO_ERR_ARG
+    assert lib.nitro_prep_stats(None, ctypes.byref(mu), ctypes.byref(om)) == nb.NITRO_ERR_ARG
+    assert lib.nitro_prep_create(None) == nb.NITRO_ERR_ARG
+    lib.nitro_prep_destroy(None)
 
 
 def test_oracle_library_builds_independently():

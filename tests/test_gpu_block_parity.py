@@ -99,6 +99,33 @@ def test_trunc_rounding_with_weight_decay_and_other_alpha():
     _run(blocks, 6, steps=3, input_shape=(8, 8, 2), eta_inv_fw=25000, eta_inv_lr=3000)
 
 
+def test_gamma_plateau_schedule_changes_updates_like_oracle():
+    """App. B schedule: gamma_inv x3 on a plateau, pushed through
+    nitro_block_set_hyper between steps; the oracle blocks take the same
+    values.  Weight decay switched on at the same time."""
+    from paper_2407_11698_gb300.schedule import GammaPlateau
+    blocks = [_b([(C, 2, 8, 8, 8, 1)], 8 * 8 * 2), _b([], 4 * 4 * 8)]
+    pair = NetPair(blocks, 6, seed=77)
+    sched = GammaPlateau(512, patience=1)
+    try:
+        for s in range(6):
+            x = synth.images(5, s, 6, (8, 8, 2))
+            y = synth.labels(5, s, 6)
+            gl, ol = pair.step(x, y)
+            assert gl == ol
+            pair.compare("step %d" % s)
+            if sched.step(0.5):                # a flat metric: every call past the first raises
+                sched.apply(pair.gb, eta_inv_fw=25000, eta_inv_lr=3000)
+                for o in pair.ob:
+                    o.gamma_inv_lr = sched.gamma_inv
+                    o.eta_inv_fw, o.eta_inv_lr = 25000, 3000
+        assert sched.gamma_inv == 512 * 3 ** 5
+        with pytest.raises(nb.NitroError):
+            pair.gb[0].set_hyper(0)
+    finally:
+        pair.close()
+
+
 def test_other_class_counts():
     blocks = [_b([(L, 16, 8, 1, 1, 0)], 16), _b([], 8)]
     _run(blocks, 9, steps=3, num_classes=3)

@@ -523,3 +523,63 @@ def test_synthetic_inputs_are_seeded():
     assert not np.array_equal(a, synth.images(1, 1, 4, (28, 28, 1)))
     lab = synth.labels(1, 0, 1000)
     assert lab.min() == 0 and lab.max() == 9
+
+
+# ------------------------------------------------------- pre-processing
+def test_prep_golden(golden):
+    for row in golden("preprocess.txt"):
+        n = row[0]
+        x, (mu, om), xh = row[1:1 + n], row[1 + n:3 + n], row[3 + n:]
+        assert O.prep_stats(x) == (mu, om)
+        assert O.prep_apply(np.array(x), mu, om).tolist() == xh
+
+
+def test_prep_shift_invariance():
+    """mu moves with a constant shift of the data, omega and x_hat do not."""
+    x = RNG.integers(0, 200, 20011)
+    mu, om = O.prep_stats(x)
+    mu2, om2 = O.prep_stats(x + 37)
+    assert (mu2, om2) == (mu + 37, om)
+    assert np.array_equal(O.prep_apply(x, mu, om), O.prep_apply(x + 37, mu2, om2))
+
+
+def test_prep_uniform_data_has_mad_51():
+    """Uniform bytes: omega ~ 64, no value reaches the clamp, and the mean
+    absolute value of x_hat is the 51 the rescaling multiplies by (App. A)."""
+    x = RNG.integers(0, 256, 1 << 20)
+    mu, om = O.prep_stats(x)
+    assert 126 <= mu <= 128 and 62 <= om <= 65
+    xh = O.prep_apply(x, mu, om).astype(np.int64)
+    assert np.abs(xh).max() < 127
+    assert abs(np.abs(xh).mean() - 51) < 1.0
+    assert abs(xh.mean()) < 1.0
+
+
+def test_prep_gaussian_data_meets_the_stated_target():
+    """App. A: the rescaling by 51 / omega (omega = mean absolute deviation,
+    ~0.8 sigma for Gaussian data) gives Gaussian data a standard deviation of
+    ~64, so ~95% of it lands in [-127, 127].  Checked on N(128.5, 30^2) bytes:
+    the realised scale 51 sd(x) / omega is within 5% of 64, and the mean and
+    standard deviation of x_hat equal those of the clipped normal that the
+    realised affine map (floor included) predicts."""
+    from scipy import integrate
+    from scipy.stats import norm
+    x = np.clip(np.rint(RNG.normal(128.5, 30.0, 1 << 20)), 0, 255)
+    mu, om = O.prep_stats(x)
+    assert abs(om - math.sqrt(2 / math.pi) * 30) <= 1.5
+    scale = 51 * x.std() / om
+    assert abs(scale / 64 - 1) < 0.05
+    shift = (x.mean() - mu) * 51 / om - 0.5          # floor lowers by 1/2 on average
+    sd = math.sqrt(scale ** 2 + 1 / 12)
+    clip = lambda y: min(max(y, -127.0), 127.0)
+    pdf = lambda y: norm.pdf(y, shift, sd)
+    m1 = integrate.quad(lambda y: clip(y) * pdf(y), shift - 10 * sd, shift + 10 * sd,
+                        points=[-127, 127], limit=200)[0]
+    m2 = integrate.quad(lambda y: clip(y) ** 2 * pdf(y), shift - 10 * sd, shift + 10 * sd,
+                        points=[-127, 127], limit=200)[0]
+    xh = O.prep_apply(x, mu, om).astype(np.float64)
+    assert abs(xh.mean() - m1) < 0.3
+    assert abs(xh.std() / math.sqrt(m2 - m1 ** 2) - 1) < 0.01
+    inside = norm.cdf(127, shift, sd) - norm.cdf(-127, shift, sd)
+    assert abs(inside - 0.95) < 0.02
+    assert abs((np.abs(xh) < 127).mean() - inside) < 0.01
