@@ -70,6 +70,12 @@ def lib():
     for name in ("nor_maxpool_fwd",):
         getattr(L, name).argtypes = [_I64] * 4 + [_P64, _P64, _P64]
     L.nor_maxpool_bwd.argtypes = [_I64] * 4 + [_P64, _P64, _P64]
+    L.nor_winpool_fwd.argtypes = [_I64] * 6 + [_P64, _P64, _P64]
+    L.nor_winpool_bwd.argtypes = [_I64] * 6 + [_P64, _P64, _P64]
+    L.nor_dropout_drop.argtypes = [ctypes.c_uint64] * 4 + [_I64]
+    L.nor_dropout_drop.restype = _I64
+    L.nor_dropout_mask.argtypes = [_I64, ctypes.c_uint64, ctypes.c_uint64, ctypes.c_uint64,
+                                   _I64, _P64]
     L.nor_integersgd.argtypes = [_I64, _P64, _P64, _I64, _I64, _I64]
     L.nor_prep_stats.argtypes = [_I64, ctypes.c_void_p, _P64, _P64]
     L.nor_prep_apply.argtypes = [_I64, ctypes.c_void_p, _I64, _I64, ctypes.c_void_p]
@@ -261,6 +267,64 @@ def maxpool_bwd(g_out, argmax, H, W):
     return g_in
 
 
+def winpool_fwd(a, kh, kw):
+    """kh x kw max-pool, stride (kh, kw), first maximum in row-major window
+    order; returns (pooled, argmax position r * kw + s)."""
+    a = _c(a)
+    B, H, W, C = a.shape
+    out = np.empty((B, H // kh, W // kw, C), dtype=np.int64)
+    am = np.empty_like(out)
+    lib().nor_winpool_fwd(B, H, W, C, int(kh), int(kw), _p(a), _p(out), _p(am))
+    return out, am
+
+
+def winpool_bwd(g_out, argmax, H, W, kh, kw):
+    g_out, argmax = _c(g_out), _c(argmax)
+    B, _, _, C = g_out.shape
+    g_in = np.empty((B, H, W, C), dtype=np.int64)
+    lib().nor_winpool_bwd(B, H, W, C, int(kh), int(kw), _p(g_out), _p(argmax), _p(g_in))
+    return g_in
+
+
+def dropout_drop(seed, step, layer, e, p16):
+    """1 if element e of forward layer ``layer`` is dropped at step ``step``."""
+    return lib().nor_dropout_drop(int(seed) & (2**64 - 1), int(step), int(layer), int(e),
+                                  int(p16))
+
+
+def dropout_mask(n, seed, step, layer, p16):
+    drop = np.empty(int(n), dtype=np.int64)
+    lib().nor_dropout_mask(int(n), int(seed) & (2**64 - 1), int(step), int(layer), int(p16),
+                           _p(drop))
+    return drop
+
+
+MAX_LR_WINDOW = 256     # positions of a learning-pool window (argmax kept in a byte)
+
+
+def lr_pool_window(C, H, W, d_lr):
+    """Window (kh, kw) of the learning-layer max-pool that brings a C x H x W
+    block output down to at most d_lr features (App. B's d^lr; Sec. 3.3 names
+    the pooled tensor z^mp).  Reading (the paper states no rule): starting
+    from 1 x 1, double the window height, then its width, alternately, while
+    C * floor(H / kh) * floor(W / kw) > d_lr and the window still fits the
+    map; a side that can no longer double leaves the other to grow.  d_lr = 0
+    means no pooling."""
+    kh = kw = 1
+    if d_lr <= 0:
+        return 1, 1
+    while C * (H // kh) * (W // kw) > d_lr:
+        if kh <= kw and 2 * kh <= H:
+            kh *= 2
+        elif 2 * kw <= W:
+            kw *= 2
+        elif 2 * kh <= H:
+            kh *= 2
+        else:
+            break
+    return kh, kw
+
+
 def integersgd(w, dw, gamma_inv, eta_inv, round_mode=FLOOR):
     """Algorithm 1 on a copy of ``w``; returns the int64 result (unchecked)."""
     w = _c(w).copy()
@@ -335,14 +399,23 @@ class LayerDesc:
 
 class OracleBlock:
     """One integer local-loss block (Sec. 3.2): forward layers, then a learning
-    layer (identity pool -> IntLinear(d -> G) -> NITRO-Scaling) trained on the
-    RSS loss against the scaled one-hot target.  A block with no forward layers
-    is the network's output block: its learning layer is the output layer."""
+    layer (max-pool to at most d_lr features, or identity -> IntLinear(d -> G)
+    -> NITRO-Scaling) trained on the RSS loss against the scaled one-hot
+    target.  A block with no forward layers is the network's output block: its
+    learning layer is the output layer.  dropout_p16 > 0 drops the outputs of
+    the block's linear forward layers during training (App. B's p_l, in units
+    of 2^-16); the mask of step t comes from the block's SplitMix64 stream,
+    and t counts the IntegerSGD steps the block has taken."""
 
     def __init__(self, layers, in_features=None, num_classes=10, alpha_inv=10,
                  gamma_inv_lr=512, eta_inv_fw=0, eta_inv_lr=0, sgd_round=FLOOR,
-                 seed=0, lr_post_update=False):
+                 seed=0, lr_post_update=False, d_lr=0, dropout_p16=0):
         self.layers = list(layers)
+        self.seed = int(seed)
+        self.dropout_p16 = int(dropout_p16)
+        if not 0 <= self.dropout_p16 <= 65536:
+            raise ValueError("dropout_p16 must lie in [0, 65536]")
+        self.t = 0
         self.G = int(num_classes)
         self.alpha_inv = int(alpha_inv)
         self.gamma_inv_lr = int(gamma_inv_lr)
@@ -361,9 +434,17 @@ class OracleBlock:
             if prev is not None and L.in_features != prev.out_features:
                 raise ValueError("layer input size does not match previous output")
             prev = L
+        # learning-layer pooling window over the block output (conv blocks)
+        self.lr_win = (1, 1)
         if self.layers:
             self.in_features = self.layers[0].in_features
-            self.d = self.layers[-1].out_features
+            last = self.layers[-1]
+            oh, ow = last.out_hw
+            self.lr_win = lr_pool_window(last.cout, oh, ow, int(d_lr))
+            kh, kw = self.lr_win
+            if kh * kw > MAX_LR_WINDOW:
+                raise ValueError("learning-pool window above %d positions" % MAX_LR_WINDOW)
+            self.d = last.cout * (oh // kh) * (ow // kw)
         else:
             if not in_features:
                 raise ValueError("an output block needs in_features")
@@ -401,6 +482,13 @@ class OracleBlock:
             else:
                 z = linear_fwd(x.reshape(B, L.cin), self.W[i])
             zs, reg, act = scale_relu(z, L.scaling_factor, self.alpha_inv)
+            if L.kind == LINEAR and self.dropout_p16:
+                # dropped outputs become 0 and carry region code 4, whose
+                # NITRO-ReLU backward passes nothing
+                drop = dropout_mask(act.size, self.seed, self.t, i,
+                                    self.dropout_p16).reshape(act.shape)
+                act = np.where(drop == 1, 0, act)
+                reg = np.where(drop == 1, 4, reg)
             self.zs.append(zs)
             self.region.append(reg)
             if L.pool:
@@ -418,8 +506,16 @@ class OracleBlock:
         """Learning-layer forward, loss, and every weight gradient of the block
         (Sec. 3.3 second phase).  Returns floor(SSE / 2)."""
         labels = np.asarray(labels, dtype=np.int64).reshape(-1)
+        self.lr_in, self.lr_argmax = None, None
         if self.layers:
             a = self.out
+            if self.lr_win != (1, 1):
+                # z^mp: the block output max-pooled for the learning layer
+                last = self.layers[-1]
+                oh, ow = last.out_hw
+                zmp, am = winpool_fwd(a.reshape(a.shape[0], oh, ow, last.cout), *self.lr_win)
+                a = zmp.reshape(a.shape[0], self.d)
+                self.lr_in, self.lr_argmax = a, am.reshape(a.shape[0], self.d)
         else:
             a = _c(a_in).reshape(labels.size, self.in_features)
             self.batch = a.shape[0]
@@ -455,6 +551,14 @@ class OracleBlock:
             self.status |= ST_OVERFLOW
         g, bad = store32(linear_dgrad(gl, wlr))
         self.status |= ST_OVERFLOW if bad else 0
+        if self.lr_in is not None:
+            # back through the learning-layer pooling to the block output
+            last = self.layers[-1]
+            oh, ow = last.out_hw
+            kh, kw = self.lr_win
+            g = winpool_bwd(g.reshape(B, oh // kh, ow // kw, last.cout),
+                            self.lr_argmax.reshape(B, oh // kh, ow // kw, last.cout),
+                            oh, ow, kh, kw).reshape(B, last.out_features)
         # down through the forward layers: pool backward, ReLU backward, STE
         # through NITRO-Scaling (Sec. 3.2.1), weight gradient, input gradient
         for i in reversed(range(len(self.layers))):
@@ -498,6 +602,7 @@ class OracleBlock:
                                        self.eta_inv_lr))
         self.Wlr = w.reshape(self.G, self.d)
         self.status |= ST_OVERFLOW if bad else 0
+        self.t += 1
 
 
 def train_step(blocks, x, labels):

@@ -310,6 +310,71 @@ void nor_maxpool_bwd(int64_t B, int64_t H, int64_t W, int64_t C,
 }
 
 /* ---------------------------------------------------------------------- */
+/* Learning-layer pooling (Sec. 3.3 training iteration: a block's output   */
+/* is downsampled by a pooling layer, z^mp, before its learning layers;    */
+/* App. B fixes the learning layers' input size d^lr).  A kh x kw max-pool */
+/* with stride (kh, kw); output floor(H/kh) x floor(W/kw).  The window is  */
+/* scanned row by row, the first maximum wins, and its position            */
+/* r * kw + s (row r, column s of the window) is recorded for backward.    */
+/* ---------------------------------------------------------------------- */
+void nor_winpool_fwd(int64_t B, int64_t H, int64_t W, int64_t C, int64_t kh, int64_t kw,
+                     const int64_t* a, int64_t* out, int64_t* argmax) {
+    int64_t Ho = H / kh, Wo = W / kw;
+    for (int64_t b = 0; b < B; ++b)
+        for (int64_t y = 0; y < Ho; ++y)
+            for (int64_t x = 0; x < Wo; ++x)
+                for (int64_t c = 0; c < C; ++c) {
+                    int64_t best = 0, bestv = 0;
+                    for (int64_t r = 0; r < kh; ++r)
+                        for (int64_t s = 0; s < kw; ++s) {
+                            int64_t v = a[((b * H + y * kh + r) * W + x * kw + s) * C + c];
+                            if ((r == 0 && s == 0) || v > bestv) { bestv = v; best = r * kw + s; }
+                        }
+                    out[((b * Ho + y) * Wo + x) * C + c] = bestv;
+                    argmax[((b * Ho + y) * Wo + x) * C + c] = best;
+                }
+}
+
+/* Backward of nor_winpool_fwd: each pooled gradient goes to the recorded  */
+/* window position; every other position, and the rows and columns the    */
+/* floor drops, get 0.                                                     */
+void nor_winpool_bwd(int64_t B, int64_t H, int64_t W, int64_t C, int64_t kh, int64_t kw,
+                     const int64_t* g_out, const int64_t* argmax, int64_t* g_in) {
+    int64_t Ho = H / kh, Wo = W / kw;
+    for (int64_t i = 0; i < B * H * W * C; ++i) g_in[i] = 0;
+    for (int64_t b = 0; b < B; ++b)
+        for (int64_t y = 0; y < Ho; ++y)
+            for (int64_t x = 0; x < Wo; ++x)
+                for (int64_t c = 0; c < C; ++c) {
+                    int64_t o = ((b * Ho + y) * Wo + x) * C + c;
+                    int64_t k = argmax[o];
+                    int64_t iy = y * kh + k / kw, ix = x * kw + k % kw;
+                    g_in[((b * H + iy) * W + ix) * C + c] = g_out[o];
+                }
+}
+
+/* ---------------------------------------------------------------------- */
+/* Dropout of the linear blocks (App. B, rate p_l).  The paper gives no    */
+/* integer form; the reading used: a dropped activation becomes 0 (the     */
+/* centre of the NITRO-ReLU output, which is shifted by mu) with no        */
+/* rescaling, and passes no gradient.  p is given in units of 2^-16        */
+/* (p16 in 0..65536).  Element e = b * out_features + j of forward layer   */
+/* `layer` at training step t is dropped when the top 16 bits of output    */
+/* 2^63 + t * 2^35 + layer * 2^31 + e of the block's SplitMix64 stream are */
+/* below p16 (t is taken modulo 2^28).                                     */
+/* ---------------------------------------------------------------------- */
+int64_t nor_dropout_drop(uint64_t seed, uint64_t step, uint64_t layer, uint64_t e, int64_t p16) {
+    uint64_t idx = (1ULL << 63) + ((step & ((1ULL << 28) - 1)) << 35) + (layer << 31) + e;
+    uint64_t u = nor_splitmix64_at(seed, idx);
+    return (int64_t)(u >> 48) < p16;
+}
+
+void nor_dropout_mask(int64_t n, uint64_t seed, uint64_t step, uint64_t layer, int64_t p16,
+                      int64_t* drop) {
+    for (int64_t e = 0; e < n; ++e) drop[e] = nor_dropout_drop(seed, step, layer, (uint64_t)e, p16);
+}
+
+/* ---------------------------------------------------------------------- */
 /* IntegerSGD, Algorithm 1.  For every weight:                             */
 /*   d = R(dw, gamma_inv);  if eta_inv != 0: d += R(w, eta_inv);  w -= d   */
 /* R is floor division (round_mode 0, the paper's notation) or truncation  */
