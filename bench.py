@@ -128,6 +128,24 @@ class ClockSampler:
                 "samples": len(sm)}
 
 
+# ------------------------------------------------------------------ ranks
+def max_over_ranks(ms, world, device):
+    """The slowest rank's time: every rank contributes its own `ms` and gets
+    back the maximum (a MAX all-reduce when world > 1)."""
+    import torch
+    t = torch.tensor([float(ms)], dtype=torch.float64, device=device)
+    if world > 1:
+        import torch.distributed as dist
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_rate(units_per_rank, world, steps, max_ms):
+    """Whole-job throughput: units processed by all ranks over `steps` steps
+    divided by the slowest rank's time (weak scaling: per-rank work fixed)."""
+    return world * units_per_rank * steps / (max_ms / 1e3)
+
+
 # ------------------------------------------------------------------ our step
 class GpuNet:
     """A chain of block handles driven through the public calls.  With
@@ -139,7 +157,8 @@ class GpuNet:
         self.torch, self.nb = torch, nb
         B = wl["batch"]
         self.B = B
-        self.blocks = [nb.Block(b["layers"], b["in_features"], seed=seed + i, max_batch=B)
+        self.blocks = [nb.Block(b["layers"], b["in_features"], seed=seed + i, max_batch=B,
+                                **wl.get("hyper", {}))
                        for i, b in enumerate(wl["blocks"])]
         from paper_2407_11698_gb300 import synth
         x = synth.images(seed, 0, B, wl["input_shape"]).reshape(B, -1)
@@ -320,12 +339,8 @@ def run_ours(args, rank, world, local_rank):
     if world > 1:
         dist.barrier()
     step_ms = [a.elapsed_time(b) for a, b in ev]
-    total_ms = sum(step_ms)
-    t = torch.tensor([total_ms], dtype=torch.float64, device="cuda")
-    if world > 1:
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-    total_ms = float(t.item())
-    value = world * net.B * args.steps / (total_ms / 1e3)
+    total_ms = max_over_ranks(sum(step_ms), world, "cuda")
+    value = job_rate(net.B, world, args.steps, total_ms)
 
     # ---------------- end to end through the public API, host buffers
     from paper_2407_11698_gb300 import synth
@@ -345,11 +360,8 @@ def run_ours(args, rank, world, local_rank):
         lh.copy_(net.loss, non_blocking=True)
     e1.record(stream)
     torch.cuda.synchronize()
-    e2e_ms = e0.elapsed_time(e1)
-    t = torch.tensor([e2e_ms], dtype=torch.float64, device="cuda")
-    if world > 1:
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-    e2e_value = world * net.B * args.steps / (float(t.item()) / 1e3)
+    e2e_value = job_rate(net.B, world, args.steps,
+                         max_over_ranks(e0.elapsed_time(e1), world, "cuda"))
 
     # ---------------- per-kernel device time inside eager steps (roofline); the
     # blocks run one after another here so that no kernel shares the GPU
@@ -440,7 +452,8 @@ def oracle_rate(wl_name, sample_batch, steps, warmup=0):
     from paper_2407_11698_gb300 import workloads as WL
     wl = WL.WORKLOADS[wl_name]
     blocks = [O.OracleBlock([O.LayerDesc(*l) for l in b["layers"]], in_features=b["in_features"],
-                            seed=20240716 + i) for i, b in enumerate(wl["blocks"])]
+                            seed=20240716 + i, **wl.get("hyper", {}))
+              for i, b in enumerate(wl["blocks"])]
     for s in range(warmup + steps):
         if s == warmup:
             t0 = time.perf_counter()

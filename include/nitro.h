@@ -91,7 +91,36 @@ typedef struct {
     int64_t eta_inv_fw, eta_inv_lr;  /* weight-decay thresholds, 0 = off     */
     int sgd_round;                   /* nitro_round for IntegerSGD           */
     int max_batch;                   /* workspace is sized for this          */
+    int d_lr;                        /* learning-layer input size d^lr; 0 =
+                                        no learning-layer pooling            */
+    int dropout_p16;                 /* dropout rate of the linear forward
+                                        layers, in units of 2^-16 (0..65536) */
 } nitro_block_desc;
+
+/* Learning-layer pooling (Sec. 3.3: the block output is downsampled by a
+ * pooling layer to z^mp before the learning layers; App. B: d^lr input
+ * features).  When d_lr > 0 and the last forward layer's output C x H' x W'
+ * holds more than d_lr values, the learning layer reads a kh x kw max-pool
+ * of it (stride (kh, kw), output floor(H'/kh) x floor(W'/kw) x C, first
+ * maximum in row-major window order, position r*kw + s recorded).  The paper
+ * states no rule for the window; this library takes: from 1 x 1, double kh,
+ * then kw, alternately, while C*floor(H'/kh)*floor(W'/kw) > d_lr and the
+ * window fits the map (a side that cannot double leaves the other to grow).
+ * The learning layer then has d = C*floor(H'/kh)*floor(W'/kw) inputs (its
+ * fan-in for the initialisation).  Windows above 256 positions return
+ * NITRO_ERR_UNSUPPORTED.  Linear outputs (1 x 1) and output blocks never
+ * pool.
+ *
+ * Dropout (App. B, rate p_l of the linear blocks).  With dropout_p16 > 0,
+ * every nitro_block_forward drops outputs of the block's linear forward
+ * layers: a dropped activation is stored as 0, its NITRO-ReLU region code
+ * becomes 4, and it passes no gradient.  The paper gives no integer form of
+ * dropout; no rescaling is applied.  Element e = b*out_features + j of forward
+ * layer l is dropped at step t when the top 16 bits of output
+ * 2^63 + t*2^35 + l*2^31 + e of SplitMix64 seeded with the block's seed are
+ * below dropout_p16.  t is the block's step counter (NITRO_T_STEP): the
+ * number of nitro_integersgd_step calls so far, modulo 2^28.  Set the rate
+ * to 0 (nitro_block_set_dropout) for inference. */
 
 typedef struct nitro_block nitro_block;
 
@@ -145,6 +174,13 @@ nitro_status nitro_integersgd_step(nitro_block* blk, void* stream);
 nitro_status nitro_block_set_hyper(nitro_block* blk, int64_t gamma_inv_lr, int64_t eta_inv_fw,
                                    int64_t eta_inv_lr);
 
+/* Replaces the dropout rate of the block's linear forward layers (0..65536,
+ * units of 2^-16; 0 = off, e.g. for inference).  Host-only: it takes effect
+ * at the next nitro_block_forward call; a CUDA graph that captured an earlier
+ * forward keeps the rate it was captured with.  NITRO_ERR_ARG if out of
+ * range (nothing changes). */
+nitro_status nitro_block_set_dropout(nitro_block* blk, int dropout_p16);
+
 /* Tensors readable / writable through get/set_tensor.  Batch-shaped tensors
  * hold the last forward/backward batch. */
 typedef enum {
@@ -153,11 +189,18 @@ typedef enum {
     NITRO_T_WLR = 2,     /* learning/output weights [G x d], int32 (layer = 0) */
     NITRO_T_DWLR = 3,    /* learning weight gradient, int64 (layer = 0)        */
     NITRO_T_ACT = 4,     /* layer output after pool, int8 [batch x out]        */
-    NITRO_T_REGION = 5,  /* NITRO-ReLU piece 0..3 per pre-pool output, int8    */
+    NITRO_T_REGION = 5,  /* NITRO-ReLU piece 0..3 per pre-pool output, int8;
+                            4 = dropped by dropout                             */
     NITRO_T_ARGMAX = 6,  /* max-pool window position 0..3 per output, int8     */
     NITRO_T_DELTA = 7,   /* gradient at the layer's pre-activation, int32      */
     NITRO_T_GRAD_L = 8,  /* loss gradient [batch x G], int32 (layer = 0)       */
-    NITRO_T_SSE = 9      /* sum of squared errors, int64 [1] (layer = 0)       */
+    NITRO_T_SSE = 9,     /* sum of squared errors, int64 [1] (layer = 0)       */
+    NITRO_T_LR_IN = 10,  /* pooled learning-layer input z^mp [batch x d], int8
+                            (layer = 0; blocks with learning-layer pooling)    */
+    NITRO_T_LR_ARGMAX = 11, /* window position r*kw + s of each z^mp value,
+                            uint8 [batch x d] (same blocks)                    */
+    NITRO_T_STEP = 12    /* step counter of the dropout masks, uint32 [1]
+                            (layer = 0); writable, for resuming                */
 } nitro_tensor;
 
 /* Size in bytes of tensor (which, layer) at the current batch. */
@@ -171,8 +214,9 @@ nitro_status nitro_block_get_tensor(nitro_block* blk, int which, int layer, void
                                     size_t bytes);
 
 /* Synchronises the device and overwrites a weight tensor (NITRO_T_W,
- * NITRO_T_DW, NITRO_T_WLR, NITRO_T_DWLR) from host memory; used to resume
- * from a checkpoint.  Bit-exact: all state is integer. */
+ * NITRO_T_DW, NITRO_T_WLR, NITRO_T_DWLR) or the step counter (NITRO_T_STEP)
+ * from host memory; used to resume from a checkpoint.  Bit-exact: all state
+ * is integer. */
 nitro_status nitro_block_set_tensor(nitro_block* blk, int which, int layer,
                                     const void* host_src, size_t bytes);
 

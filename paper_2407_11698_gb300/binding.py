@@ -20,12 +20,14 @@ NITRO_ROUND_FLOOR, NITRO_ROUND_TRUNC = 0, 1
 STATUS_BIT_OVERFLOW, STATUS_BIT_BAD_LABEL, STATUS_BIT_TIMEOUT = 1, 2, 4
 NITRO_CONTRACT_FWD, NITRO_CONTRACT_WGRAD, NITRO_CONTRACT_DGRAD = 0, 1, 2
 (NITRO_T_W, NITRO_T_DW, NITRO_T_WLR, NITRO_T_DWLR, NITRO_T_ACT, NITRO_T_REGION,
- NITRO_T_ARGMAX, NITRO_T_DELTA, NITRO_T_GRAD_L, NITRO_T_SSE) = range(10)
+ NITRO_T_ARGMAX, NITRO_T_DELTA, NITRO_T_GRAD_L, NITRO_T_SSE, NITRO_T_LR_IN, NITRO_T_LR_ARGMAX,
+ NITRO_T_STEP) = range(13)
 
 TENSOR_DTYPE = {
     NITRO_T_W: np.int32, NITRO_T_DW: np.int64, NITRO_T_WLR: np.int32, NITRO_T_DWLR: np.int64,
     NITRO_T_ACT: np.int8, NITRO_T_REGION: np.int8, NITRO_T_ARGMAX: np.int8,
     NITRO_T_DELTA: np.int32, NITRO_T_GRAD_L: np.int32, NITRO_T_SSE: np.int64,
+    NITRO_T_LR_IN: np.int8, NITRO_T_LR_ARGMAX: np.uint8, NITRO_T_STEP: np.uint32,
 }
 
 
@@ -39,7 +41,8 @@ class nitro_block_desc(ctypes.Structure):
                 ("in_features", ctypes.c_int), ("num_classes", ctypes.c_int),
                 ("alpha_inv", ctypes.c_int), ("gamma_inv_lr", ctypes.c_int64),
                 ("eta_inv_fw", ctypes.c_int64), ("eta_inv_lr", ctypes.c_int64),
-                ("sgd_round", ctypes.c_int), ("max_batch", ctypes.c_int)]
+                ("sgd_round", ctypes.c_int), ("max_batch", ctypes.c_int),
+                ("d_lr", ctypes.c_int), ("dropout_p16", ctypes.c_int)]
 
 
 class NitroError(RuntimeError):
@@ -108,6 +111,8 @@ def lib():
     L.nitro_gemm_destroy.restype = None
     L.nitro_block_set_hyper.argtypes = [_VP, ctypes.c_int64, ctypes.c_int64, ctypes.c_int64]
     L.nitro_block_set_hyper.restype = ctypes.c_int
+    L.nitro_block_set_dropout.argtypes = [_VP, ctypes.c_int]
+    L.nitro_block_set_dropout.restype = ctypes.c_int
     L.nitro_prep_create.argtypes = [ctypes.POINTER(_VP)]
     L.nitro_prep_fit.argtypes = [_VP, _VP, ctypes.c_int64, _VP]
     L.nitro_prep_apply.argtypes = [_VP, _VP, ctypes.c_int64, _VP, _VP]
@@ -188,7 +193,8 @@ def nitro_destroy_block(blk):
 
 # ---------------------------------------------------------------- helpers
 def make_block_desc(layers, in_features, num_classes=10, alpha_inv=10, gamma_inv_lr=512,
-                    eta_inv_fw=0, eta_inv_lr=0, sgd_round=NITRO_ROUND_FLOOR, max_batch=1):
+                    eta_inv_fw=0, eta_inv_lr=0, sgd_round=NITRO_ROUND_FLOOR, max_batch=1,
+                    d_lr=0, dropout_p16=0):
     """Build a ``nitro_block_desc`` from layer tuples (kind, cin, cout, h, w, pool).
     Returns (desc, keepalive) - keep the second value alive while desc is used."""
     arr = (nitro_layer_desc * max(1, len(layers)))()
@@ -196,7 +202,7 @@ def make_block_desc(layers, in_features, num_classes=10, alpha_inv=10, gamma_inv
         arr[i] = nitro_layer_desc(*[int(v) for v in l])
     d = nitro_block_desc(len(layers), arr if layers else None, int(in_features), int(num_classes),
                          int(alpha_inv), int(gamma_inv_lr), int(eta_inv_fw), int(eta_inv_lr),
-                         int(sgd_round), int(max_batch))
+                         int(sgd_round), int(max_batch), int(d_lr), int(dropout_p16))
     return d, arr
 
 
@@ -254,6 +260,11 @@ class Block:
                                          int(eta_inv_lr))
         if st != NITRO_OK:
             raise NitroError(st, "nitro_block_set_hyper")
+
+    def set_dropout(self, dropout_p16):
+        st = lib().nitro_block_set_dropout(self.h, int(dropout_p16))
+        if st != NITRO_OK:
+            raise NitroError(st, "nitro_block_set_dropout")
 
     def get(self, which, layer=0, check=True):
         """Host copy of a tensor as a flat numpy array (synchronises)."""

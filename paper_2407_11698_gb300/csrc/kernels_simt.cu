@@ -139,15 +139,22 @@ __global__ void __launch_bounds__(256) k_gemm(GemmParams p) {
 __global__ void k_fwd_epilogue(const int64_t* __restrict__ z, LayerGeom g, int B,
                                int alpha_inv, int mu, int64_t kdiv, int8_t* __restrict__ out,
                                int8_t* __restrict__ out2, int8_t* __restrict__ region,
-                               int8_t* __restrict__ argmax) {
+                               int8_t* __restrict__ argmax, DropoutArgs drop) {
     const int C = g.cout;
     if (!g.pool) {
+        // dropout (linear layers): element i = b * out_features + j of this step's mask
+        const uint32_t t = drop.p16 ? *drop.step : 0u;
         const int64_t n = (int64_t)B * g.h * g.w * C;
         for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
              i += (int64_t)gridDim.x * blockDim.x) {
             const int64_t zs = scale_floor(z[i], kdiv);
-            region[i] = (int8_t)relu_region(zs);
-            const int8_t v = (int8_t)relu_value(zs, alpha_inv, mu);
+            int rg = relu_region(zs);
+            int8_t v = (int8_t)relu_value(zs, alpha_inv, mu);
+            if (drop.p16 && dropout_drop(drop.seed, t, drop.layer, (uint64_t)i, drop.p16)) {
+                rg = kRegionDropped;
+                v = 0;
+            }
+            region[i] = (int8_t)rg;
             out[i] = v;
             if (out2) out2[i] = v;
         }
@@ -366,6 +373,104 @@ __global__ void k_grad_to_delta(DeltaSrc src, LayerGeom g, int B, int alpha_inv,
 }
 
 // ---------------------------------------------------------------------------
+// Learning-layer max-pool (Sec. 3.3, z^mp; window from d^lr, App. B): one
+// thread per pooled element, channel fastest, so a warp reads 32 consecutive
+// channels of each window row.  First maximum in row-major window order.
+// ---------------------------------------------------------------------------
+__global__ void k_lr_pool_fwd(const int8_t* __restrict__ a, int B, int H, int W, int C, int kh,
+                              int kw, int ph, int pw, int8_t* __restrict__ out,
+                              uint8_t* __restrict__ am) {
+    const int64_t n = (int64_t)B * ph * pw * C;
+    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        const int c = (int)(i % C);
+        int64_t r = i / C;
+        const int x = (int)(r % pw);
+        r /= pw;
+        const int y = (int)(r % ph);
+        const int64_t b = r / ph;
+        const int8_t* p = a + ((b * H + (int64_t)y * kh) * W + (int64_t)x * kw) * C + c;
+        int best = 0, bestv = p[0];
+        for (int u = 0; u < kh; ++u)
+            for (int v = 0; v < kw; ++v) {
+                const int val = p[((int64_t)u * W + v) * C];
+                if (val > bestv) { bestv = val; best = u * kw + v; }
+            }
+        out[i] = (int8_t)bestv;
+        am[i] = (uint8_t)best;
+    }
+}
+
+// ---------------------------------------------------------------------------
+// Learning-layer backward through the pool, into the last layer's delta.  One
+// thread per pre-pool element (b, y, x, c) of that conv layer: it receives a
+// gradient only if it won its 2x2 window (when the layer pools) and the
+// pooled position won its learning-pool window; that thread alone forms
+// delta_fw = sum_g grad_L[b][g] W_lr[g][f] of the learning feature f (modulo
+// 2^64, int32 storage rule) and applies NITRO-ReLU backward.  Every element is
+// written, so no clearing pass is needed.
+// ---------------------------------------------------------------------------
+__global__ void k_lrpool_to_delta(const int32_t* __restrict__ gl, const int32_t* __restrict__ wlr,
+                                  int G, int d, LayerGeom g, LrPoolGeom lp, int B,
+                                  const uint8_t* __restrict__ lam,
+                                  const int8_t* __restrict__ argmax,
+                                  const int8_t* __restrict__ region, FloorDiv32 alpha,
+                                  int32_t* __restrict__ delta, const uint32_t* maxabs_gl,
+                                  const uint32_t* maxabs_wlr, uint32_t* maxabs_delta,
+                                  uint32_t* status) {
+    const int C = g.cout;
+    const int64_t n = (int64_t)B * g.h * g.w * C;
+    if (blockIdx.x == 0 && threadIdx.x == 0 && int64_bound_exceeded(*maxabs_gl, *maxabs_wlr, G))
+        atomicOr(status, ST_OVERFLOW);
+    uint32_t mx = 0;
+    bool ovf = false;
+    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        const int c = (int)(i % C);
+        int64_t r = i / C;
+        const int x = (int)(r % g.w);
+        r /= g.w;
+        const int y = (int)(r % g.h);
+        const int64_t b = r / g.h;
+        int qy = y, qx = x;
+        bool hit = true;
+        if (g.pool) {
+            qy = y >> 1;
+            qx = x >> 1;
+            hit = qy < g.oh && qx < g.ow &&
+                  argmax[((b * g.oh + qy) * g.ow + qx) * C + c] == (((y & 1) << 1) | (x & 1));
+        }
+        int32_t dv = 0;
+        if (hit) {
+            const int wy = qy / lp.kh, wx = qx / lp.kw;
+            hit = wy < lp.ph && wx < lp.pw &&
+                  lam[((b * lp.ph + wy) * lp.pw + wx) * C + c] ==
+                      (qy - wy * lp.kh) * lp.kw + (qx - wx * lp.kw);
+            if (hit) {
+                const int64_t f = ((int64_t)wy * lp.pw + wx) * C + c;
+                uint64_t acc = 0;   // modulo 2^64, exact below the bound
+                for (int k = 0; k < G; ++k)
+                    acc += (uint64_t)((int64_t)gl[b * G + k] * wlr[(int64_t)k * d + f]);
+                const int64_t gv = (int64_t)acc;
+                ovf |= !fits_i32(gv);
+                const int32_t gs = (int32_t)gv;
+                const int rg = region[i];
+                dv = rg == 1 ? alpha.floor_div(gs) : (rg == 2 ? gs : 0);
+            }
+        }
+        delta[i] = dv;
+        mx = max(mx, abs_u32(dv));
+    }
+#pragma unroll
+    for (int off = 16; off; off >>= 1) mx = max(mx, __shfl_xor_sync(kFull, mx, off));
+    ovf = __any_sync(kFull, ovf);
+    if ((threadIdx.x & 31) == 0) {
+        if (mx) atomicMax(maxabs_delta, mx);
+        if (ovf) atomicOr(status, ST_OVERFLOW);
+    }
+}
+
+// ---------------------------------------------------------------------------
 // IntegerSGD (Algorithm 1); blockIdx.y selects the tensor.
 // ---------------------------------------------------------------------------
 __device__ __forceinline__ int32_t sgd_one(const SgdTensor& t, int round_trunc, int32_t w32,
@@ -441,6 +546,8 @@ __global__ void k_integersgd(SgdBatch bt) {
         if (mx) atomicMax(t.maxabs_w, mx);
         if (ovf) atomicOr(bt.status, ST_OVERFLOW);
     }
+    // one block step taken: advance the dropout step counter
+    if (bt.step && blockIdx.x == 0 && blockIdx.y == 0 && threadIdx.x == 0) *bt.step += 1u;
 }
 
 // ---------------------------------------------------------------------------
@@ -781,14 +888,52 @@ cudaError_t simt_gemm(int mode, const int8_t* act, const int32_t* grad, const in
 
 cudaError_t simt_fwd_epilogue(const int64_t* z, const LayerGeom& g, int B, int alpha_inv,
                               int mu, int8_t* out, int8_t* out2, int8_t* region,
-                              int8_t* argmax, cudaStream_t s) {
+                              int8_t* argmax, cudaStream_t s, const DropoutArgs* drop) {
     if (B <= 0) return cudaSuccess;
     const int64_t kdiv = g.kind == NITRO_CONV3X3 ? 9LL * g.cin : (int64_t)g.cin;
     const int64_t n = g.pool ? (int64_t)B * ((g.h + 1) / 2) * ((g.w + 1) / 2) * g.cout
                              : (int64_t)B * g.h * g.w * g.cout;
+    DropoutArgs da{};
+    if (drop && drop->p16) {
+        if (g.pool || !drop->step) return cudaErrorInvalidValue;
+        da = *drop;
+    }
     ProfScope ps(K_FWD_EPILOGUE, s, 0.0, 0.0);
     k_fwd_epilogue<<<grid_for(n, 256), 256, 0, s>>>(z, g, B, alpha_inv, mu, kdiv, out, out2,
-                                                    region, argmax);
+                                                    region, argmax, da);
+    return cudaGetLastError();
+}
+
+cudaError_t simt_lr_pool_fwd(const int8_t* a, int B, int H, int W, int C, int kh, int kw,
+                             int ph, int pw, int8_t* out, uint8_t* am, cudaStream_t s) {
+    const int64_t n = (int64_t)B * ph * pw * C;
+    if (n <= 0) return cudaSuccess;
+    if (kh < 1 || kw < 1 || ph * kh > H || pw * kw > W || kh * kw > 256) return cudaErrorInvalidValue;
+    ProfScope ps(K_LR_POOL, s, 0.0, (double)B * H * W * C + 2.0 * n);
+    k_lr_pool_fwd<<<grid_for(n, 256), 256, 0, s>>>(a, B, H, W, C, kh, kw, ph, pw, out, am);
+    return cudaGetLastError();
+}
+
+cudaError_t simt_lrpool_to_delta(const int32_t* gl, const int32_t* wlr, int G, int d,
+                                 const LayerGeom& g, const LrPoolGeom& lp, int B,
+                                 const uint8_t* am, const int8_t* argmax, const int8_t* region,
+                                 int alpha_inv, int32_t* delta, const uint32_t* maxabs_gl,
+                                 const uint32_t* maxabs_wlr, uint32_t* maxabs_delta,
+                                 uint32_t* status, cudaStream_t s) {
+    const int64_t n = (int64_t)B * g.h * g.w * g.cout;
+    if (n <= 0) return cudaSuccess;
+    if (g.kind != NITRO_CONV3X3 || lp.ph * lp.kh > g.oh || lp.pw * lp.kw > g.ow ||
+        (int64_t)lp.ph * lp.pw * g.cout != d || alpha_inv < 1)
+        return cudaErrorInvalidValue;
+    // bytes: region (1) and delta (4) per element, the two argmax codes per
+    // pooled position, grad_L and the columns of W_lr read
+    ProfScope ps(K_LRPOOL_TO_DELTA, s, 2.0 * B * d * G,
+                 5.0 * n + (double)B * g.oh * g.ow * g.cout * (g.pool ? 1 : 0) + (double)B * d +
+                     4.0 * G * (B + (double)d));
+    k_lrpool_to_delta<<<grid_for(n, 256), 256, 0, s>>>(
+        gl, wlr, G, d, g, lp, B, am, argmax, region,
+        FloorDiv32::make((uint32_t)alpha_inv), delta, maxabs_gl, maxabs_wlr, maxabs_delta,
+        status);
     return cudaGetLastError();
 }
 

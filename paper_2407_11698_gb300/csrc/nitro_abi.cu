@@ -46,6 +46,11 @@ struct nitro_block {
     size_t z64_elems = 0;
     uint32_t* words = nullptr;      // [0] status [1] max|grad_l| [2] max|W_lr|
                                     // [3 + i] max|W_i|  [3 + n + i] max|delta_i|
+                                    // [3 + 2n] step counter (dropout masks)
+    uint64_t seed = 0;
+    LrPoolGeom lp{1, 1, 0, 0};      // learning-layer pool window and output grid
+    int8_t* zmp = nullptr;          // [max_batch x d] pooled learning input, or null
+    uint8_t* lr_am = nullptr;       // [max_batch x d] its window positions
     unsigned long long* sse = nullptr;
     int batch = 0;
     std::vector<void*> allocs;
@@ -59,7 +64,8 @@ uint32_t* w_gl(nitro_block* b) { return b->words + 1; }
 uint32_t* w_wlr(nitro_block* b) { return b->words + 2; }
 uint32_t* w_w(nitro_block* b, int i) { return b->words + 3 + i; }
 uint32_t* w_delta(nitro_block* b, int i) { return b->words + 3 + (int)b->L.size() + i; }
-int n_words(int n_layers) { return 3 + 2 * n_layers; }
+uint32_t* w_step(nitro_block* b) { return b->words + 3 + 2 * (int)b->L.size(); }
+int n_words(int n_layers) { return 4 + 2 * n_layers; }
 
 template <typename T>
 bool dalloc(nitro_block* b, T** p, size_t count) {
@@ -76,13 +82,6 @@ void free_all(nitro_block* b) {
     for (void* p : b->host_allocs) cudaFreeHost(p);
     b->allocs.clear();
     b->host_allocs.clear();
-}
-
-uint64_t splitmix64_at(uint64_t seed, uint64_t index) {
-    uint64_t z = seed + (index + 1ULL) * 0x9E3779B97F4A7C15ULL;
-    z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ULL;
-    z = (z ^ (z >> 27)) * 0x94D049BB133111EBULL;
-    return z ^ (z >> 31);
 }
 
 int64_t isqrt64(int64_t n) {
@@ -104,6 +103,24 @@ std::vector<int32_t> draw_weights(int64_t n, int64_t fan_in, uint64_t seed, uint
     for (int64_t e = 0; e < n; ++e)
         w[(size_t)e] = (int32_t)((int64_t)(splitmix64_at(seed, (tensor_id << 40) + (uint64_t)e) % span) - b);
     return w;
+}
+
+// Learning-layer pooling window (Sec. 3.3 z^mp, App. B d^lr): grow a 1 x 1
+// window by doubling its height, then its width, alternately, while the
+// pooled C x floor(H/kh) x floor(W/kw) map holds more than d_lr values and
+// the window still fits; a side that cannot double leaves the other to grow.
+void lr_window(int64_t C, int H, int W, int d_lr, int* kh_out, int* kw_out) {
+    int kh = 1, kw = 1;
+    if (d_lr > 0) {
+        while (C * (H / kh) * (W / kw) > d_lr) {
+            if (kh <= kw && 2 * kh <= H) kh *= 2;
+            else if (2 * kw <= W) kw *= 2;
+            else if (2 * kh <= H) kh *= 2;
+            else break;
+        }
+    }
+    *kh_out = kh;
+    *kw_out = kw;
 }
 
 uint32_t host_maxabs(const int32_t* p, size_t n) {
@@ -130,6 +147,7 @@ nitro_status validate(const nitro_block_desc* d) {
     if (d->sgd_round != NITRO_ROUND_FLOOR && d->sgd_round != NITRO_ROUND_TRUNC) return NITRO_ERR_ARG;
     if (d->max_batch < 0 || d->max_batch > 1000000) return NITRO_ERR_ARG;
     if (d->in_features < 1 || d->in_features > (1 << 24)) return NITRO_ERR_ARG;
+    if (d->d_lr < 0 || d->dropout_p16 < 0 || d->dropout_p16 > 65536) return NITRO_ERR_ARG;
     int64_t prev_out = d->in_features;
     for (int i = 0; i < d->n_layers; ++i) {
         const nitro_layer_desc& l = d->layers[i];
@@ -157,6 +175,14 @@ nitro_status validate(const nitro_block_desc* d) {
         prev_out = out_f;
     }
     if ((int64_t)d->max_batch * prev_out >= ((int64_t)1 << 31)) return NITRO_ERR_ARG;
+    if (d->n_layers > 0) {
+        const nitro_layer_desc& l = d->layers[d->n_layers - 1];
+        if (l.kind == NITRO_CONV3X3) {
+            int kh, kw;
+            lr_window(l.cout, l.pool2x2 ? l.h / 2 : l.h, l.pool2x2 ? l.w / 2 : l.w, d->d_lr, &kh, &kw);
+            if (kh * kw > 256) return NITRO_ERR_UNSUPPORTED;
+        }
+    }
     return NITRO_OK;
 }
 
@@ -219,7 +245,18 @@ nitro_status nitro_init_block(const nitro_block_desc* desc, uint64_t seed, void*
         host_w.push_back(draw_weights(ly.wcount, fan_in, seed, (uint64_t)i));
         b->L.push_back(ly);
     }
+    b->seed = seed;
     b->d = desc->n_layers ? b->L.back().out_f : desc->in_features;
+    if (desc->n_layers && b->L.back().g.kind == NITRO_CONV3X3) {
+        const LayerGeom& lg = b->L.back().g;
+        int kh, kw;
+        lr_window(lg.cout, lg.oh, lg.ow, desc->d_lr, &kh, &kw);
+        if (kh * kw > 1) {
+            b->lp = LrPoolGeom{kh, kw, lg.oh / kh, lg.ow / kw};
+            b->d = (int64_t)b->lp.ph * b->lp.pw * lg.cout;
+            ok = ok && dalloc(b, &b->zmp, (size_t)MB * b->d) && dalloc(b, &b->lr_am, (size_t)MB * b->d);
+        }
+    }
     ok = ok && dalloc(b, &b->Wlr, (size_t)b->G * b->d) && dalloc(b, &b->dWlr, (size_t)b->G * b->d) &&
          dalloc(b, &b->grad_l, (size_t)MB * b->G) && dalloc(b, &b->zsum, (size_t)MB * b->G + (MB + 15) / 16 + 1) && dalloc(b, &b->z64, z_need) &&
          dalloc(b, &b->words, n_words(desc->n_layers)) && dalloc(b, &b->sse, 1);
@@ -299,9 +336,13 @@ nitro_status nitro_block_forward(nitro_block* b, const int8_t* a_in, int batch, 
             const int mode = g.kind == NITRO_CONV3X3 ? GM_CONV_FWD : GM_LIN_FWD;
             NITRO_TRY(simt_gemm(mode, x, nullptr, ly.W, b->z64, batch, g.h, g.w, g.cin, g.cout, s));
         }
-        if (!fused)
+        if (!fused) {
+            // dropout of the linear layers (App. B, p_l)
+            DropoutArgs da{b->seed, (uint32_t)b->desc.dropout_p16, i, w_step(b)};
+            const bool drop = g.kind == NITRO_LINEAR && b->desc.dropout_p16 > 0;
             NITRO_TRY(simt_fwd_epilogue(b->z64, g, batch, b->desc.alpha_inv, b->mu, ly.act, out2,
-                                        ly.region, ly.argmax, s));
+                                        ly.region, ly.argmax, s, drop ? &da : nullptr));
+        }
         nhwc_done = fused && next_nhwc != nullptr;
         x = ly.act;
     }
@@ -330,9 +371,29 @@ nitro_status nitro_block_backward(nitro_block* b, const int8_t* a_in, const int3
         return NITRO_OK;
     }
     const int8_t* a_last = n ? b->L[n - 1].act : a_in;
+    if (b->zmp) {
+        // z^mp: the block output max-pooled for the learning layer (Sec. 3.3)
+        const LayerGeom& lg = b->L[n - 1].g;
+        NITRO_TRY(simt_lr_pool_fwd(a_last, batch, lg.oh, lg.ow, lg.cout, b->lp.kh, b->lp.kw,
+                                   b->lp.ph, b->lp.pw, b->zmp, b->lr_am, s));
+        a_last = b->zmp;
+    }
     NITRO_TRY(simt_learn_fwd(a_last, b->Wlr, labels, batch, (int)d, G, b->zsum, b->grad_l, b->sse,
                              loss_dev, w_gl(b), w_status(b), s));
-    if (simt_lr_backward_ok(G)) {
+    if (b->zmp) {
+        // learning-weight gradient from z^mp, then delta_fw back through the
+        // learning pool into the last layer's delta (pre-update W_lr)
+        if (simt_lr_backward_ok(G))
+            NITRO_TRY(simt_lr_backward(a_last, b->grad_l, b->Wlr, batch, G, (int)d, nullptr,
+                                       b->desc.alpha_inv, nullptr, nullptr, nullptr, b->dWlr,
+                                       w_gl(b), w_wlr(b), nullptr, w_status(b), s));
+        else
+            NITRO_TRY(simt_learn_dw(a_last, b->grad_l, batch, (int)d, G, b->dWlr, s));
+        Layer& ly = b->L[n - 1];
+        NITRO_TRY(simt_lrpool_to_delta(b->grad_l, b->Wlr, G, (int)d, ly.g, b->lp, batch, b->lr_am,
+                                       ly.argmax, ly.region, b->desc.alpha_inv, ly.delta, w_gl(b),
+                                       w_wlr(b), w_delta(b, n - 1), w_status(b), s));
+    } else if (simt_lr_backward_ok(G)) {
         // learning-weight gradient and (below a forward layer) delta_fw -> that
         // layer's delta in one pass
         Layer* ly = n ? &b->L[n - 1] : nullptr;
@@ -345,7 +406,7 @@ nitro_status nitro_block_backward(nitro_block* b, const int8_t* a_in, const int3
     }
     if (n == 0) return NITRO_OK;
     // delta_fw = grad_L W_lr (pre-update), into the last layer
-    if (!simt_lr_backward_ok(G)) {
+    if (!b->zmp && !simt_lr_backward_ok(G)) {
         Layer& ly = b->L[n - 1];
         DeltaSrc src{};
         src.grad_l = b->grad_l; src.wlr = b->Wlr; src.G = G;
@@ -406,6 +467,12 @@ nitro_status nitro_block_set_hyper(nitro_block* b, int64_t gamma_inv_lr, int64_t
     return NITRO_OK;
 }
 
+nitro_status nitro_block_set_dropout(nitro_block* b, int dropout_p16) {
+    if (!b || dropout_p16 < 0 || dropout_p16 > 65536) return NITRO_ERR_ARG;
+    b->desc.dropout_p16 = dropout_p16;
+    return NITRO_OK;
+}
+
 nitro_status nitro_integersgd_step(nitro_block* b, void* stream) {
     if (!b) return NITRO_ERR_ARG;
     cudaStream_t s = (cudaStream_t)stream;
@@ -415,6 +482,7 @@ nitro_status nitro_integersgd_step(nitro_block* b, void* stream) {
     SgdBatch bt{};
     bt.round_trunc = b->desc.sgd_round == NITRO_ROUND_TRUNC;
     bt.status = w_status(b);
+    bt.step = w_step(b);
     for (int i = 0; i < n; ++i) {
         // the update also writes the tensor-core weight planes of the layer
         SgdTensor st{b->L[i].W, b->L[i].dW, b->L[i].wcount, gamma_fw, b->desc.eta_inv_fw,
@@ -439,6 +507,7 @@ nitro_status nitro_block_tensor_bytes(const nitro_block* b, int which, int layer
                            which == NITRO_T_REGION || which == NITRO_T_ARGMAX || which == NITRO_T_DELTA;
     if (per_layer && (layer < 0 || layer >= n)) return NITRO_ERR_ARG;
     if (!per_layer && layer != 0) return NITRO_ERR_ARG;
+    if ((which == NITRO_T_LR_IN || which == NITRO_T_LR_ARGMAX) && !b->zmp) return NITRO_ERR_ARG;
     const size_t B = (size_t)b->batch;
     switch (which) {
         case NITRO_T_W: *bytes = (size_t)b->L[layer].wcount * 4; break;
@@ -454,6 +523,9 @@ nitro_status nitro_block_tensor_bytes(const nitro_block* b, int which, int layer
         case NITRO_T_DELTA: *bytes = B * b->L[layer].pre_f * 4; break;
         case NITRO_T_GRAD_L: *bytes = B * b->G * 4; break;
         case NITRO_T_SSE: *bytes = 8; break;
+        case NITRO_T_LR_IN:
+        case NITRO_T_LR_ARGMAX: *bytes = B * b->d; break;
+        case NITRO_T_STEP: *bytes = 4; break;
         default: return NITRO_ERR_ARG;
     }
     return NITRO_OK;
@@ -471,6 +543,9 @@ static const void* tensor_ptr(nitro_block* b, int which, int layer) {
         case NITRO_T_DELTA: return b->L[layer].delta;
         case NITRO_T_GRAD_L: return b->grad_l;
         case NITRO_T_SSE: return b->sse;
+        case NITRO_T_LR_IN: return b->zmp;
+        case NITRO_T_LR_ARGMAX: return b->lr_am;
+        case NITRO_T_STEP: return w_step(b);
     }
     return nullptr;
 }
@@ -515,7 +590,8 @@ nitro_status nitro_block_get_tensor(nitro_block* b, int which, int layer, void* 
 
 nitro_status nitro_block_set_tensor(nitro_block* b, int which, int layer, const void* host_src,
                                     size_t bytes) {
-    if (which != NITRO_T_W && which != NITRO_T_DW && which != NITRO_T_WLR && which != NITRO_T_DWLR)
+    if (which != NITRO_T_W && which != NITRO_T_DW && which != NITRO_T_WLR && which != NITRO_T_DWLR &&
+        which != NITRO_T_STEP)
         return NITRO_ERR_ARG;
     size_t need = 0;
     nitro_status st = nitro_block_tensor_bytes(b, which, layer, &need);

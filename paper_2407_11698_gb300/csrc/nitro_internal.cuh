@@ -126,6 +126,34 @@ __host__ __device__ __forceinline__ uint32_t abs_u32(int32_t v) {
     return v < 0 ? (uint32_t)(-(int64_t)v) : (uint32_t)v;
 }
 
+// SplitMix64 (Steele, Lea & Flood, OOPSLA 2014), random-access form: output
+// `index` of the generator seeded with `seed` is the published finaliser
+// applied to seed + (index + 1) * 0x9E3779B97F4A7C15.
+__host__ __device__ __forceinline__ uint64_t splitmix64_at(uint64_t seed, uint64_t index) {
+    uint64_t z = seed + (index + 1ULL) * 0x9E3779B97F4A7C15ULL;
+    z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ULL;
+    z = (z ^ (z >> 27)) * 0x94D049BB133111EBULL;
+    return z ^ (z >> 31);
+}
+
+// Dropout of the linear forward layers (App. B, p_l): element e of forward
+// layer `layer` at step t is dropped when the top 16 bits of output
+// 2^63 + t 2^35 + layer 2^31 + e of the block's SplitMix64 stream are below
+// p16 (rate in units of 2^-16; t modulo 2^28, layer < 16, e < 2^31).
+constexpr int kRegionDropped = 4;   // region code of a dropped activation
+struct DropoutArgs {
+    uint64_t seed;
+    uint32_t p16;           // 0 = off
+    int layer;
+    const uint32_t* step;   // device step counter
+};
+__host__ __device__ __forceinline__ bool dropout_drop(uint64_t seed, uint32_t t, int layer,
+                                                      uint64_t e, uint32_t p16) {
+    const uint64_t idx = (1ULL << 63) + ((uint64_t)(t & ((1u << 28) - 1)) << 35) +
+                         ((uint64_t)layer << 31) + e;
+    return (uint32_t)(splitmix64_at(seed, idx) >> 48) < p16;
+}
+
 // max|A| * max|B| * k >= 2^63 : int64 exactness of an int32 x int32
 // contraction of length k is no longer guaranteed.
 __host__ __device__ __forceinline__ bool int64_bound_exceeded(uint32_t ma, uint32_t mb, int64_t k) {
@@ -167,9 +195,31 @@ cudaError_t simt_gemm(int mode, const int8_t* act, const int32_t* grad, const in
 
 // z (int64, pre-pool NHWC) -> NITRO-Scaling -> NITRO-ReLU -> region codes,
 // optional 2x2 max-pool with argmax codes, int8 outputs (out2 may be NULL).
+// With drop.p16 > 0 (linear layers, no pool) dropped outputs are stored as 0
+// with region code kRegionDropped.
 cudaError_t simt_fwd_epilogue(const int64_t* z, const LayerGeom& g, int B, int alpha_inv,
                               int mu, int8_t* out, int8_t* out2, int8_t* region,
-                              int8_t* argmax, cudaStream_t s);
+                              int8_t* argmax, cudaStream_t s, const DropoutArgs* drop = nullptr);
+
+// Learning-layer max-pool (Sec. 3.3, z^mp): a [B][H][W][C] int8 -> out
+// [B][ph][pw][C] over kh x kw windows with stride (kh, kw), first maximum in
+// row-major window order, its position r*kw + s in am.
+cudaError_t simt_lr_pool_fwd(const int8_t* a, int B, int H, int W, int C, int kh, int kw,
+                             int ph, int pw, int8_t* out, uint8_t* am, cudaStream_t s);
+
+// delta_fw = grad_l W_lr at the pooled learning features (int32 storage rule,
+// int64 bound check), routed back through the learning-layer pool (window
+// maximum am), the 2x2 max-pool of conv layer g (argmax) and NITRO-ReLU
+// backward into g's delta [B][h][w][cout]; every element is written.
+struct LrPoolGeom {
+    int kh, kw, ph, pw;
+};
+cudaError_t simt_lrpool_to_delta(const int32_t* gl, const int32_t* wlr, int G, int d,
+                                 const LayerGeom& g, const LrPoolGeom& lp, int B,
+                                 const uint8_t* am, const int8_t* argmax, const int8_t* region,
+                                 int alpha_inv, int32_t* delta, const uint32_t* maxabs_gl,
+                                 const uint32_t* maxabs_wlr, uint32_t* maxabs_delta,
+                                 uint32_t* status, cudaStream_t s);
 
 // Learning layer forward + loss: grad_l = floor(a W^T / (256 d)) - 32 onehot,
 // sse = sum grad_l^2 (mod 2^64), loss = floor(sse / 2) (if loss != NULL),
@@ -242,6 +292,7 @@ struct SgdBatch {
     int count;
     int round_trunc;
     uint32_t* status;
+    uint32_t* step;        // block step counter, incremented once per launch (or null)
 };
 cudaError_t simt_integersgd(const SgdBatch& b, cudaStream_t s);
 

@@ -37,6 +37,8 @@ enum KernelId : int {
     K_PREP_SUM,
     K_PREP_MAD,
     K_PREP_APPLY,
+    K_LR_POOL,
+    K_LRPOOL_TO_DELTA,
     K_COUNT
 };
 

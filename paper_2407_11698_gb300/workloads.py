@@ -47,6 +47,61 @@ WORKLOADS = {
                 _blk([], 4 * 4 * 256)]),
 }
 
+
+def _vgg_b(spec, hw, cin):
+    # one local-loss block per layer: (cout, pool) convs, then linear widths
+    blocks = []
+    for cout, pool in spec:
+        blocks.append(_blk([_conv(cin, cout, hw, pool)], hw * hw * cin))
+        cin, hw = cout, hw // 2 if pool else hw
+    return blocks, hw * hw * cin
+
+
+def _paper_vgg(spec):
+    blocks, flat = _vgg_b(spec, 32, 3)
+    blocks.append(_blk([_lin(flat, 1024)], flat))
+    blocks.append(_blk([], 1024))
+    return blocks
+
+
+def _paper_mlp(widths):
+    blocks = [_blk([_lin(a, b)], a) for a, b in zip(widths[:-1], widths[1:])]
+    blocks.append(_blk([], widths[-1]))
+    return blocks
+
+
+# Paper-scale networks of Table 1 with the CIFAR-10 / MNIST hyper-parameters
+# of App. B (gamma_inv = 512; Table 6's decay rates taken as eta_inv; d^lr;
+# the linear blocks' dropout p_l in units of 2^-16).  Every IntConv2D (with the
+# MaxPool2D after it) and every hidden IntLinear is a local-loss block.  Batch
+# 64 as in App. B.  Used for timing; parity runs them at smaller batches.
+PAPER_WORKLOADS = {
+    # VGG8B, CIFAR-10: d^lr 4096, lambda 25000 / 3000, p_l = 0.15
+    "vgg8b_cifar10_b64": dict(
+        input_shape=(32, 32, 3), batch=64, steps=10,
+        hyper=dict(d_lr=4096, eta_inv_fw=25000, eta_inv_lr=3000, dropout_p16=9830),
+        blocks=_paper_vgg([(128, False), (256, True), (256, False), (512, True), (512, True),
+                           (512, True)])),
+    # VGG11B, CIFAR-10: d^lr 4096, lambda 28000 / 4500, p_l = 0
+    "vgg11b_cifar10_b64": dict(
+        input_shape=(32, 32, 3), batch=64, steps=10,
+        hyper=dict(d_lr=4096, eta_inv_fw=28000, eta_inv_lr=4500),
+        blocks=_paper_vgg([(128, False), (128, False), (128, False), (256, True), (256, False),
+                           (512, True), (512, False), (512, True), (512, True)])),
+    # MLP3, MNIST: 784-1024-1024-1024-10, lambda 28000 / 5000
+    "mlp3_mnist_b64": dict(
+        input_shape=(28, 28, 1), batch=64, steps=10,
+        hyper=dict(eta_inv_fw=28000, eta_inv_lr=5000),
+        blocks=_paper_mlp([784, 1024, 1024, 1024])),
+    # MLP4, CIFAR-10: 1024-3000-3000-3000-10 (Table 1 gives a 1024-wide input:
+    # one 32 x 32 channel), lambda 19000 / 7500, p_l = 0.10
+    "mlp4_cifar10_b64": dict(
+        input_shape=(32, 32, 1), batch=64, steps=10,
+        hyper=dict(eta_inv_fw=19000, eta_inv_lr=7500, dropout_p16=6554),
+        blocks=_paper_mlp([1024, 3000, 3000, 3000])),
+}
+WORKLOADS.update(PAPER_WORKLOADS)
+
 # Kernel sweep: conv fwd / dgrad / wgrad at batch 256 and int GEMM sizes.
 SWEEP_CONV = [(256, hw, c) for hw in (32, 16, 8) for c in (64, 128, 256, 512)]
 SWEEP_GEMM = [1024, 4096, 8192]

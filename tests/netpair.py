@@ -88,6 +88,10 @@ class NetPair:
             _eq(g.get(nb.NITRO_T_DWLR, 0, check=False), o.dWlr, tag + " dWlr")
             _eq(g.get(nb.NITRO_T_GRAD_L, 0, check=False), o.grad_l, tag + " grad_l")
             _eq(g.get(nb.NITRO_T_SSE, 0, check=False), np.array([o.sse]), tag + " sse")
+            if getattr(o, "lr_in", None) is not None:
+                _eq(g.get(nb.NITRO_T_LR_IN, 0, check=False), o.lr_in, tag + " lr_in")
+                _eq(g.get(nb.NITRO_T_LR_ARGMAX, 0, check=False), o.lr_argmax, tag + " lr_argmax")
+            _eq(g.get(nb.NITRO_T_STEP, 0, check=False), np.array([o.t]), tag + " step")
             assert g.status_bits() == o.status, "%s status %d vs %d" % (tag, g.status_bits(), o.status)
 
 
@@ -101,12 +105,15 @@ def _eq(got, want, what):
             what, bad.size, want.size, bad[0], got[bad[0]], want[bad[0]]))
 
 
-def run_workload(wl, steps, seed=20240716, check_every=1, data_seed=7, concurrent=False):
-    pair = NetPair(wl["blocks"], wl["batch"], seed=seed, concurrent=concurrent)
+def run_workload(wl, steps, seed=20240716, check_every=1, data_seed=7, concurrent=False,
+                 batch=None, **hyper):
+    batch = batch or wl["batch"]
+    hyper = dict(wl.get("hyper", {}), **hyper)
+    pair = NetPair(wl["blocks"], batch, seed=seed, concurrent=concurrent, **hyper)
     try:
         for s in range(steps):
-            x = synth.images(data_seed, s, wl["batch"], wl["input_shape"])
-            y = synth.labels(data_seed, s, wl["batch"])
+            x = synth.images(data_seed, s, batch, wl["input_shape"])
+            y = synth.labels(data_seed, s, batch)
             gl, ol = pair.step(x, y)
             assert gl == ol, "step %d losses gpu %s oracle %s" % (s, gl, ol)
             if (s + 1) % check_every == 0 or s == steps - 1:

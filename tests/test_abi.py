@@ -80,13 +80,24 @@ def _bad(**kw):
     dict(layers=[(7, 1, 4, 6, 6, 0)]),                      # unknown kind
     dict(layers=[(nb.NITRO_CONV3X3, 1, 4, 6, 6, 1), (nb.NITRO_LINEAR, 37, 3, 1, 1, 0)]),
     dict(layers=[], in_features=0),
+    dict(d_lr=-1),                                          # learning-layer input size
+    dict(dropout_p16=-1),
+    dict(dropout_p16=65537),                                # rate above 1
 ])
 def test_init_rejects_bad_descriptors(lib, kw):
     st, h, _ = _bad(**kw)
     assert st == nb.NITRO_ERR_ARG and not h.value
 
 
+def test_init_rejects_learning_pool_windows_above_a_byte(lib):
+    # a 64 x 64 single-channel map brought to one feature needs a 64 x 64
+    # window: its argmax no longer fits the byte the library stores it in
+    st, h, _ = _bad(layers=[(nb.NITRO_CONV3X3, 1, 1, 64, 64, 0)], in_features=64 * 64, d_lr=1)
+    assert st == nb.NITRO_ERR_UNSUPPORTED and not h.value
+
+
 def test_null_handle_calls_are_rejected(lib):
+    assert lib.nitro_block_set_dropout(None, 0) == nb.NITRO_ERR_ARG
     assert nb.nitro_block_forward(None, None, 0, None) == nb.NITRO_ERR_ARG
     assert nb.nitro_block_backward(None, None, None, 0, None) == nb.NITRO_ERR_ARG
     assert nb.nitro_integersgd_step(None) == nb.NITRO_ERR_ARG

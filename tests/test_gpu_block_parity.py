@@ -207,6 +207,8 @@ def test_checkpoint_resume_is_bit_exact():
                 ob.W[i] = oa.W[i].copy()
             gb_.set(nb.NITRO_T_WLR, 0, ga.get(nb.NITRO_T_WLR, 0))
             ob.Wlr = oa.Wlr.copy()
+            gb_.set(nb.NITRO_T_STEP, 0, ga.get(nb.NITRO_T_STEP, 0))
+            ob.t = oa.t
         for s in range(2, 4):
             x, y = synth.images(4, s, 4, (8, 8, 1)), synth.labels(4, s, 4)
             la, _ = a.step(x, y)

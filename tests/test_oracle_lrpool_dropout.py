@@ -228,3 +228,27 @@ def test_block_lr_pool_brute_force(pool, hw, d_lr):
 def test_block_lr_pool_rejects_wide_windows():
     with pytest.raises(ValueError):
         O.OracleBlock([O.LayerDesc(O.CONV, 1, 1, 64, 64, False)], d_lr=1)
+
+
+# ------------------------------------------------------- paper-scale networks
+def test_paper_workloads_chain_and_pool_to_d_lr():
+    from paper_2407_11698_gb300 import workloads as WL
+    for name, wl in WL.PAPER_WORKLOADS.items():
+        hyper = wl.get("hyper", {})
+        blocks = [O.OracleBlock([O.LayerDesc(*l) for l in b["layers"]],
+                                in_features=b["in_features"], seed=i, **hyper)
+                  for i, b in enumerate(wl["blocks"])]
+        in_f = int(np.prod(wl["input_shape"]))
+        for blk in blocks:
+            assert blk.in_features == in_f, name
+            if blk.layers:
+                in_f = blk.layers[-1].out_features
+                if hyper.get("d_lr"):
+                    assert blk.d <= hyper["d_lr"], name
+        assert blocks[-1].layers == [] and blocks[-1].G == 10
+    # VGG8B's learning layers all see 4096 features except the 2 x 2 x 512
+    # block and the linear block (2048 and 1024 outputs)
+    ds = [O.OracleBlock([O.LayerDesc(*l) for l in b["layers"]], in_features=b["in_features"],
+                        **WL.PAPER_WORKLOADS["vgg8b_cifar10_b64"]["hyper"]).d
+          for b in WL.PAPER_WORKLOADS["vgg8b_cifar10_b64"]["blocks"][:-1]]
+    assert ds == [4096, 4096, 4096, 4096, 4096, 2048, 1024]
