@@ -855,9 +855,14 @@ cudaError_t simt_gemm(int mode, const int8_t* act, const int32_t* grad, const in
     }
     if (p.M <= 0 || p.N <= 0) return cudaSuccess;
     const int tiles_m = (p.M + kTile - 1) / kTile, tiles_n = (p.N + kTile - 1) / kTile;
+    // Split K over gridDim.z (64-bit atomics into a zeroed output, exact in any
+    // order) until the grid holds about four CTAs per SM, keeping at least
+    // 256 K per split.  Weight gradients always reduce over a long K; the
+    // forward and input gradient need it when the output has few tiles (a
+    // batch of 64 against a linear layer, a 4 x 4 conv map).
     int splits = 1;
-    if (mode == GM_CONV_WGRAD || mode == GM_LIN_WGRAD) {
-        const int64_t tiles = (int64_t)tiles_m * tiles_n;
+    const int64_t tiles = (int64_t)tiles_m * tiles_n;
+    if (mode == GM_CONV_WGRAD || mode == GM_LIN_WGRAD || tiles < 2 * 152) {
         const int64_t want = (4 * 152 + tiles - 1) / tiles;
         const int64_t maxs = (p.K + 255) / 256;
         splits = (int)(want < maxs ? want : maxs);

@@ -29,7 +29,16 @@ struct Layer {
     int8_t* argmax = nullptr;    // [max_batch x out_f] if pool
     int32_t* delta = nullptr;    // [max_batch x pre_f]
     TcLayer tc;                  // tensor-core state (limb planes, maps)
+    uint16_t* lin_a = nullptr;       // linear on tcgen05: bf16 input [max_batch x in]
+    uint16_t* lin_planes = nullptr;  // and weight limb planes [4][out][in]
 };
+
+// Linear forward on the tcgen05 GEMM: rows of 16-byte multiples for TMA
+// (in % 8 == 0), and large enough to beat the CUDA-core kernel.
+bool lin_tc_ok(const nitro_layer_desc& l) {
+    return l.kind == NITRO_LINEAR && l.cin % 8 == 0 && l.cin >= 64 &&
+           (int64_t)l.cin * l.cout >= 4096 && (int64_t)l.cin * l.cout < ((int64_t)1 << 31);
+}
 
 }  // namespace
 
@@ -240,6 +249,9 @@ nitro_status nitro_init_block(const nitro_block_desc* desc, uint64_t seed, void*
              dalloc(b, &ly.region, (size_t)MB * ly.pre_f) &&
              dalloc(b, &ly.delta, (size_t)MB * ly.pre_f);
         if (ok && l.pool2x2) ok = dalloc(b, &ly.argmax, (size_t)MB * ly.out_f);
+        if (ok && lin_tc_ok(l))
+            ok = dalloc(b, &ly.lin_a, (size_t)MB * l.cin) &&
+                 dalloc(b, &ly.lin_planes, (size_t)kMaxLimbs * ly.wcount);
         z_need = std::max(z_need, (size_t)MB * (size_t)ly.pre_f);
         z_need = std::max(z_need, (size_t)MB * (size_t)ly.in_f);
         host_w.push_back(draw_weights(ly.wcount, fan_in, seed, (uint64_t)i));
@@ -282,8 +294,11 @@ nitro_status nitro_init_block(const nitro_block_desc* desc, uint64_t seed, void*
     if (e == cudaSuccess) e = cudaMemsetAsync(b->dWlr, 0, (size_t)b->G * b->d * 8, s);
     if (e == cudaSuccess) e = cudaMemcpyAsync(b->words, words.data(), words.size() * 4, cudaMemcpyHostToDevice, s);
     if (e == cudaSuccess) e = cudaMemsetAsync(b->sse, 0, 8, s);
-    for (int i = 0; e == cudaSuccess && i < desc->n_layers; ++i)
+    for (int i = 0; e == cudaSuccess && i < desc->n_layers; ++i) {
         e = tc_refresh_weights(b->L[i].tc, b->L[i].g, b->L[i].W, w_w(b, i), s);
+        if (e == cudaSuccess && b->L[i].lin_planes)
+            e = tc_pack_limbs(b->L[i].W, b->L[i].wcount, w_w(b, i), b->L[i].lin_planes, s);
+    }
     if (e == cudaSuccess) e = cudaStreamSynchronize(s);
     if (e != cudaSuccess) {
         free_all(b);
@@ -326,6 +341,13 @@ nitro_status nitro_block_forward(nitro_block* b, const int8_t* a_in, int batch, 
             next_nhwc = b->L[i + 1].tc.act_nhwc;
         TcFwdOut fo{b->desc.alpha_inv, b->mu, ly.act, out2, ly.region, ly.argmax, next_nhwc};
         NITRO_TRY(tc_conv_forward(ly.tc, g, batch, b->z64, &fo, w_status(b), s, &done, &fused));
+        if (ly.lin_planes) {
+            // linear: z = a W^T on the tcgen05 GEMM (weight planes kept by IntegerSGD)
+            NITRO_TRY(tc_pack_int8(x, batch, g.cin, ly.lin_a, s));
+            NITRO_TRY(tc_gemm_run(ly.lin_a, ly.lin_planes, batch, g.cout, g.cin, w_w(b, i), b->z64,
+                                  w_status(b), s));
+            done = true;
+        }
         if (!done && simt_small_conv_ok(g)) {
             // narrow input (image channels): fused CUDA-core forward
             NITRO_TRY(simt_conv_small_fwd(x, ly.W, g, batch, b->desc.alpha_inv, b->mu, ly.act, out2,
@@ -489,6 +511,14 @@ nitro_status nitro_integersgd_step(nitro_block* b, void* stream) {
                      w_w(b, i), {}, {}, nullptr, 0, 0, 0, 0, {}};
         tc_weight_planes(b->L[i].tc, b->L[i].g, &st.planes, &st.plane, &st.row_k, &st.tap_k);
         st.cin = b->L[i].g.cin;
+        if (b->L[i].lin_planes) {
+            // linear planes [4][out][in]: element o*in + k at row o*9*in + tap*in with
+            // the update's (row, tap) = (o / 9, o % 9) decomposition
+            st.planes = b->L[i].lin_planes;
+            st.plane = b->L[i].wcount;
+            st.row_k = 9 * b->L[i].g.cin;
+            st.tap_k = b->L[i].g.cin;
+        }
         bt.t[bt.count++] = st;
     }
     bt.t[bt.count++] = SgdTensor{b->Wlr, b->dWlr, (int64_t)b->G * b->d, b->desc.gamma_inv_lr,
@@ -606,6 +636,10 @@ nitro_status nitro_block_set_tensor(nitro_block* b, int which, int layer, const 
         if (cudaMemcpy(word, &m, 4, cudaMemcpyHostToDevice) != cudaSuccess) return NITRO_ERR_CUDA;
         if (which == NITRO_T_W &&
             tc_refresh_weights(b->L[layer].tc, b->L[layer].g, b->L[layer].W, word, 0) != cudaSuccess)
+            return NITRO_ERR_CUDA;
+        if (which == NITRO_T_W && b->L[layer].lin_planes &&
+            tc_pack_limbs(b->L[layer].W, b->L[layer].wcount, word, b->L[layer].lin_planes, 0) !=
+                cudaSuccess)
             return NITRO_ERR_CUDA;
     }
     if (cudaDeviceSynchronize() != cudaSuccess) return NITRO_ERR_CUDA;

@@ -599,8 +599,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                     if (m < args.B) {
                         int64_t* o = args.out + (int64_t)m * args.ncols + col0;
 #pragma unroll
-                        for (int i = 0; i < NH; ++i)
-                            if (col0 + i < args.ncols) o[i] = (int64_t)acc[i];
+                        for (int i = 0; i < NH; ++i) {
+                            if (col0 + i >= args.ncols) break;
+                            if (args.atomic_out)       // K split: exact 64-bit sums
+                                atomicAdd(reinterpret_cast<unsigned long long*>(o + i),
+                                          (unsigned long long)acc[i]);
+                            else
+                                o[i] = (int64_t)acc[i];
+                        }
                     }
                 } else if (MODE == TC_WGRAD) {
                     const int m = T.mt * kBM + r;
@@ -1466,13 +1472,26 @@ cudaError_t tc_gemm_run(const uint16_t* a_bf16, const uint16_t* b_planes, int M,
     const int n = pick_n(N);
     a.tiles_m = (M + kBM - 1) / kBM;
     a.tiles_n = (N + n - 1) / n;
-    a.total_tiles = a.tiles_m * a.tiles_n;
     a.kb_total = (K + kBK - 1) / kBK;
-    a.kb_per_split = a.kb_total;
+    // few output tiles (a batch of 64 against a linear layer): split K so that
+    // about one wave of CTAs runs, at least four K-blocks per split, partial
+    // sums added with 64-bit atomics into a zeroed C
+    const int tiles = a.tiles_m * a.tiles_n;
+    int splits = sm_count() / tiles;
+    const int max_splits = (a.kb_total + 3) / 4;
+    splits = splits < 1 ? 1 : (splits > max_splits ? max_splits : splits);
+    a.kb_per_split = (a.kb_total + splits - 1) / splits;
+    splits = (a.kb_total + a.kb_per_split - 1) / a.kb_per_split;
+    a.total_tiles = tiles * splits;
+    a.atomic_out = splits > 1;
     a.max_a = nullptr;
     a.max_b = max_b;
     a.out = out;
     a.status = status;
+    if (a.atomic_out) {
+        cudaError_t e = cudaMemsetAsync(out, 0, sizeof(int64_t) * (size_t)M * N, s);
+        if (e != cudaSuccess) return e;
+    }
     CUtensorMap ma, mb;
     const uint64_t da[2] = {(uint64_t)K, (uint64_t)M};
     const uint64_t sa[1] = {(uint64_t)K};

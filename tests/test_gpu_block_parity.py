@@ -85,6 +85,16 @@ def test_conv_then_linear_in_one_block():
     _run(blocks, 5, steps=3, input_shape=(6, 6, 3))
 
 
+def test_linear_layers_on_tensor_cores():
+    # input widths that are multiples of 8 run the forward on the tcgen05 GEMM:
+    # three row tiles (batch 257), a ragged column tile, a K split (3000-wide
+    # input against few output tiles), weight decay and dropout on top
+    blocks = [_b([(L, 136, 200, 1, 1, 0), (L, 200, 72, 1, 1, 0)], 136), _b([], 72)]
+    _run(blocks, 257, steps=3, eta_inv_fw=25000, eta_inv_lr=3000, dropout_p16=6554)
+    blocks = [_b([(L, 3000, 40, 1, 1, 0)], 3000), _b([], 40)]
+    _run(blocks, 20, steps=3)
+
+
 def test_batch_of_one_and_max_batch():
     blocks = [_b([(L, 20, 9, 1, 1, 0)], 20)]
     _run(blocks, 1, steps=2)

@@ -148,7 +148,9 @@ def test_conv_sweep_sampled(torch, B, hw, c):
 
 @pytest.mark.parametrize("m,n,k,lb", [(1024, 1024, 1024, 1), (1024, 1024, 1024, 3),
                                       (4096, 4096, 4096, 1), (8192, 8192, 8192, 2),
-                                      (300, 200, 136, 4), (130, 70, 12, 2)])
+                                      (300, 200, 136, 4), (130, 70, 12, 2),
+                                      # few output tiles: K split across CTAs
+                                      (64, 3000, 3000, 2), (20, 40, 3000, 3), (64, 1024, 2048, 1)])
 def test_int_gemm(torch, m, n, k, lb):
     a = synth.int_tensor(41, (m, k), -128, 127, dtype=np.int8)
     b = synth.int_tensor(42, (n, k), *RANGES[lb], dtype=np.int32)
