@@ -1100,7 +1100,8 @@ int pick_n(int cols) { return cols % 128 == 0 ? 128 : 64; }
 
 void pixel_tiling(const LayerGeom& g, int batch, TcArgs& a) {
     if (g.w > 8) { a.wb = 16; a.hb = 8; a.bb = 1; }
-    else { a.wb = 8; a.hb = 8; a.bb = 2; }
+    else if (g.w > 4 || g.h > 4) { a.wb = 8; a.hb = 8; a.bb = 2; }
+    else { a.wb = 4; a.hb = 4; a.bb = 8; }     // 4 x 4 maps: eight whole images per tile
     a.ntx = (g.w + a.wb - 1) / a.wb;
     a.nty = (g.h + a.hb - 1) / a.hb;
     a.tiles_m = a.ntx * a.nty * ((batch + a.bb - 1) / a.bb);
@@ -1135,9 +1136,10 @@ bool tc_layer_init(TcLayer& t, const LayerGeom& g, int max_batch, bool has_dgrad
     // kernels: zero-padding them to a 64-wide K-block wastes most MMA work.
     // Inputs with 9 Cin <= 64 run as one 64-wide K-block of im2col rows.
     const bool pix_ok = g.h >= 8 && g.w >= 8;
+    const bool pix4 = g.h == 4 && g.w == 4;       // forward only: 4 x 4 x 8-image tiles
     const bool wide = g.cin >= 32;
     t.im2col = pix_ok && 9 * g.cin <= kBK && im2col_smem(g.w, g.cin) <= 48 * 1024;
-    t.fwd = pix_ok && (wide || t.im2col);
+    t.fwd = (pix_ok && (wide || t.im2col)) || (pix4 && wide);
     t.wgrad = (wide || t.im2col) && g.cout % 8 == 0;
     // the input gradient reads the forward planes, which im2col layers lay out
     // without taps

@@ -49,6 +49,8 @@ def _widen(pair, scale):
     (4, 8, 8, 64, 64, 64, True, 70001),        # three-limb weights
     (4, 8, 8, 64, 64, 64, False, 2**22),       # four-limb weights
     (130, 8, 16, 64, 64, 64, True, 1),         # batch over 128 (wgrad batch blocks)
+    (13, 4, 4, 64, 64, 128, True, 1),          # 4 x 4 maps: 8-image forward tiles, ragged batch
+    (9, 4, 4, 128, 128, 64, False, 70001),     # 4 x 4 maps, three-limb weights, N = 64 tiles
 ])
 def test_two_conv_block_parity(B, h, w, c0, c1, c2, pool, scale):
     _run_two_conv(B, h, w, c0, c1, c2, pool, scale, False)
