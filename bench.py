@@ -48,10 +48,13 @@ def parse():
     return p.parse_args()
 
 
-def ncu_traffic(kernel):
+def ncu_traffic(kernel, workload=WORKLOAD):
     """Per-launch DRAM bytes of `kernel` from the committed ncu summary, or None
-    when the kernel source changed since the counters were taken."""
+    when the kernel source changed since the counters were taken or the
+    workload is not the one the summary covers."""
     import hashlib
+    if workload != WORKLOAD:
+        return None
     try:
         src = open(os.path.join(ROOT, "paper_2407_11698_gb300", "csrc", "tc_conv.cu"), "rb").read()
         sha = hashlib.sha1(src).hexdigest()[:12]
@@ -428,7 +431,7 @@ def run_ours(args, rank, world, local_rank):
         "gpu_launches": int(launches_per_step * args.steps),
         "roofline": {"bound": bound, "kernel": dom_name, "achieved": round(achieved, 3),
                      "peak": round(peak, 2), "unit": unit, "frac": round(achieved / peak, 4),
-                     "traffic": ncu_traffic(dom_name), "peak_source": peak_note,
+                     "traffic": ncu_traffic(dom_name, args.workload), "peak_source": peak_note,
                      "per_launch_ms": round(per_launch_ms, 5),
                      "share_of_kernel_time": round(dom["ms"] / total_k, 4),
                      "issued": issued_line},

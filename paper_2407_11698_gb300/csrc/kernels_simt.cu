@@ -401,6 +401,36 @@ __global__ void k_lr_pool_fwd(const int8_t* __restrict__ a, int B, int H, int W,
     }
 }
 
+// Same, four channels per thread (C % 4 == 0, 4-byte aligned buffers): signed
+// SIMD byte maxima, and a window position replaced only where a later value
+// is strictly greater (the first maximum wins).
+__global__ void k_lr_pool_fwd4(const int8_t* __restrict__ a, int B, int H, int W, int C, int kh,
+                               int kw, int ph, int pw, FloorDiv32 dv_c4, FloorDiv32 dv_pw,
+                               FloorDiv32 dv_ph, int8_t* __restrict__ out,
+                               uint8_t* __restrict__ am) {
+    const int C4 = C >> 2;
+    const uint32_t n4 = (uint32_t)B * ph * pw * C4;
+    for (uint32_t i = blockIdx.x * blockDim.x + threadIdx.x; i < n4; i += gridDim.x * blockDim.x) {
+        const uint32_t pix = dv_c4.udiv(i);
+        const int c = (int)(i - pix * C4) * 4;
+        const uint32_t r = dv_pw.udiv(pix);
+        const int x = (int)(pix - r * pw);
+        const uint32_t b = dv_ph.udiv(r);
+        const int y = (int)(r - b * ph);
+        const int8_t* p = a + ((b * H + (uint32_t)(y * kh)) * W + (uint32_t)(x * kw)) * C + c;
+        uint32_t best = *reinterpret_cast<const uint32_t*>(p), pos = 0;
+        for (int u = 0; u < kh; ++u)
+            for (int v = 0; v < kw; ++v) {
+                const uint32_t val = *reinterpret_cast<const uint32_t*>(p + (u * W + v) * C);
+                const uint32_t gt = __vcmpgts4(val, best);
+                best = __vmaxs4(best, val);
+                pos = (pos & ~gt) | ((uint32_t)(u * kw + v) * 0x01010101u & gt);
+            }
+        reinterpret_cast<uint32_t*>(out)[i] = best;
+        reinterpret_cast<uint32_t*>(am)[i] = pos;
+    }
+}
+
 // ---------------------------------------------------------------------------
 // Learning-layer backward through the pool, into the last layer's delta.  One
 // thread per pre-pool element (b, y, x, c) of that conv layer: it receives a
@@ -460,6 +490,79 @@ __global__ void k_lrpool_to_delta(const int32_t* __restrict__ gl, const int32_t*
         }
         delta[i] = dv;
         mx = max(mx, abs_u32(dv));
+    }
+#pragma unroll
+    for (int off = 16; off; off >>= 1) mx = max(mx, __shfl_xor_sync(kFull, mx, off));
+    ovf = __any_sync(kFull, ovf);
+    if ((threadIdx.x & 31) == 0) {
+        if (mx) atomicMax(maxabs_delta, mx);
+        if (ovf) atomicOr(status, ST_OVERFLOW);
+    }
+}
+
+// Same, four channels per thread (C % 4 == 0): one 4-byte load of each code
+// array and of the region bytes, one 16-byte delta store, 32-bit index
+// arithmetic (B h w C < 2^31) through invariant dividers; the pool windows
+// are powers of two, so their divisions are shifts.
+__global__ void k_lrpool_to_delta4(const int32_t* __restrict__ gl, const int32_t* __restrict__ wlr,
+                                   int G, int d, LayerGeom g, LrPoolGeom lp, int lg_kh, int lg_kw,
+                                   int B, FloorDiv32 dv_c4, FloorDiv32 dv_w, FloorDiv32 dv_h,
+                                   const uint8_t* __restrict__ lam,
+                                   const int8_t* __restrict__ argmax,
+                                   const int8_t* __restrict__ region, FloorDiv32 alpha,
+                                   int32_t* __restrict__ delta, const uint32_t* maxabs_gl,
+                                   const uint32_t* maxabs_wlr, uint32_t* maxabs_delta,
+                                   uint32_t* status) {
+    const int C = g.cout, C4 = g.cout >> 2;
+    const uint32_t n4 = (uint32_t)B * g.h * g.w * C4;
+    if (blockIdx.x == 0 && threadIdx.x == 0 && int64_bound_exceeded(*maxabs_gl, *maxabs_wlr, G))
+        atomicOr(status, ST_OVERFLOW);
+    uint32_t mx = 0;
+    bool ovf = false;
+    for (uint32_t i = blockIdx.x * blockDim.x + threadIdx.x; i < n4; i += gridDim.x * blockDim.x) {
+        const uint32_t pix = dv_c4.udiv(i);
+        const int c = (int)(i - pix * C4) * 4;
+        const uint32_t r = dv_w.udiv(pix);
+        const int x = (int)(pix - r * g.w);
+        const uint32_t b = dv_h.udiv(r);
+        const int y = (int)(r - b * g.h);
+        int qy = y, qx = x;
+        bool any = true;
+        uint32_t am2 = 0, code2 = 0;
+        if (g.pool) {
+            qy = y >> 1;
+            qx = x >> 1;
+            any = qy < g.oh && qx < g.ow;
+            if (any) {
+                am2 = *reinterpret_cast<const uint32_t*>(argmax + ((b * g.oh + qy) * g.ow + qx) * C + c);
+                code2 = (uint32_t)(((y & 1) << 1) | (x & 1));
+            }
+        }
+        int v[4] = {0, 0, 0, 0};
+        const int wy = qy >> lg_kh, wx = qx >> lg_kw;
+        if (any && wy < lp.ph && wx < lp.pw) {
+            const uint32_t lw =
+                *reinterpret_cast<const uint32_t*>(lam + ((b * lp.ph + wy) * lp.pw + wx) * C + c);
+            const uint32_t code = (uint32_t)(((qy - (wy << lg_kh)) << lg_kw) + (qx - (wx << lg_kw)));
+            const uint32_t rw = *reinterpret_cast<const uint32_t*>(region + 4 * (size_t)i);
+            const int f0 = (wy * lp.pw + wx) * C + c;
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                const bool hit = (!g.pool || ((am2 >> (8 * j)) & 255u) == code2) &&
+                                 ((lw >> (8 * j)) & 255u) == code;
+                if (!hit) continue;
+                uint64_t acc = 0;   // modulo 2^64, exact below the bound
+                for (int k = 0; k < G; ++k)
+                    acc += (uint64_t)((int64_t)gl[b * G + k] * wlr[(int64_t)k * d + f0 + j]);
+                const int64_t gv = (int64_t)acc;
+                ovf |= !fits_i32(gv);
+                const int32_t gs = (int32_t)gv;
+                const int rg = (int8_t)(rw >> (8 * j));
+                v[j] = rg == 1 ? alpha.floor_div(gs) : (rg == 2 ? gs : 0);
+                mx = max(mx, abs_u32(v[j]));
+            }
+        }
+        reinterpret_cast<int4*>(delta)[i] = make_int4(v[0], v[1], v[2], v[3]);
     }
 #pragma unroll
     for (int off = 16; off; off >>= 1) mx = max(mx, __shfl_xor_sync(kFull, mx, off));
@@ -915,7 +1018,12 @@ cudaError_t simt_lr_pool_fwd(const int8_t* a, int B, int H, int W, int C, int kh
     if (n <= 0) return cudaSuccess;
     if (kh < 1 || kw < 1 || ph * kh > H || pw * kw > W || kh * kw > 256) return cudaErrorInvalidValue;
     ProfScope ps(K_LR_POOL, s, 0.0, (double)B * H * W * C + 2.0 * n);
-    k_lr_pool_fwd<<<grid_for(n, 256), 256, 0, s>>>(a, B, H, W, C, kh, kw, ph, pw, out, am);
+    if (C % 4 == 0 && (((uintptr_t)a | (uintptr_t)out | (uintptr_t)am) & 3) == 0)
+        k_lr_pool_fwd4<<<grid_for(n / 4, 256), 256, 0, s>>>(
+            a, B, H, W, C, kh, kw, ph, pw, FloorDiv32::make((uint32_t)(C / 4)),
+            FloorDiv32::make((uint32_t)pw), FloorDiv32::make((uint32_t)ph), out, am);
+    else
+        k_lr_pool_fwd<<<grid_for(n, 256), 256, 0, s>>>(a, B, H, W, C, kh, kw, ph, pw, out, am);
     return cudaGetLastError();
 }
 
@@ -935,10 +1043,23 @@ cudaError_t simt_lrpool_to_delta(const int32_t* gl, const int32_t* wlr, int G, i
     ProfScope ps(K_LRPOOL_TO_DELTA, s, 2.0 * B * d * G,
                  5.0 * n + (double)B * g.oh * g.ow * g.cout * (g.pool ? 1 : 0) + (double)B * d +
                      4.0 * G * (B + (double)d));
-    k_lrpool_to_delta<<<grid_for(n, 256), 256, 0, s>>>(
-        gl, wlr, G, d, g, lp, B, am, argmax, region,
-        FloorDiv32::make((uint32_t)alpha_inv), delta, maxabs_gl, maxabs_wlr, maxabs_delta,
-        status);
+    int lg_kh = 0, lg_kw = 0;
+    while ((1 << lg_kh) < lp.kh) ++lg_kh;
+    while ((1 << lg_kw) < lp.kw) ++lg_kw;
+    const bool aligned = (((uintptr_t)am | (uintptr_t)region | (uintptr_t)delta |
+                           (uintptr_t)(g.pool ? argmax : region)) & 15) == 0;
+    if (g.cout % 4 == 0 && aligned && (1 << lg_kh) == lp.kh && (1 << lg_kw) == lp.kw) {
+        k_lrpool_to_delta4<<<grid_for(n / 4, 256), 256, 0, s>>>(
+            gl, wlr, G, d, g, lp, lg_kh, lg_kw, B, FloorDiv32::make((uint32_t)(g.cout / 4)),
+            FloorDiv32::make((uint32_t)g.w), FloorDiv32::make((uint32_t)g.h), am, argmax, region,
+            FloorDiv32::make((uint32_t)alpha_inv), delta, maxabs_gl, maxabs_wlr, maxabs_delta,
+            status);
+    } else {
+        k_lrpool_to_delta<<<grid_for(n, 256), 256, 0, s>>>(
+            gl, wlr, G, d, g, lp, B, am, argmax, region,
+            FloorDiv32::make((uint32_t)alpha_inv), delta, maxabs_gl, maxabs_wlr, maxabs_delta,
+            status);
+    }
     return cudaGetLastError();
 }
 

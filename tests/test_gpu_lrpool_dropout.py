@@ -69,6 +69,9 @@ def test_last_layer_without_pool_and_ragged_map():
     _run(blocks, 5, steps=3, input_shape=(10, 10, 3), d_lr=100)
     blocks = [_b([(C, 3, 16, 8, 8, 0)], 8 * 8 * 3), _b([], 8 * 8 * 16)]
     _run(blocks, 4, steps=2, input_shape=(8, 8, 3), d_lr=64)
+    # six channels: the one-channel-per-thread routing kernel
+    blocks = [_b([(C, 3, 6, 8, 8, 1)], 8 * 8 * 3), _b([], 4 * 4 * 6)]
+    _run(blocks, 5, steps=2, input_shape=(8, 8, 3), d_lr=20)
 
 
 def test_pooled_tensor_core_layers_and_many_classes():
