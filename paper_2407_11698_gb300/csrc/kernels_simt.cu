@@ -936,6 +936,125 @@ __global__ void __launch_bounds__(256) k_lr_backward(const int8_t* __restrict__ 
     }
 }
 
+// Same, four features per thread when the last layer's channel count is a
+// multiple of 4 (four consecutive features are then four channels of one
+// output position): thread (f4, u) takes features q0 + 4 f4 .. + 3 of sample
+// b0 + u.  The W_lr slice is staged in shared memory; the argmax codes and
+// the region bytes of the four channels are read as 4-byte words and the
+// delta written with 16-byte stores.  The dW_lr partials are those of
+// k_lr_backward.
+template <int GM>
+__global__ void __launch_bounds__(256) k_lr_backward4(const int8_t* __restrict__ a,
+                                                      const int32_t* __restrict__ gl,
+                                                      const int32_t* __restrict__ wlr, int B,
+                                                      int G, int d, LayerGeom lg, FloorDiv32 alpha,
+                                                      const int8_t* __restrict__ region,
+                                                      const int8_t* __restrict__ argmax,
+                                                      int32_t* __restrict__ delta,
+                                                      unsigned long long* __restrict__ dwlr,
+                                                      const uint32_t* maxabs_gl,
+                                                      const uint32_t* maxabs_wlr,
+                                                      uint32_t* maxabs_delta, uint32_t* status) {
+    __shared__ int32_t gls[kLbSamples][GM];
+    __shared__ int8_t as[kLbSamples][kLbQ];
+    __shared__ __align__(16) int32_t wsl[GM][kLbQ];
+    const int f4 = threadIdx.x & 15, u = threadIdx.x >> 4;
+    const int q0 = blockIdx.x * kLbQ, q = q0 + 4 * f4;
+    const int b0 = blockIdx.y * kLbSamples;
+    const int nb = min(kLbSamples, B - b0);
+    for (int i = threadIdx.x; i < kLbSamples * GM; i += blockDim.x) {
+        const int uu = i / GM, g = i % GM;
+        gls[uu][g] = (uu < nb && g < G) ? gl[(int64_t)(b0 + uu) * G + g] : 0;
+    }
+    for (int i = threadIdx.x; i < kLbSamples * kLbQ; i += blockDim.x) {
+        const int uu = i / kLbQ, qq = i % kLbQ;
+        as[uu][qq] = (uu < nb && q0 + qq < d) ? a[(int64_t)(b0 + uu) * d + q0 + qq] : (int8_t)0;
+    }
+    for (int i = threadIdx.x; i < GM * kLbQ; i += blockDim.x) {
+        const int g = i / kLbQ, qq = i % kLbQ;
+        wsl[g][qq] = (g < G && q0 + qq < d) ? wlr[(int64_t)g * d + q0 + qq] : 0;
+    }
+    if (blockIdx.x == 0 && blockIdx.y == 0 && threadIdx.x == 0 &&
+        int64_bound_exceeded(*maxabs_gl, *maxabs_wlr, G))
+        atomicOr(status, ST_OVERFLOW);
+    // loads of the delta path go out with the staging loads, before the barrier
+    const bool act = q < d && u < nb;      // d % 4 == 0: all four features valid
+    int64_t base = 0, dx = 0, dy = 0;
+    uint32_t amw = 0, r00 = 0, r01 = 0, r10 = 0, r11 = 0;
+    if (act) {
+        const int c = q % lg.cout;
+        const int r = q / lg.cout;
+        const int ox = r % lg.ow, oy = r / lg.ow;
+        const int64_t img = lg.pool ? (int64_t)lg.h * lg.w * lg.cout : (int64_t)d;
+        const int64_t p00 = lg.pool ? ((int64_t)(2 * oy) * lg.w + 2 * ox) * lg.cout + c : q;
+        dx = lg.cout;
+        dy = (int64_t)lg.w * lg.cout;
+        base = (b0 + u) * img + p00;
+        r00 = *reinterpret_cast<const uint32_t*>(region + base);
+        if (lg.pool) {
+            amw = *reinterpret_cast<const uint32_t*>(argmax + (int64_t)(b0 + u) * d + q);
+            r01 = *reinterpret_cast<const uint32_t*>(region + base + dx);
+            r10 = *reinterpret_cast<const uint32_t*>(region + base + dy);
+            r11 = *reinterpret_cast<const uint32_t*>(region + base + dy + dx);
+        }
+    }
+    __syncthreads();
+    // dW_lr partials: (g, q) pairs over the CTA's samples
+    for (int i = threadIdx.x; i < G * kLbQ; i += blockDim.x) {
+        const int g = i / kLbQ, qq = i - g * kLbQ;
+        if (q0 + qq >= d) continue;
+        long long t = 0;
+#pragma unroll
+        for (int uu = 0; uu < kLbSamples; ++uu) t += (long long)gls[uu][g] * as[uu][qq];
+        if (t != 0) atomicAdd(&dwlr[(int64_t)g * d + q0 + qq], (unsigned long long)t);
+    }
+    uint32_t mx = 0;
+    bool ovf = false;
+    if (act) {
+        uint64_t acc[4] = {0, 0, 0, 0};    // modulo 2^64, exact below the bound
+#pragma unroll
+        for (int g = 0; g < GM; ++g) {
+            const int4 w4 = *reinterpret_cast<const int4*>(&wsl[g][4 * f4]);
+            const int64_t gv = gls[u][g];
+            acc[0] += (uint64_t)(gv * w4.x);
+            acc[1] += (uint64_t)(gv * w4.y);
+            acc[2] += (uint64_t)(gv * w4.z);
+            acc[3] += (uint64_t)(gv * w4.w);
+        }
+        int32_t dv[4];
+        int code[4];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const int64_t g64 = (int64_t)acc[j];
+            ovf |= !fits_i32(g64);
+            const int32_t gs = (int32_t)g64;
+            // region byte at the recorded window position of channel j
+            code[j] = lg.pool ? (int)((amw >> (8 * j)) & 3u) : 0;
+            const uint32_t rsel = code[j] == 0 ? r00 : (code[j] == 1 ? r01 : (code[j] == 2 ? r10 : r11));
+            const int rg = (int8_t)(rsel >> (8 * j));
+            // NITRO-ReLU backward: piece 1 -> floor(g / alpha_inv), piece 2 -> g, else 0
+            dv[j] = rg == 1 ? alpha.floor_div(gs) : (rg == 2 ? gs : 0);
+            mx = max(mx, abs_u32(dv[j]));
+        }
+        if (lg.pool) {
+#pragma unroll
+            for (int k = 0; k < 4; ++k)
+                *reinterpret_cast<int4*>(delta + base + (k & 1) * dx + (k >> 1) * dy) =
+                    make_int4(code[0] == k ? dv[0] : 0, code[1] == k ? dv[1] : 0,
+                              code[2] == k ? dv[2] : 0, code[3] == k ? dv[3] : 0);
+        } else {
+            *reinterpret_cast<int4*>(delta + base) = make_int4(dv[0], dv[1], dv[2], dv[3]);
+        }
+    }
+#pragma unroll
+    for (int off = 16; off; off >>= 1) mx = max(mx, __shfl_xor_sync(kFull, mx, off));
+    ovf = __any_sync(kFull, ovf);
+    if ((threadIdx.x & 31) == 0) {
+        if (mx) atomicMax(maxabs_delta, mx);
+        if (ovf) atomicOr(status, ST_OVERFLOW);
+    }
+}
+
 inline int grid_for(int64_t n, int threads, int cap = 152 * 16) {
     int64_t g = (n + threads - 1) / threads;
     return (int)(g < 1 ? 1 : (g > cap ? cap : g));
@@ -1193,6 +1312,22 @@ cudaError_t simt_lr_backward(const int8_t* a, const int32_t* gl, const int32_t* 
     const FloorDiv32 al = FloorDiv32::make((uint32_t)(alpha_inv > 0 ? alpha_inv : 1));
     auto* dw64 = reinterpret_cast<unsigned long long*>(dwlr);
     const LayerGeom g0 = lg ? *lg : LayerGeom{};
+    // four features per thread: channel counts in multiples of 4 and
+    // 16-byte aligned code and delta buffers (this library's own)
+    const bool quad = lg && lg->cout % 4 == 0 && d % 4 == 0 &&
+                      (((uintptr_t)region | (uintptr_t)delta |
+                        (uintptr_t)(lg->pool ? argmax : region)) & 15) == 0;
+    if (quad) {
+        if (G <= 10)
+            k_lr_backward4<10><<<grid, 256, 0, s>>>(a, gl, wlr, B, G, d, g0, al, region, argmax,
+                                                    delta, dw64, maxabs_gl, maxabs_wlr,
+                                                    maxabs_delta, status);
+        else
+            k_lr_backward4<kLbMaxG><<<grid, 256, 0, s>>>(a, gl, wlr, B, G, d, g0, al, region,
+                                                         argmax, delta, dw64, maxabs_gl,
+                                                         maxabs_wlr, maxabs_delta, status);
+        return cudaGetLastError();
+    }
     if (G <= 10)
         k_lr_backward<10><<<grid, 256, 0, s>>>(a, gl, wlr, B, G, d, lg != nullptr, g0, al, region,
                                                argmax, delta, dw64, maxabs_gl, maxabs_wlr,

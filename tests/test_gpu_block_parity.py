@@ -139,6 +139,7 @@ def test_gamma_plateau_schedule_changes_updates_like_oracle():
 def test_other_class_counts():
     blocks = [_b([(L, 16, 8, 1, 1, 0)], 16), _b([], 8)]
     _run(blocks, 9, steps=3, num_classes=3)
+    _run(blocks, 9, steps=2, num_classes=16)     # widest fused learning-layer backward
     _run(blocks, 9, steps=2, num_classes=40)
 
 
