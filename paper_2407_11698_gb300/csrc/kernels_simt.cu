@@ -204,40 +204,54 @@ __global__ void k_fwd_epilogue(const int64_t* __restrict__ z, LayerGeom g, int B
 // ---------------------------------------------------------------------------
 constexpr int kLrSamples = 16;   // samples per CTA
 constexpr int kLpSlice = 128;    // features per CTA
+static_assert(kLpSlice == 16 * 8, "k_learn_partial: 16 lanes of 8 features per sample");
 
 __global__ void __launch_bounds__(256) k_learn_partial(const int8_t* __restrict__ a,
                                                        const int32_t* __restrict__ wlr, int B,
-                                                       int d, int G,
+                                                       int d, int G, int vec8,
                                                        unsigned long long* __restrict__ zsum,
                                                        FloorDiv dv, const int32_t* __restrict__ labels,
                                                        int32_t* __restrict__ grad_l,
                                                        unsigned long long* sse, int64_t* loss,
                                                        uint32_t* maxabs_gl, uint32_t* status) {
-    // thread (u, k): sample u of the group, features k, k + 16, ... of the slice;
-    // the slice of W_lr is staged in shared memory, classes in chunks of kLpG
+    // thread (u, k): sample u of the group, features 8k .. 8k + 7 of the slice,
+    // read as one 8-byte word when the rows allow it (vec8: d % 8 == 0 and an
+    // 8-byte aligned a).  The slice of W_lr is staged in shared memory with
+    // feature 8k + m at column 16m + k, so the lanes of a sample read
+    // consecutive words; classes in chunks of kLpG.
     constexpr int kLpG = 16;
     __shared__ int32_t ws[kLpG][kLpSlice + 1];
     const int u = threadIdx.x >> 4, k = threadIdx.x & 15;
     const int b = blockIdx.y * kLrSamples + u;
     const int j0 = blockIdx.x * kLpSlice;
-    int av[kLpSlice / 16];
+    const int jb = j0 + 8 * k;
+    int av[8];
+    if (vec8 && b < B && jb + 8 <= d) {
+        const uint2 w = *reinterpret_cast<const uint2*>(a + (int64_t)b * d + jb);
 #pragma unroll
-    for (int m = 0; m < kLpSlice / 16; ++m) {
-        const int j = j0 + k + 16 * m;
-        av[m] = (b < B && j < d) ? a[(int64_t)b * d + j] : 0;
+        for (int m = 0; m < 4; ++m) {
+            av[m] = (int8_t)(w.x >> (8 * m));
+            av[4 + m] = (int8_t)(w.y >> (8 * m));
+        }
+    } else {
+#pragma unroll
+        for (int m = 0; m < 8; ++m) {
+            const int j = jb + m;
+            av[m] = (b < B && j < d) ? a[(int64_t)b * d + j] : 0;
+        }
     }
     for (int gc = 0; gc < G; gc += kLpG) {
         const int ng = min(kLpG, G - gc);
         if (gc) __syncthreads();
         for (int i = threadIdx.x; i < ng * kLpSlice; i += blockDim.x) {
             const int g = i / kLpSlice, j = i - g * kLpSlice;
-            ws[g][j] = j0 + j < d ? wlr[(int64_t)(gc + g) * d + j0 + j] : 0;
+            ws[g][(j & 7) * 16 + (j >> 3)] = j0 + j < d ? wlr[(int64_t)(gc + g) * d + j0 + j] : 0;
         }
         __syncthreads();
         for (int g = 0; g < ng; ++g) {
             long long t = 0;
 #pragma unroll
-            for (int m = 0; m < kLpSlice / 16; ++m) t += (long long)ws[g][k + 16 * m] * av[m];
+            for (int m = 0; m < 8; ++m) t += (long long)ws[g][16 * m + k] * av[m];
 #pragma unroll
             for (int off = 8; off; off >>= 1) t += __shfl_xor_sync(kFull, t, off);
             if (k == 0 && b < B && t != 0)
@@ -1192,7 +1206,9 @@ cudaError_t simt_learn_fwd(const int8_t* a, const int32_t* wlr, const int32_t* l
     if (e != cudaSuccess) return e;
     dim3 grid((d + kLpSlice - 1) / kLpSlice, groups);
     ProfScope ps(K_LEARN_FWD, s, 2.0 * B * d * G, 0.0);
-    k_learn_partial<<<grid, 256, 0, s>>>(a, wlr, B, d, G, reinterpret_cast<unsigned long long*>(zsum),
+    const int vec8 = d % 8 == 0 && ((uintptr_t)a & 7) == 0;
+    k_learn_partial<<<grid, 256, 0, s>>>(a, wlr, B, d, G, vec8,
+                                         reinterpret_cast<unsigned long long*>(zsum),
                                          FloorDiv::make((uint64_t)d), labels, grad_l, sse, loss,
                                          maxabs_gl, status);
     return cudaGetLastError();
