@@ -84,13 +84,16 @@ def test_pooled_tensor_core_layers_and_many_classes():
 
 def test_pooled_block_exposes_window_geometry():
     blk = nb.Block([(C, 4, 16, 16, 16, 1)], 16 * 16 * 4, seed=3, max_batch=2, d_lr=256)
+    plain = nb.Block([(C, 4, 16, 16, 16, 1)], 16 * 16 * 4, seed=3, max_batch=2)
     try:
         # 16 x 8 x 8 = 1024 -> 2 x 1 -> 2 x 2: 16 x 4 x 4 = 256 learning inputs
         assert blk.get(nb.NITRO_T_WLR, 0).size == 10 * 256
+        # a block without learning-layer pooling has no pooled input to read
         with pytest.raises(nb.NitroError):
-            nb.Block([(C, 4, 16, 16, 16, 1)], 16 * 16 * 4, seed=3, max_batch=2).get(nb.NITRO_T_LR_IN)
+            plain.get(nb.NITRO_T_LR_IN)
     finally:
         blk.close()
+        plain.close()
 
 
 # ------------------------------------------------------- dropout
