@@ -116,3 +116,24 @@ def test_tensor_core_kernels_ran(c0):
         assert names["simt_conv_fwd"] == 0 and names["simt_conv_wgrad"] == 0
     finally:
         pair.close()
+
+
+def test_linear_tensor_core_weights_from_a_checkpoint():
+    """Weights written through set_tensor reach the tensor-core linear forward
+    (input width a multiple of 8): the layer's limb planes are rebuilt from the
+    new int32 weights, here widened to three limbs on both sides."""
+    blocks = [{"layers": [(nb.NITRO_LINEAR, 136, 64, 1, 1, 0)], "in_features": 136},
+              {"layers": [], "in_features": 64}]
+    pair = NetPair(blocks, 12, seed=8)
+    try:
+        x, y = synth.images(21, 0, 12, (136,)), synth.labels(21, 0, 12)
+        gl, ol = pair.step(x, y)
+        assert gl == ol
+        _widen(pair, 70001)      # max |W| 21 after one step -> 1.47e6: three limbs
+        for s in range(1, 3):
+            x, y = synth.images(21, s, 12, (136,)), synth.labels(21, s, 12)
+            gl, ol = pair.step(x, y)
+            assert gl == ol, (s, gl, ol)
+            pair.compare("step %d" % s)
+    finally:
+        pair.close()
