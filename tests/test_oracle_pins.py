@@ -583,3 +583,54 @@ def test_prep_gaussian_data_meets_the_stated_target():
     inside = norm.cdf(127, shift, sd) - norm.cdf(-127, shift, sd)
     assert abs(inside - 0.95) < 0.02
     assert abs((np.abs(xh) < 127).mean() - inside) < 0.01
+
+
+# ---------------------------------------------------------------- whole step
+@pytest.mark.parametrize("round_mode", [O.FLOOR, O.TRUNC])
+def test_block_step_worked_by_hand(golden, round_mode):
+    # one full training step of a one-layer linear block, every intermediate
+    # and the updated weights worked by hand (tests/golden/block_step_linear.txt)
+    rows = golden("block_step_linear.txt")
+    (a, w, wlr, lab, zs, region, a1, yhat, grad_l, sse_loss, dwlr, delta, dw,
+     w_floor, wlr_new, w_trunc) = rows
+    blk = O.OracleBlock([O.LayerDesc(O.LINEAR, 2, 2)], num_classes=2, alpha_inv=10,
+                        gamma_inv_lr=512, sgd_round=round_mode, seed=1)
+    blk.W[0] = np.array(w, dtype=np.int64).reshape(2, 2)
+    blk.Wlr = np.array(wlr, dtype=np.int64).reshape(2, 2)
+    losses = O.train_step([blk], np.array([a], dtype=np.int64), np.array(lab, dtype=np.int64))
+    assert losses == [sse_loss[1]] and blk.sse == sse_loss[0]
+    assert blk.zs[0].reshape(-1).tolist() == zs
+    assert blk.region[0].reshape(-1).tolist() == region
+    assert blk.act[0].reshape(-1).tolist() == a1
+    assert blk.yhat.reshape(-1).tolist() == yhat
+    assert blk.grad_l.reshape(-1).tolist() == grad_l
+    assert blk.dWlr.reshape(-1).tolist() == dwlr
+    assert blk.delta[0].reshape(-1).tolist() == delta
+    assert blk.dW[0].reshape(-1).tolist() == dw
+    assert blk.W[0].reshape(-1).tolist() == (w_floor if round_mode == O.FLOOR else w_trunc)
+    assert blk.Wlr.reshape(-1).tolist() == wlr_new
+    assert blk.status == 0
+
+
+def test_conv_block_step_worked_by_hand(golden):
+    # the conv counterpart: padding, scaling, pool routing and the 3x3 weight
+    # gradient of one full step, worked by hand (tests/golden/block_step_conv.txt)
+    (a, w, wlr, lab, zs, region, _relu, a1, am, yhat, grad_l, sse_loss, dwlr, delta, dw,
+     w_new, wlr_new) = golden("block_step_conv.txt")
+    blk = O.OracleBlock([O.LayerDesc(O.CONV, 1, 1, 2, 2, True)], num_classes=2, alpha_inv=10,
+                        gamma_inv_lr=512, seed=1)
+    blk.W[0] = np.array(w, dtype=np.int64).reshape(1, 3, 3, 1)
+    blk.Wlr = np.array(wlr, dtype=np.int64).reshape(2, 1)
+    losses = O.train_step([blk], np.array([a], dtype=np.int64), np.array(lab, dtype=np.int64))
+    assert losses == [sse_loss[1]] and blk.sse == sse_loss[0]
+    assert blk.zs[0].reshape(-1).tolist() == zs
+    assert blk.region[0].reshape(-1).tolist() == region
+    assert blk.act[0].reshape(-1).tolist() == a1
+    assert blk.argmax[0].reshape(-1).tolist() == am
+    assert blk.yhat.reshape(-1).tolist() == yhat
+    assert blk.grad_l.reshape(-1).tolist() == grad_l
+    assert blk.dWlr.reshape(-1).tolist() == dwlr
+    assert blk.delta[0].reshape(-1).tolist() == delta
+    assert blk.dW[0].reshape(-1).tolist() == dw
+    assert blk.W[0].reshape(-1).tolist() == w_new
+    assert blk.Wlr.reshape(-1).tolist() == wlr_new
