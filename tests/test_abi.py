@@ -127,3 +127,37 @@ def test_oracle_library_builds_independently():
     out = subprocess.run(["nm", "-D", "--defined-only", path], capture_output=True, text=True,
                          check=True).stdout
     assert not any(" nitro_" in l for l in out.splitlines())
+
+
+def test_binding_structs_match_the_header(tmp_path):
+    # sizes and field offsets of the C structs, as a C compiler lays them out
+    # from include/nitro.h, against the binding's ctypes mirrors
+    import shutil
+    cc = shutil.which("gcc") or shutil.which("cc")
+    if not cc:
+        pytest.skip("no C compiler")
+    fields = {
+        "nitro_layer_desc": [f for f, _ in nb.nitro_layer_desc._fields_],
+        "nitro_block_desc": [f for f, _ in nb.nitro_block_desc._fields_],
+    }
+    src = ["#include <stdio.h>", "#include <stddef.h>", '#include "nitro.h"', "int main(void) {"]
+    for st, fs in fields.items():
+        src.append('printf("%%s size %%zu\\n", "%s", sizeof(%s));' % (st, st))
+        for f in fs:
+            src.append('printf("%%s %%s %%zu\\n", "%s", "%s", offsetof(%s, %s));' % (st, f, st, f))
+    src += ["return 0;", "}"]
+    c = tmp_path / "layout.c"
+    c.write_text("\n".join(src) + "\n")
+    exe = tmp_path / "layout"
+    subprocess.run([cc, "-I", os.path.join(ROOT, "include"), str(c), "-o", str(exe)], check=True)
+    out = subprocess.run([str(exe)], capture_output=True, text=True, check=True).stdout.split("\n")
+    got = {}
+    for line in out:
+        parts = line.split()
+        if len(parts) == 3:
+            got[(parts[0], parts[1])] = int(parts[2])
+    for st, fs in fields.items():
+        cls = getattr(nb, st)
+        assert got[(st, "size")] == ctypes.sizeof(cls), st
+        for f in fs:
+            assert got[(st, f)] == getattr(cls, f).offset, (st, f)
