@@ -161,3 +161,30 @@ def test_binding_structs_match_the_header(tmp_path):
         assert got[(st, "size")] == ctypes.sizeof(cls), st
         for f in fs:
             assert got[(st, f)] == getattr(cls, f).offset, (st, f)
+
+
+def test_binding_constants_match_the_header(tmp_path):
+    # every enum value and status bit the binding mirrors, from the header
+    import shutil
+    cc = shutil.which("gcc") or shutil.which("cc")
+    if not cc:
+        pytest.skip("no C compiler")
+    names = [n for n in dir(nb) if n.startswith("NITRO_")]
+    bits = {"STATUS_BIT_OVERFLOW": "NITRO_STATUS_BIT_OVERFLOW",
+            "STATUS_BIT_BAD_LABEL": "NITRO_STATUS_BIT_BAD_LABEL",
+            "STATUS_BIT_TIMEOUT": "NITRO_STATUS_BIT_TIMEOUT"}
+    src = ["#include <stdio.h>", '#include "nitro.h"', "int main(void) {"]
+    for n in names:
+        src.append('printf("%s %%lld\\n", (long long)%s);' % (n, n))
+    for py, c in bits.items():
+        src.append('printf("%s %%lld\\n", (long long)%s);' % (py, c))
+    src += ["return 0;", "}"]
+    c = tmp_path / "consts.c"
+    c.write_text("\n".join(src) + "\n")
+    exe = tmp_path / "consts"
+    subprocess.run([cc, "-I", os.path.join(ROOT, "include"), str(c), "-o", str(exe)], check=True)
+    out = subprocess.run([str(exe)], capture_output=True, text=True, check=True).stdout
+    got = dict((l.split()[0], int(l.split()[1])) for l in out.splitlines() if l.strip())
+    assert len(names) >= 26          # statuses, kinds, rounding, contractions, 13 tensors
+    for n in names + list(bits):
+        assert got[n] == getattr(nb, n), n
