@@ -188,3 +188,20 @@ def test_binding_constants_match_the_header(tmp_path):
     assert len(names) >= 26          # statuses, kinds, rounding, contractions, 13 tensors
     for n in names + list(bits):
         assert got[n] == getattr(nb, n), n
+
+
+def test_product_package_never_reaches_the_oracle():
+    # the library and its binding share nothing with the oracle: no Python
+    # import of it, no include of its C file, no mention of its library
+    pkg = os.path.join(ROOT, "paper_2407_11698_gb300")
+    offenders = []
+    for dirpath, _, files in os.walk(pkg):
+        for fn in files:
+            if not fn.endswith((".py", ".cu", ".cuh", ".h", ".c", ".cpp")):
+                continue
+            path = os.path.join(dirpath, fn)
+            text = open(path, encoding="utf-8").read()
+            if re.search(r"^\s*(import oracle|from oracle\b)", text, flags=re.M) or \
+                    "nitro_oracle" in text or "libnitro_oracle" in text:
+                offenders.append(os.path.relpath(path, ROOT))
+    assert not offenders, offenders
