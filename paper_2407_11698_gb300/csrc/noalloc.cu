@@ -4,10 +4,11 @@
 // a host program that owns the whole device-memory budget (a serving process
 // or game engine with its own arena), real-time loops where allocation after
 // start-up is not allowed, and code that must not stall the device (cudaMalloc
-// and cudaFree may synchronise it).  For them this entry point runs the same
-// kernels as nitro_block_forward for one conv layer, but keeps the layer's
-// int64 pre-activations in a fixed array that is part of the library image
-// instead of in a block's workspace.
+// and cudaFree may synchronise it).  For them this entry point runs one conv
+// layer's forward on the CUDA-core kernels that nitro_block_forward uses for
+// layers off the tensor path (same results), but keeps the layer's int64
+// pre-activations in a fixed array that is part of the library image instead
+// of in a block's workspace.
 //
 // The array is a file-scope __device__ variable: every GPU that loads the
 // library holds kNoallocScratchElems * 8 bytes (16 MiB) until the process
@@ -66,7 +67,8 @@ extern "C" nitro_status nitro_conv3x3_forward_noalloc(
     LayerGeom g{NITRO_CONV3X3, cin, cout, h, w, pool2x2, pool2x2 ? h / 2 : h, pool2x2 ? w / 2 : w};
     // mu_int8 of NITRO-ReLU: floor-average of the four segment means
     const int mu = (int)fdiv64(fdiv64(-127, alpha_inv) + fdiv64(-127, 2 * alpha_inv) + 63 + 127, 4);
-    // The GEMM writes every element of z, so the array needs no clearing.
+    // The GEMM overwrites every element of z (directly, or by clearing it
+    // before adding K-split partial sums), so the array needs no clearing here.
     if (simt_gemm(GM_CONV_FWD, a_in, nullptr, weights, z, batch, h, w, cin, cout, s) != cudaSuccess)
         return NITRO_ERR_CUDA;
     if (simt_fwd_epilogue(z, g, batch, alpha_inv, mu, a_out, nullptr, region, argmax, s) !=
