@@ -1,12 +1,14 @@
 // CUDA-core kernels of the NITRO-D block step: an exact int64 implicit GEMM
 // for every contraction shape (conv 3x3 fwd / dgrad / wgrad, linear fwd /
 // dgrad / wgrad), and the element-wise stages fused around it (NITRO-Scaling,
-// NITRO-ReLU and max-pool forward; max-pool, NITRO-ReLU backward and STE;
-// learning layer and RSS loss; IntegerSGD).
+// NITRO-ReLU and max-pool forward, with dropout for linear layers; max-pool,
+// NITRO-ReLU backward and STE; the learning layer, its max-pool to d_lr and
+// the RSS loss; IntegerSGD).
 //
-// These serve the layers whose contraction is too narrow for the tensor-core
-// path (first layers with 1 or 3 input channels, MLP layers, learning layers
-// with G = 10 outputs) and are the exactness reference on the device.
+// The GEMM serves the contractions the tensor-core path does not take (narrow
+// or small layers, linear weight and input gradients, linear forwards whose
+// input width is not a multiple of 8); the learning layer (G = 10 outputs) and
+// the element-wise stages always run here.
 #include <cuda_bf16.h>
 
 #include "nitro_internal.cuh"
