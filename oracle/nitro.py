@@ -2,7 +2,8 @@
 
 Every arithmetic step is a call into ``nitro_oracle.c``; this file fixes the
 order of the steps, the shapes, and the points where a value is stored into its
-declared integer type.  Those storage rules are part of the definition the GPU
+declared integer type (the learning-pool window size and the selection of
+dropped activations are plain Python on the C results).  Those storage rules are part of the definition the GPU
 library must reproduce bit for bit:
 
 * activations are int8 (NITRO-ReLU output, Sec. 3.2.2);
