@@ -196,7 +196,8 @@ typedef enum {
     NITRO_T_GRAD_L = 8,  /* loss gradient [batch x G], int32 (layer = 0)       */
     NITRO_T_SSE = 9,     /* sum of squared errors, int64 [1] (layer = 0)       */
     NITRO_T_LR_IN = 10,  /* pooled learning-layer input z^mp [batch x d], int8
-                            (layer = 0; blocks with learning-layer pooling)    */
+                            (layer = 0; blocks with learning-layer pooling,
+                            NITRO_ERR_ARG for the others)                      */
     NITRO_T_LR_ARGMAX = 11, /* window position r*kw + s of each z^mp value,
                             uint8 [batch x d] (same blocks)                    */
     NITRO_T_STEP = 12    /* step counter of the dropout masks, uint32 [1]
