@@ -34,7 +34,8 @@ def parse():
     p.add_argument("--steps", type=int, default=20)
     p.add_argument("--warmup", type=int, default=5)
     p.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    p.add_argument("--workload", default=WORKLOAD)
+    from paper_2407_11698_gb300 import workloads as WL
+    p.add_argument("--workload", default=WORKLOAD, choices=sorted(WL.WORKLOADS))
     p.add_argument("--no-graph", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--sequential-blocks", action="store_true",
