@@ -274,14 +274,18 @@ void nitro_gemm_destroy(nitro_gemm* g);
  * (conv, NITRO-Scaling, NITRO-ReLU, optional 2x2 max-pool) on caller-owned
  * buffers: a_in int8 NHWC [batch x h x w x cin], weights int32 OHWI, a_out
  * int8 [batch x h' x w' x cout], region int8 [batch x h x w x cout], argmax
- * int8 [batch x h' x w' x cout] (pool2x2 only, else may be NULL).  It calls no
+ * int8 [batch x h' x w' x cout] (pool2x2 only, else may be NULL), where
+ * h' = pool2x2 ? floor(h / 2) : h and w' = pool2x2 ? floor(w / 2) : w (an odd
+ * last row or column is dropped by the pool, as in the block path).  It calls no
  * cudaMalloc, cudaFree or allocating library routine: the int64
  * pre-activations go to a fixed 16 MiB array inside the library, so
  * batch*h*w*cout may be at most 2^21; larger sizes return NITRO_ERR_ARG and
  * queue nothing.  Every GPU that loads the library holds that array until the
  * process exits.  The first call on each device looks up the array's address
- * (cudaGetSymbolAddress, with that device current); make that first call
- * before any stream capture.  All calls share the one array: calls whose work
+ * (cudaGetSymbolAddress, with that device current) and keeps it for the life
+ * of the process; make that first call before any stream capture.  Calls
+ * after a cudaDeviceReset of that device are not supported (the library image
+ * may be reloaded elsewhere).  All calls share the one array: calls whose work
  * overlaps on the GPU (different streams, or different host threads) race
  * and give wrong results; serialise them, e.g. on one stream. */
 nitro_status nitro_conv3x3_forward_noalloc(const int8_t* a_in, const int32_t* weights, int batch,
@@ -339,6 +343,20 @@ nitro_status nitro_profile_read(int id, uint64_t* launches, double* ms, double* 
  * Synchronises on that launch's events; NITRO_ERR_ARG for i out of range. */
 int nitro_profile_record_count(void);
 nitro_status nitro_profile_record(int i, int* kernel, double* ms, double* ops, double* bytes);
+
+/* Failure-path check of the bounded device waits (SURVEY's TIMEOUT contract;
+ * the paper has no counterpart: its failure model is integer overflow).
+ * Queues on `stream` one CTA that allocates TMEM as the contraction kernels do
+ * and waits, through their bounded mbarrier wait, on a barrier that nothing
+ * ever completes.  After wait_us microseconds the wait gives up: the kernel
+ * latches the TIMEOUT bit in b's status word, the CTA's other waiting warps
+ * see its abort flag and leave, TMEM is freed and the kernel returns, so the
+ * CUDA context stays usable and the block keeps its state.  The next
+ * nitro_block_status / nitro_block_get_tensor returns NITRO_ERR_TIMEOUT until
+ * the status is cleared (nitro_block_status(b, 1)).
+ * Errors: NITRO_ERR_ARG for a null handle or wait_us outside [1, 2000000];
+ * NITRO_ERR_CUDA for a failed launch. */
+nitro_status nitro_block_diag_timeout(nitro_block* b, int wait_us, void* stream);
 
 /* Static, human-readable name of a status code. */
 const char* nitro_status_str(nitro_status s);

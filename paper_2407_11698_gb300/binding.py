@@ -113,6 +113,8 @@ def lib():
     L.nitro_block_set_hyper.restype = ctypes.c_int
     L.nitro_block_set_dropout.argtypes = [_VP, ctypes.c_int]
     L.nitro_block_set_dropout.restype = ctypes.c_int
+    L.nitro_block_diag_timeout.argtypes = [_VP, ctypes.c_int, _VP]
+    L.nitro_block_diag_timeout.restype = ctypes.c_int
     L.nitro_prep_create.argtypes = [ctypes.POINTER(_VP)]
     L.nitro_prep_fit.argtypes = [_VP, _VP, ctypes.c_int64, _VP]
     L.nitro_prep_apply.argtypes = [_VP, _VP, ctypes.c_int64, _VP, _VP]
@@ -287,6 +289,12 @@ class Block:
 
     def status(self, clear=False):
         return nitro_block_status(self.h, clear)
+
+    def diag_timeout(self, wait_us, stream=None):
+        """Queue the bounded-wait failure check (nitro_block_diag_timeout)."""
+        st = lib().nitro_block_diag_timeout(self.h, int(wait_us), _stream_ptr(stream))
+        if st != NITRO_OK:
+            raise NitroError(st, "nitro_block_diag_timeout")
 
     def status_bits(self):
         return nitro_block_status_bits(self.h)

@@ -530,6 +530,12 @@ nitro_status nitro_integersgd_step(nitro_block* b, void* stream) {
     return NITRO_OK;
 }
 
+nitro_status nitro_block_diag_timeout(nitro_block* b, int wait_us, void* stream) {
+    if (!b || wait_us < 1 || wait_us > 2000000) return NITRO_ERR_ARG;
+    NITRO_TRY(tc_timeout_probe(w_status(b), (uint64_t)wait_us * 1000ull, (cudaStream_t)stream));
+    return NITRO_OK;
+}
+
 nitro_status nitro_block_tensor_bytes(const nitro_block* b, int which, int layer, size_t* bytes) {
     if (!b || !bytes) return NITRO_ERR_ARG;
     const int n = (int)b->L.size();

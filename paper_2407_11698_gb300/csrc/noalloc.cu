@@ -14,7 +14,9 @@
 // library holds kNoallocScratchElems * 8 bytes (16 MiB) until the process
 // exits.  Host code cannot use its name as a device address, so on the first
 // call on each device the entry point looks the address up with
-// cudaGetSymbolAddress (with that device current) and caches it.
+// cudaGetSymbolAddress (with that device current) and caches it for the life
+// of the process; a cudaDeviceReset of that device is therefore not supported
+// between calls.
 #include <mutex>
 
 #include "nitro_internal.cuh"

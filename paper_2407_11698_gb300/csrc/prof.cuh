@@ -39,6 +39,7 @@ enum KernelId : int {
     K_PREP_APPLY,
     K_LR_POOL,
     K_LRPOOL_TO_DELTA,
+    K_TC_PROBE,
     K_COUNT
 };
 

@@ -64,13 +64,13 @@ __device__ __forceinline__ uint64_t global_ns() {
 // Bounded wait: false when the time limit passed (TIMEOUT raised) or another
 // role of this CTA gave up.  The first test is inline; the polling loop is not.
 __device__ __noinline__ bool mbar_wait_slow(uint32_t bar, uint32_t parity, volatile int* abort_flag,
-                                            uint32_t* status) {
+                                            uint32_t* status, uint64_t limit_ns) {
     const uint64_t t0 = global_ns();
     for (uint32_t i = 1;; ++i) {
         if (mbar_try_wait(bar, parity)) return true;
         if ((i & 63) == 0) {
             if (*abort_flag) return false;
-            if (global_ns() - t0 > kWaitNs) {
+            if (global_ns() - t0 > limit_ns) {
                 *abort_flag = 1;
                 atomicOr(status, ST_TIMEOUT);
                 return false;
@@ -79,8 +79,8 @@ __device__ __noinline__ bool mbar_wait_slow(uint32_t bar, uint32_t parity, volat
     }
 }
 __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag,
-                                          uint32_t* status) {
-    return mbar_try_wait(bar, parity) || mbar_wait_slow(bar, parity, abort_flag, status);
+                                          uint32_t* status, uint64_t limit_ns = kWaitNs) {
+    return mbar_try_wait(bar, parity) || mbar_wait_slow(bar, parity, abort_flag, status, limit_ns);
 }
 
 __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* m, uint32_t bar,
@@ -311,6 +311,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     constexpr int NBUF = C::NBUF;
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * S + 2 * NBUF);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+    int* hiskip_slot = reinterpret_cast<int*>(tmem_slot + 2);
     int8_t* relu_tab = reinterpret_cast<int8_t*>(smem + S * C::STAGE + 256);   // 255 entries
     // bf16 bits of every int8 value v, at index (v + 128) = byte ^ 0x80
     uint16_t* bf16_tab = reinterpret_cast<uint16_t*>(smem + S * C::STAGE + 512);
@@ -332,6 +333,13 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_init(tempty_bar(b), kEpiWarps);
         }
         *abort_flag = 0;
+        // Fused input gradient: the lower delta is stored as the low 32 bits of
+        // the exact sum, and limb pairs with la + lb >= 4 only add multiples
+        // of 2^32.  They matter only for deciding OVERFLOW, so once that bit
+        // is latched they are skipped.  Read once per CTA so that all roles
+        // walk the same passes (CTAs may differ; each result is the same).
+        *hiskip_slot = (MODE == TC_DGRAD && args.fuse)
+            ? ((*reinterpret_cast<volatile uint32_t*>(args.status) & ST_OVERFLOW) != 0) : 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
     // int32 x int32 contraction: flag when max|delta| max|W| 9 Cout >= 2^63
@@ -357,8 +365,9 @@ __global__ void __launch_bounds__(kThreads, 1)
 
     const int LA = args.max_a ? limb_count(*args.max_a) : 1;
     const int LB = args.max_b ? limb_count(*args.max_b) : 1;
-    const int NG = (LB + PB - 1) / PB;       // groups of B limbs per A limb
-    const int passes = LA * NG;
+    const int hiskip = *hiskip_slot;
+    // B limbs that pair with A limb la: all, or those with la + lb <= 3
+    auto lb_limit = [&](int la) { return hiskip ? min(LB, 4 - la) : LB; };
 
     if (warp == 0) {
         if (lane == 0) {
@@ -385,9 +394,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                         wa_dy[j] = t / 3 - 1;
                     }
                 }
-                for (int p = 0; p < passes; ++p) {
-                    const int la = p / NG, lb0 = (p % NG) * PB;
-                    const int nb = min(PB, LB - lb0);
+                for (int la = 0; la < LA; ++la)
+                for (int lb0 = 0; lb0 < lb_limit(la); lb0 += PB) {
+                    const int nb = min(PB, lb_limit(la) - lb0);
                     // weight gradient: K-block kb = pixel box (xt, yt) of image bk,
                     // walked incrementally
                     int wxt = 0, wyt = 0, wbk = 0;
@@ -476,11 +485,16 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int tile = blockIdx.x; tile < args.total_tiles; tile += gridDim.x) {
                 const Tile T = decode_tile(args, tile);
                 const int cpp = (T.kb1 - T.kb0 + kChunkBlocks - 1) / kChunkBlocks;
-                for (int p = 0; p < passes; ++p) {
-                    const int nb = min(PB, LB - (p % NG) * PB);
-                    // MN-major B holds [64-channel block][PB limbs]: the MMA spans all
-                    // of them (unused limbs cost MMA time, not correctness)
-                    const uint32_t idesc = (MODE == TC_WGRAD || MODE == TC_DGRAD) ? idesc_nb[PB] : idesc_nb[nb];
+                for (int la = 0; la < LA; ++la)
+                for (int lb0 = 0; lb0 < lb_limit(la); lb0 += PB) {
+                    const int nb = min(PB, lb_limit(la) - lb0);
+                    // one MMA of width nb * N over the pass's limb tiles.  MN-major B
+                    // holds [64-channel block h][PB limbs] in 8 KB blocks: the first
+                    // nb limbs of a 64-wide tile are adjacent; with two channel blocks
+                    // and nb < PB the used blocks are PB * 8 KB apart (leading byte
+                    // offset), and their accumulators land side by side.
+                    const uint32_t idesc = idesc_nb[nb];
+                    const uint32_t b_lbo = (N > 64 && nb < PB) ? PB * 64 * 128 : 64 * 128;
                     for (int c = 0; c < cpp; ++c, ++chunk) {
                         const int buf = chunk % NBUF;
                         if (!mbar_wait(tempty_bar(buf), ((chunk / NBUF) & 1) ^ 1, abort_flag,
@@ -504,7 +518,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                             constexpr bool a_mn = MODE == TC_WGRAD;
                             constexpr bool b_mn = MODE == TC_WGRAD || MODE == TC_DGRAD;
                             const uint64_t da0 = a_mn ? desc_sw128_mn(a_addr, 64 * 128) : desc_sw128(a_addr);
-                            const uint64_t db0 = b_mn ? desc_sw128_mn(b_addr, 64 * 128) : desc_sw128(b_addr);
+                            const uint64_t db0 = b_mn ? desc_sw128_mn(b_addr, b_lbo) : desc_sw128(b_addr);
 #pragma unroll
                             for (int k = 0; k < kBK / 16; ++k)
                                 umma_bf16(d, da0 + (uint64_t)k * (a_mn ? 2048 / 16 : 32 / 16),
@@ -529,21 +543,22 @@ __global__ void __launch_bounds__(kThreads, 1)
             uint64_t acc[NH];
 #pragma unroll
             for (int i = 0; i < NH; ++i) acc[i] = 0;
-            for (int p = 0; p < passes; ++p) {
-                const int lb0 = (p % NG) * PB;
-                const int nb = min(PB, LB - lb0);
-                const int shift0 = 8 * (p / NG + lb0);
+            for (int la = 0; la < LA; ++la)
+            for (int lb0 = 0; lb0 < lb_limit(la); lb0 += PB) {
+                const int nb = min(PB, lb_limit(la) - lb0);
+                const int pbw = nb < PB ? nb : PB;   // MN-major: limb blocks per channel block
+                const int shift0 = 8 * (la + lb0);
                 for (int c = 0; c < cpp; ++c, ++chunk) {
                     const int buf = chunk % NBUF;
                     if (!mbar_wait(tfull_bar(buf), (chunk / NBUF) & 1, abort_flag, args.status))
                         goto epi_done;
                     tc_fence_after();
                     // K-major B: limb-major columns; MN-major B: 64-column blocks
-                    // ordered [channel block][limb]
+                    // ordered [channel block][limb of this pass]
                     auto limb_base = [&](int jb) -> uint32_t {
                         const int hb = (half * NH) / 64;
                         const int colj = (MODE == TC_WGRAD || MODE == TC_DGRAD)
-                            ? (hb * PB + jb) * 64 + (half * NH - hb * 64)
+                            ? (hb * pbw + jb) * 64 + (half * NH - hb * 64)
                             : jb * N + half * NH;
                         return tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(buf * PB * N + colj);
                     };
@@ -828,6 +843,50 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (warp == 1) {
         tc_fence_after();
         asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(C::TCOLS)
+                     : "memory");
+    }
+}
+
+// ------------------------------------------------------------------ timeout probe
+// Exercises the failure path of the bounded waits without a fault: the CTA
+// holds TMEM like the contraction kernel, warp 0 waits on an mbarrier that
+// nothing ever completes with a short limit, gives up, raises TIMEOUT and the
+// abort flag; warps 1 and 2 wait on another such barrier under the kernel's
+// normal limit and leave when they see the flag.  TMEM is then freed and the
+// kernel returns, so the context stays usable.
+__global__ void __launch_bounds__(96, 1) k_tc_wait_probe(uint32_t* status, uint64_t limit_ns) {
+    __shared__ __align__(8) uint64_t bars[2];
+    __shared__ uint32_t tmem_slot;
+    __shared__ int abort_s;
+    volatile int* abort_flag = &abort_s;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (threadIdx.x == 0) {
+        mbar_init(smem_u32(&bars[0]), 1);
+        mbar_init(smem_u32(&bars[1]), 1);
+        *abort_flag = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    if (warp == 1) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                         smem_u32(&tmem_slot)),
+                     "r"(32)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = tmem_slot;
+    if (lane == 0) {
+        // phase 0 of a fresh barrier never completes: both waits must give up
+        if (warp == 0) mbar_wait(smem_u32(&bars[0]), 0, abort_flag, status, limit_ns);
+        else mbar_wait(smem_u32(&bars[1]), 0, abort_flag, status);
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(32)
                      : "memory");
     }
 }
@@ -1425,6 +1484,12 @@ cudaError_t tc_conv_dgrad(TcLayer& t, const LayerGeom& g, int batch, int64_t* g6
         *fused = a.fuse != 0;
     }
     return e;
+}
+
+cudaError_t tc_timeout_probe(uint32_t* status, uint64_t limit_ns, cudaStream_t s) {
+    ProfScope ps(K_TC_PROBE, s, 0.0, 0.0);
+    k_tc_wait_probe<<<1, 96, 0, s>>>(status, limit_ns);
+    return cudaGetLastError();
 }
 
 // ------------------------------------------------------------------ plain GEMM

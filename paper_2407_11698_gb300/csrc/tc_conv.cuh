@@ -128,6 +128,11 @@ cudaError_t tc_conv_dgrad(TcLayer& t, const LayerGeom& g, int batch, int64_t* g6
                           const TcDgradOut* fo, uint32_t* status, cudaStream_t s, bool* done,
                           bool* fused);
 
+// One CTA that holds TMEM and waits, through the contraction kernel's bounded
+// mbarrier wait, on a barrier nothing completes: after limit_ns it raises
+// ST_TIMEOUT in *status, frees TMEM and returns.
+cudaError_t tc_timeout_probe(uint32_t* status, uint64_t limit_ns, cudaStream_t s);
+
 // Helpers of the kernel-level entry points (contract.cu).
 cudaError_t tc_maxabs(const int32_t* x, int64_t n, uint32_t* out, cudaStream_t s);
 cudaError_t tc_pack_int8(const int8_t* x, int64_t rows, int cols, uint16_t* out, cudaStream_t s);
