@@ -528,7 +528,8 @@ __global__ void k_lrpool_to_delta4(const int32_t* __restrict__ gl, const int32_t
                                    const int8_t* __restrict__ region, FloorDiv32 alpha,
                                    int32_t* __restrict__ delta, const uint32_t* maxabs_gl,
                                    const uint32_t* maxabs_wlr, uint32_t* maxabs_delta,
-                                   uint32_t* status) {
+                                   uint32_t* status, uint16_t* __restrict__ planes,
+                                   int64_t plane) {
     const int C = g.cout, C4 = g.cout >> 2;
     const uint32_t n4 = (uint32_t)B * g.h * g.w * C4;
     if (blockIdx.x == 0 && threadIdx.x == 0 && int64_bound_exceeded(*maxabs_gl, *maxabs_wlr, G))
@@ -579,6 +580,7 @@ __global__ void k_lrpool_to_delta4(const int32_t* __restrict__ gl, const int32_t
             }
         }
         reinterpret_cast<int4*>(delta)[i] = make_int4(v[0], v[1], v[2], v[3]);
+        if (planes) store_delta_planes4(planes + 4 * (int64_t)i, plane, v[0], v[1], v[2], v[3]);
     }
 #pragma unroll
     for (int off = 16; off; off >>= 1) mx = max(mx, __shfl_xor_sync(kFull, mx, off));
@@ -970,7 +972,9 @@ __global__ void __launch_bounds__(256) k_lr_backward4(const int8_t* __restrict__
                                                       unsigned long long* __restrict__ dwlr,
                                                       const uint32_t* maxabs_gl,
                                                       const uint32_t* maxabs_wlr,
-                                                      uint32_t* maxabs_delta, uint32_t* status) {
+                                                      uint32_t* maxabs_delta, uint32_t* status,
+                                                      uint16_t* __restrict__ planes,
+                                                      int64_t plane) {
     __shared__ int32_t gls[kLbSamples][GM];
     __shared__ int8_t as[kLbSamples][kLbQ];
     __shared__ __align__(16) int32_t wsl[GM][kLbQ];
@@ -1054,12 +1058,16 @@ __global__ void __launch_bounds__(256) k_lr_backward4(const int8_t* __restrict__
         }
         if (lg.pool) {
 #pragma unroll
-            for (int k = 0; k < 4; ++k)
-                *reinterpret_cast<int4*>(delta + base + (k & 1) * dx + (k >> 1) * dy) =
-                    make_int4(code[0] == k ? dv[0] : 0, code[1] == k ? dv[1] : 0,
-                              code[2] == k ? dv[2] : 0, code[3] == k ? dv[3] : 0);
+            for (int k = 0; k < 4; ++k) {
+                const int64_t o = base + (k & 1) * dx + (k >> 1) * dy;
+                const int4 w = make_int4(code[0] == k ? dv[0] : 0, code[1] == k ? dv[1] : 0,
+                                         code[2] == k ? dv[2] : 0, code[3] == k ? dv[3] : 0);
+                *reinterpret_cast<int4*>(delta + o) = w;
+                if (planes) store_delta_planes4(planes + o, plane, w.x, w.y, w.z, w.w);
+            }
         } else {
             *reinterpret_cast<int4*>(delta + base) = make_int4(dv[0], dv[1], dv[2], dv[3]);
+            if (planes) store_delta_planes4(planes + base, plane, dv[0], dv[1], dv[2], dv[3]);
         }
     }
 #pragma unroll
@@ -1167,7 +1175,9 @@ cudaError_t simt_lrpool_to_delta(const int32_t* gl, const int32_t* wlr, int G, i
                                  const uint8_t* am, const int8_t* argmax, const int8_t* region,
                                  int alpha_inv, int32_t* delta, const uint32_t* maxabs_gl,
                                  const uint32_t* maxabs_wlr, uint32_t* maxabs_delta,
-                                 uint32_t* status, cudaStream_t s) {
+                                 uint32_t* status, cudaStream_t s, uint16_t* planes,
+                                 int64_t plane, bool* planes_done) {
+    if (planes_done) *planes_done = false;
     const int64_t n = (int64_t)B * g.h * g.w * g.cout;
     if (n <= 0) return cudaSuccess;
     if (g.kind != NITRO_CONV3X3 || lp.ph * lp.kh > g.oh || lp.pw * lp.kw > g.ow ||
@@ -1188,7 +1198,8 @@ cudaError_t simt_lrpool_to_delta(const int32_t* gl, const int32_t* wlr, int G, i
             gl, wlr, G, d, g, lp, lg_kh, lg_kw, B, FloorDiv32::make((uint32_t)(g.cout / 4)),
             FloorDiv32::make((uint32_t)g.w), FloorDiv32::make((uint32_t)g.h), am, argmax, region,
             FloorDiv32::make((uint32_t)alpha_inv), delta, maxabs_gl, maxabs_wlr, maxabs_delta,
-            status);
+            status, planes, plane);
+        if (planes_done) *planes_done = planes != nullptr;
     } else {
         k_lrpool_to_delta<<<grid_for(n, 256), 256, 0, s>>>(
             gl, wlr, G, d, g, lp, B, am, argmax, region,
@@ -1318,10 +1329,13 @@ cudaError_t simt_lr_backward(const int8_t* a, const int32_t* gl, const int32_t* 
                              int d, const LayerGeom* lg, int alpha_inv, const int8_t* region,
                              const int8_t* argmax, int32_t* delta, int64_t* dwlr,
                              const uint32_t* maxabs_gl, const uint32_t* maxabs_wlr,
-                             uint32_t* maxabs_delta, uint32_t* status, cudaStream_t s) {
+                             uint32_t* maxabs_delta, uint32_t* status, cudaStream_t s,
+                             uint16_t* planes, int64_t plane, bool* planes_done) {
+    if (planes_done) *planes_done = false;
     cudaError_t e = cudaMemsetAsync(dwlr, 0, sizeof(int64_t) * (size_t)G * d, s);
     if (e != cudaSuccess || B <= 0) return e;
-    if (lg && lg->pool && ((lg->h & 1) || (lg->w & 1))) {   // rows / columns the pool dropped
+    const bool dropped = lg && lg->pool && ((lg->h & 1) || (lg->w & 1));
+    if (dropped) {   // rows / columns the pool dropped
         e = cudaMemsetAsync(delta, 0, sizeof(int32_t) * (size_t)B * lg->h * lg->w * lg->cout, s);
         if (e != cudaSuccess) return e;
     }
@@ -1336,14 +1350,20 @@ cudaError_t simt_lr_backward(const int8_t* a, const int32_t* gl, const int32_t* 
                       (((uintptr_t)region | (uintptr_t)delta |
                         (uintptr_t)(lg->pool ? argmax : region)) & 15) == 0;
     if (quad) {
+        if (planes && dropped) {
+            e = cudaMemsetAsync(planes, 0, 2 * (size_t)plane * 4, s);
+            if (e != cudaSuccess) return e;
+        }
         if (G <= 10)
             k_lr_backward4<10><<<grid, 256, 0, s>>>(a, gl, wlr, B, G, d, g0, al, region, argmax,
                                                     delta, dw64, maxabs_gl, maxabs_wlr,
-                                                    maxabs_delta, status);
+                                                    maxabs_delta, status, planes, plane);
         else
             k_lr_backward4<kLbMaxG><<<grid, 256, 0, s>>>(a, gl, wlr, B, G, d, g0, al, region,
                                                          argmax, delta, dw64, maxabs_gl,
-                                                         maxabs_wlr, maxabs_delta, status);
+                                                         maxabs_wlr, maxabs_delta, status, planes,
+                                                         plane);
+        if (planes_done) *planes_done = planes != nullptr;
         return cudaGetLastError();
     }
     if (G <= 10)

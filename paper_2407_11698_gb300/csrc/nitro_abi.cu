@@ -393,6 +393,17 @@ nitro_status nitro_block_backward(nitro_block* b, const int8_t* a_in, const int3
         return NITRO_OK;
     }
     const int8_t* a_last = n ? b->L[n - 1].act : a_in;
+    // layers whose delta limb planes were written by the kernel producing delta
+    std::vector<char> planes_done(n > 0 ? n : 1, 0);
+    bool pd = false;
+    auto delta_planes = [&](int i, uint16_t** p, int64_t* plane) {
+        const Layer& ly = b->L[i];
+        *p = tc_delta_planes(ly.tc);
+        *plane = (int64_t)batch * ly.g.h * ly.g.w * ly.g.cout;
+    };
+    uint16_t* last_planes = nullptr;
+    int64_t last_plane = 0;
+    if (n) delta_planes(n - 1, &last_planes, &last_plane);
     if (b->zmp) {
         // z^mp: the block output max-pooled for the learning layer (Sec. 3.3)
         const LayerGeom& lg = b->L[n - 1].g;
@@ -414,7 +425,9 @@ nitro_status nitro_block_backward(nitro_block* b, const int8_t* a_in, const int3
         Layer& ly = b->L[n - 1];
         NITRO_TRY(simt_lrpool_to_delta(b->grad_l, b->Wlr, G, (int)d, ly.g, b->lp, batch, b->lr_am,
                                        ly.argmax, ly.region, b->desc.alpha_inv, ly.delta, w_gl(b),
-                                       w_wlr(b), w_delta(b, n - 1), w_status(b), s));
+                                       w_wlr(b), w_delta(b, n - 1), w_status(b), s, last_planes,
+                                       last_plane, &pd));
+        planes_done[n - 1] = pd;
     } else if (simt_lr_backward_ok(G)) {
         // learning-weight gradient and (below a forward layer) delta_fw -> that
         // layer's delta in one pass
@@ -422,7 +435,9 @@ nitro_status nitro_block_backward(nitro_block* b, const int8_t* a_in, const int3
         NITRO_TRY(simt_lr_backward(a_last, b->grad_l, b->Wlr, batch, G, (int)d, ly ? &ly->g : nullptr,
                                    b->desc.alpha_inv, ly ? ly->region : nullptr,
                                    ly ? ly->argmax : nullptr, ly ? ly->delta : nullptr, b->dWlr,
-                                   w_gl(b), w_wlr(b), n ? w_delta(b, n - 1) : nullptr, w_status(b), s));
+                                   w_gl(b), w_wlr(b), n ? w_delta(b, n - 1) : nullptr, w_status(b), s,
+                                   last_planes, last_plane, &pd));
+        if (n) planes_done[n - 1] = pd;
     } else {
         NITRO_TRY(simt_learn_dw(a_last, b->grad_l, batch, (int)d, G, b->dWlr, s));
     }
@@ -441,7 +456,8 @@ nitro_status nitro_block_backward(nitro_block* b, const int8_t* a_in, const int3
         const LayerGeom& g = ly.g;
         const int8_t* x = i ? b->L[i - 1].act : a_in;
         bool done = false;
-        NITRO_TRY(tc_conv_wgrad(ly.tc, g, ly.delta, w_delta(b, i), batch, ly.dW, w_status(b), s, &done));
+        NITRO_TRY(tc_conv_wgrad(ly.tc, g, ly.delta, w_delta(b, i), batch, ly.dW, w_status(b), s, &done,
+                                planes_done[i] != 0));
         if (!done && simt_small_conv_ok(g)) {
             NITRO_TRY(simt_conv_small_wgrad(x, ly.delta, g, batch, ly.dW, s));
             done = true;
@@ -455,7 +471,7 @@ nitro_status nitro_block_backward(nitro_block* b, const int8_t* a_in, const int3
         bool fused = false;
         Layer& lo = b->L[i - 1];
         TcDgradOut fo{b->desc.alpha_inv, w_delta(b, i), w_w(b, i), lo.g.h, lo.g.w, lo.g.pool,
-                      lo.region, lo.argmax, lo.delta, w_delta(b, i - 1)};
+                      lo.region, lo.argmax, lo.delta, w_delta(b, i - 1), tc_delta_planes(lo.tc)};
         // the fused epilogue needs the lower layer to be a conv on the same grid
         const bool can_fuse = lo.g.kind == NITRO_CONV3X3 && lo.g.oh == g.h && lo.g.ow == g.w;
         NITRO_TRY(tc_conv_dgrad(ly.tc, g, batch, b->z64, can_fuse ? &fo : nullptr, w_status(b), s,
@@ -464,7 +480,10 @@ nitro_status nitro_block_backward(nitro_block* b, const int8_t* a_in, const int3
             const int mode = g.kind == NITRO_CONV3X3 ? GM_CONV_DGRAD : GM_LIN_DGRAD;
             NITRO_TRY(simt_gemm(mode, nullptr, ly.delta, ly.W, b->z64, batch, g.h, g.w, g.cin, g.cout, s));
         }
-        if (fused) continue;
+        if (fused) {
+            planes_done[i - 1] = fo.low_planes != nullptr;
+            continue;
+        }
         DeltaSrc src{};
         src.g64 = b->z64;
         src.maxabs_a = w_delta(b, i); src.maxabs_b = w_w(b, i);

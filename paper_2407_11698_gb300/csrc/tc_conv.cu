@@ -27,8 +27,16 @@ enum TcMode : int { TC_FWD = 0, TC_WGRAD = 1, TC_DGRAD = 2, TC_GEMM = 3 };
 constexpr int kBM = 128;              // rows per tile (TMEM lanes)
 constexpr int kBK = 64;               // K elements per block (one 128-byte row)
 constexpr int kChunkBlocks = 16;      // 16 x 64 = 1024 products per exact chunk
-constexpr int kEpiWarps = 16;         // 4 per TMEM lane quadrant
-constexpr int kThreads = 64 + 32 * kEpiWarps;   // TMA warp, MMA warp, epilogue
+// Warp roles: warpgroup 0 = TMA warp, MMA warp and two idle warps; warpgroups
+// 1 and 2 = the epilogue, two warps per TMEM lane quadrant, each holding half
+// of the N columns as int64 accumulators.  The warpgroups split the register
+// file with setmaxnreg: 128 x kRegsProducer + 256 x kRegsEpilogue must not
+// exceed kThreads x the registers the kernel is launched with (checked on the
+// host before the first launch).
+constexpr int kEpiWarp0 = 4;          // first epilogue warp
+constexpr int kEpiWarps = 8;          // 2 per TMEM lane quadrant
+constexpr int kThreads = 32 * (kEpiWarp0 + kEpiWarps);
+constexpr int kRegsProducer = 48, kRegsEpilogue = 224;
 constexpr uint64_t kWaitNs = 2000000000ull;   // 2 s bound on any wait
 
 // ------------------------------------------------------------------ PTX
@@ -62,8 +70,9 @@ __device__ __forceinline__ uint64_t global_ns() {
 }
 
 // Bounded wait: false when the time limit passed (TIMEOUT raised) or another
-// role of this CTA gave up.  The first test is inline; the polling loop is not.
-__device__ __noinline__ bool mbar_wait_slow(uint32_t bar, uint32_t parity, volatile int* abort_flag,
+// role of this CTA gave up.  Inlined: a function call cannot sit inside the
+// register-split (setmaxnreg) regions of the contraction kernel.
+__device__ __forceinline__ bool mbar_wait_slow(uint32_t bar, uint32_t parity, volatile int* abort_flag,
                                             uint32_t* status, uint64_t limit_ns) {
     const uint64_t t0 = global_ns();
     for (uint32_t i = 1;; ++i) {
@@ -180,15 +189,20 @@ __device__ __forceinline__ void tmem_ld16_nowait(uint32_t taddr, uint32_t* r) {
           "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
         : "r"(taddr));
 }
-__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
-    asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, "
-        "%11, %12, %13, %14, %15}, [%16];"
-        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
-          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
-          "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
-        : "r"(taddr));
+
+// Wait for this thread's outstanding tcgen05.ld, then mark the n destination
+// registers as written here, so that no use of them is placed before the wait.
+__device__ __forceinline__ void reg_touch16(uint32_t* r) {
+    asm volatile(""
+                 : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]),
+                   "+r"(r[6]), "+r"(r[7]), "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]),
+                   "+r"(r[12]), "+r"(r[13]), "+r"(r[14]), "+r"(r[15]));
+}
+template <int n>
+__device__ __forceinline__ void tmem_wait_ld(uint32_t* r) {
     asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+    for (int j = 0; j < n / 16; ++j) reg_touch16(r + 16 * j);
 }
 
 // Limbs of a tensor with max |x| = m.  The split is canonical: limbs 0..2 are
@@ -240,6 +254,8 @@ struct TcArgs {
     const int8_t* low_argmax;
     int32_t* low_delta;
     uint32_t* low_maxabs;
+    uint16_t* low_planes;      // the lower delta's bf16 limb planes, or null
+    int64_t low_plane;
 };
 
 // 16 int8 values (4 packed words) -> one 16-byte store
@@ -302,7 +318,7 @@ __global__ void __launch_bounds__(kThreads, 1)
               const TcArgs args) {
     using C = TcCfg<N, PB>;
     constexpr int S = C::S;
-    constexpr int NH = N / 4;            // columns per epilogue warp
+    constexpr int NH = N / 2;            // columns per epilogue warp
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
@@ -347,10 +363,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         int64_bound_exceeded(*args.bound_a, *args.bound_b, 9LL * args.Cout))
         atomicOr(args.status, ST_OVERFLOW);
     // NITRO-ReLU value of every z* in [-127, 127] (fused forward epilogue)
-    if (MODE == TC_FWD && args.fuse && threadIdx.x >= 64 && threadIdx.x < 64 + 255)
-        relu_tab[threadIdx.x - 64] = (int8_t)relu_value((int64_t)threadIdx.x - 64 - 127, args.alpha, args.mu);
-    if (MODE == TC_FWD && args.fuse && threadIdx.x >= 320 && threadIdx.x < 320 + 256)
-        bf16_tab[threadIdx.x - 320] = __bfloat16_as_ushort(__float2bfloat16_rn((float)((int)threadIdx.x - 320 - 128)));
+    if (MODE == TC_FWD && args.fuse) {
+        for (int i = threadIdx.x; i < 255; i += kThreads)
+            relu_tab[i] = (int8_t)relu_value((int64_t)i - 127, args.alpha, args.mu);
+        for (int i = threadIdx.x; i < 256; i += kThreads)
+            bf16_tab[i] = __bfloat16_as_ushort(__float2bfloat16_rn((float)(i - 128)));
+    }
     if (warp == 1) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
                          smem_u32(tmem_slot)),
@@ -369,6 +387,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     // B limbs that pair with A limb la: all, or those with la + lb <= 3
     auto lb_limit = [&](int la) { return hiskip ? min(LB, 4 - la) : LB; };
 
+    if (warp < kEpiWarp0) {
+    // warpgroup 0 gives registers back, then splits into its roles
+    asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kRegsProducer));
     if (warp == 0) {
         if (lane == 0) {
             // ---------------- TMA producer
@@ -532,10 +553,12 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
         mma_done:;
         }
+    }
     } else {
-        // ---------------- epilogue: warps 2..17
-        const int q = warp & 3;             // TMEM lane quadrant this warp may read
-        const int half = (warp - 2) >> 2;   // which quarter of the N columns
+        // ---------------- epilogue: warpgroups 1 and 2
+        asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(kRegsEpilogue));
+        const int q = warp & 3;                     // TMEM lane quadrant this warp may read
+        const int half = (warp - kEpiWarp0) >> 2;   // which half of the N columns
         int chunk = 0;
         for (int tile = blockIdx.x; tile < args.total_tiles; tile += gridDim.x) {
             const Tile T = decode_tile(args, tile);
@@ -580,25 +603,18 @@ __global__ void __launch_bounds__(kThreads, 1)
                             }
                         }
                     };
-                    if (NH == 16) {
-                        // 16 columns per limb: two limbs per TMEM round trip
-                        for (int jb = 0; jb < nb; jb += 2) {
-                            uint32_t r0[16], r1[16];
-                            tmem_ld16_nowait(limb_base(jb), r0);
-                            if (jb + 1 < nb) tmem_ld16_nowait(limb_base(jb + 1), r1);
-                            asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-                            accumulate(r0, 0, shift0 + 8 * jb);
-                            if (jb + 1 < nb) accumulate(r1, 0, shift0 + 8 * (jb + 1));
-                        }
-                    } else {
-                        for (int jb = 0; jb < nb; ++jb) {
-                            const uint32_t base = limb_base(jb);
+                    // 32 columns of one limb per TMEM round trip: two loads
+                    // issued back to back, then one wait
+                    for (int jb = 0; jb < nb; ++jb) {
+                        const uint32_t base = limb_base(jb);
 #pragma unroll
-                            for (int j = 0; j < NH / 16; ++j) {
-                                uint32_t r[16];
-                                tmem_ld16(base + 16 * j, r);
-                                accumulate(r, j, shift0 + 8 * jb);
-                            }
+                        for (int j2 = 0; j2 < NH / 32; ++j2) {
+                            uint32_t r[32];
+                            tmem_ld16_nowait(base + 32 * j2, r);
+                            tmem_ld16_nowait(base + 32 * j2 + 16, r + 16);
+                            tmem_wait_ld<32>(r);
+                            accumulate(r, 2 * j2, shift0 + 8 * jb);
+                            accumulate(r + 16, 2 * j2 + 1, shift0 + 8 * jb);
                         }
                     }
                     tc_fence_before();
@@ -656,78 +672,73 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const int64_t zlo = args.z_lo;
                     const uint64_t zrange = (uint64_t)(args.z_hi - args.z_lo);
                     const FloorDiv32 sf32 = args.sf32;
-                    uint32_t vpk[NH / 4], rpk[NH / 4];
-#pragma unroll
-                    for (int g4 = 0; g4 < NH / 4; ++g4) {
-                        uint32_t vp = 0, rp = 0;
-#pragma unroll
-                        for (int u = 0; u < 4; ++u) {
-                            // z* = floor(z / SF) = floor((z >> 8) / 9Cin).  Inside
-                            // [-127 SF, 128 SF) it fits 32 bits and indexes the NITRO-ReLU
-                            // table; outside, the value is flat (table ends) and only the
-                            // sign picks the piece.
-                            const uint64_t z = acc[4 * g4 + u];
-                            const bool inside = z - (uint64_t)zlo < zrange;
-                            const bool neg = (int32_t)(z >> 32) < 0;
-                            const int zq = sf32.floor_div((int32_t)((int64_t)z >> 8));
-                            const int idx = inside ? zq + 127 : (neg ? 0 : 254);
-                            const int reg = inside ? (neg ? 1 : 2) : (neg ? 0 : 3);
-                            rp |= (uint32_t)reg << (8 * u);
-                            vp |= (uint32_t)(uint8_t)relu_tab[idx] << (8 * u);
-                        }
-                        vpk[g4] = vp;
-                        rpk[g4] = rp;
-                    }
                     const int64_t pix = ((int64_t)b * args.H + y) * args.W + x;
-                    if (valid) {
+                    const bool anchor = valid && !(x & 1) && !(y & 1) && x + 1 < args.W && y + 1 < args.H;
+                    const int64_t opix = ((int64_t)b * args.oh + (y >> 1)) * args.ow + (x >> 1);
+                    const int dys = args.wb;
+                    // one group of 16 columns at a time (only its packed words live)
 #pragma unroll
-                        for (int k = 0; k < NH / 16; ++k)
-                            if (col0 + 16 * k < C) st16(args.region + pix * C + col0 + 16 * k, rpk + 4 * k);
-                    }
-                    if (!args.pool) {
-                        if (valid) {
+                    for (int k = 0; k < NH / 16; ++k) {
+                        if (col0 + 16 * k >= C) break;   // uniform across the warp
+                        uint32_t vpk[4], rpk[4];
 #pragma unroll
-                            for (int k = 0; k < NH / 16; ++k) {
-                                if (col0 + 16 * k >= C) break;
-                                const int64_t o = pix * C + col0 + 16 * k;
-                                st16(args.act + o, vpk + 4 * k);
-                                if (args.out2) st16(args.out2 + o, vpk + 4 * k);
-                                if (args.next_nhwc) st16_bf16(args.next_nhwc + o, vpk + 4 * k, bf16_tab);
+                        for (int g4 = 0; g4 < 4; ++g4) {
+                            uint32_t vp = 0, rp = 0;
+#pragma unroll
+                            for (int u = 0; u < 4; ++u) {
+                                // z* = floor(z / SF) = floor((z >> 8) / 9Cin).  Inside
+                                // [-127 SF, 128 SF) it fits 32 bits and indexes the
+                                // NITRO-ReLU table; outside, the value is flat (table
+                                // ends) and only the sign picks the piece.
+                                const uint64_t z = acc[16 * k + 4 * g4 + u];
+                                const bool inside = z - (uint64_t)zlo < zrange;
+                                const bool neg = (int32_t)(z >> 32) < 0;
+                                const int zq = sf32.floor_div((int32_t)((int64_t)z >> 8));
+                                const int idx = inside ? zq + 127 : (neg ? 0 : 254);
+                                const int reg = inside ? (neg ? 1 : 2) : (neg ? 0 : 3);
+                                rp |= (uint32_t)reg << (8 * u);
+                                vp |= (uint32_t)(uint8_t)relu_tab[idx] << (8 * u);
                             }
+                            vpk[g4] = vp;
+                            rpk[g4] = rp;
                         }
-                    } else {
-                        const int dys = args.wb;
-                        uint32_t opk[NH / 4], apk[NH / 4];
+                        const int c16 = col0 + 16 * k;
+                        if (valid) st16(args.region + pix * C + c16, rpk);
+                        if (!args.pool) {
+                            if (valid) {
+                                const int64_t o = pix * C + c16;
+                                st16(args.act + o, vpk);
+                                if (args.out2) st16(args.out2 + o, vpk);
+                                if (args.next_nhwc) st16_bf16(args.next_nhwc + o, vpk, bf16_tab);
+                            }
+                        } else {
+                            uint32_t opk[4], apk[4];
 #pragma unroll
-                        for (int g4 = 0; g4 < NH / 4; ++g4) {
-                            const uint32_t v00 = vpk[g4];
-                            const uint32_t v01 = __shfl_xor_sync(0xffffffffu, v00, 1);
-                            const uint32_t v10 = __shfl_xor_sync(0xffffffffu, v00, dys);
-                            const uint32_t v11 = __shfl_xor_sync(0xffffffffu, v00, dys ^ 1);
-                            // four windows at once, a byte each: signed maxima, then
-                            // the first position (order (0,0), (0,1), (1,0), (1,1))
-                            // that holds the maximum
-                            const uint32_t best = __vmaxs4(__vmaxs4(v00, v01), __vmaxs4(v10, v11));
-                            const uint32_t e0 = __vcmpeq4(v00, best);
-                            const uint32_t e1 = __vcmpeq4(v01, best);
-                            const uint32_t e2 = __vcmpeq4(v10, best);
-                            uint32_t ap = 0x03030303u;
-                            ap = (ap & ~e2) | (0x02020202u & e2);
-                            ap = (ap & ~e1) | (0x01010101u & e1);
-                            ap &= ~e0;
-                            opk[g4] = best;
-                            apk[g4] = ap;
-                        }
-                        if (valid && !(x & 1) && !(y & 1) && x + 1 < args.W && y + 1 < args.H) {
-                            const int64_t opix = ((int64_t)b * args.oh + (y >> 1)) * args.ow + (x >> 1);
-#pragma unroll
-                            for (int k = 0; k < NH / 16; ++k) {
-                                if (col0 + 16 * k >= C) break;
-                                const int64_t o = opix * C + col0 + 16 * k;
-                                st16(args.act + o, opk + 4 * k);
-                                if (args.out2) st16(args.out2 + o, opk + 4 * k);
-                                st16(args.argmax + o, apk + 4 * k);
-                                if (args.next_nhwc) st16_bf16(args.next_nhwc + o, opk + 4 * k, bf16_tab);
+                            for (int g4 = 0; g4 < 4; ++g4) {
+                                const uint32_t v00 = vpk[g4];
+                                const uint32_t v01 = __shfl_xor_sync(0xffffffffu, v00, 1);
+                                const uint32_t v10 = __shfl_xor_sync(0xffffffffu, v00, dys);
+                                const uint32_t v11 = __shfl_xor_sync(0xffffffffu, v00, dys ^ 1);
+                                // four windows at once, a byte each: signed maxima, then
+                                // the first position (order (0,0), (0,1), (1,0), (1,1))
+                                // that holds the maximum
+                                const uint32_t best = __vmaxs4(__vmaxs4(v00, v01), __vmaxs4(v10, v11));
+                                const uint32_t e0 = __vcmpeq4(v00, best);
+                                const uint32_t e1 = __vcmpeq4(v01, best);
+                                const uint32_t e2 = __vcmpeq4(v10, best);
+                                uint32_t ap = 0x03030303u;
+                                ap = (ap & ~e2) | (0x02020202u & e2);
+                                ap = (ap & ~e1) | (0x01010101u & e1);
+                                ap &= ~e0;
+                                opk[g4] = best;
+                                apk[g4] = ap;
+                            }
+                            if (anchor) {
+                                const int64_t o = opix * C + c16;
+                                st16(args.act + o, opk);
+                                if (args.out2) st16(args.out2 + o, opk);
+                                st16(args.argmax + o, apk);
+                                if (args.next_nhwc) st16_bf16(args.next_nhwc + o, opk, bf16_tab);
                             }
                         }
                     }
@@ -799,6 +810,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                                     }
                                     *reinterpret_cast<int4*>(args.low_delta + ppix[k] * Cl + c0) =
                                         make_int4(dv[0], dv[1], dv[2], dv[3]);
+                                    if (args.low_planes)
+                                        store_delta_planes4(args.low_planes + ppix[k] * Cl + c0,
+                                                            args.low_plane, dv[0], dv[1], dv[2], dv[3]);
                                 }
                             }
                         }
@@ -1126,8 +1140,16 @@ cudaError_t launch_gemm(const CUtensorMap& a, const CUtensorMap& b, const TcArgs
         return cudaErrorInvalidValue;
     static bool attr_set = false;
     if (!attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(k_tc_gemm<MODE, N, PB>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+        // the setmaxnreg split must fit the registers the CTA is launched with,
+        // else setmaxnreg.inc would wait forever: never launch such a build
+        cudaFuncAttributes fa{};
+        cudaError_t e = cudaFuncGetAttributes(&fa, k_tc_gemm<MODE, N, PB>);
+        if (e != cudaSuccess) return e;
+        if (fa.maxThreadsPerBlock < kThreads ||
+            128 * kRegsProducer + 32 * kEpiWarps * kRegsEpilogue > kThreads * fa.numRegs)
+            return cudaErrorInvalidConfiguration;
+        e = cudaFuncSetAttribute(k_tc_gemm<MODE, N, PB>,
+                                 cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
         if (e != cudaSuccess) return e;
         attr_set = true;
     }
@@ -1342,12 +1364,13 @@ cudaError_t tc_conv_forward(TcLayer& t, const LayerGeom& g, int batch, int64_t* 
 }
 
 cudaError_t tc_pack_delta(TcLayer& t, const LayerGeom& g, const int32_t* delta,
-                          const uint32_t* maxabs_delta, int batch, cudaStream_t s) {
+                          const uint32_t* maxabs_delta, int batch, cudaStream_t s,
+                          bool planes_done) {
     if (batch <= 0 || (!t.wgrad && !t.dgrad)) return cudaSuccess;
-    // limb planes of delta (NHWC, read by the wgrad and dgrad passes); the
-    // launch also records the limb count for the GEMMs
+    // limb planes of delta (NHWC, read by the wgrad and dgrad passes), unless
+    // the kernel that produced delta wrote them
     const int64_t n = (int64_t)batch * g.h * g.w * g.cout;   // cout % 8 == 0
-    {
+    if (!planes_done) {
         ProfScope ps(K_TC_PACK_D, s, 0.0, (double)n * 4 * 2);
         k_pack_delta_nhwc<<<grid1d(n / 8), 256, 0, s>>>(delta, n, ((uintptr_t)delta & 15) == 0,
                                                        maxabs_delta, t.d_nhwc);
@@ -1359,10 +1382,10 @@ cudaError_t tc_pack_delta(TcLayer& t, const LayerGeom& g, const int32_t* delta,
 
 cudaError_t tc_conv_wgrad(TcLayer& t, const LayerGeom& g, const int32_t* delta,
                           const uint32_t* maxabs_delta, int batch, int64_t* dW,
-                          uint32_t* status, cudaStream_t s, bool* done) {
+                          uint32_t* status, cudaStream_t s, bool* done, bool planes_done) {
     *done = false;
     if (batch <= 0 || (!t.wgrad && !t.dgrad)) return cudaSuccess;
-    cudaError_t pe = tc_pack_delta(t, g, delta, maxabs_delta, batch, s);
+    cudaError_t pe = tc_pack_delta(t, g, delta, maxabs_delta, batch, s, planes_done);
     if (pe != cudaSuccess) return pe;
     if (!t.wgrad) return cudaSuccess;
     const int hw = g.h * g.w;
@@ -1455,10 +1478,16 @@ cudaError_t tc_conv_dgrad(TcLayer& t, const LayerGeom& g, int batch, int64_t* g6
         a.low_argmax = fo->low_argmax;
         a.low_delta = fo->low_delta;
         a.low_maxabs = fo->low_maxabs;
+        a.low_planes = fo->low_planes;
+        a.low_plane = (int64_t)batch * fo->low_h * fo->low_w * g.cin;
         if (fo->low_pool && ((fo->low_h & 1) || (fo->low_w & 1))) {   // rows the pool dropped
             cudaError_t e = cudaMemsetAsync(fo->low_delta, 0,
                                             sizeof(int32_t) * (size_t)batch * fo->low_h * fo->low_w * g.cin, s);
             if (e != cudaSuccess) return e;
+            if (fo->low_planes) {
+                e = cudaMemsetAsync(fo->low_planes, 0, 2 * (size_t)a.low_plane * kMaxLimbs, s);
+                if (e != cudaSuccess) return e;
+            }
         }
     }
     CUtensorMap ma, mb;

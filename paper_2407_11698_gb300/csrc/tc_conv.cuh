@@ -97,15 +97,24 @@ cudaError_t tc_conv_forward(TcLayer& t, const LayerGeom& g, int batch, int64_t* 
                             bool* fused);
 
 // Splits delta into NHWC limb planes for the wgrad and dgrad passes (limb
-// count from *maxabs_delta, recorded on the device for the GEMMs).
+// count from *maxabs_delta), unless planes_done (the producer of delta wrote
+// all four planes, see store_delta_planes4); then refreshes the host hint of
+// max |delta|.
 cudaError_t tc_pack_delta(TcLayer& t, const LayerGeom& g, const int32_t* delta,
-                          const uint32_t* maxabs_delta, int batch, cudaStream_t s);
+                          const uint32_t* maxabs_delta, int batch, cudaStream_t s,
+                          bool planes_done = false);
+
+// Where a producer of this layer's delta writes its limb planes: d_nhwc
+// [4][batch][h][w][cout] (plane stride batch h w cout), or null when no
+// contraction of the layer reads them.
+inline uint16_t* tc_delta_planes(const TcLayer& t) { return (t.wgrad || t.dgrad) ? t.d_nhwc : nullptr; }
 
 // tc_pack_delta, then, if wgrad runs on tcgen05, dW = sum_p delta (x)
 // im2col(a).  Must precede tc_conv_dgrad.
 cudaError_t tc_conv_wgrad(TcLayer& t, const LayerGeom& g, const int32_t* delta,
                           const uint32_t* maxabs_delta, int batch, int64_t* dW,
-                          uint32_t* status, cudaStream_t s, bool* done);
+                          uint32_t* status, cudaStream_t s, bool* done,
+                          bool planes_done = false);
 
 // Where the input gradient goes when the dgrad epilogue is fused: through the
 // lower layer's max-pool backward and NITRO-ReLU backward into its delta.
@@ -118,6 +127,7 @@ struct TcDgradOut {
     const int8_t* low_argmax;
     int32_t* low_delta;             // [B][low_h][low_w][Cin] int32
     uint32_t* low_maxabs;           // max|lower delta| (atomic max)
+    uint16_t* low_planes;           // lower delta's limb planes (tc_delta_planes), or null
 };
 
 // g[p][ci] = sum_(t,co) delta[p - tap t][co] W[co][t][ci] on tcgen05
