@@ -221,6 +221,19 @@ nitro_status nitro_block_get_tensor(nitro_block* blk, int which, int layer, void
 nitro_status nitro_block_set_tensor(nitro_block* blk, int which, int layer,
                                     const void* host_src, size_t bytes);
 
+/* Device address of the block's int64 weight gradient (NITRO_T_DW of a
+ * layer, or NITRO_T_DWLR with layer 0) and its size in bytes, for a
+ * data-parallel exchange step between nitro_block_backward and
+ * nitro_integersgd_step (Algorithm 1 applied once to the gradient summed over
+ * replicas: the sum of int64 gradients is exact modulo 2^64 in any order, and
+ * the floor of the update comes after it).  The memory stays owned by the
+ * block and valid until nitro_destroy_block; the caller may read and
+ * overwrite it in stream order between those two calls.  Does not
+ * synchronise.  Errors: NITRO_ERR_ARG for a null handle or pointer, another
+ * tensor, or a layer out of range. */
+nitro_status nitro_block_grad_device(nitro_block* blk, int which, int layer, void** dev_ptr,
+                                     size_t* bytes);
+
 /* Synchronises the device and returns the latched status as nitro_status
  * (TIMEOUT before OVERFLOW before a bad label = ARG); clears it if clear. */
 nitro_status nitro_block_status(nitro_block* blk, int clear);

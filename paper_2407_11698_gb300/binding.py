@@ -115,6 +115,9 @@ def lib():
     L.nitro_block_set_dropout.restype = ctypes.c_int
     L.nitro_block_diag_timeout.argtypes = [_VP, ctypes.c_int, _VP]
     L.nitro_block_diag_timeout.restype = ctypes.c_int
+    L.nitro_block_grad_device.argtypes = [_VP, ctypes.c_int, ctypes.c_int, ctypes.POINTER(_VP),
+                                          ctypes.POINTER(ctypes.c_size_t)]
+    L.nitro_block_grad_device.restype = ctypes.c_int
     L.nitro_prep_create.argtypes = [ctypes.POINTER(_VP)]
     L.nitro_prep_fit.argtypes = [_VP, _VP, ctypes.c_int64, _VP]
     L.nitro_prep_apply.argtypes = [_VP, _VP, ctypes.c_int64, _VP, _VP]
@@ -208,6 +211,16 @@ def make_block_desc(layers, in_features, num_classes=10, alpha_inv=10, gamma_inv
     return d, arr
 
 
+class _DeviceArray:
+    """A 1-D device buffer described by __cuda_array_interface__ (so torch can
+    view library-owned memory without copying it)."""
+
+    def __init__(self, ptr, n, typestr):
+        self.__cuda_array_interface__ = {"shape": (int(n),), "typestr": typestr,
+                                         "data": (int(ptr or 0), False), "version": 3,
+                                         "strides": None}
+
+
 def _stream_ptr(stream):
     if stream is None:
         import torch
@@ -289,6 +302,17 @@ class Block:
 
     def status(self, clear=False):
         return nitro_block_status(self.h, clear)
+
+    def grad_device(self, which, layer=0):
+        """The block's int64 weight gradient (NITRO_T_DW / NITRO_T_DWLR) as a
+        flat torch CUDA tensor that views the block's own memory (no copy)."""
+        import torch
+        p, n = _VP(), ctypes.c_size_t()
+        st = lib().nitro_block_grad_device(self.h, int(which), int(layer), ctypes.byref(p),
+                                           ctypes.byref(n))
+        if st != NITRO_OK:
+            raise NitroError(st, "nitro_block_grad_device")
+        return torch.as_tensor(_DeviceArray(p.value, n.value // 8, "<i8"), device="cuda")
 
     def diag_timeout(self, wait_us, stream=None):
         """Queue the bounded-wait failure check (nitro_block_diag_timeout)."""

@@ -605,6 +605,19 @@ static const void* tensor_ptr(nitro_block* b, int which, int layer) {
     return nullptr;
 }
 
+nitro_status nitro_block_grad_device(nitro_block* b, int which, int layer, void** dev_ptr,
+                                     size_t* bytes) {
+    if (!b || !dev_ptr) return NITRO_ERR_ARG;
+    *dev_ptr = nullptr;
+    if (which != NITRO_T_DW && which != NITRO_T_DWLR) return NITRO_ERR_ARG;
+    size_t need = 0;
+    nitro_status st = nitro_block_tensor_bytes(b, which, layer, &need);
+    if (st != NITRO_OK) return st;
+    *dev_ptr = const_cast<void*>(tensor_ptr(b, which, layer));
+    if (bytes) *bytes = need;
+    return NITRO_OK;
+}
+
 static nitro_status latched(uint32_t bits) {
     if (bits & ST_TIMEOUT) return NITRO_ERR_TIMEOUT;
     if (bits & ST_OVERFLOW) return NITRO_ERR_OVERFLOW;
