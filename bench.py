@@ -40,6 +40,9 @@ def parse():
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--sequential-blocks", action="store_true",
                    help="run all blocks on one stream (default: a stream per block)")
+    p.add_argument("--separate-update", action="store_true",
+                   help="backward and IntegerSGD as two calls (default: one call, the update "
+                        "fused into the tensor-core weight-gradient kernels)")
     p.add_argument("--profile-steps", type=int, default=3)
     p.add_argument("--sweep", action="store_true",
                    help="time the kernel sweep (conv contractions, integer GEMM, IntegerSGD, "
@@ -157,8 +160,9 @@ class GpuNet:
     only for block i's forward, so block i's backward and update overlap the
     blocks after it (blocks exchange no gradients, Sec. 3.3)."""
 
-    def __init__(self, wl, seed, torch, nb, concurrent=True):
+    def __init__(self, wl, seed, torch, nb, concurrent=True, fused_update=True):
         self.torch, self.nb = torch, nb
+        self.fused_update = fused_update
         B = wl["batch"]
         self.B = B
         self.blocks = [nb.Block(b["layers"], b["in_features"], seed=seed + i, max_batch=B,
@@ -186,6 +190,10 @@ class GpuNet:
         if not self.streams or sequential:
             for i, g in enumerate(self.blocks):
                 g.forward(acts[i], acts[i + 1] if g.layers else None)
+            if self.fused_update:
+                for i, g in enumerate(self.blocks):
+                    g.backward_update(acts[i], y, loss[i:i + 1])
+                return
             for i, g in enumerate(self.blocks):
                 g.backward(acts[i], y, loss[i:i + 1])
             for g in self.blocks:
@@ -198,8 +206,11 @@ class GpuNet:
                 s.wait_event(self.fwd_done[i - 1])   # the block's input activations
             g.forward(acts[i], acts[i + 1] if g.layers else None, stream=s)
             self.fwd_done[i].record(s)
-            g.backward(acts[i], y, loss[i:i + 1], stream=s)
-            g.sgd(stream=s)
+            if self.fused_update:
+                g.backward_update(acts[i], y, loss[i:i + 1], stream=s)
+            else:
+                g.backward(acts[i], y, loss[i:i + 1], stream=s)
+                g.sgd(stream=s)
         for s in self.streams:
             main.wait_stream(s)
 
@@ -241,9 +252,13 @@ def issued_profile(nb, net, flush, steps, torch):
         for i in reversed(range(len(g.layers))):
             if g.layers[i][0] != nb.NITRO_CONV3X3:
                 continue
-            bwd.append(("tc_conv_wgrad", bi, i))
-            if i > 0:
-                bwd.append(("tc_conv_dgrad", bi, i))
+            # the fused update runs a layer's input gradient before its weight
+            # gradient (the input gradient reads the pre-update weights)
+            order = (("tc_conv_dgrad", "tc_conv_wgrad") if net.fused_update
+                     else ("tc_conv_wgrad", "tc_conv_dgrad"))
+            for name in order:
+                if name == "tc_conv_wgrad" or i > 0:
+                    bwd.append((name, bi, i))
 
     def maxabs(bi, which, i):
         return np.abs(net.blocks[bi].get(which, i, check=False).astype(np.int64)).max()
@@ -289,7 +304,8 @@ def run_ours(args, rank, world, local_rank):
     torch.cuda.set_device(local_rank)
     nb.lib()
     wl = WL.WORKLOADS[args.workload]
-    net = GpuNet(wl, 20240716 + 7 * rank, torch, nb, concurrent=not args.sequential_blocks)
+    net = GpuNet(wl, 20240716 + 7 * rank, torch, nb, concurrent=not args.sequential_blocks,
+                 fused_update=not args.separate_update)
     stream = torch.cuda.current_stream()
     flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device="cuda")
 
@@ -427,6 +443,8 @@ def run_ours(args, rank, world, local_rank):
                    "input": "x".join(str(v) for v in wl["input_shape"]) + " int8 uniform [-128,127]",
                    "blocks": len(wl["blocks"]), "cuda_graph": graph is not None,
                    "block_streams": "one" if args.sequential_blocks else "one per block",
+                   "update": ("separate IntegerSGD call" if args.separate_update
+                              else "fused into the tensor-core weight-gradient kernels"),
                    "l2": "flushed (512 MiB write) between timed steps",
                    "parallelism": "replicas" if world > 1 else "single"},
         "e2e": {"value": round(e2e_value, 2), "unit": "images/s",

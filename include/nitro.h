@@ -162,6 +162,20 @@ nitro_status nitro_block_backward(nitro_block* blk, const int8_t* a_in, const in
  * learning layer gamma_inv_lr and eta_inv_lr. */
 nitro_status nitro_integersgd_step(nitro_block* blk, void* stream);
 
+/* nitro_block_backward followed by nitro_integersgd_step, with the same
+ * results bit for bit (Sec. 3.3: a block's backward and its update depend on
+ * no other block).  The conv layers whose weight gradient runs on the tensor
+ * cores apply Algorithm 1 inside that kernel, to each output tile once its
+ * sum is final: their new weights and limb planes are written without a
+ * second pass over the gradients, and their input gradient (which reads the
+ * pre-update weights) runs before the update.  The weight gradients stay
+ * readable (nitro_block_get_tensor) after the call.  A data-parallel
+ * exchange of the gradients needs the two separate calls instead.
+ * Errors: as nitro_block_backward. */
+nitro_status nitro_block_backward_update(nitro_block* blk, const int8_t* a_in,
+                                         const int32_t* labels, int batch, int64_t* loss_dev,
+                                         void* stream);
+
 /* Replaces the IntegerSGD hyper-parameters of a block (Algorithm 1):
  * gamma_inv_lr (the forward layers use 2^6*G*gamma_inv_lr, Sec. 3.3.5),
  * eta_inv_fw and eta_inv_lr.  App. B multiplies the inverse learning rate by 3

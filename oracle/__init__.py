@@ -16,5 +16,5 @@ from .nitro import (  # noqa: F401
     relu_bwd, isqrt, init_bound, splitmix64_at, conv3x3_fwd, conv3x3_dgrad,
     conv3x3_wgrad, linear_fwd, linear_dgrad, linear_wgrad, maxpool_fwd, maxpool_bwd,
     integersgd, amplification_factor, num_threads, prep_stats, prep_apply,
-    winpool_fwd, winpool_bwd, dropout_drop, dropout_mask, lr_pool_window,
+    winpool_fwd, winpool_bwd, dropout_drop, dropout_mask, lr_pool_window, scale_relu,
 )

@@ -69,6 +69,7 @@ def lib():
     L.nitro_block_forward.argtypes = [_VP, _VP, ctypes.c_int, _VP, _VP]
     L.nitro_block_backward.argtypes = [_VP, _VP, _VP, ctypes.c_int, _VP, _VP]
     L.nitro_integersgd_step.argtypes = [_VP, _VP]
+    L.nitro_block_backward_update.argtypes = [_VP, _VP, _VP, ctypes.c_int, _VP, _VP]
     L.nitro_block_tensor_bytes.argtypes = [_VP, ctypes.c_int, ctypes.c_int,
                                            ctypes.POINTER(ctypes.c_size_t)]
     L.nitro_block_get_tensor.argtypes = [_VP, ctypes.c_int, ctypes.c_int, _VP, ctypes.c_size_t]
@@ -129,7 +130,7 @@ def lib():
                  "nitro_prep_create", "nitro_prep_fit", "nitro_prep_apply", "nitro_prep_stats"):
         getattr(L, name).restype = ctypes.c_int
     for name in ("nitro_init_block", "nitro_block_forward", "nitro_block_backward",
-                 "nitro_integersgd_step", "nitro_block_tensor_bytes", "nitro_block_get_tensor",
+                 "nitro_block_backward_update", "nitro_integersgd_step", "nitro_block_tensor_bytes", "nitro_block_get_tensor",
                  "nitro_block_set_tensor", "nitro_block_status"):
         getattr(L, name).restype = ctypes.c_int
     _lib = L
@@ -161,6 +162,10 @@ def nitro_block_backward(blk, a_in, labels, batch, loss_dev, stream=None):
 
 def nitro_integersgd_step(blk, stream=None):
     return lib().nitro_integersgd_step(blk, stream)
+
+
+def nitro_block_backward_update(blk, a_in, labels, batch, loss_dev, stream=None):
+    return lib().nitro_block_backward_update(blk, a_in, labels, int(batch), loss_dev, stream)
 
 
 def nitro_block_tensor_bytes(blk, which, layer=0):
@@ -263,6 +268,15 @@ class Block:
                                   _stream_ptr(stream))
         if st != NITRO_OK:
             raise NitroError(st, "nitro_block_backward")
+        return loss
+
+    def backward_update(self, a_in, labels, loss=None, stream=None):
+        """backward() then sgd() in one call, the update fused into the
+        tensor-core weight-gradient kernels (same results)."""
+        st = nitro_block_backward_update(self.h, _ptr(a_in), _ptr(labels), labels.shape[0],
+                                         _ptr(loss), _stream_ptr(stream))
+        if st != NITRO_OK:
+            raise NitroError(st, "nitro_block_backward_update")
         return loss
 
     def sgd(self, stream=None):

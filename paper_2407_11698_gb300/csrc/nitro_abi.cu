@@ -374,9 +374,18 @@ nitro_status nitro_block_forward(nitro_block* b, const int8_t* a_in, int batch, 
     return NITRO_OK;
 }
 
-nitro_status nitro_block_backward(nitro_block* b, const int8_t* a_in, const int32_t* labels,
-                                  int batch, int64_t* loss_dev, void* stream) {
+}  // extern "C"
+
+namespace {
+
+// The block's backward (Sec. 3.3, second phase).  With `updated` != null the
+// layers whose weight gradient runs on tcgen05 also apply IntegerSGD inside
+// that kernel (their input gradient, which needs the pre-update weights, runs
+// first) and are marked in *updated; the caller updates the rest.
+nitro_status block_backward(nitro_block* b, const int8_t* a_in, const int32_t* labels, int batch,
+                            int64_t* loss_dev, void* stream, std::vector<char>* updated) {
     if (!b || batch < 0 || batch != b->batch) return NITRO_ERR_ARG;
+    if (updated) updated->assign(b->L.size(), 0);
     if (batch > 0 && (!labels || !a_in)) return NITRO_ERR_ARG;
     cudaStream_t s = (cudaStream_t)stream;
     const int n = (int)b->L.size();
@@ -451,22 +460,52 @@ nitro_status nitro_block_backward(nitro_block* b, const int8_t* a_in, const int3
         NITRO_TRY(simt_grad_to_delta(src, ly.g, batch, b->desc.alpha_inv, ly.region, ly.argmax,
                                      ly.delta, w_delta(b, n - 1), w_status(b), s));
     }
+    const int64_t gamma_fw = 64LL * b->G * b->desc.gamma_inv_lr;
     for (int i = n - 1; i >= 0; --i) {
         Layer& ly = b->L[i];
         const LayerGeom& g = ly.g;
         const int8_t* x = i ? b->L[i - 1].act : a_in;
         bool done = false;
-        NITRO_TRY(tc_conv_wgrad(ly.tc, g, ly.delta, w_delta(b, i), batch, ly.dW, w_status(b), s, &done,
-                                planes_done[i] != 0));
-        if (!done && simt_small_conv_ok(g)) {
-            NITRO_TRY(simt_conv_small_wgrad(x, ly.delta, g, batch, ly.dW, s));
-            done = true;
+        // fused update: the input gradient reads the pre-update weights, so it
+        // runs first (after the delta split), then the weight gradient with
+        // IntegerSGD; otherwise weight gradient first, as the split requires
+        const bool fuse_sgd = updated && ly.tc.wgrad;
+        auto wgrad = [&]() -> nitro_status {
+            if (fuse_sgd) {
+                NITRO_TRY(cudaMemsetAsync(w_w(b, i), 0, 4, s));
+                TcSgd sg{gamma_fw, b->desc.eta_inv_fw, b->desc.sgd_round == NITRO_ROUND_TRUNC, ly.W,
+                         w_w(b, i)};
+                NITRO_TRY(tc_conv_wgrad(ly.tc, g, ly.delta, w_delta(b, i), batch, ly.dW, w_status(b), s,
+                                        &done, true, &sg));
+                (*updated)[i] = done;
+                if (done) NITRO_TRY(tc_weights_hint(ly.tc, s));
+            } else {
+                NITRO_TRY(tc_conv_wgrad(ly.tc, g, ly.delta, w_delta(b, i), batch, ly.dW, w_status(b), s,
+                                        &done, planes_done[i] != 0));
+            }
+            if (!done && simt_small_conv_ok(g)) {
+                NITRO_TRY(simt_conv_small_wgrad(x, ly.delta, g, batch, ly.dW, s));
+                done = true;
+            }
+            if (!done) {
+                const int mode = g.kind == NITRO_CONV3X3 ? GM_CONV_WGRAD : GM_LIN_WGRAD;
+                NITRO_TRY(simt_gemm(mode, x, ly.delta, nullptr, ly.dW, batch, g.h, g.w, g.cin, g.cout, s));
+            }
+            return NITRO_OK;
+        };
+        if (fuse_sgd) {
+            NITRO_TRY(tc_pack_delta(ly.tc, g, ly.delta, w_delta(b, i), batch, s, planes_done[i] != 0));
+        } else {
+            nitro_status st = wgrad();
+            if (st != NITRO_OK) return st;
         }
-        if (!done) {
-            const int mode = g.kind == NITRO_CONV3X3 ? GM_CONV_WGRAD : GM_LIN_WGRAD;
-            NITRO_TRY(simt_gemm(mode, x, ly.delta, nullptr, ly.dW, batch, g.h, g.w, g.cin, g.cout, s));
+        if (i == 0) {
+            if (fuse_sgd) {
+                nitro_status st = wgrad();
+                if (st != NITRO_OK) return st;
+            }
+            break;
         }
-        if (i == 0) break;
         done = false;
         bool fused = false;
         Layer& lo = b->L[i - 1];
@@ -482,16 +521,76 @@ nitro_status nitro_block_backward(nitro_block* b, const int8_t* a_in, const int3
         }
         if (fused) {
             planes_done[i - 1] = fo.low_planes != nullptr;
-            continue;
+        } else {
+            DeltaSrc src{};
+            src.g64 = b->z64;
+            src.maxabs_a = w_delta(b, i); src.maxabs_b = w_w(b, i);
+            src.bound_k = g.kind == NITRO_CONV3X3 ? 9LL * g.cout : (int64_t)g.cout;
+            NITRO_TRY(simt_grad_to_delta(src, lo.g, batch, b->desc.alpha_inv, lo.region, lo.argmax,
+                                         lo.delta, w_delta(b, i - 1), w_status(b), s));
         }
-        DeltaSrc src{};
-        src.g64 = b->z64;
-        src.maxabs_a = w_delta(b, i); src.maxabs_b = w_w(b, i);
-        src.bound_k = g.kind == NITRO_CONV3X3 ? 9LL * g.cout : (int64_t)g.cout;
-        NITRO_TRY(simt_grad_to_delta(src, lo.g, batch, b->desc.alpha_inv, lo.region, lo.argmax,
-                                     lo.delta, w_delta(b, i - 1), w_status(b), s));
+        if (fuse_sgd) {
+            nitro_status st = wgrad();
+            if (st != NITRO_OK) return st;
+        }
     }
     return NITRO_OK;
+}
+
+// IntegerSGD of every tensor of the block not yet updated (skip[i] marks a
+// forward layer updated inside its weight-gradient kernel).
+nitro_status block_sgd(nitro_block* b, void* stream, const std::vector<char>* skip) {
+    if (!b) return NITRO_ERR_ARG;
+    cudaStream_t s = (cudaStream_t)stream;
+    const int n = (int)b->L.size();
+    // gamma_inv^fw = AF * gamma_inv^lr, AF = 2^6 * G (Sec. 3.3.5)
+    const int64_t gamma_fw = 64LL * b->G * b->desc.gamma_inv_lr;
+    SgdBatch bt{};
+    bt.round_trunc = b->desc.sgd_round == NITRO_ROUND_TRUNC;
+    bt.status = w_status(b);
+    bt.step = w_step(b);
+    for (int i = 0; i < n; ++i) {
+        if (skip && (*skip)[i]) continue;
+        // the update also writes the tensor-core weight planes of the layer
+        SgdTensor st{b->L[i].W, b->L[i].dW, b->L[i].wcount, gamma_fw, b->desc.eta_inv_fw,
+                     w_w(b, i), {}, {}, nullptr, 0, 0, 0, 0, {}};
+        tc_weight_planes(b->L[i].tc, b->L[i].g, &st.planes, &st.plane, &st.row_k, &st.tap_k);
+        st.cin = b->L[i].g.cin;
+        if (b->L[i].lin_planes) {
+            // linear planes [4][out][in]: element o*in + k at row o*9*in + tap*in with
+            // the update's (row, tap) = (o / 9, o % 9) decomposition
+            st.planes = b->L[i].lin_planes;
+            st.plane = b->L[i].wcount;
+            st.row_k = 9 * b->L[i].g.cin;
+            st.tap_k = b->L[i].g.cin;
+        }
+        NITRO_TRY(cudaMemsetAsync(w_w(b, i), 0, 4, s));
+        bt.t[bt.count++] = st;
+    }
+    bt.t[bt.count++] = SgdTensor{b->Wlr, b->dWlr, (int64_t)b->G * b->d, b->desc.gamma_inv_lr,
+                                 b->desc.eta_inv_lr, w_wlr(b), {}, {}, nullptr, 0, 0, 0, 0, {}};
+    NITRO_TRY(cudaMemsetAsync(w_wlr(b), 0, 4, s));
+    NITRO_TRY(simt_integersgd(bt, s));
+    for (int i = 0; i < n; ++i)
+        if (!(skip && (*skip)[i])) NITRO_TRY(tc_weights_hint(b->L[i].tc, s));
+    return NITRO_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+nitro_status nitro_block_backward(nitro_block* b, const int8_t* a_in, const int32_t* labels,
+                                  int batch, int64_t* loss_dev, void* stream) {
+    return block_backward(b, a_in, labels, batch, loss_dev, stream, nullptr);
+}
+
+nitro_status nitro_block_backward_update(nitro_block* b, const int8_t* a_in, const int32_t* labels,
+                                         int batch, int64_t* loss_dev, void* stream) {
+    std::vector<char> updated;
+    nitro_status st = block_backward(b, a_in, labels, batch, loss_dev, stream, &updated);
+    if (st != NITRO_OK) return st;
+    return block_sgd(b, stream, &updated);
 }
 
 nitro_status nitro_block_set_hyper(nitro_block* b, int64_t gamma_inv_lr, int64_t eta_inv_fw,
@@ -515,38 +614,7 @@ nitro_status nitro_block_set_dropout(nitro_block* b, int dropout_p16) {
 }
 
 nitro_status nitro_integersgd_step(nitro_block* b, void* stream) {
-    if (!b) return NITRO_ERR_ARG;
-    cudaStream_t s = (cudaStream_t)stream;
-    const int n = (int)b->L.size();
-    // gamma_inv^fw = AF * gamma_inv^lr, AF = 2^6 * G (Sec. 3.3.5)
-    const int64_t gamma_fw = 64LL * b->G * b->desc.gamma_inv_lr;
-    SgdBatch bt{};
-    bt.round_trunc = b->desc.sgd_round == NITRO_ROUND_TRUNC;
-    bt.status = w_status(b);
-    bt.step = w_step(b);
-    for (int i = 0; i < n; ++i) {
-        // the update also writes the tensor-core weight planes of the layer
-        SgdTensor st{b->L[i].W, b->L[i].dW, b->L[i].wcount, gamma_fw, b->desc.eta_inv_fw,
-                     w_w(b, i), {}, {}, nullptr, 0, 0, 0, 0, {}};
-        tc_weight_planes(b->L[i].tc, b->L[i].g, &st.planes, &st.plane, &st.row_k, &st.tap_k);
-        st.cin = b->L[i].g.cin;
-        if (b->L[i].lin_planes) {
-            // linear planes [4][out][in]: element o*in + k at row o*9*in + tap*in with
-            // the update's (row, tap) = (o / 9, o % 9) decomposition
-            st.planes = b->L[i].lin_planes;
-            st.plane = b->L[i].wcount;
-            st.row_k = 9 * b->L[i].g.cin;
-            st.tap_k = b->L[i].g.cin;
-        }
-        bt.t[bt.count++] = st;
-    }
-    bt.t[bt.count++] = SgdTensor{b->Wlr, b->dWlr, (int64_t)b->G * b->d, b->desc.gamma_inv_lr,
-                                 b->desc.eta_inv_lr, w_wlr(b), {}, {}, nullptr, 0, 0, 0, 0, {}};
-    NITRO_TRY(cudaMemsetAsync(w_wlr(b), 0, 4, s));
-    if (n) NITRO_TRY(cudaMemsetAsync(w_w(b, 0), 0, 4 * n, s));
-    NITRO_TRY(simt_integersgd(bt, s));
-    for (int i = 0; i < n; ++i) NITRO_TRY(tc_weights_hint(b->L[i].tc, s));
-    return NITRO_OK;
+    return block_sgd(b, stream, nullptr);
 }
 
 nitro_status nitro_block_diag_timeout(nitro_block* b, int wait_us, void* stream) {

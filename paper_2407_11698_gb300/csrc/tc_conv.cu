@@ -256,6 +256,17 @@ struct TcArgs {
     uint32_t* low_maxabs;
     uint16_t* low_planes;      // the lower delta's bf16 limb planes, or null
     int64_t low_plane;
+    // weight gradient with IntegerSGD applied to the finished sums
+    int sgd;
+    int splits;                // K splits per output tile
+    int* tickets;              // per (tile, epilogue warp) arrivals, zero between launches
+    int32_t* wt;               // the layer's weights [Cout][9][Cin]
+    uint16_t* wp;              // weight limb planes [4][Cout][row_k], or null
+    int64_t w_plane;
+    int row_k, tap_k;
+    FloorDiv gdiv, ediv;       // gamma_inv, eta_inv (eta_inv = 0: no decay)
+    int decay, trunc;
+    uint32_t* maxabs_w;        // max |new W| (atomic max, zeroed by the caller)
 };
 
 // 16 int8 values (4 packed words) -> one 16-byte store
@@ -644,9 +655,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const int t = m / args.cin_k, ci = m - t * args.cin_k;
                     // im2col rows: row m is already the (tap, ci) index t Cin + ci
                     const bool ok = args.taps == 1 ? m < 9 * args.Cin : (t < 9 && ci < args.Cin);
+                    const int64_t wrow = args.taps == 1 ? (int64_t)m : (int64_t)t * args.Cin + ci;
+                    const int64_t cstride = 9LL * args.Cin;
                     if (ok) {
-                        int64_t* o = args.out + (args.taps == 1 ? (int64_t)m : (int64_t)t * args.Cin + ci);
-                        const int64_t cstride = 9LL * args.Cin;
+                        int64_t* o = args.out + wrow;
 #pragma unroll
                         for (int i = 0; i < NH; ++i) {
                             if (col0 + i >= args.ncols) break;
@@ -654,6 +666,77 @@ __global__ void __launch_bounds__(kThreads, 1)
                                 o + (int64_t)(col0 + i) * cstride);
                             if (args.atomic_out) atomicAdd(dst, (unsigned long long)acc[i]);
                             else *dst = acc[i];
+                        }
+                    }
+                    if (args.sgd) {
+                        // IntegerSGD (Algorithm 1) on this warp's 32 rows x NH columns
+                        // once their sums are final.  With a K split the warp of the
+                        // same slot that arrives last (per-slot ticket, after its
+                        // atomics are fenced) reads the sums back; no CTA-wide barrier
+                        // is involved, so a warp that gave up on a wait blocks nobody.
+                        bool mine = true;
+                        if (args.atomic_out) {
+                            __threadfence();
+                            __syncwarp();
+                            int* ticket = args.tickets + ((int64_t)T.mt * args.tiles_n + T.nt) * kEpiWarps +
+                                          (warp - kEpiWarp0);
+                            int tk = 0;
+                            if (lane == 0) tk = atomicAdd(ticket, 1);
+                            tk = __shfl_sync(0xffffffffu, tk, 0);
+                            mine = tk == args.splits - 1;
+                            if (mine) {
+                                if (lane == 0) *ticket = 0;   // ready for the next launch
+                                __threadfence();
+                            }
+                        }
+                        if (mine) {
+                            uint32_t mx = 0;
+                            bool ovf = false;
+                            if (ok) {
+                                const int tt = args.taps == 1 ? 0 : t;
+#pragma unroll
+                                for (int i = 0; i < NH; ++i) {
+                                    const int co = col0 + i;
+                                    if (co >= args.ncols) break;
+                                    const int64_t e = (int64_t)co * cstride + wrow;
+                                    const int64_t g = args.atomic_out
+                                        ? (int64_t)__ldcg(reinterpret_cast<const unsigned long long*>(args.out + e))
+                                        : (int64_t)acc[i];
+                                    const int64_t w = args.wt[e];
+                                    int64_t d = args.trunc ? args.gdiv.trunc_div(g) : args.gdiv.floor_div(g);
+                                    if (args.decay) d += args.trunc ? args.ediv.trunc_div(w) : args.ediv.floor_div(w);
+                                    const int64_t nw = w - d;
+                                    ovf |= !fits_i32(nw);
+                                    const int32_t s32 = (int32_t)nw;
+                                    args.wt[e] = s32;
+                                    mx = max(mx, abs_u32(s32));
+                                    if (args.wp) {
+                                        // limb planes of the new weight, entry (t, ci) of row co
+                                        uint16_t* pp = args.wp + (int64_t)co * args.row_k +
+                                                       (args.taps == 1 ? (int64_t)m : (int64_t)tt * args.tap_k + ci);
+                                        int32_t x = s32;
+#pragma unroll
+                                        for (int l = 0; l < 4; ++l) {
+                                            int dg;
+                                            if (l < 3) {
+                                                const int rr = x & 255;
+                                                dg = rr - ((rr >> 7) << 8);
+                                                x = (x >> 8) + (rr >> 7);
+                                            } else {
+                                                dg = x;
+                                            }
+                                            pp[l * args.w_plane] = (uint16_t)(__float_as_uint((float)dg) >> 16);
+                                        }
+                                    }
+                                }
+                            }
+#pragma unroll
+                            for (int off = 16; off; off >>= 1) mx = max(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+                            ovf = __any_sync(0xffffffffu, ovf);
+                            if (lane == 0) {
+                                if (mx) atomicMax(args.maxabs_w, mx);
+                                if (ovf) atomicOr(args.status, ST_OVERFLOW);
+                            }
                         }
                     }
                 } else if (MODE == TC_FWD && args.fuse) {
@@ -1234,6 +1317,10 @@ bool tc_layer_init(TcLayer& t, const LayerGeom& g, int max_batch, bool has_dgrad
     if (ok && (t.wgrad || t.dgrad))
         ok = dalloc(allocs, &t.d_nhwc, (size_t)kMaxLimbs * max_batch * hw * g.cout);
     if (ok && (t.fwd || t.dgrad)) ok = dalloc(allocs, &t.w_planes, (size_t)kMaxLimbs * nwk);
+    // weight-gradient output tiles: ceil(taps * cin_k / 128) x ceil(cout / 64) at most
+    const size_t ntk = (size_t)((t.im2col ? kBK : 9 * t.cin_k) + kBM - 1) / kBM * ((g.cout + 63) / 64) * kEpiWarps;
+    if (ok && t.wgrad) ok = dalloc(allocs, &t.tickets, ntk);
+    if (ok && t.tickets) ok = cudaMemset(t.tickets, 0, ntk * sizeof(int)) == cudaSuccess;
     if (ok) {
         void* h = nullptr;
         ok = cudaMallocHost(&h, 2 * sizeof(uint32_t)) == cudaSuccess;
@@ -1382,7 +1469,8 @@ cudaError_t tc_pack_delta(TcLayer& t, const LayerGeom& g, const int32_t* delta,
 
 cudaError_t tc_conv_wgrad(TcLayer& t, const LayerGeom& g, const int32_t* delta,
                           const uint32_t* maxabs_delta, int batch, int64_t* dW,
-                          uint32_t* status, cudaStream_t s, bool* done, bool planes_done) {
+                          uint32_t* status, cudaStream_t s, bool* done, bool planes_done,
+                          const TcSgd* sgd) {
     *done = false;
     if (batch <= 0 || (!t.wgrad && !t.dgrad)) return cudaSuccess;
     cudaError_t pe = tc_pack_delta(t, g, delta, maxabs_delta, batch, s, planes_done);
@@ -1419,6 +1507,21 @@ cudaError_t tc_conv_wgrad(TcLayer& t, const LayerGeom& g, const int32_t* delta,
     a.out = dW;
     a.status = status;
     a.atomic_out = splits > 1;
+    if (sgd) {
+        if (!t.tickets || sgd->gamma_inv < 1 || sgd->eta_inv < 0) return cudaErrorInvalidValue;
+        a.sgd = 1;
+        a.splits = splits;
+        a.tickets = t.tickets;
+        a.wt = sgd->W;
+        a.maxabs_w = sgd->maxabs_w;
+        a.gdiv = FloorDiv::make((uint64_t)sgd->gamma_inv);
+        a.decay = sgd->eta_inv > 0;
+        a.ediv = FloorDiv::make(sgd->eta_inv > 0 ? (uint64_t)sgd->eta_inv : 1);
+        a.trunc = sgd->trunc;
+        int64_t plane = 0;
+        tc_weight_planes(t, g, &a.wp, &plane, &a.row_k, &a.tap_k);
+        a.w_plane = plane;
+    }
     CUtensorMap ma, mb;
     const uint64_t da[4] = {(uint64_t)t.cin8, (uint64_t)g.w, (uint64_t)g.h, (uint64_t)batch};
     const uint64_t sa[3] = {(uint64_t)t.cin8, (uint64_t)g.w * t.cin8, (uint64_t)hw * t.cin8};

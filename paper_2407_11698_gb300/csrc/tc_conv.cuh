@@ -48,6 +48,20 @@ struct TcLayer {
     // pinned host copies of the two words, refreshed asynchronously; possibly
     // stale, used only to pick a kernel variant (any choice is exact)
     uint32_t* max_host = nullptr;
+    // arrival tickets of the weight gradient's fused IntegerSGD, one per
+    // (output tile, epilogue warp), zero between launches
+    int* tickets = nullptr;
+};
+
+// IntegerSGD folded into the weight-gradient kernel (Algorithm 1 with the
+// forward layers' gamma_inv and eta_inv): the kernel updates W and its limb
+// planes and atomically maxes max |W| into *maxabs_w, which the caller zeroes
+// first.  The weight gradient is still written to dW.
+struct TcSgd {
+    int64_t gamma_inv, eta_inv;   // eta_inv = 0: no decay
+    int trunc;                    // NITRO_ROUND_TRUNC
+    int32_t* W;
+    uint32_t* maxabs_w;
 };
 
 // Decides which passes of a layer run on tensor cores and allocates their
@@ -111,10 +125,12 @@ inline uint16_t* tc_delta_planes(const TcLayer& t) { return (t.wgrad || t.dgrad)
 
 // tc_pack_delta, then, if wgrad runs on tcgen05, dW = sum_p delta (x)
 // im2col(a).  Must precede tc_conv_dgrad.
+// With sgd != null (and only if the weight gradient runs on tcgen05: check
+// *done) the kernel also applies IntegerSGD, see TcSgd.
 cudaError_t tc_conv_wgrad(TcLayer& t, const LayerGeom& g, const int32_t* delta,
                           const uint32_t* maxabs_delta, int batch, int64_t* dW,
                           uint32_t* status, cudaStream_t s, bool* done,
-                          bool planes_done = false);
+                          bool planes_done = false, const TcSgd* sgd = nullptr);
 
 // Where the input gradient goes when the dgrad epilogue is fused: through the
 // lower layer's max-pool backward and NITRO-ReLU backward into its delta.

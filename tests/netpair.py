@@ -13,10 +13,11 @@ def _torch():
 
 
 class NetPair:
-    def __init__(self, blocks, batch, seed=1000, concurrent=False, **hyper):
+    def __init__(self, blocks, batch, seed=1000, concurrent=False, fused_update=False, **hyper):
         self.batch = batch
         self.spec = blocks
         self.concurrent = concurrent   # a stream per block, as bench.py drives them
+        self.fused_update = fused_update   # backward and update in one call
         self.ob = [O.OracleBlock([O.LayerDesc(*l) for l in b["layers"]],
                                  in_features=b["in_features"], seed=seed + i, **hyper)
                    for i, b in enumerate(blocks)]
@@ -50,17 +51,24 @@ class NetPair:
                     s.wait_event(done[i - 1])
                 g.forward(acts[i], acts[i + 1] if g.layers else None, stream=s)
                 done[i].record(s)
-                g.backward(acts[i], ys, losses[i], stream=s)
-                g.sgd(stream=s)
+                if self.fused_update:
+                    g.backward_update(acts[i], ys, losses[i], stream=s)
+                else:
+                    g.backward(acts[i], ys, losses[i], stream=s)
+                    g.sgd(stream=s)
             for s in streams:
                 main.wait_stream(s)
         else:
             for i, g in enumerate(self.gb):
                 g.forward(acts[i], acts[i + 1] if g.layers else None)
-            for i, g in enumerate(self.gb):
-                g.backward(acts[i], ys, losses[i])
-            for g in self.gb:
-                g.sgd()
+            if self.fused_update:
+                for i, g in enumerate(self.gb):
+                    g.backward_update(acts[i], ys, losses[i])
+            else:
+                for i, g in enumerate(self.gb):
+                    g.backward(acts[i], ys, losses[i])
+                for g in self.gb:
+                    g.sgd()
         torch.cuda.synchronize()
         return [int(l.item()) for l in losses]
 
@@ -106,10 +114,11 @@ def _eq(got, want, what):
 
 
 def run_workload(wl, steps, seed=20240716, check_every=1, data_seed=7, concurrent=False,
-                 batch=None, **hyper):
+                 batch=None, fused_update=False, **hyper):
     batch = batch or wl["batch"]
     hyper = dict(wl.get("hyper", {}), **hyper)
-    pair = NetPair(wl["blocks"], batch, seed=seed, concurrent=concurrent, **hyper)
+    pair = NetPair(wl["blocks"], batch, seed=seed, concurrent=concurrent,
+                   fused_update=fused_update, **hyper)
     try:
         for s in range(steps):
             x = synth.images(data_seed, s, batch, wl["input_shape"])
