@@ -11,6 +11,8 @@
 // the element-wise stages always run here.
 #include <cuda_bf16.h>
 
+#include <algorithm>
+
 #include "nitro_internal.cuh"
 #include "prof.cuh"
 
@@ -196,102 +198,113 @@ __global__ void k_fwd_epilogue(const int64_t* __restrict__ z, LayerGeom g, int B
 }
 
 // ---------------------------------------------------------------------------
-// Learning layer forward + RSS loss, in one kernel.  A CTA (128-feature
-// slice, 16 samples) adds its partial sums of z[b][g] = sum_j a[b][j] W_lr[g][j]
-// into zsum with int64 atomics (exact, order independent).  The last CTA of
-// a sample group (per-group ticket) turns that group's z into
-// y_hat = floor(z / (256 d)) and grad_L = y_hat - 32 onehot and adds its part
-// of the SSE; the last of those (final ticket) writes the loss.
-// Tickets live behind zsum: zsum[B G + y] per group, zsum[B G + groups].
+// Learning layer forward + RSS loss, in two short kernels with no atomics
+// between them.  k_learn_partial: CTA (s, y) covers the 16 samples of group y
+// and the 128-feature chunks s, s + S, s + 2S, ... of the d features (S
+// slices), and writes its partial sums of z[b][g] = sum_j a[b][j] W_lr[g][j]
+// to part[s][b][g] with plain stores.  k_learn_finish: one thread per (b, g)
+// adds the S partials (exact int64), forms y_hat = floor(z / (256 d)) and
+// grad_L = y_hat - 32 onehot, and adds its share of the SSE; the last CTA
+// (ticket) writes the loss.
 // ---------------------------------------------------------------------------
 constexpr int kLrSamples = 16;   // samples per CTA
-constexpr int kLpSlice = 128;    // features per CTA
+constexpr int kLpSlice = 128;    // features per chunk
+constexpr int kLpMaxSlices = 128;
 static_assert(kLpSlice == 16 * 8, "k_learn_partial: 16 lanes of 8 features per sample");
 
 __global__ void __launch_bounds__(256) k_learn_partial(const int8_t* __restrict__ a,
                                                        const int32_t* __restrict__ wlr, int B,
                                                        int d, int G, int vec8,
-                                                       unsigned long long* __restrict__ zsum,
-                                                       FloorDiv dv, const int32_t* __restrict__ labels,
-                                                       int32_t* __restrict__ grad_l,
-                                                       unsigned long long* sse, int64_t* loss,
-                                                       uint32_t* maxabs_gl, uint32_t* status) {
-    // thread (u, k): sample u of the group, features 8k .. 8k + 7 of the slice,
+                                                       long long* __restrict__ part) {
+    // thread (u, k): sample u of the group, features 8k .. 8k + 7 of a chunk,
     // read as one 8-byte word when the rows allow it (vec8: d % 8 == 0 and an
-    // 8-byte aligned a).  The slice of W_lr is staged in shared memory with
+    // 8-byte aligned a).  A chunk of W_lr is staged in shared memory with
     // feature 8k + m at column 16m + k, so the lanes of a sample read
-    // consecutive words; classes in chunks of kLpG.
+    // consecutive words; classes in groups of kLpG.
     constexpr int kLpG = 16;
     __shared__ int32_t ws[kLpG][kLpSlice + 1];
     const int u = threadIdx.x >> 4, k = threadIdx.x & 15;
     const int b = blockIdx.y * kLrSamples + u;
-    const int j0 = blockIdx.x * kLpSlice;
-    const int jb = j0 + 8 * k;
-    int av[8];
-    if (vec8 && b < B && jb + 8 <= d) {
-        const uint2 w = *reinterpret_cast<const uint2*>(a + (int64_t)b * d + jb);
-#pragma unroll
-        for (int m = 0; m < 4; ++m) {
-            av[m] = (int8_t)(w.x >> (8 * m));
-            av[4 + m] = (int8_t)(w.y >> (8 * m));
-        }
-    } else {
-#pragma unroll
-        for (int m = 0; m < 8; ++m) {
-            const int j = jb + m;
-            av[m] = (b < B && j < d) ? a[(int64_t)b * d + j] : 0;
-        }
-    }
+    const int S = gridDim.x;
     for (int gc = 0; gc < G; gc += kLpG) {
         const int ng = min(kLpG, G - gc);
-        if (gc) __syncthreads();
-        for (int i = threadIdx.x; i < ng * kLpSlice; i += blockDim.x) {
-            const int g = i / kLpSlice, j = i - g * kLpSlice;
-            ws[g][(j & 7) * 16 + (j >> 3)] = j0 + j < d ? wlr[(int64_t)(gc + g) * d + j0 + j] : 0;
+        long long t[kLpG];
+#pragma unroll
+        for (int g = 0; g < kLpG; ++g) t[g] = 0;
+        for (int j0 = blockIdx.x * kLpSlice; j0 < d; j0 += S * kLpSlice) {
+            const int jb = j0 + 8 * k;
+            int av[8];
+            if (vec8 && b < B && jb + 8 <= d) {
+                const uint2 w = *reinterpret_cast<const uint2*>(a + (int64_t)b * d + jb);
+#pragma unroll
+                for (int m = 0; m < 4; ++m) {
+                    av[m] = (int8_t)(w.x >> (8 * m));
+                    av[4 + m] = (int8_t)(w.y >> (8 * m));
+                }
+            } else {
+#pragma unroll
+                for (int m = 0; m < 8; ++m) {
+                    const int j = jb + m;
+                    av[m] = (b < B && j < d) ? a[(int64_t)b * d + j] : 0;
+                }
+            }
+            __syncthreads();   // readers of the previous chunk are done
+            for (int i = threadIdx.x; i < ng * kLpSlice; i += blockDim.x) {
+                const int g = i / kLpSlice, j = i - g * kLpSlice;
+                ws[g][(j & 7) * 16 + (j >> 3)] = j0 + j < d ? wlr[(int64_t)(gc + g) * d + j0 + j] : 0;
+            }
+            __syncthreads();
+#pragma unroll
+            for (int g = 0; g < kLpG; ++g) {
+                if (g >= ng) break;
+#pragma unroll
+                for (int m = 0; m < 8; ++m) t[g] += (long long)ws[g][16 * m + k] * av[m];
+            }
         }
-        __syncthreads();
-        for (int g = 0; g < ng; ++g) {
-            long long t = 0;
 #pragma unroll
-            for (int m = 0; m < 8; ++m) t += (long long)ws[g][16 * m + k] * av[m];
+        for (int g = 0; g < kLpG; ++g) {
+            if (g >= ng) break;
+            long long v = t[g];
 #pragma unroll
-            for (int off = 8; off; off >>= 1) t += __shfl_xor_sync(kFull, t, off);
-            if (k == 0 && b < B && t != 0)
-                atomicAdd(&zsum[(int64_t)b * G + gc + g], (unsigned long long)t);
+            for (int off = 8; off; off >>= 1) v += __shfl_xor_sync(kFull, v, off);
+            if (k == 0 && b < B) part[((int64_t)blockIdx.x * B + b) * G + gc + g] = v;
         }
     }
-    __shared__ int last;
+}
+
+__global__ void __launch_bounds__(256) k_learn_finish(const long long* __restrict__ part, int S,
+                                                      int B, int G, FloorDiv dv,
+                                                      const int32_t* __restrict__ labels,
+                                                      int32_t* __restrict__ grad_l,
+                                                      unsigned long long* sse, int64_t* loss,
+                                                      uint32_t* maxabs_gl, uint32_t* status,
+                                                      unsigned int* ticket) {
     __shared__ unsigned long long red_s[8];
     __shared__ uint32_t red_m[8];
     __shared__ int flags;
-    unsigned long long* tickets = zsum + (int64_t)B * G;
-    if (k == 0) __threadfence();     // the lanes that added into zsum
+    if (threadIdx.x == 0) flags = 0;
     __syncthreads();
-    if (threadIdx.x == 0) {
-        flags = 0;
-        last = atomicAdd(&tickets[blockIdx.y], 1ull) == (unsigned long long)gridDim.x - 1;
-    }
-    __syncthreads();
-    if (!last) return;
-    __threadfence();
-    // this sample group's z is complete: y_hat, grad_L, its share of the SSE
+    const int i = blockIdx.x * blockDim.x + threadIdx.x;
+    const int n = B * G;
     unsigned long long ss = 0;
     uint32_t mx = 0;
     int fl = 0;
-    const int nb = min(kLrSamples, B - (int)blockIdx.y * kLrSamples);
-    for (int i = threadIdx.x; i < nb * G; i += blockDim.x) {
-        const int bb = blockIdx.y * kLrSamples + i / G, g = i % G;
+    if (i < n) {
+        unsigned long long z = 0;     // exact: partial sums of at most 2^31 products
+#pragma unroll 8
+        for (int s2 = 0; s2 < S; ++s2) z += (unsigned long long)part[(int64_t)s2 * n + i];
+        const int bb = i / G, g = i - bb * G;
         const int lab = labels[bb];
         const bool bad = lab < 0 || lab >= G;
         if (bad && g == 0) fl |= ST_BAD_LABEL;
         // NITRO-Scaling, SF = 2^8 d: floor(floor(z / 256) / d)
-        const int64_t yhat = dv.floor_div((int64_t)__ldcg(zsum + (int64_t)bb * G + g) >> 8);
+        const int64_t yhat = dv.floor_div((int64_t)z >> 8);
         const int64_t v = yhat - ((!bad && g == lab) ? 32 : 0);
         if (!fits_i32(v)) fl |= ST_OVERFLOW;
         const int32_t sv = (int32_t)v;
-        grad_l[(int64_t)bb * G + g] = sv;
-        ss += (unsigned long long)((int64_t)sv * sv);
-        mx = max(mx, abs_u32(sv));
+        grad_l[i] = sv;
+        ss = (unsigned long long)((int64_t)sv * sv);
+        mx = abs_u32(sv);
     }
 #pragma unroll
     for (int off = 16; off; off >>= 1) {
@@ -310,10 +323,11 @@ __global__ void __launch_bounds__(256) k_learn_partial(const int8_t* __restrict_
         if (m) atomicMax(maxabs_gl, m);
         if (flags) atomicOr(status, (uint32_t)flags);
         __threadfence();
-        if (atomicAdd(&tickets[gridDim.y], 1ull) == (unsigned long long)gridDim.y - 1) {
+        if (atomicAdd(ticket, 1u) == gridDim.x - 1) {
             __threadfence();
             const unsigned long long tot = atomicAdd(sse, 0ull);
             if (loss) *loss = fdiv64((int64_t)tot, 2);
+            *ticket = 0;                                     // ready for the next launch
         }
     }
 }
@@ -1209,21 +1223,31 @@ cudaError_t simt_lrpool_to_delta(const int32_t* gl, const int32_t* wlr, int G, i
     return cudaGetLastError();
 }
 
+size_t simt_learn_scratch(int max_batch, int d, int G) {
+    const int S = std::min(kLpMaxSlices, (d + kLpSlice - 1) / kLpSlice);
+    return (size_t)S * max_batch * G + 1;
+}
+
 cudaError_t simt_learn_fwd(const int8_t* a, const int32_t* wlr, const int32_t* labels, int B,
-                           int d, int G, int64_t* zsum, int32_t* grad_l, unsigned long long* sse,
+                           int d, int G, int64_t* scratch, int32_t* grad_l, unsigned long long* sse,
                            int64_t* loss, uint32_t* maxabs_gl, uint32_t* status, cudaStream_t s) {
     if (B <= 0) return cudaSuccess;
     const int groups = (B + kLrSamples - 1) / kLrSamples;
-    // partial sums, then the per-group tickets and the final ticket
-    cudaError_t e = cudaMemsetAsync(zsum, 0, sizeof(int64_t) * ((size_t)B * G + groups + 1), s);
+    const int S = std::min(kLpMaxSlices, (d + kLpSlice - 1) / kLpSlice);
+    // word 0: the finish kernel's ticket (zero between launches); then the partials
+    unsigned int* ticket = reinterpret_cast<unsigned int*>(scratch);
+    long long* part = reinterpret_cast<long long*>(scratch + 1);
+    {
+        ProfScope ps(K_LEARN_FWD, s, 2.0 * B * d * G, 0.0);
+        const int vec8 = d % 8 == 0 && ((uintptr_t)a & 7) == 0;
+        k_learn_partial<<<dim3(S, groups), 256, 0, s>>>(a, wlr, B, d, G, vec8, part);
+    }
+    cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    dim3 grid((d + kLpSlice - 1) / kLpSlice, groups);
-    ProfScope ps(K_LEARN_FWD, s, 2.0 * B * d * G, 0.0);
-    const int vec8 = d % 8 == 0 && ((uintptr_t)a & 7) == 0;
-    k_learn_partial<<<grid, 256, 0, s>>>(a, wlr, B, d, G, vec8,
-                                         reinterpret_cast<unsigned long long*>(zsum),
-                                         FloorDiv::make((uint64_t)d), labels, grad_l, sse, loss,
-                                         maxabs_gl, status);
+    ProfScope ps(K_FINISH_LOSS, s, 0.0, 0.0);
+    k_learn_finish<<<(B * G + 255) / 256, 256, 0, s>>>(part, S, B, G, FloorDiv::make((uint64_t)d),
+                                                      labels, grad_l, sse, loss, maxabs_gl,
+                                                      status, ticket);
     return cudaGetLastError();
 }
 

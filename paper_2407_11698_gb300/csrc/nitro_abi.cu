@@ -50,7 +50,7 @@ struct nitro_block {
     int32_t* Wlr = nullptr;
     int64_t* dWlr = nullptr;
     int32_t* grad_l = nullptr;      // [max_batch x G]
-    int64_t* zsum = nullptr;        // [max_batch x G] learning-layer pre-activations, then a ticket
+    int64_t* zsum = nullptr;        // learning-layer partial sums and ticket (simt_learn_scratch)
     int64_t* z64 = nullptr;         // scratch, int64 pre-activations / dgrad outputs
     size_t z64_elems = 0;
     uint32_t* words = nullptr;      // [0] status [1] max|grad_l| [2] max|W_lr|
@@ -270,7 +270,7 @@ nitro_status nitro_init_block(const nitro_block_desc* desc, uint64_t seed, void*
         }
     }
     ok = ok && dalloc(b, &b->Wlr, (size_t)b->G * b->d) && dalloc(b, &b->dWlr, (size_t)b->G * b->d) &&
-         dalloc(b, &b->grad_l, (size_t)MB * b->G) && dalloc(b, &b->zsum, (size_t)MB * b->G + (MB + 15) / 16 + 1) && dalloc(b, &b->z64, z_need) &&
+         dalloc(b, &b->grad_l, (size_t)MB * b->G) && dalloc(b, &b->zsum, simt_learn_scratch(MB, (int)b->d, b->G)) && dalloc(b, &b->z64, z_need) &&
          dalloc(b, &b->words, n_words(desc->n_layers)) && dalloc(b, &b->sse, 1);
     b->z64_elems = z_need;
     for (int i = 0; ok && i < desc->n_layers; ++i)
@@ -294,6 +294,8 @@ nitro_status nitro_init_block(const nitro_block_desc* desc, uint64_t seed, void*
     if (e == cudaSuccess) e = cudaMemsetAsync(b->dWlr, 0, (size_t)b->G * b->d * 8, s);
     if (e == cudaSuccess) e = cudaMemcpyAsync(b->words, words.data(), words.size() * 4, cudaMemcpyHostToDevice, s);
     if (e == cudaSuccess) e = cudaMemsetAsync(b->sse, 0, 8, s);
+    if (e == cudaSuccess)
+        e = cudaMemsetAsync(b->zsum, 0, 8 * simt_learn_scratch(MB, (int)b->d, b->G), s);
     for (int i = 0; e == cudaSuccess && i < desc->n_layers; ++i) {
         e = tc_refresh_weights(b->L[i].tc, b->L[i].g, b->L[i].W, w_w(b, i), s);
         if (e == cudaSuccess && b->L[i].lin_planes)

@@ -694,38 +694,52 @@ __global__ void __launch_bounds__(kThreads, 1)
                             bool ovf = false;
                             if (ok) {
                                 const int tt = args.taps == 1 ? 0 : t;
+                                const int64_t pcol = args.taps == 1 ? (int64_t)m : (int64_t)tt * args.tap_k + ci;
+                                // 16 columns at a time: all loads of a group are issued
+                                // before any store, so a group costs one memory round trip
 #pragma unroll
-                                for (int i = 0; i < NH; ++i) {
-                                    const int co = col0 + i;
-                                    if (co >= args.ncols) break;
-                                    const int64_t e = (int64_t)co * cstride + wrow;
-                                    const int64_t g = args.atomic_out
-                                        ? (int64_t)__ldcg(reinterpret_cast<const unsigned long long*>(args.out + e))
-                                        : (int64_t)acc[i];
-                                    const int64_t w = args.wt[e];
-                                    int64_t d = args.trunc ? args.gdiv.trunc_div(g) : args.gdiv.floor_div(g);
-                                    if (args.decay) d += args.trunc ? args.ediv.trunc_div(w) : args.ediv.floor_div(w);
-                                    const int64_t nw = w - d;
-                                    ovf |= !fits_i32(nw);
-                                    const int32_t s32 = (int32_t)nw;
-                                    args.wt[e] = s32;
-                                    mx = max(mx, abs_u32(s32));
-                                    if (args.wp) {
-                                        // limb planes of the new weight, entry (t, ci) of row co
-                                        uint16_t* pp = args.wp + (int64_t)co * args.row_k +
-                                                       (args.taps == 1 ? (int64_t)m : (int64_t)tt * args.tap_k + ci);
-                                        int32_t x = s32;
+                                for (int i0 = 0; i0 < NH; i0 += 16) {
+                                    if (col0 + i0 >= args.ncols) break;   // uniform across the warp
+                                    int64_t gv[16];
+                                    int32_t wv[16];
 #pragma unroll
-                                        for (int l = 0; l < 4; ++l) {
-                                            int dg;
-                                            if (l < 3) {
-                                                const int rr = x & 255;
-                                                dg = rr - ((rr >> 7) << 8);
-                                                x = (x >> 8) + (rr >> 7);
-                                            } else {
-                                                dg = x;
+                                    for (int i = 0; i < 16; ++i) {
+                                        const int co = min(col0 + i0 + i, args.ncols - 1);
+                                        const int64_t e = (int64_t)co * cstride + wrow;
+                                        gv[i] = args.atomic_out
+                                            ? (int64_t)__ldcg(reinterpret_cast<const unsigned long long*>(args.out + e))
+                                            : (int64_t)acc[i0 + i];
+                                        wv[i] = __ldcg(args.wt + e);
+                                    }
+#pragma unroll
+                                    for (int i = 0; i < 16; ++i) {
+                                        const int co = col0 + i0 + i;
+                                        if (co >= args.ncols) break;
+                                        const int64_t e = (int64_t)co * cstride + wrow;
+                                        const int64_t w = wv[i];
+                                        int64_t d = args.trunc ? args.gdiv.trunc_div(gv[i]) : args.gdiv.floor_div(gv[i]);
+                                        if (args.decay) d += args.trunc ? args.ediv.trunc_div(w) : args.ediv.floor_div(w);
+                                        const int64_t nw = w - d;
+                                        ovf |= !fits_i32(nw);
+                                        const int32_t s32 = (int32_t)nw;
+                                        args.wt[e] = s32;
+                                        mx = max(mx, abs_u32(s32));
+                                        if (args.wp) {
+                                            // limb planes of the new weight, entry (t, ci) of row co
+                                            uint16_t* pp = args.wp + (int64_t)co * args.row_k + pcol;
+                                            int32_t x = s32;
+#pragma unroll
+                                            for (int l = 0; l < 4; ++l) {
+                                                int dg;
+                                                if (l < 3) {
+                                                    const int rr = x & 255;
+                                                    dg = rr - ((rr >> 7) << 8);
+                                                    x = (x >> 8) + (rr >> 7);
+                                                } else {
+                                                    dg = x;
+                                                }
+                                                pp[l * args.w_plane] = (uint16_t)(__float_as_uint((float)dg) >> 16);
                                             }
-                                            pp[l * args.w_plane] = (uint16_t)(__float_as_uint((float)dg) >> 16);
                                         }
                                     }
                                 }
@@ -848,54 +862,73 @@ __global__ void __launch_bounds__(kThreads, 1)
                             ppix[k] = args.low_pool
                                 ? ((int64_t)b * args.low_h + 2 * y + (k >> 1)) * args.low_w + 2 * x + (k & 1)
                                 : opix;
-                        // per 16 channels: the argmax and region words of every window
-                        // position are loaded first (16-byte loads), then the gradient,
-                        // its floor quotient by alpha_inv and the stores, 4 channels at
-                        // a time
+                        // the int32 values first (storage rule), then the argmax and
+                        // region words of all the thread's channels and window positions
+                        // in one batch of 16-byte loads, then per 4 channels the floor
+                        // quotient by alpha_inv, the routing and the stores
+                        constexpr int NG16 = NH / 16;
+                        int32_t gsv[NH];
 #pragma unroll
-                        for (int k16 = 0; k16 < NH / 16; ++k16) {
-                            const int c16 = col0 + 16 * k16;
-                            if (c16 >= Cl) break;
-                            const uint4 amv = args.low_pool
-                                ? *reinterpret_cast<const uint4*>(args.low_argmax + opix * Cl + c16)
-                                : make_uint4(0, 0, 0, 0);
-                            uint4 rgv[4];
+                        for (int i = 0; i < NH; ++i) {
+                            const int64_t gv = (int64_t)acc[i];
+                            ovf |= col0 + i < Cl && !fits_i32(gv);
+                            gsv[i] = (int32_t)gv;
+                        }
+                        // two groups of 16 channels per batch of code loads
 #pragma unroll
-                            for (int k = 0; k < 4; ++k)
-                                rgv[k] = k < npos ? *reinterpret_cast<const uint4*>(args.low_region + ppix[k] * Cl + c16)
-                                                  : make_uint4(0, 0, 0, 0);
-                            const uint32_t amw4[4] = {amv.x, amv.y, amv.z, amv.w};
+                        for (int kp = 0; kp < NG16; kp += 2) {
+                            if (col0 + 16 * kp >= Cl) break;   // uniform across the warp
+                            uint4 amv[2], rgv[2][4];
 #pragma unroll
-                            for (int e4 = 0; e4 < 4; ++e4) {
-                                const int c0 = c16 + 4 * e4;
-                                int32_t gs[4], gq[4];   // gradient and floor(gradient / alpha_inv)
+                            for (int h = 0; h < 2; ++h) {
+                                const int c16 = col0 + 16 * (kp + h);
+                                const bool in = c16 < Cl;
+                                amv[h] = (args.low_pool && in)
+                                    ? *reinterpret_cast<const uint4*>(args.low_argmax + opix * Cl + c16)
+                                    : make_uint4(0, 0, 0, 0);
 #pragma unroll
-                                for (int e = 0; e < 4; ++e) {
-                                    const int64_t gv = (int64_t)acc[16 * k16 + 4 * e4 + e];
-                                    ovf |= !fits_i32(gv);
-                                    gs[e] = (int32_t)gv;
-                                    gq[e] = args.alpha32.floor_div(gs[e]);
-                                }
-                                const uint32_t amw = amw4[e4];
+                                for (int k = 0; k < 4; ++k)
+                                    rgv[h][k] = (k < npos && in)
+                                        ? *reinterpret_cast<const uint4*>(args.low_region + ppix[k] * Cl + c16)
+                                        : make_uint4(0, 0, 0, 0);
+                            }
 #pragma unroll
-                                for (int k = 0; k < 4; ++k) {
-                                    if (k >= npos) break;
-                                    const uint32_t rw[4] = {rgv[k].x, rgv[k].y, rgv[k].z, rgv[k].w};
-                                    const uint32_t rgw = rw[e4];
-                                    int32_t dv[4];
+                            for (int h = 0; h < 2; ++h) {
+                                const int k16 = kp + h;
+                                const int c16 = col0 + 16 * k16;
+                                if (c16 >= Cl) break;
+                                const uint32_t amw4[4] = {amv[h].x, amv[h].y, amv[h].z, amv[h].w};
+#pragma unroll
+                                for (int e4 = 0; e4 < 4; ++e4) {
+                                    const int c0 = c16 + 4 * e4;
+                                    int32_t gs[4], gq[4];   // gradient and floor(gradient / alpha_inv)
 #pragma unroll
                                     for (int e = 0; e < 4; ++e) {
-                                        const int reg = (int)((rgw >> (8 * e)) & 255u);
-                                        const int am = (int)((amw >> (8 * e)) & 255u);
-                                        const int32_t v = am != k ? 0 : (reg == 1 ? gq[e] : (reg == 2 ? gs[e] : 0));
-                                        dv[e] = v;
-                                        mx = max(mx, abs_u32(v));
+                                        gs[e] = gsv[16 * k16 + 4 * e4 + e];
+                                        gq[e] = args.alpha32.floor_div(gs[e]);
                                     }
-                                    *reinterpret_cast<int4*>(args.low_delta + ppix[k] * Cl + c0) =
-                                        make_int4(dv[0], dv[1], dv[2], dv[3]);
-                                    if (args.low_planes)
-                                        store_delta_planes4(args.low_planes + ppix[k] * Cl + c0,
-                                                            args.low_plane, dv[0], dv[1], dv[2], dv[3]);
+                                    const uint32_t amw = amw4[e4];
+#pragma unroll
+                                    for (int k = 0; k < 4; ++k) {
+                                        if (k >= npos) break;
+                                        const uint32_t rw[4] = {rgv[h][k].x, rgv[h][k].y, rgv[h][k].z,
+                                                                rgv[h][k].w};
+                                        const uint32_t rgw = rw[e4];
+                                        int32_t dv[4];
+#pragma unroll
+                                        for (int e = 0; e < 4; ++e) {
+                                            const int reg = (int)((rgw >> (8 * e)) & 255u);
+                                            const int am = (int)((amw >> (8 * e)) & 255u);
+                                            const int32_t v = am != k ? 0 : (reg == 1 ? gq[e] : (reg == 2 ? gs[e] : 0));
+                                            dv[e] = v;
+                                            mx = max(mx, abs_u32(v));
+                                        }
+                                        *reinterpret_cast<int4*>(args.low_delta + ppix[k] * Cl + c0) =
+                                            make_int4(dv[0], dv[1], dv[2], dv[3]);
+                                        if (args.low_planes)
+                                            store_delta_planes4(args.low_planes + ppix[k] * Cl + c0,
+                                                                args.low_plane, dv[0], dv[1], dv[2], dv[3]);
+                                    }
                                 }
                             }
                         }
