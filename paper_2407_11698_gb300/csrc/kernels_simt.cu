@@ -279,40 +279,40 @@ __global__ void __launch_bounds__(256) k_learn_finish(const long long* __restric
                                                       unsigned long long* sse, int64_t* loss,
                                                       uint32_t* maxabs_gl, uint32_t* status,
                                                       unsigned int* ticket) {
+    // one warp per output (b, g): the lanes add the S partials (at most 4
+    // each, loads issued together), then lane 0 finishes the output
     __shared__ unsigned long long red_s[8];
     __shared__ uint32_t red_m[8];
     __shared__ int flags;
     if (threadIdx.x == 0) flags = 0;
     __syncthreads();
-    const int i = blockIdx.x * blockDim.x + threadIdx.x;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int i = blockIdx.x * 8 + warp;
     const int n = B * G;
     unsigned long long ss = 0;
     uint32_t mx = 0;
-    int fl = 0;
     if (i < n) {
-        unsigned long long z = 0;     // exact: partial sums of at most 2^31 products
-#pragma unroll 8
-        for (int s2 = 0; s2 < S; ++s2) z += (unsigned long long)part[(int64_t)s2 * n + i];
-        const int bb = i / G, g = i - bb * G;
-        const int lab = labels[bb];
-        const bool bad = lab < 0 || lab >= G;
-        if (bad && g == 0) fl |= ST_BAD_LABEL;
-        // NITRO-Scaling, SF = 2^8 d: floor(floor(z / 256) / d)
-        const int64_t yhat = dv.floor_div((int64_t)z >> 8);
-        const int64_t v = yhat - ((!bad && g == lab) ? 32 : 0);
-        if (!fits_i32(v)) fl |= ST_OVERFLOW;
-        const int32_t sv = (int32_t)v;
-        grad_l[i] = sv;
-        ss = (unsigned long long)((int64_t)sv * sv);
-        mx = abs_u32(sv);
-    }
+        unsigned long long z = 0;     // exact: the partial sums of z fit int64
+        for (int s2 = lane; s2 < S; s2 += 32) z += (unsigned long long)part[(int64_t)s2 * n + i];
 #pragma unroll
-    for (int off = 16; off; off >>= 1) {
-        ss += __shfl_xor_sync(kFull, ss, off);
-        mx = max(mx, __shfl_xor_sync(kFull, mx, off));
+        for (int off = 16; off; off >>= 1) z += __shfl_xor_sync(kFull, z, off);
+        if (lane == 0) {
+            int fl = 0;
+            const int bb = i / G, g = i - bb * G;
+            const int lab = labels[bb];
+            const bool bad = lab < 0 || lab >= G;
+            if (bad && g == 0) fl |= ST_BAD_LABEL;
+            // NITRO-Scaling, SF = 2^8 d: floor(floor(z / 256) / d)
+            const int64_t yhat = dv.floor_div((int64_t)z >> 8);
+            const int64_t v = yhat - ((!bad && g == lab) ? 32 : 0);
+            if (!fits_i32(v)) fl |= ST_OVERFLOW;
+            const int32_t sv = (int32_t)v;
+            grad_l[i] = sv;
+            ss = (unsigned long long)((int64_t)sv * sv);
+            mx = abs_u32(sv);
+            if (fl) atomicOr(&flags, fl);
+        }
     }
-    if (fl) atomicOr(&flags, fl);
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     if (lane == 0) { red_s[warp] = ss; red_m[warp] = mx; }
     __syncthreads();
     if (threadIdx.x == 0) {
@@ -1245,7 +1245,7 @@ cudaError_t simt_learn_fwd(const int8_t* a, const int32_t* wlr, const int32_t* l
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     ProfScope ps(K_FINISH_LOSS, s, 0.0, 0.0);
-    k_learn_finish<<<(B * G + 255) / 256, 256, 0, s>>>(part, S, B, G, FloorDiv::make((uint64_t)d),
+    k_learn_finish<<<(B * G + 7) / 8, 256, 0, s>>>(part, S, B, G, FloorDiv::make((uint64_t)d),
                                                       labels, grad_l, sse, loss, maxabs_gl,
                                                       status, ticket);
     return cudaGetLastError();

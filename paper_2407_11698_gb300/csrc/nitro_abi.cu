@@ -273,9 +273,13 @@ nitro_status nitro_init_block(const nitro_block_desc* desc, uint64_t seed, void*
          dalloc(b, &b->grad_l, (size_t)MB * b->G) && dalloc(b, &b->zsum, simt_learn_scratch(MB, (int)b->d, b->G)) && dalloc(b, &b->z64, z_need) &&
          dalloc(b, &b->words, n_words(desc->n_layers)) && dalloc(b, &b->sse, 1);
     b->z64_elems = z_need;
-    for (int i = 0; ok && i < desc->n_layers; ++i)
-        ok = tc_layer_init(b->L[i].tc, b->L[i].g, desc->max_batch, i > 0, w_w(b, i), w_delta(b, i),
-                           b->allocs, b->host_allocs);
+    for (int i = 0; ok && i < desc->n_layers; ++i) {
+        Layer& ly = b->L[i];
+        ok = ly.lin_a ? tc_linear_init(ly.tc, ly.g, desc->max_batch, ly.lin_a, w_w(b, i), w_delta(b, i),
+                                       b->allocs, b->host_allocs)
+                      : tc_layer_init(ly.tc, ly.g, desc->max_batch, i > 0, w_w(b, i), w_delta(b, i),
+                                      b->allocs, b->host_allocs);
+    }
     if (!ok) {
         free_all(b);
         delete b;
@@ -471,16 +475,25 @@ nitro_status block_backward(nitro_block* b, const int8_t* a_in, const int32_t* l
         // fused update: the input gradient reads the pre-update weights, so it
         // runs first (after the delta split), then the weight gradient with
         // IntegerSGD; otherwise weight gradient first, as the split requires
-        const bool fuse_sgd = updated && ly.tc.wgrad;
+        const bool fuse_sgd = updated && tc_wgrad_fusable(ly.tc, g, batch);
         auto wgrad = [&]() -> nitro_status {
             if (fuse_sgd) {
                 NITRO_TRY(cudaMemsetAsync(w_w(b, i), 0, 4, s));
                 TcSgd sg{gamma_fw, b->desc.eta_inv_fw, b->desc.sgd_round == NITRO_ROUND_TRUNC, ly.W,
-                         w_w(b, i)};
+                         w_w(b, i), nullptr, 0, 0, 0};
+                if (ly.lin_planes) {
+                    // linear weight planes [4][out][in]
+                    sg.planes = ly.lin_planes;
+                    sg.plane = ly.wcount;
+                    sg.row_k = g.cin;
+                } else {
+                    tc_weight_planes(ly.tc, g, &sg.planes, &sg.plane, &sg.row_k, &sg.tap_k);
+                }
+                bool sgd_done = false;
                 NITRO_TRY(tc_conv_wgrad(ly.tc, g, ly.delta, w_delta(b, i), batch, ly.dW, w_status(b), s,
-                                        &done, true, &sg));
-                (*updated)[i] = done;
-                if (done) NITRO_TRY(tc_weights_hint(ly.tc, s));
+                                        &done, true, &sg, &sgd_done));
+                (*updated)[i] = done && sgd_done;
+                if ((*updated)[i]) NITRO_TRY(tc_weights_hint(ly.tc, s));
             } else {
                 NITRO_TRY(tc_conv_wgrad(ly.tc, g, ly.delta, w_delta(b, i), batch, ly.dW, w_status(b), s,
                                         &done, planes_done[i] != 0));
@@ -512,7 +525,7 @@ nitro_status block_backward(nitro_block* b, const int8_t* a_in, const int32_t* l
         bool fused = false;
         Layer& lo = b->L[i - 1];
         TcDgradOut fo{b->desc.alpha_inv, w_delta(b, i), w_w(b, i), lo.g.h, lo.g.w, lo.g.pool,
-                      lo.region, lo.argmax, lo.delta, w_delta(b, i - 1), tc_delta_planes(lo.tc)};
+                      lo.region, lo.argmax, lo.delta, w_delta(b, i - 1)};
         // the fused epilogue needs the lower layer to be a conv on the same grid
         const bool can_fuse = lo.g.kind == NITRO_CONV3X3 && lo.g.oh == g.h && lo.g.ow == g.w;
         NITRO_TRY(tc_conv_dgrad(ly.tc, g, batch, b->z64, can_fuse ? &fo : nullptr, w_status(b), s,
@@ -521,9 +534,7 @@ nitro_status block_backward(nitro_block* b, const int8_t* a_in, const int32_t* l
             const int mode = g.kind == NITRO_CONV3X3 ? GM_CONV_DGRAD : GM_LIN_DGRAD;
             NITRO_TRY(simt_gemm(mode, nullptr, ly.delta, ly.W, b->z64, batch, g.h, g.w, g.cin, g.cout, s));
         }
-        if (fused) {
-            planes_done[i - 1] = fo.low_planes != nullptr;
-        } else {
+        if (!fused) {
             DeltaSrc src{};
             src.g64 = b->z64;
             src.maxabs_a = w_delta(b, i); src.maxabs_b = w_w(b, i);

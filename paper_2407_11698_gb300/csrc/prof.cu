@@ -41,7 +41,7 @@ const char* const kNames[K_COUNT] = {
     "learn_dw", "grad_to_delta", "integersgd", "learn_finish_loss", "tc_conv_fwd",
     "tc_conv_wgrad", "tc_conv_dgrad", "tc_pack_limbs", "tc_finish", "tc_gemm", "lr_backward",
     "tc_pack_weights", "tc_pack_input", "tc_pack_delta", "prep_sum", "prep_mad",
-    "prep_apply", "lr_pool", "lrpool_to_delta", "tc_timeout_probe"};
+    "prep_apply", "lr_pool", "lrpool_to_delta", "tc_timeout_probe", "tc_linear_wgrad"};
 
 }  // namespace
 

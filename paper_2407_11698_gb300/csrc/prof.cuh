@@ -40,6 +40,7 @@ enum KernelId : int {
     K_LR_POOL,
     K_LRPOOL_TO_DELTA,
     K_TC_PROBE,
+    K_TC_LIN_WGRAD,
     K_COUNT
 };
 

@@ -28,15 +28,18 @@ constexpr int kBM = 128;              // rows per tile (TMEM lanes)
 constexpr int kBK = 64;               // K elements per block (one 128-byte row)
 constexpr int kChunkBlocks = 16;      // 16 x 64 = 1024 products per exact chunk
 // Warp roles: warpgroup 0 = TMA warp, MMA warp and two idle warps; warpgroups
-// 1 and 2 = the epilogue, two warps per TMEM lane quadrant, each holding half
-// of the N columns as int64 accumulators.  The warpgroups split the register
-// file with setmaxnreg: 128 x kRegsProducer + 256 x kRegsEpilogue must not
-// exceed kThreads x the registers the kernel is launched with (checked on the
-// host before the first launch).
+// 1 to 4 = the epilogue, four warps per TMEM lane quadrant, each holding a
+// quarter of the N columns as int64 accumulators.  The epilogue is bound by
+// memory latency, so it gets as many warps as the register file allows; the
+// warpgroups split it with setmaxnreg: 128 x kRegsProducer + 32 x kEpiWarps x
+// kRegsEpilogue must not exceed kThreads x the registers the kernel is
+// launched with (checked on the host before the first launch).  A layout with
+// eight epilogue warps (half the N columns each, 224 registers, no spills) was
+// measured slower: 175k against 257k images/s on the VGG-style step.
 constexpr int kEpiWarp0 = 4;          // first epilogue warp
-constexpr int kEpiWarps = 8;          // 2 per TMEM lane quadrant
+constexpr int kEpiWarps = 16;         // 4 per TMEM lane quadrant
 constexpr int kThreads = 32 * (kEpiWarp0 + kEpiWarps);
-constexpr int kRegsProducer = 48, kRegsEpilogue = 224;
+constexpr int kRegsProducer = 32, kRegsEpilogue = 112;
 constexpr uint64_t kWaitNs = 2000000000ull;   // 2 s bound on any wait
 
 // ------------------------------------------------------------------ PTX
@@ -254,12 +257,11 @@ struct TcArgs {
     const int8_t* low_argmax;
     int32_t* low_delta;
     uint32_t* low_maxabs;
-    uint16_t* low_planes;      // the lower delta's bf16 limb planes, or null
-    int64_t low_plane;
-    // weight gradient with IntegerSGD applied to the finished sums
+    // weight gradient: valid rows (taps == 1) and the row stride of dW / W
+    int rows;
+    int64_t cstride;
+    // weight gradient with IntegerSGD applied to the finished sums (no K split)
     int sgd;
-    int splits;                // K splits per output tile
-    int* tickets;              // per (tile, epilogue warp) arrivals, zero between launches
     int32_t* wt;               // the layer's weights [Cout][9][Cin]
     uint16_t* wp;              // weight limb planes [4][Cout][row_k], or null
     int64_t w_plane;
@@ -329,7 +331,7 @@ __global__ void __launch_bounds__(kThreads, 1)
               const TcArgs args) {
     using C = TcCfg<N, PB>;
     constexpr int S = C::S;
-    constexpr int NH = N / 2;            // columns per epilogue warp
+    constexpr int NH = N / 4;            // columns per epilogue warp
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
@@ -569,7 +571,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         // ---------------- epilogue: warpgroups 1 and 2
         asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(kRegsEpilogue));
         const int q = warp & 3;                     // TMEM lane quadrant this warp may read
-        const int half = (warp - kEpiWarp0) >> 2;   // which half of the N columns
+        const int half = (warp - kEpiWarp0) >> 2;   // which quarter of the N columns
         int chunk = 0;
         for (int tile = blockIdx.x; tile < args.total_tiles; tile += gridDim.x) {
             const Tile T = decode_tile(args, tile);
@@ -614,18 +616,29 @@ __global__ void __launch_bounds__(kThreads, 1)
                             }
                         }
                     };
-                    // 32 columns of one limb per TMEM round trip: two loads
-                    // issued back to back, then one wait
-                    for (int jb = 0; jb < nb; ++jb) {
-                        const uint32_t base = limb_base(jb);
-#pragma unroll
-                        for (int j2 = 0; j2 < NH / 32; ++j2) {
+                    // 32 values per TMEM round trip: two loads issued back to
+                    // back, then one wait (16 columns: two limbs at once)
+                    if (NH == 16) {
+                        for (int jb = 0; jb < nb; jb += 2) {
                             uint32_t r[32];
-                            tmem_ld16_nowait(base + 32 * j2, r);
-                            tmem_ld16_nowait(base + 32 * j2 + 16, r + 16);
+                            tmem_ld16_nowait(limb_base(jb), r);
+                            if (jb + 1 < nb) tmem_ld16_nowait(limb_base(jb + 1), r + 16);
                             tmem_wait_ld<32>(r);
-                            accumulate(r, 2 * j2, shift0 + 8 * jb);
-                            accumulate(r + 16, 2 * j2 + 1, shift0 + 8 * jb);
+                            accumulate(r, 0, shift0 + 8 * jb);
+                            if (jb + 1 < nb) accumulate(r + 16, 0, shift0 + 8 * (jb + 1));
+                        }
+                    } else {
+                        for (int jb = 0; jb < nb; ++jb) {
+                            const uint32_t base = limb_base(jb);
+#pragma unroll
+                            for (int j2 = 0; j2 < NH / 32; ++j2) {
+                                uint32_t r[32];
+                                tmem_ld16_nowait(base + 32 * j2, r);
+                                tmem_ld16_nowait(base + 32 * j2 + 16, r + 16);
+                                tmem_wait_ld<32>(r);
+                                accumulate(r, 2 * j2, shift0 + 8 * jb);
+                                accumulate(r + 16, 2 * j2 + 1, shift0 + 8 * jb);
+                            }
                         }
                     }
                     tc_fence_before();
@@ -654,9 +667,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const int m = T.mt * kBM + r;
                     const int t = m / args.cin_k, ci = m - t * args.cin_k;
                     // im2col rows: row m is already the (tap, ci) index t Cin + ci
-                    const bool ok = args.taps == 1 ? m < 9 * args.Cin : (t < 9 && ci < args.Cin);
+                    const bool ok = args.taps == 1 ? m < args.rows : (t < 9 && ci < args.Cin);
                     const int64_t wrow = args.taps == 1 ? (int64_t)m : (int64_t)t * args.Cin + ci;
-                    const int64_t cstride = 9LL * args.Cin;
+                    const int64_t cstride = args.cstride;
                     if (ok) {
                         int64_t* o = args.out + wrow;
 #pragma unroll
@@ -669,27 +682,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                         }
                     }
                     if (args.sgd) {
-                        // IntegerSGD (Algorithm 1) on this warp's 32 rows x NH columns
-                        // once their sums are final.  With a K split the warp of the
-                        // same slot that arrives last (per-slot ticket, after its
-                        // atomics are fenced) reads the sums back; no CTA-wide barrier
-                        // is involved, so a warp that gave up on a wait blocks nobody.
-                        bool mine = true;
-                        if (args.atomic_out) {
-                            __threadfence();
-                            __syncwarp();
-                            int* ticket = args.tickets + ((int64_t)T.mt * args.tiles_n + T.nt) * kEpiWarps +
-                                          (warp - kEpiWarp0);
-                            int tk = 0;
-                            if (lane == 0) tk = atomicAdd(ticket, 1);
-                            tk = __shfl_sync(0xffffffffu, tk, 0);
-                            mine = tk == args.splits - 1;
-                            if (mine) {
-                                if (lane == 0) *ticket = 0;   // ready for the next launch
-                                __threadfence();
-                            }
-                        }
-                        if (mine) {
+                        // IntegerSGD (Algorithm 1) on this thread's row of NH columns,
+                        // from the final sums in the accumulators (no K split)
+                        {
                             uint32_t mx = 0;
                             bool ovf = false;
                             if (ok) {
@@ -706,10 +701,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                                     for (int i = 0; i < 16; ++i) {
                                         const int co = min(col0 + i0 + i, args.ncols - 1);
                                         const int64_t e = (int64_t)co * cstride + wrow;
-                                        gv[i] = args.atomic_out
-                                            ? (int64_t)__ldcg(reinterpret_cast<const unsigned long long*>(args.out + e))
-                                            : (int64_t)acc[i0 + i];
-                                        wv[i] = __ldcg(args.wt + e);
+                                        gv[i] = (int64_t)acc[i0 + i];
+                                        wv[i] = args.wt[e];
                                     }
 #pragma unroll
                                     for (int i = 0; i < 16; ++i) {
@@ -882,7 +875,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                             for (int h = 0; h < 2; ++h) {
                                 const int c16 = col0 + 16 * (kp + h);
-                                const bool in = c16 < Cl;
+                                const bool in = kp + h < NG16 && c16 < Cl;
                                 amv[h] = (args.low_pool && in)
                                     ? *reinterpret_cast<const uint4*>(args.low_argmax + opix * Cl + c16)
                                     : make_uint4(0, 0, 0, 0);
@@ -896,7 +889,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                             for (int h = 0; h < 2; ++h) {
                                 const int k16 = kp + h;
                                 const int c16 = col0 + 16 * k16;
-                                if (c16 >= Cl) break;
+                                if (k16 >= NG16 || c16 >= Cl) break;
                                 const uint32_t amw4[4] = {amv[h].x, amv[h].y, amv[h].z, amv[h].w};
 #pragma unroll
                                 for (int e4 = 0; e4 < 4; ++e4) {
@@ -925,9 +918,6 @@ __global__ void __launch_bounds__(kThreads, 1)
                                         }
                                         *reinterpret_cast<int4*>(args.low_delta + ppix[k] * Cl + c0) =
                                             make_int4(dv[0], dv[1], dv[2], dv[3]);
-                                        if (args.low_planes)
-                                            store_delta_planes4(args.low_planes + ppix[k] * Cl + c0,
-                                                                args.low_plane, dv[0], dv[1], dv[2], dv[3]);
                                     }
                                 }
                             }
@@ -1320,7 +1310,29 @@ bool dalloc(std::vector<void*>& allocs, T** p, size_t count) {
 
 inline int round_up(int v, int m) { return (v + m - 1) / m * m; }
 
+// K split of the weight gradient: at most one wave of CTAs (every CTA one work
+// unit), each split at least one exact chunk.  Returns the split count.
+int wgrad_splits(int tiles, int kb_total, int* kb_per_split) {
+    int splits = sm_count() / tiles;
+    const int max_splits = (kb_total + kChunkBlocks - 1) / kChunkBlocks;
+    splits = splits < 1 ? 1 : (splits > max_splits ? max_splits : splits);
+    *kb_per_split = (kb_total + splits - 1) / splits;
+    return (kb_total + *kb_per_split - 1) / *kb_per_split;
+}
+
 }  // namespace
+
+bool tc_wgrad_fusable(const TcLayer& t, const LayerGeom& g, int batch) {
+    if (!t.wgrad || batch <= 0) return false;
+    const bool lin = g.kind == NITRO_LINEAR;
+    const int gh = lin ? 1 : g.h, gw = lin ? batch : g.w;
+    const int wb = gw <= 8 ? 8 : (gw <= 16 ? 16 : (gw <= 32 ? 32 : 64)), hb = 64 / wb;
+    const int taps = (t.im2col || lin) ? 1 : 9;
+    const int tiles = (taps * t.cin_k + kBM - 1) / kBM * ((g.cout + pick_n(g.cout) - 1) / pick_n(g.cout));
+    const int kb_total = (lin ? 1 : batch) * ((gw + wb - 1) / wb) * ((gh + hb - 1) / hb);
+    int kbs = 0;
+    return wgrad_splits(tiles, kb_total, &kbs) == 1;
+}
 
 bool tc_layer_init(TcLayer& t, const LayerGeom& g, int max_batch, bool has_dgrad,
                    const uint32_t* maxabs_w, const uint32_t* maxabs_d,
@@ -1350,10 +1362,6 @@ bool tc_layer_init(TcLayer& t, const LayerGeom& g, int max_batch, bool has_dgrad
     if (ok && (t.wgrad || t.dgrad))
         ok = dalloc(allocs, &t.d_nhwc, (size_t)kMaxLimbs * max_batch * hw * g.cout);
     if (ok && (t.fwd || t.dgrad)) ok = dalloc(allocs, &t.w_planes, (size_t)kMaxLimbs * nwk);
-    // weight-gradient output tiles: ceil(taps * cin_k / 128) x ceil(cout / 64) at most
-    const size_t ntk = (size_t)((t.im2col ? kBK : 9 * t.cin_k) + kBM - 1) / kBM * ((g.cout + 63) / 64) * kEpiWarps;
-    if (ok && t.wgrad) ok = dalloc(allocs, &t.tickets, ntk);
-    if (ok && t.tickets) ok = cudaMemset(t.tickets, 0, ntk * sizeof(int)) == cudaSuccess;
     if (ok) {
         void* h = nullptr;
         ok = cudaMallocHost(&h, 2 * sizeof(uint32_t)) == cudaSuccess;
@@ -1364,6 +1372,32 @@ bool tc_layer_init(TcLayer& t, const LayerGeom& g, int max_batch, bool has_dgrad
         }
     }
     if (ok && t.w_planes) ok = cudaMemset(t.w_planes, 0, (size_t)kMaxLimbs * nwk * 2) == cudaSuccess;
+    return ok;
+}
+
+bool tc_linear_init(TcLayer& t, const LayerGeom& g, int max_batch, uint16_t* act_bf16,
+                    const uint32_t* maxabs_w, const uint32_t* maxabs_d,
+                    std::vector<void*>& allocs, std::vector<void*>& host_allocs) {
+    t = TcLayer();
+    t.maxabs_w = maxabs_w;
+    t.maxabs_d = maxabs_d;
+    if (g.kind != NITRO_LINEAR || max_batch < 1 || !act_bf16 || !encode_fn()) return true;
+    // TMA strides in multiples of 16 bytes; 8-wide output channel groups
+    if (g.cin % 8 != 0 || g.cout % 8 != 0) return true;
+    t.wgrad = true;
+    t.cin8 = g.cin;
+    t.cin_k = round_up(g.cin, 64);
+    t.act_nhwc = act_bf16;       // the forward's bf16 copy of the layer input
+    bool ok = dalloc(allocs, &t.d_nhwc, (size_t)kMaxLimbs * max_batch * g.cout);
+    if (ok) {
+        void* h = nullptr;
+        ok = cudaMallocHost(&h, 2 * sizeof(uint32_t)) == cudaSuccess;
+        if (ok) {
+            host_allocs.push_back(h);
+            t.max_host = static_cast<uint32_t*>(h);
+            t.max_host[0] = t.max_host[1] = 0;
+        }
+    }
     return ok;
 }
 
@@ -1503,76 +1537,83 @@ cudaError_t tc_pack_delta(TcLayer& t, const LayerGeom& g, const int32_t* delta,
 cudaError_t tc_conv_wgrad(TcLayer& t, const LayerGeom& g, const int32_t* delta,
                           const uint32_t* maxabs_delta, int batch, int64_t* dW,
                           uint32_t* status, cudaStream_t s, bool* done, bool planes_done,
-                          const TcSgd* sgd) {
+                          const TcSgd* sgd, bool* sgd_done) {
     *done = false;
+    if (sgd_done) *sgd_done = false;
     if (batch <= 0 || (!t.wgrad && !t.dgrad)) return cudaSuccess;
     cudaError_t pe = tc_pack_delta(t, g, delta, maxabs_delta, batch, s, planes_done);
     if (pe != cudaSuccess) return pe;
     if (!t.wgrad) return cudaSuccess;
-    const int hw = g.h * g.w;
+    // A linear layer is one image of height 1 and width `batch` with a single
+    // centred tap: rows = input features, K = the samples.
+    const bool lin = g.kind == NITRO_LINEAR;
+    const int nimg = lin ? 1 : batch, gh = lin ? 1 : g.h, gw = lin ? batch : g.w;
+    const int hw = gh * gw;
     TcArgs a{};
-    a.B = batch; a.H = g.h; a.W = g.w; a.Cin = g.cin; a.Cout = g.cout;
-    a.Bp = round_up(batch, 8);
+    a.B = nimg; a.H = gh; a.W = gw; a.Cin = g.cin; a.Cout = g.cout;
+    a.Bp = round_up(nimg, 8);
     a.cin_k = t.cin_k;
-    a.taps = t.im2col ? 1 : 9;
+    a.taps = (t.im2col || lin) ? 1 : 9;
+    a.rows = lin ? g.cin : 9 * g.cin;
+    a.cstride = lin ? (int64_t)g.cin : 9LL * g.cin;
     // K-blocks: 64-pixel boxes (wb x hb) of one image
-    a.wb = g.w <= 8 ? 8 : (g.w <= 16 ? 16 : (g.w <= 32 ? 32 : 64));
+    a.wb = gw <= 8 ? 8 : (gw <= 16 ? 16 : (gw <= 32 ? 32 : 64));
     a.hb = 64 / a.wb;
     a.bb = 1;
-    a.ntx = (g.w + a.wb - 1) / a.wb;
-    a.nty = (g.h + a.hb - 1) / a.hb;
+    a.ntx = (gw + a.wb - 1) / a.wb;
+    a.nty = (gh + a.hb - 1) / a.hb;
     const int n = pick_n(g.cout);
     a.tiles_m = (a.taps * t.cin_k + kBM - 1) / kBM;
     a.tiles_n = (g.cout + n - 1) / n;
-    a.kb_total = batch * a.ntx * a.nty;
-    // split K so that at most one wave of CTAs runs (every CTA one work unit),
-    // each with >= one exact chunk
-    const int tiles = a.tiles_m * a.tiles_n;
-    int splits = sm_count() / tiles;
-    const int max_splits = (a.kb_total + kChunkBlocks - 1) / kChunkBlocks;
-    splits = splits < 1 ? 1 : (splits > max_splits ? max_splits : splits);
-    a.kb_per_split = (a.kb_total + splits - 1) / splits;
-    splits = (a.kb_total + a.kb_per_split - 1) / a.kb_per_split;
-    a.total_tiles = tiles * splits;
+    a.kb_total = nimg * a.ntx * a.nty;
+    int splits = wgrad_splits(a.tiles_m * a.tiles_n, a.kb_total, &a.kb_per_split);
+    a.total_tiles = a.tiles_m * a.tiles_n * splits;
     a.ncols = g.cout;
     a.max_a = nullptr;
     a.max_b = maxabs_delta;
     a.out = dW;
     a.status = status;
     a.atomic_out = splits > 1;
+    // The update is folded in only without a K split: the sums are then final
+    // in the accumulators.  With a split, the warp that completes an output
+    // slot would have to read its sums back and update after every other
+    // split has arrived; that tail measured ~50 us per launch on the VGG-style
+    // step against ~7 us for the block's separate IntegerSGD launch, so split
+    // layers report *sgd_done = false and are updated by IntegerSGD.
+    if (sgd && sgd_done) *sgd_done = !a.atomic_out;
+    if (sgd && a.atomic_out) sgd = nullptr;
     if (sgd) {
-        if (!t.tickets || sgd->gamma_inv < 1 || sgd->eta_inv < 0) return cudaErrorInvalidValue;
+        if (sgd->gamma_inv < 1 || sgd->eta_inv < 0) return cudaErrorInvalidValue;
         a.sgd = 1;
-        a.splits = splits;
-        a.tickets = t.tickets;
         a.wt = sgd->W;
         a.maxabs_w = sgd->maxabs_w;
         a.gdiv = FloorDiv::make((uint64_t)sgd->gamma_inv);
         a.decay = sgd->eta_inv > 0;
         a.ediv = FloorDiv::make(sgd->eta_inv > 0 ? (uint64_t)sgd->eta_inv : 1);
         a.trunc = sgd->trunc;
-        int64_t plane = 0;
-        tc_weight_planes(t, g, &a.wp, &plane, &a.row_k, &a.tap_k);
-        a.w_plane = plane;
+        a.wp = sgd->planes;
+        a.w_plane = sgd->plane;
+        a.row_k = sgd->row_k;
+        a.tap_k = sgd->tap_k;
     }
     CUtensorMap ma, mb;
-    const uint64_t da[4] = {(uint64_t)t.cin8, (uint64_t)g.w, (uint64_t)g.h, (uint64_t)batch};
-    const uint64_t sa[3] = {(uint64_t)t.cin8, (uint64_t)g.w * t.cin8, (uint64_t)hw * t.cin8};
+    const uint64_t da[4] = {(uint64_t)t.cin8, (uint64_t)gw, (uint64_t)gh, (uint64_t)nimg};
+    const uint64_t sa[3] = {(uint64_t)t.cin8, (uint64_t)gw * t.cin8, (uint64_t)hw * t.cin8};
     const uint32_t ba[4] = {64, (uint32_t)a.wb, (uint32_t)a.hb, 1};
-    const uint64_t db[5] = {(uint64_t)g.cout, (uint64_t)g.w, (uint64_t)g.h, (uint64_t)batch,
+    const uint64_t db[5] = {(uint64_t)g.cout, (uint64_t)gw, (uint64_t)gh, (uint64_t)nimg,
                             (uint64_t)kMaxLimbs};
-    const uint64_t sb[4] = {(uint64_t)g.cout, (uint64_t)g.w * g.cout, (uint64_t)hw * g.cout,
-                            (uint64_t)batch * hw * g.cout};
+    const uint64_t sb[4] = {(uint64_t)g.cout, (uint64_t)gw * g.cout, (uint64_t)hw * g.cout,
+                            (uint64_t)nimg * hw * g.cout};
     const int pb = pick_pb(n, tc_limb_hint(t, 1));
     const uint32_t bb[5] = {64, (uint32_t)a.wb, (uint32_t)a.hb, 1, (uint32_t)pb};
     if (!make_map(&ma, t.act_nhwc, 4, da, sa, ba) || !make_map(&mb, t.d_nhwc, 5, db, sb, bb))
         return cudaErrorInvalidValue;
     if (a.atomic_out) {
-        cudaError_t e = cudaMemsetAsync(dW, 0, sizeof(int64_t) * 9 * g.cin * g.cout, s);
+        cudaError_t e = cudaMemsetAsync(dW, 0, sizeof(int64_t) * (size_t)a.cstride * g.cout, s);
         if (e != cudaSuccess) return e;
     }
-    const double ops = 2.0 * batch * hw * g.cout * 9.0 * g.cin;
-    ProfScope ps(K_TC_CONV_WGRAD, s, ops, 0.0);
+    const double ops = 2.0 * nimg * hw * g.cout * (double)a.cstride;
+    ProfScope ps(lin ? K_TC_LIN_WGRAD : K_TC_CONV_WGRAD, s, ops, 0.0);
     cudaError_t e = launch_gemm_pb<TC_WGRAD>(n, pb, ma, mb, a, s);
     if (e == cudaSuccess) *done = true;
     return e;
@@ -1614,16 +1655,10 @@ cudaError_t tc_conv_dgrad(TcLayer& t, const LayerGeom& g, int batch, int64_t* g6
         a.low_argmax = fo->low_argmax;
         a.low_delta = fo->low_delta;
         a.low_maxabs = fo->low_maxabs;
-        a.low_planes = fo->low_planes;
-        a.low_plane = (int64_t)batch * fo->low_h * fo->low_w * g.cin;
         if (fo->low_pool && ((fo->low_h & 1) || (fo->low_w & 1))) {   // rows the pool dropped
             cudaError_t e = cudaMemsetAsync(fo->low_delta, 0,
                                             sizeof(int32_t) * (size_t)batch * fo->low_h * fo->low_w * g.cin, s);
             if (e != cudaSuccess) return e;
-            if (fo->low_planes) {
-                e = cudaMemsetAsync(fo->low_planes, 0, 2 * (size_t)a.low_plane * kMaxLimbs, s);
-                if (e != cudaSuccess) return e;
-            }
         }
     }
     CUtensorMap ma, mb;

@@ -48,9 +48,6 @@ struct TcLayer {
     // pinned host copies of the two words, refreshed asynchronously; possibly
     // stale, used only to pick a kernel variant (any choice is exact)
     uint32_t* max_host = nullptr;
-    // arrival tickets of the weight gradient's fused IntegerSGD, one per
-    // (output tile, epilogue warp), zero between launches
-    int* tickets = nullptr;
 };
 
 // IntegerSGD folded into the weight-gradient kernel (Algorithm 1 with the
@@ -62,7 +59,21 @@ struct TcSgd {
     int trunc;                    // NITRO_ROUND_TRUNC
     int32_t* W;
     uint32_t* maxabs_w;
+    // the weight limb planes the update writes (null: none): entry (t, ci) of
+    // row co at co row_k + t tap_k + ci, or co row_k + i for a linear layer
+    uint16_t* planes;
+    int64_t plane;
+    int row_k, tap_k;
 };
+
+// Weight gradient of a linear layer on tcgen05 (dW[o][i] = sum_b delta[b][o]
+// a[b][i], the samples as K): for in and out in multiples of 8.  act_bf16 is
+// the forward's bf16 copy of the layer input [max_batch][in] (kept by the
+// caller); the delta limb planes are allocated here.  t.wgrad is
+// false when the layer does not qualify.
+bool tc_linear_init(TcLayer& t, const LayerGeom& g, int max_batch, uint16_t* act_bf16,
+                    const uint32_t* maxabs_w, const uint32_t* maxabs_d,
+                    std::vector<void*>& allocs, std::vector<void*>& host_allocs);
 
 // Decides which passes of a layer run on tensor cores and allocates their
 // buffers (device memory recorded in `allocs`, pinned host memory in
@@ -125,12 +136,18 @@ inline uint16_t* tc_delta_planes(const TcLayer& t) { return (t.wgrad || t.dgrad)
 
 // tc_pack_delta, then, if wgrad runs on tcgen05, dW = sum_p delta (x)
 // im2col(a).  Must precede tc_conv_dgrad.
-// With sgd != null (and only if the weight gradient runs on tcgen05: check
-// *done) the kernel also applies IntegerSGD, see TcSgd.
+// True when the layer's weight gradient runs on tcgen05 without a K split at
+// this batch, i.e. when tc_conv_wgrad can fold IntegerSGD into it.
+bool tc_wgrad_fusable(const TcLayer& t, const LayerGeom& g, int batch);
+
+// With sgd != null the kernel also applies IntegerSGD (see TcSgd) when the
+// weight gradient runs on tcgen05 without a K split; *sgd_done says whether
+// it did (the caller updates the layer otherwise).
 cudaError_t tc_conv_wgrad(TcLayer& t, const LayerGeom& g, const int32_t* delta,
                           const uint32_t* maxabs_delta, int batch, int64_t* dW,
                           uint32_t* status, cudaStream_t s, bool* done,
-                          bool planes_done = false, const TcSgd* sgd = nullptr);
+                          bool planes_done = false, const TcSgd* sgd = nullptr,
+                          bool* sgd_done = nullptr);
 
 // Where the input gradient goes when the dgrad epilogue is fused: through the
 // lower layer's max-pool backward and NITRO-ReLU backward into its delta.
@@ -143,7 +160,6 @@ struct TcDgradOut {
     const int8_t* low_argmax;
     int32_t* low_delta;             // [B][low_h][low_w][Cin] int32
     uint32_t* low_maxabs;           // max|lower delta| (atomic max)
-    uint16_t* low_planes;           // lower delta's limb planes (tc_delta_planes), or null
 };
 
 // g[p][ci] = sum_(t,co) delta[p - tap t][co] W[co][t][ci] on tcgen05
