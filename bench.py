@@ -40,9 +40,10 @@ def parse():
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--sequential-blocks", action="store_true",
                    help="run all blocks on one stream (default: a stream per block)")
-    p.add_argument("--separate-update", action="store_true",
-                   help="backward and IntegerSGD as two calls (default: one call, the update "
-                        "fused into the tensor-core weight-gradient kernels)")
+    p.add_argument("--fused-update", action="store_true",
+                   help="backward and IntegerSGD in one call (nitro_block_backward_update: the "
+                        "update folded into weight-gradient kernels without a K split); "
+                        "default: the two calls, measured faster")
     p.add_argument("--profile-steps", type=int, default=3)
     p.add_argument("--sweep", action="store_true",
                    help="time the kernel sweep (conv contractions, integer GEMM, IntegerSGD, "
@@ -160,7 +161,7 @@ class GpuNet:
     only for block i's forward, so block i's backward and update overlap the
     blocks after it (blocks exchange no gradients, Sec. 3.3)."""
 
-    def __init__(self, wl, seed, torch, nb, concurrent=True, fused_update=True):
+    def __init__(self, wl, seed, torch, nb, concurrent=True, fused_update=False):
         self.torch, self.nb = torch, nb
         self.fused_update = fused_update
         B = wl["batch"]
@@ -240,8 +241,9 @@ def issued_profile(nb, net, flush, steps, torch):
     counts (activations 1; W and delta from the layers' max |.|, W read before
     the step, delta after it).  Launches map to layers by order: every conv's
     forward in network order, then per block, last layer first, its weight
-    gradient and (above the block's first layer) its input gradient.  Returns
-    {kernel: {"issued_ops", "ms"}} or None when the launches do not match."""
+    gradient and (above the block's first layer) its input gradient (the order
+    of the separate update).  Returns {kernel: {"issued_ops", "ms"}} or None
+    when the launches do not match."""
     import ctypes
     import numpy as np
     L = nb.lib()
@@ -252,13 +254,9 @@ def issued_profile(nb, net, flush, steps, torch):
         for i in reversed(range(len(g.layers))):
             if g.layers[i][0] != nb.NITRO_CONV3X3:
                 continue
-            # the fused update runs a layer's input gradient before its weight
-            # gradient (the input gradient reads the pre-update weights)
-            order = (("tc_conv_dgrad", "tc_conv_wgrad") if net.fused_update
-                     else ("tc_conv_wgrad", "tc_conv_dgrad"))
-            for name in order:
-                if name == "tc_conv_wgrad" or i > 0:
-                    bwd.append((name, bi, i))
+            bwd.append(("tc_conv_wgrad", bi, i))
+            if i > 0:
+                bwd.append(("tc_conv_dgrad", bi, i))
 
     def maxabs(bi, which, i):
         return np.abs(net.blocks[bi].get(which, i, check=False).astype(np.int64)).max()
@@ -305,7 +303,7 @@ def run_ours(args, rank, world, local_rank):
     nb.lib()
     wl = WL.WORKLOADS[args.workload]
     net = GpuNet(wl, 20240716 + 7 * rank, torch, nb, concurrent=not args.sequential_blocks,
-                 fused_update=not args.separate_update)
+                 fused_update=args.fused_update)
     stream = torch.cuda.current_stream()
     flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device="cuda")
 
@@ -443,8 +441,8 @@ def run_ours(args, rank, world, local_rank):
                    "input": "x".join(str(v) for v in wl["input_shape"]) + " int8 uniform [-128,127]",
                    "blocks": len(wl["blocks"]), "cuda_graph": graph is not None,
                    "block_streams": "one" if args.sequential_blocks else "one per block",
-                   "update": ("separate IntegerSGD call" if args.separate_update
-                              else "fused into the tensor-core weight-gradient kernels"),
+                   "update": ("nitro_block_backward_update (folded into un-split weight "
+                              "gradients)" if args.fused_update else "separate IntegerSGD call"),
                    "l2": "flushed (512 MiB write) between timed steps",
                    "parallelism": "replicas" if world > 1 else "single"},
         "e2e": {"value": round(e2e_value, 2), "unit": "images/s",

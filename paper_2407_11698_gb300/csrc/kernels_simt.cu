@@ -198,121 +198,110 @@ __global__ void k_fwd_epilogue(const int64_t* __restrict__ z, LayerGeom g, int B
 }
 
 // ---------------------------------------------------------------------------
-// Learning layer forward + RSS loss, in two short kernels with no atomics
-// between them.  k_learn_partial: CTA (s, y) covers the 16 samples of group y
-// and the 128-feature chunks s, s + S, s + 2S, ... of the d features (S
-// slices), and writes its partial sums of z[b][g] = sum_j a[b][j] W_lr[g][j]
-// to part[s][b][g] with plain stores.  k_learn_finish: one thread per (b, g)
-// adds the S partials (exact int64), forms y_hat = floor(z / (256 d)) and
-// grad_L = y_hat - 32 onehot, and adds its share of the SSE; the last CTA
-// (ticket) writes the loss.
+// Learning layer forward + RSS loss, in one kernel.  A CTA (128-feature
+// slice, 16 samples) adds its partial sums of z[b][g] = sum_j a[b][j] W_lr[g][j]
+// into zsum with int64 atomics (exact, order independent).  The last CTA of
+// a sample group (per-group ticket) turns that group's z into
+// y_hat = floor(z / (256 d)) and grad_L = y_hat - 32 onehot and adds its part
+// of the SSE; the last of those (final ticket) writes the loss.
+// Tickets live behind zsum: zsum[B G + y] per group, zsum[B G + groups].
 // ---------------------------------------------------------------------------
 constexpr int kLrSamples = 16;   // samples per CTA
-constexpr int kLpSlice = 128;    // features per chunk
-constexpr int kLpMaxSlices = 128;
+constexpr int kLpSlice = 128;    // features per CTA
 static_assert(kLpSlice == 16 * 8, "k_learn_partial: 16 lanes of 8 features per sample");
 
 __global__ void __launch_bounds__(256) k_learn_partial(const int8_t* __restrict__ a,
                                                        const int32_t* __restrict__ wlr, int B,
                                                        int d, int G, int vec8,
-                                                       long long* __restrict__ part) {
-    // thread (u, k): sample u of the group, features 8k .. 8k + 7 of a chunk,
+                                                       unsigned long long* __restrict__ zsum,
+                                                       FloorDiv dv, const int32_t* __restrict__ labels,
+                                                       int32_t* __restrict__ grad_l,
+                                                       unsigned long long* sse, int64_t* loss,
+                                                       uint32_t* maxabs_gl, uint32_t* status) {
+    // thread (u, k): sample u of the group, features 8k .. 8k + 7 of the slice,
     // read as one 8-byte word when the rows allow it (vec8: d % 8 == 0 and an
-    // 8-byte aligned a).  A chunk of W_lr is staged in shared memory with
+    // 8-byte aligned a).  The slice of W_lr is staged in shared memory with
     // feature 8k + m at column 16m + k, so the lanes of a sample read
-    // consecutive words; classes in groups of kLpG.
+    // consecutive words; classes in chunks of kLpG.
     constexpr int kLpG = 16;
     __shared__ int32_t ws[kLpG][kLpSlice + 1];
     const int u = threadIdx.x >> 4, k = threadIdx.x & 15;
     const int b = blockIdx.y * kLrSamples + u;
-    const int S = gridDim.x;
-    for (int gc = 0; gc < G; gc += kLpG) {
-        const int ng = min(kLpG, G - gc);
-        long long t[kLpG];
+    const int j0 = blockIdx.x * kLpSlice;
+    const int jb = j0 + 8 * k;
+    int av[8];
+    if (vec8 && b < B && jb + 8 <= d) {
+        const uint2 w = *reinterpret_cast<const uint2*>(a + (int64_t)b * d + jb);
 #pragma unroll
-        for (int g = 0; g < kLpG; ++g) t[g] = 0;
-        for (int j0 = blockIdx.x * kLpSlice; j0 < d; j0 += S * kLpSlice) {
-            const int jb = j0 + 8 * k;
-            int av[8];
-            if (vec8 && b < B && jb + 8 <= d) {
-                const uint2 w = *reinterpret_cast<const uint2*>(a + (int64_t)b * d + jb);
-#pragma unroll
-                for (int m = 0; m < 4; ++m) {
-                    av[m] = (int8_t)(w.x >> (8 * m));
-                    av[4 + m] = (int8_t)(w.y >> (8 * m));
-                }
-            } else {
-#pragma unroll
-                for (int m = 0; m < 8; ++m) {
-                    const int j = jb + m;
-                    av[m] = (b < B && j < d) ? a[(int64_t)b * d + j] : 0;
-                }
-            }
-            __syncthreads();   // readers of the previous chunk are done
-            for (int i = threadIdx.x; i < ng * kLpSlice; i += blockDim.x) {
-                const int g = i / kLpSlice, j = i - g * kLpSlice;
-                ws[g][(j & 7) * 16 + (j >> 3)] = j0 + j < d ? wlr[(int64_t)(gc + g) * d + j0 + j] : 0;
-            }
-            __syncthreads();
-#pragma unroll
-            for (int g = 0; g < kLpG; ++g) {
-                if (g >= ng) break;
-#pragma unroll
-                for (int m = 0; m < 8; ++m) t[g] += (long long)ws[g][16 * m + k] * av[m];
-            }
+        for (int m = 0; m < 4; ++m) {
+            av[m] = (int8_t)(w.x >> (8 * m));
+            av[4 + m] = (int8_t)(w.y >> (8 * m));
         }
+    } else {
 #pragma unroll
-        for (int g = 0; g < kLpG; ++g) {
-            if (g >= ng) break;
-            long long v = t[g];
-#pragma unroll
-            for (int off = 8; off; off >>= 1) v += __shfl_xor_sync(kFull, v, off);
-            if (k == 0 && b < B) part[((int64_t)blockIdx.x * B + b) * G + gc + g] = v;
+        for (int m = 0; m < 8; ++m) {
+            const int j = jb + m;
+            av[m] = (b < B && j < d) ? a[(int64_t)b * d + j] : 0;
         }
     }
-}
-
-__global__ void __launch_bounds__(256) k_learn_finish(const long long* __restrict__ part, int S,
-                                                      int B, int G, FloorDiv dv,
-                                                      const int32_t* __restrict__ labels,
-                                                      int32_t* __restrict__ grad_l,
-                                                      unsigned long long* sse, int64_t* loss,
-                                                      uint32_t* maxabs_gl, uint32_t* status,
-                                                      unsigned int* ticket) {
-    // one warp per output (b, g): the lanes add the S partials (at most 4
-    // each, loads issued together), then lane 0 finishes the output
+    for (int gc = 0; gc < G; gc += kLpG) {
+        const int ng = min(kLpG, G - gc);
+        if (gc) __syncthreads();
+        for (int i = threadIdx.x; i < ng * kLpSlice; i += blockDim.x) {
+            const int g = i / kLpSlice, j = i - g * kLpSlice;
+            ws[g][(j & 7) * 16 + (j >> 3)] = j0 + j < d ? wlr[(int64_t)(gc + g) * d + j0 + j] : 0;
+        }
+        __syncthreads();
+        for (int g = 0; g < ng; ++g) {
+            long long t = 0;
+#pragma unroll
+            for (int m = 0; m < 8; ++m) t += (long long)ws[g][16 * m + k] * av[m];
+#pragma unroll
+            for (int off = 8; off; off >>= 1) t += __shfl_xor_sync(kFull, t, off);
+            if (k == 0 && b < B && t != 0)
+                atomicAdd(&zsum[(int64_t)b * G + gc + g], (unsigned long long)t);
+        }
+    }
+    __shared__ int last;
     __shared__ unsigned long long red_s[8];
     __shared__ uint32_t red_m[8];
     __shared__ int flags;
-    if (threadIdx.x == 0) flags = 0;
+    unsigned long long* tickets = zsum + (int64_t)B * G;
+    if (k == 0) __threadfence();     // the lanes that added into zsum
     __syncthreads();
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int i = blockIdx.x * 8 + warp;
-    const int n = B * G;
+    if (threadIdx.x == 0) {
+        flags = 0;
+        last = atomicAdd(&tickets[blockIdx.y], 1ull) == (unsigned long long)gridDim.x - 1;
+    }
+    __syncthreads();
+    if (!last) return;
+    __threadfence();
+    // this sample group's z is complete: y_hat, grad_L, its share of the SSE
     unsigned long long ss = 0;
     uint32_t mx = 0;
-    if (i < n) {
-        unsigned long long z = 0;     // exact: the partial sums of z fit int64
-        for (int s2 = lane; s2 < S; s2 += 32) z += (unsigned long long)part[(int64_t)s2 * n + i];
-#pragma unroll
-        for (int off = 16; off; off >>= 1) z += __shfl_xor_sync(kFull, z, off);
-        if (lane == 0) {
-            int fl = 0;
-            const int bb = i / G, g = i - bb * G;
-            const int lab = labels[bb];
-            const bool bad = lab < 0 || lab >= G;
-            if (bad && g == 0) fl |= ST_BAD_LABEL;
-            // NITRO-Scaling, SF = 2^8 d: floor(floor(z / 256) / d)
-            const int64_t yhat = dv.floor_div((int64_t)z >> 8);
-            const int64_t v = yhat - ((!bad && g == lab) ? 32 : 0);
-            if (!fits_i32(v)) fl |= ST_OVERFLOW;
-            const int32_t sv = (int32_t)v;
-            grad_l[i] = sv;
-            ss = (unsigned long long)((int64_t)sv * sv);
-            mx = abs_u32(sv);
-            if (fl) atomicOr(&flags, fl);
-        }
+    int fl = 0;
+    const int nb = min(kLrSamples, B - (int)blockIdx.y * kLrSamples);
+    for (int i = threadIdx.x; i < nb * G; i += blockDim.x) {
+        const int bb = blockIdx.y * kLrSamples + i / G, g = i % G;
+        const int lab = labels[bb];
+        const bool bad = lab < 0 || lab >= G;
+        if (bad && g == 0) fl |= ST_BAD_LABEL;
+        // NITRO-Scaling, SF = 2^8 d: floor(floor(z / 256) / d)
+        const int64_t yhat = dv.floor_div((int64_t)__ldcg(zsum + (int64_t)bb * G + g) >> 8);
+        const int64_t v = yhat - ((!bad && g == lab) ? 32 : 0);
+        if (!fits_i32(v)) fl |= ST_OVERFLOW;
+        const int32_t sv = (int32_t)v;
+        grad_l[(int64_t)bb * G + g] = sv;
+        ss += (unsigned long long)((int64_t)sv * sv);
+        mx = max(mx, abs_u32(sv));
     }
+#pragma unroll
+    for (int off = 16; off; off >>= 1) {
+        ss += __shfl_xor_sync(kFull, ss, off);
+        mx = max(mx, __shfl_xor_sync(kFull, mx, off));
+    }
+    if (fl) atomicOr(&flags, fl);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     if (lane == 0) { red_s[warp] = ss; red_m[warp] = mx; }
     __syncthreads();
     if (threadIdx.x == 0) {
@@ -323,11 +312,10 @@ __global__ void __launch_bounds__(256) k_learn_finish(const long long* __restric
         if (m) atomicMax(maxabs_gl, m);
         if (flags) atomicOr(status, (uint32_t)flags);
         __threadfence();
-        if (atomicAdd(ticket, 1u) == gridDim.x - 1) {
+        if (atomicAdd(&tickets[gridDim.y], 1ull) == (unsigned long long)gridDim.y - 1) {
             __threadfence();
             const unsigned long long tot = atomicAdd(sse, 0ull);
             if (loss) *loss = fdiv64((int64_t)tot, 2);
-            *ticket = 0;                                     // ready for the next launch
         }
     }
 }
@@ -542,8 +530,7 @@ __global__ void k_lrpool_to_delta4(const int32_t* __restrict__ gl, const int32_t
                                    const int8_t* __restrict__ region, FloorDiv32 alpha,
                                    int32_t* __restrict__ delta, const uint32_t* maxabs_gl,
                                    const uint32_t* maxabs_wlr, uint32_t* maxabs_delta,
-                                   uint32_t* status, uint16_t* __restrict__ planes,
-                                   int64_t plane) {
+                                   uint32_t* status) {
     const int C = g.cout, C4 = g.cout >> 2;
     const uint32_t n4 = (uint32_t)B * g.h * g.w * C4;
     if (blockIdx.x == 0 && threadIdx.x == 0 && int64_bound_exceeded(*maxabs_gl, *maxabs_wlr, G))
@@ -594,7 +581,6 @@ __global__ void k_lrpool_to_delta4(const int32_t* __restrict__ gl, const int32_t
             }
         }
         reinterpret_cast<int4*>(delta)[i] = make_int4(v[0], v[1], v[2], v[3]);
-        if (planes) store_delta_planes4(planes + 4 * (int64_t)i, plane, v[0], v[1], v[2], v[3]);
     }
 #pragma unroll
     for (int off = 16; off; off >>= 1) mx = max(mx, __shfl_xor_sync(kFull, mx, off));
@@ -986,9 +972,7 @@ __global__ void __launch_bounds__(256) k_lr_backward4(const int8_t* __restrict__
                                                       unsigned long long* __restrict__ dwlr,
                                                       const uint32_t* maxabs_gl,
                                                       const uint32_t* maxabs_wlr,
-                                                      uint32_t* maxabs_delta, uint32_t* status,
-                                                      uint16_t* __restrict__ planes,
-                                                      int64_t plane) {
+                                                      uint32_t* maxabs_delta, uint32_t* status) {
     __shared__ int32_t gls[kLbSamples][GM];
     __shared__ int8_t as[kLbSamples][kLbQ];
     __shared__ __align__(16) int32_t wsl[GM][kLbQ];
@@ -1072,16 +1056,12 @@ __global__ void __launch_bounds__(256) k_lr_backward4(const int8_t* __restrict__
         }
         if (lg.pool) {
 #pragma unroll
-            for (int k = 0; k < 4; ++k) {
-                const int64_t o = base + (k & 1) * dx + (k >> 1) * dy;
-                const int4 w = make_int4(code[0] == k ? dv[0] : 0, code[1] == k ? dv[1] : 0,
-                                         code[2] == k ? dv[2] : 0, code[3] == k ? dv[3] : 0);
-                *reinterpret_cast<int4*>(delta + o) = w;
-                if (planes) store_delta_planes4(planes + o, plane, w.x, w.y, w.z, w.w);
-            }
+            for (int k = 0; k < 4; ++k)
+                *reinterpret_cast<int4*>(delta + base + (k & 1) * dx + (k >> 1) * dy) =
+                    make_int4(code[0] == k ? dv[0] : 0, code[1] == k ? dv[1] : 0,
+                              code[2] == k ? dv[2] : 0, code[3] == k ? dv[3] : 0);
         } else {
             *reinterpret_cast<int4*>(delta + base) = make_int4(dv[0], dv[1], dv[2], dv[3]);
-            if (planes) store_delta_planes4(planes + base, plane, dv[0], dv[1], dv[2], dv[3]);
         }
     }
 #pragma unroll
@@ -1189,9 +1169,7 @@ cudaError_t simt_lrpool_to_delta(const int32_t* gl, const int32_t* wlr, int G, i
                                  const uint8_t* am, const int8_t* argmax, const int8_t* region,
                                  int alpha_inv, int32_t* delta, const uint32_t* maxabs_gl,
                                  const uint32_t* maxabs_wlr, uint32_t* maxabs_delta,
-                                 uint32_t* status, cudaStream_t s, uint16_t* planes,
-                                 int64_t plane, bool* planes_done) {
-    if (planes_done) *planes_done = false;
+                                 uint32_t* status, cudaStream_t s) {
     const int64_t n = (int64_t)B * g.h * g.w * g.cout;
     if (n <= 0) return cudaSuccess;
     if (g.kind != NITRO_CONV3X3 || lp.ph * lp.kh > g.oh || lp.pw * lp.kw > g.ow ||
@@ -1212,8 +1190,7 @@ cudaError_t simt_lrpool_to_delta(const int32_t* gl, const int32_t* wlr, int G, i
             gl, wlr, G, d, g, lp, lg_kh, lg_kw, B, FloorDiv32::make((uint32_t)(g.cout / 4)),
             FloorDiv32::make((uint32_t)g.w), FloorDiv32::make((uint32_t)g.h), am, argmax, region,
             FloorDiv32::make((uint32_t)alpha_inv), delta, maxabs_gl, maxabs_wlr, maxabs_delta,
-            status, planes, plane);
-        if (planes_done) *planes_done = planes != nullptr;
+            status);
     } else {
         k_lrpool_to_delta<<<grid_for(n, 256), 256, 0, s>>>(
             gl, wlr, G, d, g, lp, B, am, argmax, region,
@@ -1224,30 +1201,25 @@ cudaError_t simt_lrpool_to_delta(const int32_t* gl, const int32_t* wlr, int G, i
 }
 
 size_t simt_learn_scratch(int max_batch, int d, int G) {
-    const int S = std::min(kLpMaxSlices, (d + kLpSlice - 1) / kLpSlice);
-    return (size_t)S * max_batch * G + 1;
+    (void)d;
+    return (size_t)max_batch * G + (max_batch + kLrSamples - 1) / kLrSamples + 1;
 }
 
 cudaError_t simt_learn_fwd(const int8_t* a, const int32_t* wlr, const int32_t* labels, int B,
-                           int d, int G, int64_t* scratch, int32_t* grad_l, unsigned long long* sse,
+                           int d, int G, int64_t* zsum, int32_t* grad_l, unsigned long long* sse,
                            int64_t* loss, uint32_t* maxabs_gl, uint32_t* status, cudaStream_t s) {
     if (B <= 0) return cudaSuccess;
     const int groups = (B + kLrSamples - 1) / kLrSamples;
-    const int S = std::min(kLpMaxSlices, (d + kLpSlice - 1) / kLpSlice);
-    // word 0: the finish kernel's ticket (zero between launches); then the partials
-    unsigned int* ticket = reinterpret_cast<unsigned int*>(scratch);
-    long long* part = reinterpret_cast<long long*>(scratch + 1);
-    {
-        ProfScope ps(K_LEARN_FWD, s, 2.0 * B * d * G, 0.0);
-        const int vec8 = d % 8 == 0 && ((uintptr_t)a & 7) == 0;
-        k_learn_partial<<<dim3(S, groups), 256, 0, s>>>(a, wlr, B, d, G, vec8, part);
-    }
-    cudaError_t e = cudaGetLastError();
+    // partial sums, then the per-group tickets and the final ticket
+    cudaError_t e = cudaMemsetAsync(zsum, 0, sizeof(int64_t) * ((size_t)B * G + groups + 1), s);
     if (e != cudaSuccess) return e;
-    ProfScope ps(K_FINISH_LOSS, s, 0.0, 0.0);
-    k_learn_finish<<<(B * G + 7) / 8, 256, 0, s>>>(part, S, B, G, FloorDiv::make((uint64_t)d),
-                                                      labels, grad_l, sse, loss, maxabs_gl,
-                                                      status, ticket);
+    dim3 grid((d + kLpSlice - 1) / kLpSlice, groups);
+    ProfScope ps(K_LEARN_FWD, s, 2.0 * B * d * G, 0.0);
+    const int vec8 = d % 8 == 0 && ((uintptr_t)a & 7) == 0;
+    k_learn_partial<<<grid, 256, 0, s>>>(a, wlr, B, d, G, vec8,
+                                         reinterpret_cast<unsigned long long*>(zsum),
+                                         FloorDiv::make((uint64_t)d), labels, grad_l, sse, loss,
+                                         maxabs_gl, status);
     return cudaGetLastError();
 }
 
@@ -1353,13 +1325,10 @@ cudaError_t simt_lr_backward(const int8_t* a, const int32_t* gl, const int32_t* 
                              int d, const LayerGeom* lg, int alpha_inv, const int8_t* region,
                              const int8_t* argmax, int32_t* delta, int64_t* dwlr,
                              const uint32_t* maxabs_gl, const uint32_t* maxabs_wlr,
-                             uint32_t* maxabs_delta, uint32_t* status, cudaStream_t s,
-                             uint16_t* planes, int64_t plane, bool* planes_done) {
-    if (planes_done) *planes_done = false;
+                             uint32_t* maxabs_delta, uint32_t* status, cudaStream_t s) {
     cudaError_t e = cudaMemsetAsync(dwlr, 0, sizeof(int64_t) * (size_t)G * d, s);
     if (e != cudaSuccess || B <= 0) return e;
-    const bool dropped = lg && lg->pool && ((lg->h & 1) || (lg->w & 1));
-    if (dropped) {   // rows / columns the pool dropped
+    if (lg && lg->pool && ((lg->h & 1) || (lg->w & 1))) {   // rows / columns the pool dropped
         e = cudaMemsetAsync(delta, 0, sizeof(int32_t) * (size_t)B * lg->h * lg->w * lg->cout, s);
         if (e != cudaSuccess) return e;
     }
@@ -1374,20 +1343,14 @@ cudaError_t simt_lr_backward(const int8_t* a, const int32_t* gl, const int32_t* 
                       (((uintptr_t)region | (uintptr_t)delta |
                         (uintptr_t)(lg->pool ? argmax : region)) & 15) == 0;
     if (quad) {
-        if (planes && dropped) {
-            e = cudaMemsetAsync(planes, 0, 2 * (size_t)plane * 4, s);
-            if (e != cudaSuccess) return e;
-        }
         if (G <= 10)
             k_lr_backward4<10><<<grid, 256, 0, s>>>(a, gl, wlr, B, G, d, g0, al, region, argmax,
                                                     delta, dw64, maxabs_gl, maxabs_wlr,
-                                                    maxabs_delta, status, planes, plane);
+                                                    maxabs_delta, status);
         else
             k_lr_backward4<kLbMaxG><<<grid, 256, 0, s>>>(a, gl, wlr, B, G, d, g0, al, region,
                                                          argmax, delta, dw64, maxabs_gl,
-                                                         maxabs_wlr, maxabs_delta, status, planes,
-                                                         plane);
-        if (planes_done) *planes_done = planes != nullptr;
+                                                         maxabs_wlr, maxabs_delta, status);
         return cudaGetLastError();
     }
     if (G <= 10)

@@ -408,17 +408,6 @@ nitro_status block_backward(nitro_block* b, const int8_t* a_in, const int32_t* l
         return NITRO_OK;
     }
     const int8_t* a_last = n ? b->L[n - 1].act : a_in;
-    // layers whose delta limb planes were written by the kernel producing delta
-    std::vector<char> planes_done(n > 0 ? n : 1, 0);
-    bool pd = false;
-    auto delta_planes = [&](int i, uint16_t** p, int64_t* plane) {
-        const Layer& ly = b->L[i];
-        *p = tc_delta_planes(ly.tc);
-        *plane = (int64_t)batch * ly.g.h * ly.g.w * ly.g.cout;
-    };
-    uint16_t* last_planes = nullptr;
-    int64_t last_plane = 0;
-    if (n) delta_planes(n - 1, &last_planes, &last_plane);
     if (b->zmp) {
         // z^mp: the block output max-pooled for the learning layer (Sec. 3.3)
         const LayerGeom& lg = b->L[n - 1].g;
@@ -440,9 +429,7 @@ nitro_status block_backward(nitro_block* b, const int8_t* a_in, const int32_t* l
         Layer& ly = b->L[n - 1];
         NITRO_TRY(simt_lrpool_to_delta(b->grad_l, b->Wlr, G, (int)d, ly.g, b->lp, batch, b->lr_am,
                                        ly.argmax, ly.region, b->desc.alpha_inv, ly.delta, w_gl(b),
-                                       w_wlr(b), w_delta(b, n - 1), w_status(b), s, last_planes,
-                                       last_plane, &pd));
-        planes_done[n - 1] = pd;
+                                       w_wlr(b), w_delta(b, n - 1), w_status(b), s));
     } else if (simt_lr_backward_ok(G)) {
         // learning-weight gradient and (below a forward layer) delta_fw -> that
         // layer's delta in one pass
@@ -450,9 +437,7 @@ nitro_status block_backward(nitro_block* b, const int8_t* a_in, const int32_t* l
         NITRO_TRY(simt_lr_backward(a_last, b->grad_l, b->Wlr, batch, G, (int)d, ly ? &ly->g : nullptr,
                                    b->desc.alpha_inv, ly ? ly->region : nullptr,
                                    ly ? ly->argmax : nullptr, ly ? ly->delta : nullptr, b->dWlr,
-                                   w_gl(b), w_wlr(b), n ? w_delta(b, n - 1) : nullptr, w_status(b), s,
-                                   last_planes, last_plane, &pd));
-        if (n) planes_done[n - 1] = pd;
+                                   w_gl(b), w_wlr(b), n ? w_delta(b, n - 1) : nullptr, w_status(b), s));
     } else {
         NITRO_TRY(simt_learn_dw(a_last, b->grad_l, batch, (int)d, G, b->dWlr, s));
     }
@@ -496,7 +481,7 @@ nitro_status block_backward(nitro_block* b, const int8_t* a_in, const int32_t* l
                 if ((*updated)[i]) NITRO_TRY(tc_weights_hint(ly.tc, s));
             } else {
                 NITRO_TRY(tc_conv_wgrad(ly.tc, g, ly.delta, w_delta(b, i), batch, ly.dW, w_status(b), s,
-                                        &done, planes_done[i] != 0));
+                                        &done));
             }
             if (!done && simt_small_conv_ok(g)) {
                 NITRO_TRY(simt_conv_small_wgrad(x, ly.delta, g, batch, ly.dW, s));
@@ -509,7 +494,7 @@ nitro_status block_backward(nitro_block* b, const int8_t* a_in, const int32_t* l
             return NITRO_OK;
         };
         if (fuse_sgd) {
-            NITRO_TRY(tc_pack_delta(ly.tc, g, ly.delta, w_delta(b, i), batch, s, planes_done[i] != 0));
+            NITRO_TRY(tc_pack_delta(ly.tc, g, ly.delta, w_delta(b, i), batch, s));
         } else {
             nitro_status st = wgrad();
             if (st != NITRO_OK) return st;

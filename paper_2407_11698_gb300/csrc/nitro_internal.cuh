@@ -154,38 +154,6 @@ __host__ __device__ __forceinline__ bool dropout_drop(uint64_t seed, uint32_t t,
     return (uint32_t)(splitmix64_at(seed, idx) >> 48) < p16;
 }
 
-// Canonical limb split of four int32 deltas into the bf16 limb planes the
-// tensor-core contractions read: limbs 0..2 are the digits
-// ((x + 128) & 255) - 128 of successive base-256 remainders, limb 3 the rest
-// (in [-128, 128]); every limb is exact in bf16 (the top half of its fp32
-// bits).  Plane l of the four values is one 8-byte store at p + l * plane
-// (p and the plane stride in bytes 8-byte aligned).  Producers of a delta
-// call this next to their int32 stores, so no separate split pass is needed.
-#ifdef __CUDACC__
-__device__ __forceinline__ void store_delta_planes4(uint16_t* p, int64_t plane, int32_t v0,
-                                                    int32_t v1, int32_t v2, int32_t v3) {
-    int32_t v[4] = {v0, v1, v2, v3};
-#pragma unroll
-    for (int l = 0; l < 4; ++l) {
-        uint32_t h[4];
-#pragma unroll
-        for (int k = 0; k < 4; ++k) {
-            int dg;
-            if (l < 3) {
-                // v = 256 q + r: digit r or r - 256, remainder q or q + 1
-                const int r = v[k] & 255;
-                dg = r - ((r >> 7) << 8);
-                v[k] = (v[k] >> 8) + (r >> 7);
-            } else {
-                dg = v[k];
-            }
-            h[k] = __float_as_uint((float)dg) >> 16;
-        }
-        *reinterpret_cast<uint2*>(p + l * plane) = make_uint2(h[0] | (h[1] << 16), h[2] | (h[3] << 16));
-    }
-}
-#endif
-
 // max|A| * max|B| * k >= 2^63 : int64 exactness of an int32 x int32
 // contraction of length k is no longer guaranteed.
 __host__ __device__ __forceinline__ bool int64_bound_exceeded(uint32_t ma, uint32_t mb, int64_t k) {
@@ -246,16 +214,12 @@ cudaError_t simt_lr_pool_fwd(const int8_t* a, int B, int H, int W, int C, int kh
 struct LrPoolGeom {
     int kh, kw, ph, pw;
 };
-// With planes != null the four-channel kernel also writes delta's bf16 limb
-// planes [4][B][h][w][cout] (plane stride `plane` elements) and sets
-// *planes_done; otherwise *planes_done is false.
 cudaError_t simt_lrpool_to_delta(const int32_t* gl, const int32_t* wlr, int G, int d,
                                  const LayerGeom& g, const LrPoolGeom& lp, int B,
                                  const uint8_t* am, const int8_t* argmax, const int8_t* region,
                                  int alpha_inv, int32_t* delta, const uint32_t* maxabs_gl,
                                  const uint32_t* maxabs_wlr, uint32_t* maxabs_delta,
-                                 uint32_t* status, cudaStream_t s, uint16_t* planes = nullptr,
-                                 int64_t plane = 0, bool* planes_done = nullptr);
+                                 uint32_t* status, cudaStream_t s);
 
 // Learning layer forward + loss: grad_l = floor(a W^T / (256 d)) - 32 onehot,
 // sse = sum grad_l^2 (mod 2^64), loss = floor(sse / 2) (if loss != NULL),
@@ -304,15 +268,11 @@ cudaError_t simt_conv_small_wgrad(const int8_t* x, const int32_t* d, const Layer
 // rule, the int64 bound check, max-pool and NITRO-ReLU backward.  d: features
 // of the block output.
 bool simt_lr_backward_ok(int G);
-// planes / plane / planes_done: as for simt_lrpool_to_delta (four-feature
-// kernel only).
 cudaError_t simt_lr_backward(const int8_t* a, const int32_t* gl, const int32_t* wlr, int B, int G,
                              int d, const LayerGeom* lg, int alpha_inv, const int8_t* region,
                              const int8_t* argmax, int32_t* delta, int64_t* dwlr,
                              const uint32_t* maxabs_gl, const uint32_t* maxabs_wlr,
-                             uint32_t* maxabs_delta, uint32_t* status, cudaStream_t s,
-                             uint16_t* planes = nullptr, int64_t plane = 0,
-                             bool* planes_done = nullptr);
+                             uint32_t* maxabs_delta, uint32_t* status, cudaStream_t s);
 
 // IntegerSGD (Algorithm 1) over up to kMaxSgdTensors tensors in one launch.
 constexpr int kMaxSgdTensors = 16;

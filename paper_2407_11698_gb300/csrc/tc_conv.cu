@@ -518,7 +518,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             int it = 0, chunk = 0;
             for (int tile = blockIdx.x; tile < args.total_tiles; tile += gridDim.x) {
                 const Tile T = decode_tile(args, tile);
+                // chunks of equal length (at most kChunkBlocks K-blocks each), so
+                // that no short chunk costs a full drain for little MMA work
                 const int cpp = (T.kb1 - T.kb0 + kChunkBlocks - 1) / kChunkBlocks;
+                const int csz = cpp ? (T.kb1 - T.kb0 + cpp - 1) / cpp : 0;
                 for (int la = 0; la < LA; ++la)
                 for (int lb0 = 0; lb0 < lb_limit(la); lb0 += PB) {
                     const int nb = min(PB, lb_limit(la) - lb0);
@@ -536,8 +539,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                             goto mma_done;
                         tc_fence_after();
                         const uint32_t d = tmem + (uint32_t)(buf * PB * N);
-                        const int c0 = T.kb0 + c * kChunkBlocks;
-                        const int c1 = min(T.kb1, c0 + kChunkBlocks);
+                        const int c0 = T.kb0 + c * csz;
+                        const int c1 = min(T.kb1, c0 + csz);
                         for (int kb = c0; kb < c1; ++kb, ++it) {
                             const int s = it % S;
                             if (!mbar_wait(full_bar(s), (it / S) & 1, abort_flag, args.status))
@@ -1522,7 +1525,7 @@ cudaError_t tc_pack_delta(TcLayer& t, const LayerGeom& g, const int32_t* delta,
                           bool planes_done) {
     if (batch <= 0 || (!t.wgrad && !t.dgrad)) return cudaSuccess;
     // limb planes of delta (NHWC, read by the wgrad and dgrad passes), unless
-    // the kernel that produced delta wrote them
+    // an earlier call split this delta already
     const int64_t n = (int64_t)batch * g.h * g.w * g.cout;   // cout % 8 == 0
     if (!planes_done) {
         ProfScope ps(K_TC_PACK_D, s, 0.0, (double)n * 4 * 2);

@@ -122,17 +122,13 @@ cudaError_t tc_conv_forward(TcLayer& t, const LayerGeom& g, int batch, int64_t* 
                             bool* fused);
 
 // Splits delta into NHWC limb planes for the wgrad and dgrad passes (limb
-// count from *maxabs_delta), unless planes_done (the producer of delta wrote
-// all four planes, see store_delta_planes4); then refreshes the host hint of
-// max |delta|.
+// count from *maxabs_delta), unless planes_done (an earlier call split this
+// delta already); then refreshes the host hint of max |delta|.  Writing the
+// planes from the kernels that produce delta instead (the dgrad epilogue,
+// the learning-layer backward) was measured slower than this pass.
 cudaError_t tc_pack_delta(TcLayer& t, const LayerGeom& g, const int32_t* delta,
                           const uint32_t* maxabs_delta, int batch, cudaStream_t s,
                           bool planes_done = false);
-
-// Where a producer of this layer's delta writes its limb planes: d_nhwc
-// [4][batch][h][w][cout] (plane stride batch h w cout), or null when no
-// contraction of the layer reads them.
-inline uint16_t* tc_delta_planes(const TcLayer& t) { return (t.wgrad || t.dgrad) ? t.d_nhwc : nullptr; }
 
 // tc_pack_delta, then, if wgrad runs on tcgen05, dW = sum_p delta (x)
 // im2col(a).  Must precede tc_conv_dgrad.
