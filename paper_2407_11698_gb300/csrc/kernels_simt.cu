@@ -205,6 +205,10 @@ __global__ void k_fwd_epilogue(const int64_t* __restrict__ z, LayerGeom g, int B
 // y_hat = floor(z / (256 d)) and grad_L = y_hat - 32 onehot and adds its part
 // of the SSE; the last of those (final ticket) writes the loss.
 // Tickets live behind zsum: zsum[B G + y] per group, zsum[B G + groups].
+// Splitting this into a partial-sum kernel and a separate finish kernel
+// (per-slice partials with plain stores, or the atomic partials with a
+// one-read-per-output finish) was measured no faster: the second launch costs
+// what the fence and tickets save.
 // ---------------------------------------------------------------------------
 constexpr int kLrSamples = 16;   // samples per CTA
 constexpr int kLpSlice = 128;    // features per CTA
@@ -961,8 +965,8 @@ __global__ void __launch_bounds__(256) k_lr_backward(const int8_t* __restrict__ 
 // the region bytes of the four channels are read as 4-byte words and the
 // delta written with 16-byte stores.  The dW_lr partials are those of
 // k_lr_backward.
-template <int GM>
-__global__ void __launch_bounds__(256) k_lr_backward4(const int8_t* __restrict__ a,
+template <int GM, int NS>   // NS samples per CTA, 16 NS threads
+__global__ void __launch_bounds__(16 * NS) k_lr_backward4(const int8_t* __restrict__ a,
                                                       const int32_t* __restrict__ gl,
                                                       const int32_t* __restrict__ wlr, int B,
                                                       int G, int d, LayerGeom lg, FloorDiv32 alpha,
@@ -973,18 +977,18 @@ __global__ void __launch_bounds__(256) k_lr_backward4(const int8_t* __restrict__
                                                       const uint32_t* maxabs_gl,
                                                       const uint32_t* maxabs_wlr,
                                                       uint32_t* maxabs_delta, uint32_t* status) {
-    __shared__ int32_t gls[kLbSamples][GM];
-    __shared__ int8_t as[kLbSamples][kLbQ];
+    __shared__ int32_t gls[NS][GM];
+    __shared__ int8_t as[NS][kLbQ];
     __shared__ __align__(16) int32_t wsl[GM][kLbQ];
     const int f4 = threadIdx.x & 15, u = threadIdx.x >> 4;
     const int q0 = blockIdx.x * kLbQ, q = q0 + 4 * f4;
-    const int b0 = blockIdx.y * kLbSamples;
-    const int nb = min(kLbSamples, B - b0);
-    for (int i = threadIdx.x; i < kLbSamples * GM; i += blockDim.x) {
+    const int b0 = blockIdx.y * NS;
+    const int nb = min(NS, B - b0);
+    for (int i = threadIdx.x; i < NS * GM; i += blockDim.x) {
         const int uu = i / GM, g = i % GM;
         gls[uu][g] = (uu < nb && g < G) ? gl[(int64_t)(b0 + uu) * G + g] : 0;
     }
-    for (int i = threadIdx.x; i < kLbSamples * kLbQ; i += blockDim.x) {
+    for (int i = threadIdx.x; i < NS * kLbQ; i += blockDim.x) {
         const int uu = i / kLbQ, qq = i % kLbQ;
         as[uu][qq] = (uu < nb && q0 + qq < d) ? a[(int64_t)(b0 + uu) * d + q0 + qq] : (int8_t)0;
     }
@@ -1023,7 +1027,7 @@ __global__ void __launch_bounds__(256) k_lr_backward4(const int8_t* __restrict__
         if (q0 + qq >= d) continue;
         long long t = 0;
 #pragma unroll
-        for (int uu = 0; uu < kLbSamples; ++uu) t += (long long)gls[uu][g] * as[uu][qq];
+        for (int uu = 0; uu < NS; ++uu) t += (long long)gls[uu][g] * as[uu][qq];
         if (t != 0) atomicAdd(&dwlr[(int64_t)g * d + q0 + qq], (unsigned long long)t);
     }
     uint32_t mx = 0;
@@ -1333,6 +1337,10 @@ cudaError_t simt_lr_backward(const int8_t* a, const int32_t* gl, const int32_t* 
         if (e != cudaSuccess) return e;
     }
     dim3 grid((d + kLbQ - 1) / kLbQ, (B + kLbSamples - 1) / kLbSamples);
+    // the four-feature kernel takes 32 samples per CTA (half the weight-gradient
+    // atomics of 16) when the batch fills them
+    constexpr int kLb4Samples = 32;
+    dim3 grid4((d + kLbQ - 1) / kLbQ, (B + kLb4Samples - 1) / kLb4Samples);
     ProfScope ps(K_LR_BACKWARD, s, (lg ? 4.0 : 2.0) * B * d * G, 0.0);
     const FloorDiv32 al = FloorDiv32::make((uint32_t)(alpha_inv > 0 ? alpha_inv : 1));
     auto* dw64 = reinterpret_cast<unsigned long long*>(dwlr);
@@ -1344,13 +1352,13 @@ cudaError_t simt_lr_backward(const int8_t* a, const int32_t* gl, const int32_t* 
                         (uintptr_t)(lg->pool ? argmax : region)) & 15) == 0;
     if (quad) {
         if (G <= 10)
-            k_lr_backward4<10><<<grid, 256, 0, s>>>(a, gl, wlr, B, G, d, g0, al, region, argmax,
-                                                    delta, dw64, maxabs_gl, maxabs_wlr,
-                                                    maxabs_delta, status);
+            k_lr_backward4<10, kLb4Samples><<<grid4, 16 * kLb4Samples, 0, s>>>(
+                a, gl, wlr, B, G, d, g0, al, region, argmax, delta, dw64, maxabs_gl, maxabs_wlr,
+                maxabs_delta, status);
         else
-            k_lr_backward4<kLbMaxG><<<grid, 256, 0, s>>>(a, gl, wlr, B, G, d, g0, al, region,
-                                                         argmax, delta, dw64, maxabs_gl,
-                                                         maxabs_wlr, maxabs_delta, status);
+            k_lr_backward4<kLbMaxG, kLb4Samples><<<grid4, 16 * kLb4Samples, 0, s>>>(
+                a, gl, wlr, B, G, d, g0, al, region, argmax, delta, dw64, maxabs_gl, maxabs_wlr,
+                maxabs_delta, status);
         return cudaGetLastError();
     }
     if (G <= 10)

@@ -224,9 +224,8 @@ cudaError_t simt_lrpool_to_delta(const int32_t* gl, const int32_t* wlr, int G, i
 // Learning layer forward + loss: grad_l = floor(a W^T / (256 d)) - 32 onehot,
 // sse = sum grad_l^2 (mod 2^64), loss = floor(sse / 2) (if loss != NULL),
 // max|grad_l| into *maxabs_gl, status bits.  scratch: int64 buffer of
-// simt_learn_scratch(max_batch, d, G) words, zeroed once before first use
-// (its first word is a ticket the kernels leave at zero); *sse must be zero
-// on entry.
+// simt_learn_scratch(max_batch, d, G) words (partial sums and tickets,
+// cleared by each call); *sse must be zero on entry.
 size_t simt_learn_scratch(int max_batch, int d, int G);
 cudaError_t simt_learn_fwd(const int8_t* a, const int32_t* wlr, const int32_t* labels, int B,
                            int d, int G, int64_t* scratch, int32_t* grad_l, unsigned long long* sse,
