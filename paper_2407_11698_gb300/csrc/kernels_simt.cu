@@ -633,6 +633,31 @@ __device__ __forceinline__ void sgd_planes(const SgdTensor& t, int64_t i, int32_
     }
 }
 
+// Four consecutive updated weights into their limb planes when the planes are
+// laid out like W (linear layers; convs with Cin a multiple of 64): the same
+// split, one 8-byte store per plane at p + l * plane.
+__device__ __forceinline__ void sgd_planes4(uint16_t* p, int64_t plane, int4 w) {
+    int32_t v[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+    for (int l = 0; l < 4; ++l) {
+        uint32_t h[4];
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            int dg;
+            if (l < 3) {
+                // v = 256 q + r: digit r or r - 256, remainder q or q + 1
+                const int r = v[k] & 255;
+                dg = r - ((r >> 7) << 8);
+                v[k] = (v[k] >> 8) + (r >> 7);
+            } else {
+                dg = v[k];
+            }
+            h[k] = __float_as_uint((float)dg) >> 16;
+        }
+        *reinterpret_cast<uint2*>(p + l * plane) = make_uint2(h[0] | (h[1] << 16), h[2] | (h[3] << 16));
+    }
+}
+
 // Four consecutive weights per thread (16-byte loads of W, two of dW; the
 // tensors are this library's own 256-byte aligned buffers), the tail singly.
 __global__ void k_integersgd(SgdBatch bt) {
@@ -651,7 +676,9 @@ __global__ void k_integersgd(SgdBatch bt) {
         o.z = sgd_one(t, bt.round_trunc, w.z, g1.x, mx, ovf);
         o.w = sgd_one(t, bt.round_trunc, w.w, g1.y, mx, ovf);
         reinterpret_cast<int4*>(t.w)[i] = o;
-        if (t.planes) {
+        if (t.planes && t.contig) {
+            sgd_planes4(t.planes + 4 * i, t.plane, o);
+        } else if (t.planes) {
             sgd_planes(t, 4 * i, o.x);
             sgd_planes(t, 4 * i + 1, o.y);
             sgd_planes(t, 4 * i + 2, o.z);
@@ -1262,6 +1289,10 @@ cudaError_t simt_integersgd(const SgdBatch& b_in, cudaStream_t s) {
         if (b.t[i].planes) {
             if (b.t[i].cin < 1 || b.t[i].n >= ((int64_t)1 << 31)) return cudaErrorInvalidValue;
             b.t[i].cin_div = FloorDiv32::make((uint32_t)b.t[i].cin);
+            // planes laid out like W: entry (t, ci) of row co at co 9 cin + t cin + ci,
+            // 8-byte aligned for every group of four (plane stride a multiple of 4)
+            b.t[i].contig = b.t[i].row_k == 9 * b.t[i].tap_k && b.t[i].tap_k == b.t[i].cin &&
+                            b.t[i].plane % 4 == 0 && ((uintptr_t)b.t[i].planes & 7) == 0;
         }
     }
     dim3 grid(grid_for((nmax + 3) / 4, 256, 152 * 4), b.count);

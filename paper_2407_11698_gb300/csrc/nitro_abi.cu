@@ -53,9 +53,12 @@ struct nitro_block {
     int64_t* zsum = nullptr;        // learning-layer partial sums and ticket (simt_learn_scratch)
     int64_t* z64 = nullptr;         // scratch, int64 pre-activations / dgrad outputs
     size_t z64_elems = 0;
-    uint32_t* words = nullptr;      // [0] status [1] max|grad_l| [2] max|W_lr|
-                                    // [3 + i] max|W_i|  [3 + n + i] max|delta_i|
-                                    // [3 + 2n] step counter (dropout masks)
+    uint32_t* words = nullptr;      // [0] status [1] step counter (dropout masks)
+                                    // [2] max|W_lr| [3 + i] max|W_i|    (reset by the update)
+                                    // [3 + n] max|grad_l| [4 + n + i] max|delta_i|, then the
+                                    // SSE (8-byte aligned)              (reset by the backward)
+    uint32_t* words_host = nullptr; // pinned copy of the words, refreshed once per step: the
+                                    // limb-count hints that pick kernel variants
     uint64_t seed = 0;
     LrPoolGeom lp{1, 1, 0, 0};      // learning-layer pool window and output grid
     int8_t* zmp = nullptr;          // [max_batch x d] pooled learning input, or null
@@ -69,12 +72,13 @@ struct nitro_block {
 namespace {
 
 uint32_t* w_status(nitro_block* b) { return b->words; }
-uint32_t* w_gl(nitro_block* b) { return b->words + 1; }
+uint32_t* w_step(nitro_block* b) { return b->words + 1; }
 uint32_t* w_wlr(nitro_block* b) { return b->words + 2; }
 uint32_t* w_w(nitro_block* b, int i) { return b->words + 3 + i; }
-uint32_t* w_delta(nitro_block* b, int i) { return b->words + 3 + (int)b->L.size() + i; }
-uint32_t* w_step(nitro_block* b) { return b->words + 3 + 2 * (int)b->L.size(); }
-int n_words(int n_layers) { return 4 + 2 * n_layers; }
+uint32_t* w_gl(nitro_block* b) { return b->words + 3 + (int)b->L.size(); }
+uint32_t* w_delta(nitro_block* b, int i) { return b->words + 4 + (int)b->L.size() + i; }
+int sse_word(int n_layers) { return (4 + 2 * n_layers + 1) & ~1; }   // 8-byte aligned
+int n_words(int n_layers) { return sse_word(n_layers) + 2; }
 
 template <typename T>
 bool dalloc(nitro_block* b, T** p, size_t count) {
@@ -271,7 +275,16 @@ nitro_status nitro_init_block(const nitro_block_desc* desc, uint64_t seed, void*
     }
     ok = ok && dalloc(b, &b->Wlr, (size_t)b->G * b->d) && dalloc(b, &b->dWlr, (size_t)b->G * b->d) &&
          dalloc(b, &b->grad_l, (size_t)MB * b->G) && dalloc(b, &b->zsum, simt_learn_scratch(MB, (int)b->d, b->G)) && dalloc(b, &b->z64, z_need) &&
-         dalloc(b, &b->words, n_words(desc->n_layers)) && dalloc(b, &b->sse, 1);
+         dalloc(b, &b->words, n_words(desc->n_layers));
+    if (ok) {
+        b->sse = reinterpret_cast<unsigned long long*>(b->words + sse_word(desc->n_layers));
+        void* h = nullptr;
+        ok = cudaMallocHost(&h, sizeof(uint32_t) * n_words(desc->n_layers)) == cudaSuccess;
+        if (ok) {
+            b->host_allocs.push_back(h);
+            b->words_host = static_cast<uint32_t*>(h);
+        }
+    }
     b->z64_elems = z_need;
     for (int i = 0; ok && i < desc->n_layers; ++i) {
         Layer& ly = b->L[i];
@@ -279,6 +292,9 @@ nitro_status nitro_init_block(const nitro_block_desc* desc, uint64_t seed, void*
                                        b->allocs, b->host_allocs)
                       : tc_layer_init(ly.tc, ly.g, desc->max_batch, i > 0, w_w(b, i), w_delta(b, i),
                                       b->allocs, b->host_allocs);
+        // one copy of all the block's words per step refreshes the layers' hints
+        if (ok) tc_use_external_hints(ly.tc, b->words_host + 3 + i,
+                                      b->words_host + 4 + desc->n_layers + i);
     }
     if (!ok) {
         free_all(b);
@@ -306,6 +322,7 @@ nitro_status nitro_init_block(const nitro_block_desc* desc, uint64_t seed, void*
             e = tc_pack_limbs(b->L[i].W, b->L[i].wcount, w_w(b, i), b->L[i].lin_planes, s);
     }
     if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    if (e == cudaSuccess) std::memcpy(b->words_host, words.data(), words.size() * 4);
     if (e != cudaSuccess) {
         free_all(b);
         delete b;
@@ -397,10 +414,8 @@ nitro_status block_backward(nitro_block* b, const int8_t* a_in, const int32_t* l
     const int n = (int)b->L.size();
     const int G = b->G;
     const int64_t d = b->d;
-    // reset per-step accumulators and range words
-    NITRO_TRY(cudaMemsetAsync(b->sse, 0, sizeof(unsigned long long), s));
-    NITRO_TRY(cudaMemsetAsync(w_gl(b), 0, 4, s));
-    if (n) NITRO_TRY(cudaMemsetAsync(w_delta(b, 0), 0, 4 * n, s));
+    // reset the per-step range words and the SSE (one contiguous range)
+    NITRO_TRY(cudaMemsetAsync(w_gl(b), 0, 4 * (size_t)(n_words(n) - (3 + n)), s));
     if (batch == 0) {
         NITRO_TRY(cudaMemsetAsync(b->dWlr, 0, (size_t)G * d * 8, s));
         for (int i = 0; i < n; ++i) NITRO_TRY(cudaMemsetAsync(b->L[i].dW, 0, (size_t)b->L[i].wcount * 8, s));
@@ -478,7 +493,7 @@ nitro_status block_backward(nitro_block* b, const int8_t* a_in, const int32_t* l
                 NITRO_TRY(tc_conv_wgrad(ly.tc, g, ly.delta, w_delta(b, i), batch, ly.dW, w_status(b), s,
                                         &done, true, &sg, &sgd_done));
                 (*updated)[i] = done && sgd_done;
-                if ((*updated)[i]) NITRO_TRY(tc_weights_hint(ly.tc, s));
+
             } else {
                 NITRO_TRY(tc_conv_wgrad(ly.tc, g, ly.delta, w_delta(b, i), batch, ly.dW, w_status(b), s,
                                         &done));
@@ -562,15 +577,17 @@ nitro_status block_sgd(nitro_block* b, void* stream, const std::vector<char>* sk
             st.row_k = 9 * b->L[i].g.cin;
             st.tap_k = b->L[i].g.cin;
         }
-        NITRO_TRY(cudaMemsetAsync(w_w(b, i), 0, 4, s));
+        if (skip) NITRO_TRY(cudaMemsetAsync(w_w(b, i), 0, 4, s));
         bt.t[bt.count++] = st;
     }
     bt.t[bt.count++] = SgdTensor{b->Wlr, b->dWlr, (int64_t)b->G * b->d, b->desc.gamma_inv_lr,
                                  b->desc.eta_inv_lr, w_wlr(b), {}, {}, nullptr, 0, 0, 0, 0, {}};
-    NITRO_TRY(cudaMemsetAsync(w_wlr(b), 0, 4, s));
+    // max |W_lr| and every updated layer's max |W| start from zero: one range
+    // unless some layers were updated in their weight-gradient kernels
+    NITRO_TRY(cudaMemsetAsync(w_wlr(b), 0, 4 * (size_t)(skip ? 1 : 1 + n), s));
     NITRO_TRY(simt_integersgd(bt, s));
-    for (int i = 0; i < n; ++i)
-        if (!(skip && (*skip)[i])) NITRO_TRY(tc_weights_hint(b->L[i].tc, s));
+    // the kernel-variant hints of the next step: one copy of all the words
+    NITRO_TRY(cudaMemcpyAsync(b->words_host, b->words, 4 * (size_t)n_words(n), cudaMemcpyDeviceToHost, s));
     return NITRO_OK;
 }
 
@@ -747,6 +764,10 @@ nitro_status nitro_block_set_tensor(nitro_block* b, int which, int layer, const 
             return NITRO_ERR_CUDA;
     }
     if (cudaDeviceSynchronize() != cudaSuccess) return NITRO_ERR_CUDA;
+    // the kernel-variant hints follow the new weights
+    if (cudaMemcpy(b->words_host, b->words, 4 * (size_t)n_words((int)b->L.size()), cudaMemcpyDeviceToHost) !=
+        cudaSuccess)
+        return NITRO_ERR_CUDA;
     return NITRO_OK;
 }
 

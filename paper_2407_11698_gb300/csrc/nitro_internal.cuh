@@ -288,6 +288,7 @@ struct SgdTensor {
     int64_t plane;
     int row_k, tap_k, cin;
     FloorDiv32 cin_div;    // filled by simt_integersgd
+    bool contig;           // planes laid out like W (filled by simt_integersgd)
 };
 struct SgdBatch {
     SgdTensor t[kMaxSgdTensors];

@@ -1405,11 +1405,15 @@ bool tc_linear_init(TcLayer& t, const LayerGeom& g, int max_batch, uint16_t* act
 }
 
 int tc_limb_hint(const TcLayer& t, int which) {
+    if (!t.own_hints) {
+        const uint32_t* h = which ? t.hint_d : t.hint_w;
+        return h ? limb_count(*h) : 1;
+    }
     return t.max_host ? limb_count(t.max_host[which]) : 1;
 }
 
 cudaError_t tc_weights_hint(TcLayer& t, cudaStream_t s) {
-    if (!t.w_planes || !t.maxabs_w) return cudaSuccess;
+    if (!t.w_planes || !t.maxabs_w || !t.own_hints) return cudaSuccess;
     // host copy of max |W|, read later as a kernel-variant hint only
     return cudaMemcpyAsync(t.max_host, t.maxabs_w, sizeof(uint32_t), cudaMemcpyDeviceToHost, s);
 }
@@ -1433,7 +1437,7 @@ cudaError_t tc_refresh_weights(TcLayer& t, const LayerGeom& g, const int32_t* W,
                                                  t.w_planes);
     }
     cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
+    if (e != cudaSuccess || !t.own_hints) return e;
     return cudaMemcpyAsync(t.max_host, maxabs_w, sizeof(uint32_t), cudaMemcpyDeviceToHost, s);
 }
 
@@ -1533,7 +1537,7 @@ cudaError_t tc_pack_delta(TcLayer& t, const LayerGeom& g, const int32_t* delta,
                                                        maxabs_delta, t.d_nhwc);
     }
     cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
+    if (e != cudaSuccess || !t.own_hints) return e;
     return cudaMemcpyAsync(t.max_host + 1, maxabs_delta, sizeof(uint32_t), cudaMemcpyDeviceToHost, s);
 }
 

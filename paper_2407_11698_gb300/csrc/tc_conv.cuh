@@ -46,9 +46,23 @@ struct TcLayer {
     const uint32_t* maxabs_w = nullptr;
     const uint32_t* maxabs_d = nullptr;
     // pinned host copies of the two words, refreshed asynchronously; possibly
-    // stale, used only to pick a kernel variant (any choice is exact)
+    // stale, used only to pick a kernel variant (any choice is exact).  By
+    // default the layer keeps its own copies (max_host) and refreshes them
+    // itself; tc_use_external_hints points them into a caller's mirror that
+    // the caller refreshes.
     uint32_t* max_host = nullptr;
+    const uint32_t* hint_w = nullptr;
+    const uint32_t* hint_d = nullptr;
+    bool own_hints = true;
 };
+
+// Read the layer's limb-count hints from hint_w / hint_d (pinned host words
+// the caller refreshes) instead of copying them from the device per layer.
+inline void tc_use_external_hints(TcLayer& t, const uint32_t* hint_w, const uint32_t* hint_d) {
+    t.hint_w = hint_w;
+    t.hint_d = hint_d;
+    t.own_hints = false;
+}
 
 // IntegerSGD folded into the weight-gradient kernel (Algorithm 1 with the
 // forward layers' gamma_inv and eta_inv): the kernel updates W and its limb
