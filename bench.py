@@ -624,16 +624,18 @@ def run_sweep(args):
         gm.close()
         del a, b8, c
         torch.cuda.empty_cache()
-    # IntegerSGD alone: one linear layer of n x n weights, 16 bytes per weight
-    # (W read + write, dW read), against the measured HBM copy bandwidth
+    # IntegerSGD alone: one linear layer of n x n weights (16 bytes per weight:
+    # W read + write, dW read; + 8 for the four bf16 limb planes the update
+    # writes for the tensor-core forward) and its learning layer, against the
+    # measured HBM copy bandwidth
     hbm = peaks["hbm_gbs"]
     for n in ((4096, 16384) if "sgd" in parts else ()):
         blk = nb.Block([(nb.NITRO_LINEAR, n, n, 1, 1, 0)], n, seed=1, max_batch=1)
         ms, prof = timed(lambda: blk.sgd(), 5)
-        k = prof.get("integersgd", {"ms": float("nan"), "launches": 1})
+        k = prof.get("integersgd", {"ms": float("nan"), "launches": 1, "bytes": 0.0})
         kms = k["ms"] / max(1, k["launches"])
         params = n * n + 10 * n
-        byts = 16.0 * params
+        byts = k["bytes"] / max(1, k["launches"])
         print(json.dumps({"sweep": "integersgd", "params": params, "bytes": byts,
                           "kernel_ms": round(kms, 5), "call_ms": round(ms, 5),
                           "kernel_gbs": round(byts / kms / 1e6, 1),
