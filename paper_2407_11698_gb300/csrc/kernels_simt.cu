@@ -86,6 +86,7 @@ __device__ __forceinline__ int32_t load_b(const GemmParams& p, int n, int k) {
 // with 64-bit integer atomics (exact and order-independent).
 template <int MODE>
 __global__ void __launch_bounds__(256) k_gemm(GemmParams p) {
+    pdl_wait();
     __shared__ int32_t As[kTK][kTile + 4];
     __shared__ int32_t Bs[kTK][kTile + 4];
     const int m0 = blockIdx.y * kTile, n0 = blockIdx.x * kTile;
@@ -144,6 +145,7 @@ __global__ void k_fwd_epilogue(const int64_t* __restrict__ z, LayerGeom g, int B
                                int alpha_inv, int mu, int64_t kdiv, int8_t* __restrict__ out,
                                int8_t* __restrict__ out2, int8_t* __restrict__ region,
                                int8_t* __restrict__ argmax, DropoutArgs drop) {
+    pdl_wait();
     const int C = g.cout;
     if (!g.pool) {
         // dropout (linear layers): element i = b * out_features + j of this step's mask
@@ -222,6 +224,7 @@ __global__ void __launch_bounds__(256) k_learn_partial(const int8_t* __restrict_
                                                        int32_t* __restrict__ grad_l,
                                                        unsigned long long* sse, int64_t* loss,
                                                        uint32_t* maxabs_gl, uint32_t* status) {
+    pdl_wait();
     // thread (u, k): sample u of the group, features 8k .. 8k + 7 of the slice,
     // read as one 8-byte word when the rows allow it (vec8: d % 8 == 0 and an
     // 8-byte aligned a).  The slice of W_lr is staged in shared memory with
@@ -327,6 +330,7 @@ __global__ void __launch_bounds__(256) k_learn_partial(const int8_t* __restrict_
 // dW_lr[g][j] = sum_b grad_l[b][g] * a[b][j]
 __global__ void k_learn_dw(const int8_t* __restrict__ a, const int32_t* __restrict__ grad_l,
                            int B, int d, int G, int64_t* __restrict__ dwlr) {
+    pdl_wait();
     const int j = blockIdx.x * blockDim.x + threadIdx.x;
     const int g = blockIdx.y;
     if (j >= d) return;
@@ -343,6 +347,7 @@ __global__ void k_grad_to_delta(DeltaSrc src, LayerGeom g, int B, int alpha_inv,
                                 const int8_t* __restrict__ region,
                                 const int8_t* __restrict__ argmax, int32_t* __restrict__ delta,
                                 uint32_t* maxabs_delta, uint32_t* status) {
+    pdl_wait();
     const int64_t out_f = (int64_t)g.oh * g.ow * g.cout;
     const int64_t n = (int64_t)B * out_f;
     if (blockIdx.x == 0 && threadIdx.x == 0 &&
@@ -402,6 +407,7 @@ __global__ void k_grad_to_delta(DeltaSrc src, LayerGeom g, int B, int alpha_inv,
 __global__ void k_lr_pool_fwd(const int8_t* __restrict__ a, int B, int H, int W, int C, int kh,
                               int kw, int ph, int pw, int8_t* __restrict__ out,
                               uint8_t* __restrict__ am) {
+    pdl_wait();
     const int64_t n = (int64_t)B * ph * pw * C;
     for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
          i += (int64_t)gridDim.x * blockDim.x) {
@@ -430,6 +436,7 @@ __global__ void k_lr_pool_fwd4(const int8_t* __restrict__ a, int B, int H, int W
                                int kw, int ph, int pw, FloorDiv32 dv_c4, FloorDiv32 dv_pw,
                                FloorDiv32 dv_ph, int8_t* __restrict__ out,
                                uint8_t* __restrict__ am) {
+    pdl_wait();
     const int C4 = C >> 2;
     const uint32_t n4 = (uint32_t)B * ph * pw * C4;
     for (uint32_t i = blockIdx.x * blockDim.x + threadIdx.x; i < n4; i += gridDim.x * blockDim.x) {
@@ -470,6 +477,7 @@ __global__ void k_lrpool_to_delta(const int32_t* __restrict__ gl, const int32_t*
                                   int32_t* __restrict__ delta, const uint32_t* maxabs_gl,
                                   const uint32_t* maxabs_wlr, uint32_t* maxabs_delta,
                                   uint32_t* status) {
+    pdl_wait();
     const int C = g.cout;
     const int64_t n = (int64_t)B * g.h * g.w * C;
     if (blockIdx.x == 0 && threadIdx.x == 0 && int64_bound_exceeded(*maxabs_gl, *maxabs_wlr, G))
@@ -535,6 +543,7 @@ __global__ void k_lrpool_to_delta4(const int32_t* __restrict__ gl, const int32_t
                                    int32_t* __restrict__ delta, const uint32_t* maxabs_gl,
                                    const uint32_t* maxabs_wlr, uint32_t* maxabs_delta,
                                    uint32_t* status) {
+    pdl_wait();
     const int C = g.cout, C4 = g.cout >> 2;
     const uint32_t n4 = (uint32_t)B * g.h * g.w * C4;
     if (blockIdx.x == 0 && threadIdx.x == 0 && int64_bound_exceeded(*maxabs_gl, *maxabs_wlr, G))
@@ -661,6 +670,7 @@ __device__ __forceinline__ void sgd_planes4(uint16_t* p, int64_t plane, int4 w) 
 // Four consecutive weights per thread (16-byte loads of W, two of dW; the
 // tensors are this library's own 256-byte aligned buffers), the tail singly.
 __global__ void k_integersgd(SgdBatch bt) {
+    pdl_wait();
     const SgdTensor t = bt.t[blockIdx.y];
     uint32_t mx = 0;
     bool ovf = false;
@@ -727,6 +737,7 @@ struct SmallFwdArgs {
 };
 
 __global__ void __launch_bounds__(256) k_conv_small_fwd(const SmallFwdArgs a) {
+    pdl_wait();
     extern __shared__ int32_t wsm[];                 // Cout * 9 * Cin
     __shared__ int8_t relu_tab[256];
     const int nw = a.Cout * 9 * a.Cin;
@@ -825,6 +836,7 @@ __global__ void __launch_bounds__(256) k_conv_small_wgrad(const int8_t* __restri
                                                           const int32_t* __restrict__ d, int B,
                                                           int H, int W, int Cin, int Cout,
                                                           unsigned long long* __restrict__ dw) {
+    pdl_wait();
     extern __shared__ int32_t sm[];
     const int rows = min(kWgRows, H - blockIdx.x * kWgRows);
     const int y0 = blockIdx.x * kWgRows, b = blockIdx.y;
@@ -884,6 +896,7 @@ __global__ void __launch_bounds__(256) k_lr_backward(const int8_t* __restrict__ 
                                                      const uint32_t* maxabs_gl,
                                                      const uint32_t* maxabs_wlr,
                                                      uint32_t* maxabs_delta, uint32_t* status) {
+    pdl_wait();
     __shared__ int32_t gls[kLbSamples][GM];
     __shared__ int8_t as[kLbSamples][kLbQ];
     const int ql = threadIdx.x % kLbQ, sl = threadIdx.x / kLbQ;
@@ -1004,6 +1017,7 @@ __global__ void __launch_bounds__(16 * NS) k_lr_backward4(const int8_t* __restri
                                                       const uint32_t* maxabs_gl,
                                                       const uint32_t* maxabs_wlr,
                                                       uint32_t* maxabs_delta, uint32_t* status) {
+    pdl_wait();
     __shared__ int32_t gls[NS][GM];
     __shared__ int8_t as[NS][kLbQ];
     __shared__ __align__(16) int32_t wsl[GM][kLbQ];
@@ -1152,12 +1166,12 @@ cudaError_t simt_gemm(int mode, const int8_t* act, const int32_t* grad, const in
                                 K_SIMT_LIN_FWD, K_SIMT_LIN_DGRAD, K_SIMT_LIN_WGRAD};
     ProfScope ps(kIds[mode], s, 2.0 * p.M * p.N * p.K, 0.0);
     switch (mode) {
-        case GM_CONV_FWD: k_gemm<GM_CONV_FWD><<<grid, 256, 0, s>>>(p); break;
-        case GM_CONV_DGRAD: k_gemm<GM_CONV_DGRAD><<<grid, 256, 0, s>>>(p); break;
-        case GM_CONV_WGRAD: k_gemm<GM_CONV_WGRAD><<<grid, 256, 0, s>>>(p); break;
-        case GM_LIN_FWD: k_gemm<GM_LIN_FWD><<<grid, 256, 0, s>>>(p); break;
-        case GM_LIN_DGRAD: k_gemm<GM_LIN_DGRAD><<<grid, 256, 0, s>>>(p); break;
-        default: k_gemm<GM_LIN_WGRAD><<<grid, 256, 0, s>>>(p); break;
+        case GM_CONV_FWD: launch_k(k_gemm<GM_CONV_FWD>, grid, 256, 0, s, p); break;
+        case GM_CONV_DGRAD: launch_k(k_gemm<GM_CONV_DGRAD>, grid, 256, 0, s, p); break;
+        case GM_CONV_WGRAD: launch_k(k_gemm<GM_CONV_WGRAD>, grid, 256, 0, s, p); break;
+        case GM_LIN_FWD: launch_k(k_gemm<GM_LIN_FWD>, grid, 256, 0, s, p); break;
+        case GM_LIN_DGRAD: launch_k(k_gemm<GM_LIN_DGRAD>, grid, 256, 0, s, p); break;
+        default: launch_k(k_gemm<GM_LIN_WGRAD>, grid, 256, 0, s, p); break;
     }
     return cudaGetLastError();
 }
@@ -1175,7 +1189,7 @@ cudaError_t simt_fwd_epilogue(const int64_t* z, const LayerGeom& g, int B, int a
         da = *drop;
     }
     ProfScope ps(K_FWD_EPILOGUE, s, 0.0, 0.0);
-    k_fwd_epilogue<<<grid_for(n, 256), 256, 0, s>>>(z, g, B, alpha_inv, mu, kdiv, out, out2,
+    launch_k(k_fwd_epilogue, grid_for(n, 256), 256, 0, s, z, g, B, alpha_inv, mu, kdiv, out, out2,
                                                     region, argmax, da);
     return cudaGetLastError();
 }
@@ -1187,11 +1201,11 @@ cudaError_t simt_lr_pool_fwd(const int8_t* a, int B, int H, int W, int C, int kh
     if (kh < 1 || kw < 1 || ph * kh > H || pw * kw > W || kh * kw > 256) return cudaErrorInvalidValue;
     ProfScope ps(K_LR_POOL, s, 0.0, (double)B * H * W * C + 2.0 * n);
     if (C % 4 == 0 && (((uintptr_t)a | (uintptr_t)out | (uintptr_t)am) & 3) == 0)
-        k_lr_pool_fwd4<<<grid_for(n / 4, 256), 256, 0, s>>>(
+        launch_k(k_lr_pool_fwd4, grid_for(n / 4, 256), 256, 0, s,
             a, B, H, W, C, kh, kw, ph, pw, FloorDiv32::make((uint32_t)(C / 4)),
             FloorDiv32::make((uint32_t)pw), FloorDiv32::make((uint32_t)ph), out, am);
     else
-        k_lr_pool_fwd<<<grid_for(n, 256), 256, 0, s>>>(a, B, H, W, C, kh, kw, ph, pw, out, am);
+        launch_k(k_lr_pool_fwd, grid_for(n, 256), 256, 0, s, a, B, H, W, C, kh, kw, ph, pw, out, am);
     return cudaGetLastError();
 }
 
@@ -1217,13 +1231,13 @@ cudaError_t simt_lrpool_to_delta(const int32_t* gl, const int32_t* wlr, int G, i
     const bool aligned = (((uintptr_t)am | (uintptr_t)region | (uintptr_t)delta |
                            (uintptr_t)(g.pool ? argmax : region)) & 15) == 0;
     if (g.cout % 4 == 0 && aligned && (1 << lg_kh) == lp.kh && (1 << lg_kw) == lp.kw) {
-        k_lrpool_to_delta4<<<grid_for(n / 4, 256), 256, 0, s>>>(
+        launch_k(k_lrpool_to_delta4, grid_for(n / 4, 256), 256, 0, s,
             gl, wlr, G, d, g, lp, lg_kh, lg_kw, B, FloorDiv32::make((uint32_t)(g.cout / 4)),
             FloorDiv32::make((uint32_t)g.w), FloorDiv32::make((uint32_t)g.h), am, argmax, region,
             FloorDiv32::make((uint32_t)alpha_inv), delta, maxabs_gl, maxabs_wlr, maxabs_delta,
             status);
     } else {
-        k_lrpool_to_delta<<<grid_for(n, 256), 256, 0, s>>>(
+        launch_k(k_lrpool_to_delta, grid_for(n, 256), 256, 0, s,
             gl, wlr, G, d, g, lp, B, am, argmax, region,
             FloorDiv32::make((uint32_t)alpha_inv), delta, maxabs_gl, maxabs_wlr, maxabs_delta,
             status);
@@ -1247,7 +1261,7 @@ cudaError_t simt_learn_fwd(const int8_t* a, const int32_t* wlr, const int32_t* l
     dim3 grid((d + kLpSlice - 1) / kLpSlice, groups);
     ProfScope ps(K_LEARN_FWD, s, 2.0 * B * d * G, 0.0);
     const int vec8 = d % 8 == 0 && ((uintptr_t)a & 7) == 0;
-    k_learn_partial<<<grid, 256, 0, s>>>(a, wlr, B, d, G, vec8,
+    launch_k(k_learn_partial, grid, 256, 0, s, a, wlr, B, d, G, vec8,
                                          reinterpret_cast<unsigned long long*>(zsum),
                                          FloorDiv::make((uint64_t)d), labels, grad_l, sse, loss,
                                          maxabs_gl, status);
@@ -1258,7 +1272,7 @@ cudaError_t simt_learn_dw(const int8_t* a, const int32_t* grad_l, int B, int d, 
                           int64_t* dwlr, cudaStream_t s) {
     dim3 grid((d + 255) / 256, G);
     ProfScope ps(K_LEARN_DW, s, 2.0 * B * d * G, 0.0);
-    k_learn_dw<<<grid, 256, 0, s>>>(a, grad_l, B, d, G, dwlr);
+    launch_k(k_learn_dw, grid, 256, 0, s, a, grad_l, B, d, G, dwlr);
     return cudaGetLastError();
 }
 
@@ -1272,7 +1286,7 @@ cudaError_t simt_grad_to_delta(const DeltaSrc& src, const LayerGeom& g, int B, i
     }
     const int64_t n = (int64_t)B * g.oh * g.ow * g.cout;
     ProfScope ps(K_GRAD_TO_DELTA, s, 0.0, 0.0);
-    k_grad_to_delta<<<grid_for(n, 256), 256, 0, s>>>(src, g, B, alpha_inv, region, argmax, delta,
+    launch_k(k_grad_to_delta, grid_for(n, 256), 256, 0, s, src, g, B, alpha_inv, region, argmax, delta,
                                                      maxabs_delta, status);
     return cudaGetLastError();
 }
@@ -1300,7 +1314,7 @@ cudaError_t simt_integersgd(const SgdBatch& b_in, cudaStream_t s) {
     for (int i = 0; i < b.count; ++i)
         bytes += (b.t[i].planes ? 24.0 : 16.0) * b.t[i].n;   // W r+w, dW r (+ 4 bf16 planes)
     ProfScope ps(K_INTEGERSGD, s, 0.0, bytes);
-    k_integersgd<<<grid, 256, 0, s>>>(b);
+    launch_k(k_integersgd, grid, 256, 0, s, b);
     return cudaGetLastError();
 }
 
@@ -1332,7 +1346,7 @@ cudaError_t simt_conv_small_fwd(const int8_t* x, const int32_t* w, const LayerGe
     const int64_t n = (int64_t)B * ((g.h + step - 1) / step) * ((g.w + step - 1) / step) * (g.cout / kSmallCo);
     const size_t smem = sizeof(int32_t) * (size_t)g.cout * 9 * g.cin;
     ProfScope ps(K_SIMT_CONV_FWD, s, 2.0 * B * g.h * g.w * g.cout * 9.0 * g.cin, 0.0);
-    k_conv_small_fwd<<<grid_for(n, 256, 152 * 32), 256, smem, s>>>(a);
+    launch_k(k_conv_small_fwd, grid_for(n, 256, 152 * 32), 256, smem, s, a);
     return cudaGetLastError();
 }
 
@@ -1349,7 +1363,7 @@ cudaError_t simt_conv_small_wgrad(const int8_t* x, const int32_t* d, const Layer
         if (e != cudaSuccess) return e;
     }
     ProfScope ps(K_SIMT_CONV_WGRAD, s, 2.0 * B * g.h * g.w * g.cout * 9.0 * g.cin, 0.0);
-    k_conv_small_wgrad<<<grid, 256, smem, s>>>(x, d, B, g.h, g.w, g.cin, g.cout,
+    launch_k(k_conv_small_wgrad, grid, 256, smem, s, x, d, B, g.h, g.w, g.cin, g.cout,
                                                reinterpret_cast<unsigned long long*>(dw));
     return cudaGetLastError();
 }
@@ -1383,21 +1397,21 @@ cudaError_t simt_lr_backward(const int8_t* a, const int32_t* gl, const int32_t* 
                         (uintptr_t)(lg->pool ? argmax : region)) & 15) == 0;
     if (quad) {
         if (G <= 10)
-            k_lr_backward4<10, kLb4Samples><<<grid4, 16 * kLb4Samples, 0, s>>>(
+            launch_k(k_lr_backward4<10, kLb4Samples>, grid4, 16 * kLb4Samples, 0, s,
                 a, gl, wlr, B, G, d, g0, al, region, argmax, delta, dw64, maxabs_gl, maxabs_wlr,
                 maxabs_delta, status);
         else
-            k_lr_backward4<kLbMaxG, kLb4Samples><<<grid4, 16 * kLb4Samples, 0, s>>>(
+            launch_k(k_lr_backward4<kLbMaxG, kLb4Samples>, grid4, 16 * kLb4Samples, 0, s,
                 a, gl, wlr, B, G, d, g0, al, region, argmax, delta, dw64, maxabs_gl, maxabs_wlr,
                 maxabs_delta, status);
         return cudaGetLastError();
     }
     if (G <= 10)
-        k_lr_backward<10><<<grid, 256, 0, s>>>(a, gl, wlr, B, G, d, lg != nullptr, g0, al, region,
+        launch_k(k_lr_backward<10>, grid, 256, 0, s, a, gl, wlr, B, G, d, lg != nullptr, g0, al, region,
                                                argmax, delta, dw64, maxabs_gl, maxabs_wlr,
                                                maxabs_delta, status);
     else
-        k_lr_backward<kLbMaxG><<<grid, 256, 0, s>>>(a, gl, wlr, B, G, d, lg != nullptr, g0, al,
+        launch_k(k_lr_backward<kLbMaxG>, grid, 256, 0, s, a, gl, wlr, B, G, d, lg != nullptr, g0, al,
                                                     region, argmax, delta, dw64, maxabs_gl,
                                                     maxabs_wlr, maxabs_delta, status);
     return cudaGetLastError();

@@ -2,6 +2,7 @@
 #pragma once
 
 #include <cstdint>
+#include <utility>
 #include <cuda_runtime.h>
 
 #include "nitro.h"
@@ -299,5 +300,44 @@ struct SgdBatch {
 };
 cudaError_t simt_integersgd(const SgdBatch& b, cudaStream_t s);
 
+
+// ---------------------------------------------------------------------------
+// Programmatic dependent launch.  A kernel queued with launch_k may start
+// (get SMs, set up shared memory, barriers and TMEM) while the kernel before
+// it in the stream is still finishing; every kernel so queued executes
+// pdl_wait() in each thread before its first access to global memory, which
+// blocks until the previous kernel has completed and its writes are visible.
+// pdl_trigger() lets the next kernel of the stream start launching; it only
+// takes effect once every CTA of this kernel has executed it or exited.
+// Both are no-ops for a kernel queued without the attribute.  Only the
+// contraction kernel triggers, once its MMAs are issued: an early trigger
+// lets the next kernel's waiting CTAs hold SMs that kernels of the other
+// block streams would use (measured slower on the VGG-style step), and the
+// other kernels trigger implicitly when their CTAs exit.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+// Whether launch_k queues kernels with the programmatic-serialization
+// attribute (on unless the environment sets NITRO_PDL=0; read once).
+bool pdl_enabled();
+
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_k(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                            cudaStream_t s, Args&&... args) {
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = pdl_enabled() ? 1 : 0;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
 
 }  // namespace nitro

@@ -1,6 +1,8 @@
 // Launch counter and per-kernel CUDA-event timing (see prof.cuh) plus the
-// diagnostic ABI calls that read them.
+// diagnostic ABI calls that read them; the launch policy switch (programmatic
+// dependent launch, NITRO_PDL=0 turns it off).
 #include <atomic>
+#include <cstdlib>
 #include <mutex>
 #include <vector>
 
@@ -46,6 +48,14 @@ const char* const kNames[K_COUNT] = {
 }  // namespace
 
 const char* kernel_name(int id) { return (id >= 0 && id < K_COUNT) ? kNames[id] : "?"; }
+
+bool pdl_enabled() {
+    static const bool on = [] {
+        const char* e = std::getenv("NITRO_PDL");
+        return !(e && e[0] == '0');
+    }();
+    return on;
+}
 
 ProfScope::ProfScope(int id, cudaStream_t s, double ops, double bytes) : slot_(-1), s_(s) {
     g_launches.fetch_add(1, std::memory_order_relaxed);

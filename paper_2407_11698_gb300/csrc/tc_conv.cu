@@ -362,19 +362,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_init(tempty_bar(b), kEpiWarps);
         }
         *abort_flag = 0;
-        // Fused input gradient: the lower delta is stored as the low 32 bits of
-        // the exact sum, and limb pairs with la + lb >= 4 only add multiples
-        // of 2^32.  They matter only for deciding OVERFLOW, so once that bit
-        // is latched they are skipped.  Read once per CTA so that all roles
-        // walk the same passes (CTAs may differ; each result is the same).
-        *hiskip_slot = (MODE == TC_DGRAD && args.fuse)
-            ? ((*reinterpret_cast<volatile uint32_t*>(args.status) & ST_OVERFLOW) != 0) : 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
-    // int32 x int32 contraction: flag when max|delta| max|W| 9 Cout >= 2^63
-    if (MODE == TC_DGRAD && args.fuse && blockIdx.x == 0 && threadIdx.x == 64 &&
-        int64_bound_exceeded(*args.bound_a, *args.bound_b, 9LL * args.Cout))
-        atomicOr(args.status, ST_OVERFLOW);
     // NITRO-ReLU value of every z* in [-127, 127] (fused forward epilogue)
     if (MODE == TC_FWD && args.fuse) {
         for (int i = threadIdx.x; i < 255; i += kThreads)
@@ -389,6 +378,27 @@ __global__ void __launch_bounds__(kThreads, 1)
                      : "memory");
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
     }
+    if (warp == 0 && lane == 0) {
+        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmA)) : "memory");
+        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmB)) : "memory");
+    }
+    // The set-up above touches only shared memory, TMEM and the kernel's own
+    // tensor maps, so it may overlap the end of the previous kernel in the
+    // stream; from here on the kernel reads what that kernel wrote.
+    pdl_wait();
+    if (threadIdx.x == 0) {
+        // Fused input gradient: the lower delta is stored as the low 32 bits of
+        // the exact sum, and limb pairs with la + lb >= 4 only add multiples
+        // of 2^32.  They matter only for deciding OVERFLOW, so once that bit
+        // is latched they are skipped.  Read once per CTA so that all roles
+        // walk the same passes (CTAs may differ; each result is the same).
+        *hiskip_slot = (MODE == TC_DGRAD && args.fuse)
+            ? ((*reinterpret_cast<volatile uint32_t*>(args.status) & ST_OVERFLOW) != 0) : 0;
+    }
+    // int32 x int32 contraction: flag when max|delta| max|W| 9 Cout >= 2^63
+    if (MODE == TC_DGRAD && args.fuse && blockIdx.x == 0 && threadIdx.x == 64 &&
+        int64_bound_exceeded(*args.bound_a, *args.bound_b, 9LL * args.Cout))
+        atomicOr(args.status, ST_OVERFLOW);
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -568,6 +578,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
             }
         mma_done:;
+            // every MMA of this CTA is issued: the next kernel in the stream
+            // may start launching (its CTAs take SMs as this kernel's CTAs exit)
+            pdl_trigger();
         }
     }
     } else {
@@ -1022,6 +1035,7 @@ __device__ __forceinline__ uint16_t bf16_bits(int v) {
 // int8 NHWC [P][C] -> bf16 NHWC [P][Cp] copy, zero in channels C..Cp-1
 __global__ void k_pack_act_nhwc(const int8_t* __restrict__ x, int64_t P, int C, int Cp,
                                 uint16_t* __restrict__ out) {
+    pdl_wait();
     const int64_t n = P * Cp;
     for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
          i += (int64_t)gridDim.x * blockDim.x) {
@@ -1039,6 +1053,7 @@ __global__ void k_pack_act_nhwc(const int8_t* __restrict__ x, int64_t P, int C, 
 __global__ void __launch_bounds__(256) k_pack_im2col(const int8_t* __restrict__ x, int B, int H,
                                                      int W, int Cin,
                                                      uint16_t* __restrict__ out) {
+    pdl_wait();
     extern __shared__ int8_t win[];            // [3][W + 2][Cin]
     __shared__ int tab[kBK];                   // window offset of entry k, or -1
     const int rowlen = (W + 2) * Cin;
@@ -1087,6 +1102,7 @@ inline size_t im2col_smem(int W, int Cin) { return (size_t)3 * (W + 2) * Cin; }
 // thread (one 8-byte load, one 16-byte store)
 __global__ void k_pack_act_nhwc8(const int8_t* __restrict__ x, int64_t n8,
                                  uint16_t* __restrict__ out) {
+    pdl_wait();
     for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n8;
          i += (int64_t)gridDim.x * blockDim.x) {
         const uint2 v = reinterpret_cast<const uint2*>(x)[i];
@@ -1108,6 +1124,7 @@ __global__ void k_pack_act_nhwc8(const int8_t* __restrict__ x, int64_t n8,
 __global__ void __launch_bounds__(256) k_pack_delta_nhwc(const int32_t* __restrict__ d, int64_t n,
                                                          int vec, const uint32_t* maxabs,
                                                          uint16_t* __restrict__ out) {
+    pdl_wait();
     const int L = limb_count(*maxabs);
     const int64_t n8 = n / 8;
     for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n8;
@@ -1153,6 +1170,7 @@ __global__ void __launch_bounds__(256) k_pack_delta_nhwc(const int32_t* __restri
 // rounded up to 64, or row_k = 64, tap_k = Cin for im2col rows)
 __global__ void k_pack_weights(const int32_t* __restrict__ W, int Cout, int Cin, int row_k,
                                int tap_k, const uint32_t* maxabs, uint16_t* __restrict__ wp) {
+    pdl_wait();
     const int L = limb_count(*maxabs);
     const int64_t n = (int64_t)Cout * 9 * Cin;
     const int64_t nk = (int64_t)Cout * row_k;
@@ -1263,7 +1281,7 @@ cudaError_t launch_gemm(const CUtensorMap& a, const CUtensorMap& b, const TcArgs
         attr_set = true;
     }
     const int grid = args.total_tiles < sm_count() ? args.total_tiles : sm_count();
-    k_tc_gemm<MODE, N, PB><<<grid, kThreads, C::SMEM, s>>>(a, b, args);
+    launch_k(k_tc_gemm<MODE, N, PB>, grid, kThreads, C::SMEM, s, a, b, args);
     return cudaGetLastError();
 }
 
@@ -1433,7 +1451,7 @@ cudaError_t tc_refresh_weights(TcLayer& t, const LayerGeom& g, const int32_t* W,
     {
         ProfScope ps(K_TC_PACK_W, s, 0.0, (double)n * 4 * 2);
         const int row_k = t.im2col ? kBK : 9 * t.cin_k, tap_k = t.im2col ? g.cin : t.cin_k;
-        k_pack_weights<<<grid1d(n), 256, 0, s>>>(W, g.cout, g.cin, row_k, tap_k, maxabs_w,
+        launch_k(k_pack_weights, grid1d(n), 256, 0, s, W, g.cout, g.cin, row_k, tap_k, maxabs_w,
                                                  t.w_planes);
     }
     cudaError_t e = cudaGetLastError();
@@ -1449,16 +1467,16 @@ cudaError_t tc_pack_input(TcLayer& t, const LayerGeom& g, const int8_t* x, int b
         ProfScope ps(K_TC_PACK_X, s, 0.0, (double)P * (g.cin + 2 * kBK));
         const int64_t rows = (int64_t)batch * g.h;
         const int grid = (int)(rows < 152 * 8 ? rows : 152 * 8);
-        k_pack_im2col<<<grid, 256, im2col_smem(g.w, g.cin), s>>>(x, batch, g.h, g.w, g.cin,
+        launch_k(k_pack_im2col, grid, 256, im2col_smem(g.w, g.cin), s, x, batch, g.h, g.w, g.cin,
                                                                  t.act_nhwc);
         return cudaGetLastError();
     }
     ProfScope ps(K_TC_PACK_X, s, 0.0, (double)P * (g.cin + 2 * t.cin8));
     if (g.cin == t.cin8 && g.cin % 8 == 0 && ((uintptr_t)x & 7) == 0) {
-        k_pack_act_nhwc8<<<grid1d(P * g.cin / 8), 256, 0, s>>>(x, P * g.cin / 8, t.act_nhwc);
+        launch_k(k_pack_act_nhwc8, grid1d(P * g.cin / 8), 256, 0, s, x, P * g.cin / 8, t.act_nhwc);
         return cudaGetLastError();
     }
-    k_pack_act_nhwc<<<grid1d(P * t.cin8), 256, 0, s>>>(x, P, g.cin, t.cin8, t.act_nhwc);
+    launch_k(k_pack_act_nhwc, grid1d(P * t.cin8), 256, 0, s, x, P, g.cin, t.cin8, t.act_nhwc);
     return cudaGetLastError();
 }
 
@@ -1533,7 +1551,7 @@ cudaError_t tc_pack_delta(TcLayer& t, const LayerGeom& g, const int32_t* delta,
     const int64_t n = (int64_t)batch * g.h * g.w * g.cout;   // cout % 8 == 0
     if (!planes_done) {
         ProfScope ps(K_TC_PACK_D, s, 0.0, (double)n * 4 * 2);
-        k_pack_delta_nhwc<<<grid1d(n / 8), 256, 0, s>>>(delta, n, ((uintptr_t)delta & 15) == 0,
+        launch_k(k_pack_delta_nhwc, grid1d(n / 8), 256, 0, s, delta, n, ((uintptr_t)delta & 15) == 0,
                                                        maxabs_delta, t.d_nhwc);
     }
     cudaError_t e = cudaGetLastError();
@@ -1702,6 +1720,7 @@ cudaError_t tc_timeout_probe(uint32_t* status, uint64_t limit_ns, cudaStream_t s
 // ------------------------------------------------------------------ plain GEMM
 namespace {
 __global__ void k_maxabs(const int32_t* __restrict__ x, int64_t n, uint32_t* out) {
+    pdl_wait();
     uint32_t m = 0;
     for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
          i += (int64_t)gridDim.x * blockDim.x)
@@ -1716,14 +1735,14 @@ cudaError_t tc_maxabs(const int32_t* x, int64_t n, uint32_t* out, cudaStream_t s
     cudaError_t e = cudaMemsetAsync(out, 0, sizeof(uint32_t), s);
     if (e != cudaSuccess || n <= 0) return e;
     ProfScope ps(K_TC_PACK, s, 0.0, (double)n * 4);
-    k_maxabs<<<grid1d(n), 256, 0, s>>>(x, n, out);
+    launch_k(k_maxabs, grid1d(n), 256, 0, s, x, n, out);
     return cudaGetLastError();
 }
 
 cudaError_t tc_pack_int8(const int8_t* x, int64_t rows, int cols, uint16_t* out, cudaStream_t s) {
     if (rows <= 0) return cudaSuccess;
     ProfScope ps(K_TC_PACK, s, 0.0, (double)rows * cols * 3);
-    k_pack_act_nhwc<<<grid1d(rows * cols), 256, 0, s>>>(x, rows, cols, cols, out);
+    launch_k(k_pack_act_nhwc, grid1d(rows * cols), 256, 0, s, x, rows, cols, cols, out);
     return cudaGetLastError();
 }
 
@@ -1731,7 +1750,7 @@ cudaError_t tc_pack_limbs(const int32_t* x, int64_t n, const uint32_t* maxabs, u
                           cudaStream_t s) {
     if (n <= 0) return cudaSuccess;
     ProfScope ps(K_TC_PACK, s, 0.0, (double)n * 4 * 2);
-    k_pack_delta_nhwc<<<grid1d(n / 8), 256, 0, s>>>(x, n, ((uintptr_t)x & 15) == 0, maxabs, planes);
+    launch_k(k_pack_delta_nhwc, grid1d(n / 8), 256, 0, s, x, n, ((uintptr_t)x & 15) == 0, maxabs, planes);
     return cudaGetLastError();
 }
 
