@@ -168,3 +168,54 @@ def test_int_gemm(torch, m, n, k, lb):
         assert gm.status() == nb.NITRO_OK
     finally:
         gm.close()
+
+
+# every limb at -128 (the canonical split's top limb of an int32 stops at -127)
+_ALL_LIMBS_MIN = -128 * (1 + 256 + 65536) - 127 * 2**24
+
+
+@pytest.mark.parametrize("k", [1024, 576, 3000])
+def test_extreme_limb_products_gemm(torch, k):
+    # half of the output columns see products of 2^14 in every limb pair, so the
+    # exact chunk sums reach 2^24 (1024 products per chunk at k = 1024); the
+    # other half stays small: drains with both large and small accumulator
+    # values, on either side of the 2^22 range of the add-based conversion
+    m, n = 256, 192
+    a = np.full((m, k), -128, dtype=np.int8)
+    a[1::7] = 127
+    b = synth.int_tensor(45, (n, k), -90, 90, dtype=np.int32)
+    b[: n // 2] = _ALL_LIMBS_MIN
+    b[n // 2: n // 2 + 8] = -128
+    gm = nb.IntGemm(m, n, k)
+    try:
+        c = torch.empty((m, n), dtype=torch.int64, device="cuda")
+        gm.run(_dev(torch, a, np.int8), _dev(torch, b, np.int32), c)
+        assert np.array_equal(c.cpu().numpy(), O.linear_fwd(a.astype(np.int64), b.astype(np.int64)))
+        assert gm.status() == nb.NITRO_OK
+    finally:
+        gm.close()
+
+
+def test_extreme_limb_products_conv(torch):
+    # the three conv contractions with operands whose limbs all sit at -128 in
+    # half of the channels (chunk sums of 576 products of 2^14 = 9.4e6 > 2^22)
+    B, h, w, c = 2, 8, 8, 128
+    a = np.full((B, h, w, c), -128, dtype=np.int64)
+    W = synth.int_tensor(46, (c, 3, 3, c), -90, 90)
+    W[: c // 2] = _ALL_LIMBS_MIN
+    d = synth.int_tensor(47, (B, h, w, c), -90, 90)
+    d[..., : c // 2] = _ALL_LIMBS_MIN
+    conv = nb.Conv3x3(B, h, w, c, c)
+    try:
+        ad, Wd, dd = _dev(torch, a, np.int8), _dev(torch, W, np.int32), _dev(torch, d, np.int32)
+        z = torch.empty((B, h, w, c), dtype=torch.int64, device="cuda")
+        conv.contract(nb.NITRO_CONTRACT_FWD, ad, Wd, z)
+        assert np.array_equal(z.cpu().numpy(), O.conv3x3_fwd(a, W))
+        dw = torch.empty((c, 3, 3, c), dtype=torch.int64, device="cuda")
+        conv.contract(nb.NITRO_CONTRACT_WGRAD, ad, dd, dw)
+        assert np.array_equal(dw.cpu().numpy(), O.conv3x3_wgrad(a, d))
+        g = torch.empty((B, h, w, c), dtype=torch.int64, device="cuda")
+        conv.contract(nb.NITRO_CONTRACT_DGRAD, dd, Wd, g)
+        assert np.array_equal(g.cpu().numpy(), O.conv3x3_dgrad(d, W))
+    finally:
+        conv.close()
