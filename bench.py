@@ -443,6 +443,8 @@ def run_ours(args, rank, world, local_rank):
                    "block_streams": "one" if args.sequential_blocks else "one per block",
                    "update": ("nitro_block_backward_update (folded into un-split weight "
                               "gradients)" if args.fused_update else "separate IntegerSGD call"),
+                   "launch": ("programmatic dependent launch" if os.environ.get("NITRO_PDL", "1") != "0"
+                              else "stream-ordered"),
                    "l2": "flushed (512 MiB write) between timed steps",
                    "parallelism": "replicas" if world > 1 else "single"},
         "e2e": {"value": round(e2e_value, 2), "unit": "images/s",
