@@ -525,7 +525,21 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
             for (int j = 1; j <= PB; ++j)
                 idesc_nb[j] = idesc_bf16(kBM, j * N, MODE == TC_WGRAD, MODE == TC_WGRAD || MODE == TC_DGRAD);
-            int it = 0, chunk = 0;
+            // K-major: a K-step of 16 is 32 bytes along each row; MN-major: 16
+            // rows, two 1024-byte row groups, and 64-wide blocks along M / N 8 KB
+            // apart.  Only the address field (bytes / 16, below 2^14 since shared
+            // memory is below 256 KB) moves per K-step and per ring stage, so the
+            // descriptors of stage 0 are built once and offset per K-block.
+            constexpr bool a_mn = MODE == TC_WGRAD;
+            constexpr bool b_mn = MODE == TC_WGRAD || MODE == TC_DGRAD;
+            constexpr uint32_t kStepA = a_mn ? 2048 / 16 : 32 / 16;
+            constexpr uint32_t kStepB = b_mn ? 2048 / 16 : 32 / 16;
+            constexpr uint32_t kStageD = C::STAGE / 16;
+            const uint32_t s0 = smem_u32(smem);
+            const uint64_t da_base = a_mn ? desc_sw128_mn(s0, 64 * 128) : desc_sw128(s0);
+            int st = 0;          // ring stage of the next K-block
+            uint32_t ph = 0;     // and the parity of the phase it waits for
+            int chunk = 0;
             for (int tile = blockIdx.x; tile < args.total_tiles; tile += gridDim.x) {
                 const Tile T = decode_tile(args, tile);
                 // chunks of equal length (at most kChunkBlocks K-blocks each), so
@@ -542,6 +556,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                     // offset), and their accumulators land side by side.
                     const uint32_t idesc = idesc_nb[nb];
                     const uint32_t b_lbo = (N > 64 && nb < PB) ? PB * 64 * 128 : 64 * 128;
+                    const uint64_t db_base = b_mn ? desc_sw128_mn(s0 + C::A_BYTES, b_lbo)
+                                                  : desc_sw128(s0 + C::A_BYTES);
                     for (int c = 0; c < cpp; ++c, ++chunk) {
                         const int buf = chunk % NBUF;
                         if (!mbar_wait(tempty_bar(buf), ((chunk / NBUF) & 1) ^ 1, abort_flag,
@@ -551,27 +567,21 @@ __global__ void __launch_bounds__(kThreads, 1)
                         const uint32_t d = tmem + (uint32_t)(buf * PB * N);
                         const int c0 = T.kb0 + c * csz;
                         const int c1 = min(T.kb1, c0 + csz);
-                        for (int kb = c0; kb < c1; ++kb, ++it) {
-                            const int s = it % S;
-                            if (!mbar_wait(full_bar(s), (it / S) & 1, abort_flag, args.status))
+                        for (int kb = c0; kb < c1; ++kb) {
+                            if (!mbar_wait(full_bar(st), ph, abort_flag, args.status))
                                 goto mma_done;
                             tc_fence_after();
-                            const uint32_t a_addr = smem_u32(smem + s * C::STAGE);
-                            const uint32_t b_addr = a_addr + C::A_BYTES;
-                            // K-major: a K-step of 16 is 32 bytes along each row;
-                            // MN-major: 16 rows, two 1024-byte row groups, and
-                            // 64-wide blocks along M / N 8 KB apart.  Only the
-                            // address field (bytes / 16, below 2^14) moves per step.
-                            constexpr bool a_mn = MODE == TC_WGRAD;
-                            constexpr bool b_mn = MODE == TC_WGRAD || MODE == TC_DGRAD;
-                            const uint64_t da0 = a_mn ? desc_sw128_mn(a_addr, 64 * 128) : desc_sw128(a_addr);
-                            const uint64_t db0 = b_mn ? desc_sw128_mn(b_addr, b_lbo) : desc_sw128(b_addr);
+                            const uint64_t so = (uint64_t)((uint32_t)st * kStageD);
+                            const uint64_t da0 = da_base + so, db0 = db_base + so;
+                            umma_bf16(d, da0, db0, idesc, kb > c0 ? 1u : 0u);
 #pragma unroll
-                            for (int k = 0; k < kBK / 16; ++k)
-                                umma_bf16(d, da0 + (uint64_t)k * (a_mn ? 2048 / 16 : 32 / 16),
-                                          db0 + (uint64_t)k * (b_mn ? 2048 / 16 : 32 / 16), idesc,
-                                          (kb > c0 || k > 0) ? 1u : 0u);
-                            umma_commit(empty_bar(s));
+                            for (int k = 1; k < kBK / 16; ++k)
+                                umma_bf16(d, da0 + k * kStepA, db0 + k * kStepB, idesc, 1u);
+                            umma_commit(empty_bar(st));
+                            if (++st == S) {
+                                st = 0;
+                                ph ^= 1u;
+                            }
                         }
                         umma_commit(tfull_bar(buf));
                     }
