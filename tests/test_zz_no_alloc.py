@@ -100,3 +100,43 @@ def test_noalloc_rejects_sizes_beyond_its_array(torch):
     st = nb.nitro_conv3x3_forward_noalloc(None, None, 64, 32, 32, 64, 64, 0, 10, None, None, None,
                                           nb._stream_ptr(None))
     assert st == nb.NITRO_ERR_ARG
+
+
+def test_noalloc_call_captures_into_a_cuda_graph(torch):
+    # a stream capture in global mode rejects device allocation, so a call
+    # that allocated (or freed) would fail to capture; replays of the captured
+    # call must give the oracle's outputs for whatever input the buffer holds
+    B, h, wd, cin, cout, pool, alpha = 4, 16, 16, 32, 64, 1, 10
+    w = synth.int_tensor(81, (cout, 3, 3, cin), -30000, 30000, dtype=np.int32)
+    wd_dev = torch.from_numpy(w.reshape(-1)).cuda()
+    x = torch.empty((B, h * wd * cin), dtype=torch.int8, device="cuda")
+    oh, ow = h // 2, wd // 2
+    out = torch.empty((B, oh * ow * cout), dtype=torch.int8, device="cuda")
+    region = torch.empty((B, h * wd * cout), dtype=torch.int8, device="cuda")
+    am = torch.empty((B, oh * ow * cout), dtype=torch.int8, device="cuda")
+
+    def call(stream):
+        return nb.nitro_conv3x3_forward_noalloc(nb._ptr(x), nb._ptr(wd_dev), B, h, wd, cin, cout,
+                                                pool, alpha, nb._ptr(out), nb._ptr(region),
+                                                nb._ptr(am), nb._stream_ptr(stream))
+
+    x.copy_(torch.from_numpy(synth.images(12, 0, B, (h, wd, cin)).reshape(B, -1)))
+    assert call(None) == nb.NITRO_OK      # the first call looks the array's address up
+    torch.cuda.synchronize()
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.stream(side):
+        with torch.cuda.graph(graph, stream=side):
+            st = call(side)
+    torch.cuda.current_stream().wait_stream(side)
+    assert st == nb.NITRO_OK, nb.status_str(st)
+    for k in range(1, 3):
+        xh = synth.images(12, k, B, (h, wd, cin)).reshape(B, -1)
+        x.copy_(torch.from_numpy(xh))
+        graph.replay()
+        torch.cuda.synchronize()
+        got = (out.cpu().numpy().reshape(-1), region.cpu().numpy().reshape(-1),
+               am.cpu().numpy().reshape(-1))
+        _same(got, _oracle_forward(xh.astype(np.int64), w.astype(np.int64), B, h, wd, cin, cout,
+                                   pool, alpha), "replay %d vs oracle" % k)
