@@ -54,7 +54,7 @@ typedef enum {
     NITRO_ERR_OVERFLOW = 2,     /* a value did not fit its storage type     */
     NITRO_ERR_TIMEOUT = 3,      /* a bounded device wait gave up            */
     NITRO_ERR_CUDA = 4,         /* a CUDA runtime call failed               */
-    NITRO_ERR_UNSUPPORTED = 5   /* valid but not supported by this build    */
+    NITRO_ERR_UNSUPPORTED = 5   /* valid but not supported by the library   */
 } nitro_status;
 
 typedef enum { NITRO_ROUND_FLOOR = 0, NITRO_ROUND_TRUNC = 1 } nitro_round;
@@ -371,8 +371,8 @@ nitro_status nitro_profile_read(int id, uint64_t* launches, double* ms, double* 
 int nitro_profile_record_count(void);
 nitro_status nitro_profile_record(int i, int* kernel, double* ms, double* ops, double* bytes);
 
-/* Failure-path check of the bounded device waits (SURVEY's TIMEOUT contract;
- * the paper has no counterpart: its failure model is integer overflow).
+/* Failure-path check of the bounded device waits (the library's TIMEOUT
+ * status; the paper has no counterpart: its failure model is integer overflow).
  * Queues on `stream` one CTA that allocates TMEM as the contraction kernels do
  * and waits, through their bounded mbarrier wait, on a barrier that nothing
  * ever completes.  After wait_us microseconds the wait gives up: the kernel
