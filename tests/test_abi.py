@@ -106,6 +106,13 @@ def test_null_handle_calls_are_rejected(lib):
     nb.nitro_destroy_block(None)
     st, _ = nb.nitro_block_tensor_bytes(None, nb.NITRO_T_W, 0)
     assert st == nb.NITRO_ERR_ARG
+    # the entry points added for the folded update, the data-parallel exchange
+    # and the bounded-wait check reject a null handle before any device work
+    assert nb.nitro_block_backward_update(None, None, None, 0, None) == nb.NITRO_ERR_ARG
+    p, n = ctypes.c_void_p(), ctypes.c_size_t()
+    assert lib.nitro_block_grad_device(None, nb.NITRO_T_DW, 0, ctypes.byref(p),
+                                       ctypes.byref(n)) == nb.NITRO_ERR_ARG
+    assert lib.nitro_block_diag_timeout(None, 1000, None) == nb.NITRO_ERR_ARG
 
 
 def test_prep_null_handle_and_bad_sizes_are_rejected(lib):
