@@ -82,6 +82,13 @@ def test_pooled_tensor_core_layers_and_many_classes():
     _run(blocks, 8, steps=3, input_shape=(16, 16, 3), d_lr=128, num_classes=20)
 
 
+def test_learning_pool_with_thirteen_classes():
+    # G = 13: the routing kernel's batched loads for up to 16 classes (G = 10
+    # and G = 20 take the other two forms above)
+    blocks = [_b([(C, 3, 16, 16, 16, 1)], 16 * 16 * 3), _b([], 8 * 8 * 16)]
+    _run(blocks, 6, steps=3, input_shape=(16, 16, 3), d_lr=256, num_classes=13)
+
+
 def test_pooled_block_exposes_window_geometry():
     blk = nb.Block([(C, 4, 16, 16, 16, 1)], 16 * 16 * 4, seed=3, max_batch=2, d_lr=256)
     plain = nb.Block([(C, 4, 16, 16, 16, 1)], 16 * 16 * 4, seed=3, max_batch=2)
